@@ -1,0 +1,419 @@
+#!/usr/bin/env python
+"""Benchmark: batched re-aggregation of streamed fragments by nested ancestry.
+
+Workload (default): the throughput stream -- 16,000,000 fragments, depth 4
+(one source per root, Zipf(1.2) fanout capped at 256 per level), int32
+payloads of 1-64 tokens, 1M-fragment batches, ~18% of the leaf-parent groups
+spanning a batch boundary, concatenation at the leaf-parent level.
+
+One step = the whole stream (16 pushes of 1M fragments, every group completes)
+through the C ABI, then one drain.  Inputs are resident in HBM before the
+timed region; they are far larger than L2 (tags 512 MB, payload 2.1 GB), so no
+flush is needed between steps.  Prints ONE JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the CPU oracle (the plain arrival-order definition) on
+this host's cores over a bounded sample of the same stream; it is the
+baseline arm, not a second implementation of the library.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "fragments/sec and payload GB/s (fraction of HBM peak) at 1 GB300; p50 batch latency"
+UNIT = "fragments/s"
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def stream_caps(s):
+    import numpy as np
+    D, n = s.depth, s.n
+    st = s.batch_starts()
+    pay_b = [int(s.off[st[b + 1]] - s.off[st[b]]) for b in range(s.n_batches)]
+    groups = sum(len(np.unique(s.tags[l] >> np.uint64(32))) for l in range(D))
+    return dict(
+        max_batch_fragments=int(max(s.batch_sizes)),
+        max_batch_payload=max(1, max(pay_b)),
+        max_open_groups=min(1 << 24, groups),
+        arena_elems=min((1 << 32) - 1, 2 * int(s.payload.size) + 4 * n),
+        out_records=groups + 16,
+        out_payload_elems=int(s.payload.size) + 16,
+        out_topk=groups * max(list(s.topk_k) + [1]) + 16,
+        max_emit_children=n + 16,
+    )
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index=0):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def algorithmic_bytes(s):
+    """Bytes the method itself must move for the stream: tags 8D, offsets 4
+    and score 4 per fragment, payload read + write, 48 B per record and 8 B
+    per top-k pair."""
+    import numpy as np
+    D, n = s.depth, s.n
+    groups = sum(len(np.unique(s.tags[l] >> np.uint64(32))) for l in range(D))
+    has_score = s.score is not None
+    topk_pairs = 0  # the default workload has no top-k level
+    return n * (8 * D + 4 + (4 if has_score else 0)) + 8 * int(s.payload.size) + 48 * groups + 8 * topk_pairs
+
+
+def run_reference(args, s, rank, world):
+    """The oracle on host cores, each step a bounded sample of the stream."""
+    import oracle
+    oracle.build()
+    if rank != 0:
+        return None
+    per_step = min(s.n, int(args.ref_sample))
+    st = s.batch_starts()
+    import numpy as np
+    # the first `per_step` fragments of batch 0, as one batch
+    b0 = s.batch(0)
+    n = min(per_step, b0["n"])
+    sample = dict(n=n, tags=np.ascontiguousarray(b0["tags"][:, :n]), off=b0["off"][:n + 1],
+                  payload=b0["payload"][:int(b0["off"][n])],
+                  score=None if b0["score"] is None else b0["score"][:n])
+
+    def step():
+        o = oracle.Oracle.for_stream(s)
+        o.push_batch(sample)
+        d = o.drain()
+        o.close()
+        return d
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    value = n * args.steps / dt
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
+        "data": "synthetic", "config": {"workload": s.name, "fragments": s.n, "depth": s.depth,
+                                        "batch": int(s.batch_sizes[0])},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"first {n} fragments of batch 0 of the {s.name} stream, "
+                                   f"one batch per step, single thread"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    return line
+
+
+def cpu_baseline(s, budget_s=20.0):
+    """Oracle fragments/s on a bounded sample (batches in order until the
+    budget is spent), one host thread."""
+    import oracle
+    oracle.build()
+    o = oracle.Oracle.for_stream(s)
+    done, t0 = 0, time.perf_counter()
+    nb = 0
+    for b in range(s.n_batches):
+        bt = s.batch(b)
+        o.push_batch(bt)
+        o.drain()
+        done += bt["n"]
+        nb += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    o.close()
+    return {"value": done / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"first {nb} batch(es) ({done} fragments) of the {s.name} stream in "
+                      f"arrival order, single thread, {dt:.1f} s"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="throughput")
+    ap.add_argument("--small", action="store_true", help="scaled-down stream (quick checks)")
+    ap.add_argument("--ref-sample", type=float, default=250_000)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--latency-batches", type=int, default=16)
+    args = ap.parse_args()
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    from gen import make_stream
+    s = make_stream(args.workload, small=args.small)
+
+    if args.impl == "reference":
+        line = run_reference(args, s, rank, world)
+        if rank == 0 and line is not None:
+            print(json.dumps(line), flush=True)
+        return
+
+    import numpy as np
+    import torch
+    import paper_2403_04311_gb300 as alto
+
+    torch.cuda.set_device(local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    stream = torch.cuda.current_stream()
+    caps = stream_caps(s)
+    agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, stream=stream, **caps)
+    batches = [alto.to_device(s.batch(b)) for b in range(s.n_batches)]
+    torch.cuda.synchronize()
+
+    def step():
+        for db in batches:
+            st = agg.push(db.tags, db.off, db.payload, db.score)
+            if st != alto.OK:
+                raise RuntimeError(f"push failed: {alto.STATUS_NAMES.get(st, st)}")
+        d = agg.drain()
+        if d.status != alto.OK:
+            raise RuntimeError(f"drain failed: {alto.STATUS_NAMES.get(d.status, d.status)}")
+        return d
+
+    for _ in range(max(args.warmup, 1)):
+        d = step()
+    n_records_step = int(d.records.numel() // 48)
+    n_payload_step = int(d.payload.numel())
+
+    # ---- timed region: device-resident inputs -------------------------------
+    sampler = ClockSampler(local_rank)
+    agg.profile(True)
+    barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for _ in range(args.steps):
+        step()
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clocks = sampler.stop()
+    _st, prof = agg.profile_read()
+    agg.profile(False)
+    ms = t_start.elapsed_time(t_end)
+    if dist is not None:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_per_step = ms / args.steps
+    frags_per_step = s.n
+    value = frags_per_step * world * args.steps / (ms / 1e3)
+    payload_bytes = 8.0 * float(s.payload.size)  # read + write of every token
+    alg_bytes = algorithmic_bytes(s)
+    hbm_gbs, peak_kind = peaks()
+
+    # roofline of the dominant kernel (largest summed device time)
+    stage_ms = prof["stage_ms"]
+    dom = max(stage_ms, key=lambda k: stage_ms[k])
+    pushes = max(1, prof["pushes"])
+    # algorithmic bytes per launch of each single-kernel or byte-defined stage
+    stage_bytes = {
+        "gather": 8.0 * n_payload_step / s.n_batches,
+        "carry_over": None,
+        "ingest": (8.0 * 1 + 8.0 * (s.depth > 1) + 8.0) * s.n / s.n_batches,
+    }
+    if stage_bytes.get(dom) is None:
+        dom_for_roof = "gather"
+    else:
+        dom_for_roof = dom
+    per_launch_ms = stage_ms[dom_for_roof] / pushes
+    achieved = stage_bytes[dom_for_roof] / (per_launch_ms / 1e3) / 1e9 if per_launch_ms > 0 else 0.0
+    traffic = None
+    tf = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tf):
+        try:
+            traffic = json.load(open(tf)).get(dom_for_roof)
+        except Exception:
+            traffic = None
+
+    # ---- end to end: host buffers through the public API ---------------------
+    host = []
+    for b in range(s.n_batches):
+        hb = s.batch(b)
+        host.append({
+            "tags": torch.from_numpy(hb["tags"].view(np.int64)).pin_memory(),
+            "off": torch.from_numpy(hb["off"].view(np.int32)).pin_memory(),
+            "payload": torch.from_numpy(hb["payload"]).pin_memory(),
+            "score": None if hb["score"] is None else torch.from_numpy(hb["score"]).pin_memory(),
+        })
+    dev = [alto.DeviceBatch(n=db.n, tags=torch.empty_like(db.tags), off=torch.empty_like(db.off),
+                            payload=torch.empty_like(db.payload),
+                            score=None if db.score is None else torch.empty_like(db.score))
+           for db in batches]
+    del batches
+    rec_host = torch.empty(n_records_step * 48 + 64, dtype=torch.uint8).pin_memory()
+    pay_host = torch.empty(n_payload_step + 16, dtype=torch.int32).pin_memory()
+    h2d = sum(h["tags"].numel() * 8 + h["off"].numel() * 4 + h["payload"].numel() * 4 +
+              (h["score"].numel() * 4 if h["score"] is not None else 0) for h in host)
+
+    def e2e_step():
+        for hb, db in zip(host, dev):
+            db.tags.copy_(hb["tags"], non_blocking=True)
+            db.off.copy_(hb["off"], non_blocking=True)
+            db.payload.copy_(hb["payload"], non_blocking=True)
+            if hb["score"] is not None:
+                db.score.copy_(hb["score"], non_blocking=True)
+            st = agg.push(db.tags, db.off, db.payload, db.score)
+            if st != alto.OK:
+                raise RuntimeError(f"push failed: {st}")
+        d = agg.drain()
+        nr = d.records.numel()
+        npay = d.payload.numel()
+        rec_host[:nr].copy_(d.records, non_blocking=True)
+        pay_host[:npay].copy_(d.payload, non_blocking=True)
+        torch.cuda.synchronize()
+        return nr + npay * 4
+
+    e2e_step()
+    barrier()
+    torch.cuda.synchronize()
+    e_start = torch.cuda.Event(enable_timing=True)
+    e_end = torch.cuda.Event(enable_timing=True)
+    e_steps = max(1, min(args.steps, 5))
+    e_start.record(stream)
+    d2h = 0
+    for _ in range(e_steps):
+        d2h = e2e_step()
+    e_end.record(stream)
+    torch.cuda.synchronize()
+    e_ms = e_start.elapsed_time(e_end)
+    if dist is not None:
+        t = torch.tensor([e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e_ms = float(t.item())
+    e2e_value = frags_per_step * world * e_steps / (e_ms / 1e3)
+
+    # ---- per-batch latency: push + drain, host clock -------------------------
+    lat = []
+    for hb_i in range(min(args.latency_batches, 2 * s.n_batches)):
+        db = dev[hb_i % len(dev)]
+        t0 = time.perf_counter()
+        agg.push(db.tags, db.off, db.payload, db.score)
+        agg.drain()
+        lat.append((time.perf_counter() - t0) * 1e6)
+    lat_s = sorted(lat)
+    p50 = lat_s[len(lat_s) // 2]
+    p99 = lat_s[min(len(lat_s) - 1, int(0.99 * len(lat_s)))]
+    agg.close()
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        cpu = cpu_baseline(s)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+        "config": {"workload": s.name, "fragments": s.n, "depth": s.depth,
+                   "batch": int(s.batch_sizes[0]), "payload_tokens": int(s.payload.size),
+                   "span_fraction": s.meta.get("span_fraction"),
+                   "l2": "inputs larger than L2 (no flush)", "parallelism": f"replicas x{world}"},
+        "payload_gbps": payload_bytes * world * args.steps / (ms / 1e3) / 1e9,
+        "algorithmic_gbps": alg_bytes * world * args.steps / (ms / 1e3) / 1e9,
+        "hbm_frac_path": alg_bytes * args.steps / (ms / 1e3) / 1e9 / hbm_gbs,
+        "p50_batch_latency_us": p50, "p99_batch_latency_us": p99,
+        "roofline": {"bound": "hbm", "kernel": dom_for_roof, "dominant_stage": dom,
+                     "achieved": achieved, "peak": hbm_gbs, "unit": "GB/s",
+                     "frac": achieved / hbm_gbs, "peak_kind": peak_kind, "traffic": traffic},
+        "stage_ms_per_step": {k: v / args.steps for k, v in stage_ms.items()},
+        "gpu_launches": int(prof["launches"]),
+        "clocks": clocks,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(d2h)},
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

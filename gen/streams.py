@@ -34,6 +34,8 @@ scaled-down stream with the same structure.
 from __future__ import annotations
 
 import heapq
+import os
+from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass, field
 
 import numpy as np
@@ -47,6 +49,28 @@ S_NONE, S_MAX, S_TOPK = 0, 1, 2
 CONFIG_NAMES = ("tiny", "tiny64", "factcheck", "throughput", "tokens", "adversarial")
 
 _U32 = np.uint64(0xFFFFFFFF)
+
+
+_CHUNK = 1 << 24
+
+
+def _integers(rng, low, high, size, dtype=np.int32):
+    """Uniform integers drawn in parallel chunks from child seed sequences of
+    one seed drawn from ``rng`` (deterministic, independent of thread count)."""
+    if size <= _CHUNK:
+        return rng.integers(low, high, size=size, dtype=dtype)
+    seed = int(rng.integers(0, 2**63))
+    n_chunks = (size + _CHUNK - 1) // _CHUNK
+    children = np.random.SeedSequence(seed).spawn(n_chunks)
+    out = np.empty(size, dtype=dtype)
+
+    def fill(k):
+        a, b = k * _CHUNK, min(size, (k + 1) * _CHUNK)
+        out[a:b] = np.random.default_rng(children[k]).integers(low, high, size=b - a, dtype=dtype)
+
+    with ThreadPoolExecutor(max_workers=min(n_chunks, os.cpu_count() or 1)) as ex:
+        list(ex.map(fill, range(n_chunks)))
+    return out
 
 
 def pack_tags(pid, child, last):
@@ -169,13 +193,17 @@ def stream_from_leaves(name, gidx, cidx, order, lens, rng, *, payload_op, score_
     D = len(gidx)
     flags = _last_flags(gidx, cidx)
     tags = np.empty((D, len(order)), dtype=np.uint64)
-    for l in range(D):
-        ids = _ids(rng, int(gidx[l].max()) + 1 if len(gidx[l]) else 1)
-        tags[l] = pack_tags(ids[gidx[l][order]], cidx[l][order], flags[l][order])
+    id_tables = [_ids(rng, int(gidx[l].max()) + 1 if len(gidx[l]) else 1) for l in range(D)]
+
+    def level(l):
+        tags[l] = pack_tags(id_tables[l][gidx[l][order]], cidx[l][order], flags[l][order])
+
+    with ThreadPoolExecutor(max_workers=D) as ex:
+        list(ex.map(level, range(D)))
     lens = np.asarray(lens, dtype=np.int64)[order]
     off = np.zeros(len(order) + 1, dtype=np.int64)
     np.cumsum(lens, out=off[1:])
-    payload = rng.integers(0, TOKEN_VOCAB, size=int(off[-1]), dtype=np.int32)
+    payload = _integers(rng, 0, TOKEN_VOCAB, int(off[-1]))
     score = rng.standard_normal(len(order), dtype=np.float32) if with_score else None
     n = len(order)
     nb = n // batch
@@ -297,8 +325,8 @@ def make_throughput(n_leaves=16_000_000, seed=3, batch=1_000_000, target_span=0.
     R = int(root.max()) + 1
     root_sizes = np.bincount(root, minlength=R)
     # random order of leaves inside each root
-    u = rng.random(n)
-    within = np.lexsort((u, root))
+    u = rng.integers(0, 2**32, size=n, dtype=np.uint64)
+    within = np.argsort((root.astype(np.uint64) << np.uint64(32)) | u, kind="stable")
     rank_in_root = np.empty(n, dtype=np.int64)
     rstart = np.cumsum(root_sizes) - root_sizes
     rank_in_root[within] = np.arange(n, dtype=np.int64) - rstart[root[within]]

@@ -1,0 +1,240 @@
+/*
+ * alto_agg -- batched re-aggregation of streamed fragments by nested ancestry
+ * on one GPU (NVIDIA GB300, sm_103a).
+ *
+ * The operation follows Alto (arxiv 2403.04311):
+ *   - Sec. 4.2: every parallel-map (pmap) entry pushes one ancestry tag on
+ *     each element -- the id of the parent element and the element's index in
+ *     the parent's stream -- and every pmap exit pops one tag and aggregates
+ *     the outputs of that call.  A fragment therefore carries D tags, one per
+ *     nesting level, outermost first.
+ *   - Sec. 3.1: a stream is known to be complete only when its end-of-output
+ *     delimiter arrives.  Here the delimiter is the last-flag bit on the tag of
+ *     the stream's final child.
+ *   - Sec. 3.2 / Sec. 4.1: the outputs of a pmap are reconstituted in the
+ *     original stream order.  Sec. 3.3: an aggregate operator collects one
+ *     stream's items into one output object.  Sec. 4.3: all elements with the
+ *     same ancestry are routed to the same aggregation point.
+ *
+ * Data model.  Tag l of a fragment is packed into a u64 as
+ *     parent_id << 32 | last << 31 | child_index        (child_index < 2^31)
+ * The fragment is child `child_index` of group (l, parent_id).  For l < D-1
+ * that child is the group (l+1, parent_id of tag l+1); for l = D-1 the child
+ * is the fragment itself (a leaf, complete on arrival).  parent_ids are unique
+ * per level over the aggregator's lifetime, and a group always sits under the
+ * same tag one level up.  A group is complete when some child carries the
+ * last flag (index `last`), every child 0..last is present, and every child is
+ * complete.  Completed groups are emitted, at every level, as one record each:
+ *   - CONCAT (at most one level M): the payloads of the subtree's leaves
+ *     concatenated in child-index path order;
+ *   - MAX: the record's score is the largest leaf score of the subtree;
+ *   - TOPK(k): also the k children with the largest score (a child's score is
+ *     the largest leaf score of its subtree), ties to the smaller child index.
+ * Scores are compared under IEEE-754 totalOrder (-0.0 < +0.0); NaN is
+ * rejected.  Groups with no operation still emit a record (empty payload).
+ *
+ * Emission order.  Within a push, records come in (completion_seq ascending,
+ * level descending) order, where completion_seq is the global arrival index of
+ * the fragment that completed the group (the largest arrival index in its
+ * subtree).  Records of successive pushes follow one another.  Batches are
+ * taken in push order; fragments of a batch in array order.
+ *
+ * Streams.  Every call takes a CUDA stream (a cudaStream_t passed as void*).
+ * push_batch only enqueues work; drain is the only call that synchronises.
+ * Device buffers passed to push_batch are borrowed until the work enqueued on
+ * that stream has completed, exactly like cudaMemcpyAsync.  A handle is not
+ * thread-safe.
+ *
+ * Errors.  Every call returns an alto_status.  Argument errors found on the
+ * host are returned at once and leave the handle usable.  Errors found on the
+ * device are latched: the first batch with an error poisons the handle, the
+ * next drain returns the error (with no records), and every later call
+ * returns it too; destroy still succeeds.  When one batch holds several
+ * defects the reported class is the first of EINVAL, EDUP, EINCONSIST, ELAST,
+ * ENOSPC, ETIMEOUT.  Device detection covers: offsets that decrease or end
+ * beyond n_payload, NaN scores (EINVAL); a leaf (group, child index) given
+ * twice in one batch, and -- for CONCAT groups -- a repeated or missing child
+ * found when the group completes (EDUP); a group seen under two different
+ * parent tags, or two different child groups in one slot within one batch
+ * (EINCONSIST); two different last children, or a child index above the last
+ * (ELAST); table, arena or output capacity exceeded (ENOSPC); a device-side
+ * wait that ran past its iteration cap (ETIMEOUT).  Inputs outside that scope
+ * (for example a fragment for a group that was already emitted) give
+ * undefined records but never a fault or a hang.
+ */
+#ifndef ALTO_AGG_H
+#define ALTO_AGG_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int alto_status;
+
+#define ALTO_OK 0
+#define ALTO_EINVAL (-1)     /* bad argument, offsets or NaN score */
+#define ALTO_ENOMEM (-2)     /* device allocation failed */
+#define ALTO_ENOSPC (-3)     /* table, arena or output capacity exceeded */
+#define ALTO_EDUP (-4)       /* the same leaf slot given twice */
+#define ALTO_ELAST (-5)      /* conflicting last child, or a child past it */
+#define ALTO_EINCONSIST (-6) /* a group under two parent tags / a slot with two children */
+#define ALTO_ECLOSED (-7)    /* fragment for an emitted group (not detected on the device) */
+#define ALTO_ETIMEOUT (-8)   /* a device-side wait hit its iteration cap */
+#define ALTO_ECUDA (-9)      /* a CUDA runtime call failed */
+
+#define ALTO_MAX_DEPTH 8
+#define ALTO_MAX_TOPK 32
+
+#define ALTO_PAYLOAD_NONE 0
+#define ALTO_PAYLOAD_CONCAT 1
+#define ALTO_SCORE_NONE 0
+#define ALTO_SCORE_MAX 1
+#define ALTO_SCORE_TOPK 2
+
+/* Aggregator configuration (Sec. 5: the controller is told which queues are
+ * pmap entry/exit points and which data is aggregated; here: the nesting
+ * depth and what each level's exit computes).  Zero capacities take the
+ * defaults noted. */
+typedef struct alto_agg_config {
+  int32_t depth;                          /* D, number of tags, 1..8 */
+  int32_t payload_op[ALTO_MAX_DEPTH];     /* per level: NONE or CONCAT (at most one level) */
+  int32_t score_op[ALTO_MAX_DEPTH];       /* per level: NONE, MAX or TOPK */
+  int32_t topk_k[ALTO_MAX_DEPTH];         /* per TOPK level: 1..32 */
+  int64_t max_batch_fragments;            /* largest n of one push (required, < 2^30) */
+  int64_t max_batch_payload;              /* largest n_payload of one push (required) */
+  int64_t max_open_groups;                /* groups alive at once (default 2^20) */
+  int64_t arena_elems;                    /* int32 elements buffered for open CONCAT groups (default 2^26) */
+  int64_t out_records;                    /* records held between drains (default 4*max_batch_fragments) */
+  int64_t out_payload_elems;              /* payload elements held between drains (default 4*max_batch_payload) */
+  int64_t out_topk;                       /* top-k pairs held between drains (default out_records) */
+  int64_t max_emit_children;              /* children of CONCAT groups completing in one push (default 4*max_batch_fragments) */
+  int64_t spin_limit;                     /* device wait cap in polls (default 2^20) */
+} alto_agg_config;
+
+/* Device memory provider.  alloc returns device memory of at least `bytes`
+ * usable on `stream` (or NULL); free releases it.  A NULL allocator means
+ * cudaMallocAsync / cudaFreeAsync on the given stream. */
+typedef struct alto_allocator {
+  void* ctx;
+  void* (*alloc)(void* ctx, size_t bytes, void* stream);
+  void (*free)(void* ctx, void* ptr, void* stream);
+} alto_allocator;
+
+/* One batch of fragments, all pointers to device memory.
+ *   tags        [depth][n] u64, level-major: tag l of fragment i at tags[l*n + i]
+ *   payload_off [n+1] u32 element offsets into payload; fragment i's payload is
+ *               payload[payload_off[i] .. payload_off[i+1]); must not decrease,
+ *               and payload_off[n] <= n_payload
+ *   payload     [n_payload] int32 tokens
+ *   score       [n] f32, required iff some level has a score op, else ignored */
+typedef struct alto_batch {
+  int64_t n;
+  int32_t depth;
+  int32_t reserved;
+  const uint64_t* tags;
+  const uint32_t* payload_off;
+  int64_t n_payload;
+  const int32_t* payload;
+  const float* score;
+} alto_batch;
+
+/* One completed group (48 bytes).  payload_off / topk_off index the drain's
+ * payload and top-k arrays.  score is the subtree's largest leaf score for
+ * levels with a score op, else 0.  ops = payload_op | score_op << 2. */
+typedef struct alto_record {
+  uint64_t completion_seq;
+  uint64_t payload_off;
+  uint64_t payload_len;
+  uint64_t topk_off;
+  uint32_t parent_id;
+  uint32_t n_children;
+  uint8_t level;
+  uint8_t ops;
+  uint16_t topk_n;
+  float score;
+} alto_record;
+
+/* A selected child: best score first, ties to the smaller child index. */
+typedef struct alto_topk_pair {
+  uint32_t child_index;
+  float score;
+} alto_topk_pair;
+
+/* Everything completed since the previous drain.  All pointers are device
+ * memory owned by the handle, valid until the next push, drain or destroy. */
+typedef struct alto_drain {
+  int64_t n_records;
+  const alto_record* records;
+  int64_t n_payload;
+  const int32_t* payload;
+  int64_t n_topk;
+  const alto_topk_pair* topk;
+  uint64_t first_batch;   /* index of the first batch pushed since the previous drain */
+  uint64_t n_batches;     /* batches pushed since the previous drain */
+} alto_drain;
+
+typedef struct alto_agg alto_agg_t;
+
+/* Sec. 5 (the controller handles pmap tracking): allocate the open-group
+ * table, the arena, scratch and the output ring for `cfg` through `alloc`
+ * (NULL: cudaMallocAsync on `stream`), and return the handle in *out.
+ * Errors: EINVAL (bad config; *out untouched), ENOMEM, ECUDA. */
+alto_status alto_agg_create(const alto_agg_config* cfg, const alto_allocator* alloc,
+                            void* stream, alto_agg_t** out);
+
+/* Sec. 4.2-4.3: route the batch's fragments to their groups by ancestry,
+ * merge them with the groups left open by earlier batches, decide completion
+ * level by level, and append the records of every group completed by this
+ * batch to the handle's output ring (Sec. 3.3).  Enqueues on `stream`, never
+ * synchronises.  n = 0 is a no-op batch.  Host-side errors (returned at once,
+ * handle still usable): EINVAL for a NULL handle or batch, depth mismatch,
+ * n < 0 or n > max_batch_fragments, n_payload outside 0..max_batch_payload,
+ * NULL tags/offsets with n > 0, NULL payload with n_payload > 0, NULL score
+ * when a score op is configured.  A latched device error is returned as is. */
+alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream);
+
+/* Synchronise `stream` and return, in *out, every record completed since the
+ * previous drain (Sec. 3.3 aggregate output), in emission order, with its
+ * payload and top-k pairs.  Returns the latched status; after an error *out
+ * holds no records. */
+alto_status alto_agg_drain(alto_agg_t* h, void* stream, alto_drain* out);
+
+/* Open groups and buffered arena elements right now (synchronises stream). */
+alto_status alto_agg_stats(alto_agg_t* h, void* stream, int64_t* open_groups,
+                           int64_t* arena_elems_used);
+
+/* Measurement hooks.  The paper has no counterpart: they exist so that the
+ * benchmark can time the pipeline's stages on the device while it runs.
+ * With profiling on, every push records a CUDA event at each stage boundary
+ * on its stream; alto_agg_profile_read synchronises the handle's last push
+ * stream and sums the elapsed times.  Stages, in push order:
+ *   0 ingest (validate, table lookup, leaf-slot check)   1 leaf sort
+ *   2 leaf segments + reduce                             3 upper levels
+ *   4 emission order + offsets                            5 arena carry-over
+ *   6 dense child placement + length scan                 7 payload gather
+ *   8 records, frees, table sweep
+ * `launches` counts every kernel the pushes launched (also when profiling is
+ * off).  enable = 1 starts a fresh count, 0 stops recording events. */
+#define ALTO_NUM_STAGES 9
+typedef struct alto_profile {
+  int64_t pushes;                          /* pushes since the last enable */
+  int64_t launches;                        /* kernels those pushes launched */
+  double stage_ms[ALTO_NUM_STAGES];        /* summed device time per stage */
+  int64_t stage_launches[ALTO_NUM_STAGES]; /* kernels per stage, summed */
+} alto_profile;
+
+alto_status alto_agg_profile(alto_agg_t* h, int enable);
+alto_status alto_agg_profile_read(alto_agg_t* h, alto_profile* out);
+
+/* Free everything the handle owns; open groups are discarded.  NULL is OK.
+ * Always succeeds on a valid or poisoned handle. */
+alto_status alto_agg_destroy(alto_agg_t* h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ALTO_AGG_H */

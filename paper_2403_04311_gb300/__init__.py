@@ -1,0 +1,16 @@
+"""GB300-native re-aggregation of streamed fragments by nested ancestry.
+
+The hot path (Alto, arxiv 2403.04311, Sec. 3.1-4.3) is a CUDA library for
+sm_103a behind a four-call C ABI (``include/alto_agg.h``); this package builds
+it in-tree and binds it with ctypes.  There is no CPU implementation here.
+"""
+from ._binding import (  # noqa: F401
+    EXPORTS, OK, EINVAL, ENOMEM, ENOSPC, EDUP, ELAST, EINCONSIST, ECLOSED, ETIMEOUT, ECUDA,
+    STATUS_NAMES, PAYLOAD_NONE, PAYLOAD_CONCAT, SCORE_NONE, SCORE_MAX, SCORE_TOPK,
+    RECORD_DTYPE, PAIR_DTYPE, Aggregator, Drain, alto_agg_config, alto_allocator, alto_batch,
+    alto_drain, alto_agg_create, alto_agg_push_batch, alto_agg_drain, alto_agg_stats,
+    alto_agg_destroy, alto_agg_profile, alto_agg_profile_read, load_library, make_config,
+    STAGE_NAMES,
+)
+from ._build import build  # noqa: F401
+from .device_batches import DeviceBatch, to_device  # noqa: F401

@@ -1,0 +1,305 @@
+"""ctypes binding of the alto_agg C ABI (include/alto_agg.h).
+
+Argument marshalling only: every step of the aggregation runs in the CUDA
+library.  PyTorch supplies device memory (its caching allocator, through the
+ABI's allocator callbacks) and streams.  Loading fails loudly when the
+compiled library is missing -- there is no other implementation to fall back
+to.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import numpy as np
+
+from . import _build
+
+MAX_DEPTH = 8
+OK, EINVAL, ENOMEM, ENOSPC, EDUP, ELAST, EINCONSIST, ECLOSED, ETIMEOUT, ECUDA = (
+    0, -1, -2, -3, -4, -5, -6, -7, -8, -9)
+STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ENOMEM: "ENOMEM", ENOSPC: "ENOSPC", EDUP: "EDUP",
+                ELAST: "ELAST", EINCONSIST: "EINCONSIST", ECLOSED: "ECLOSED",
+                ETIMEOUT: "ETIMEOUT", ECUDA: "ECUDA"}
+PAYLOAD_NONE, PAYLOAD_CONCAT = 0, 1
+SCORE_NONE, SCORE_MAX, SCORE_TOPK = 0, 1, 2
+
+RECORD_DTYPE = np.dtype([
+    ("completion_seq", "<u8"), ("payload_off", "<u8"), ("payload_len", "<u8"),
+    ("topk_off", "<u8"), ("parent_id", "<u4"), ("n_children", "<u4"),
+    ("level", "u1"), ("ops", "u1"), ("topk_n", "<u2"), ("score", "<f4"),
+])
+PAIR_DTYPE = np.dtype([("child_index", "<u4"), ("score", "<f4")])
+
+
+class alto_agg_config(ctypes.Structure):
+    _fields_ = [
+        ("depth", ctypes.c_int32),
+        ("payload_op", ctypes.c_int32 * MAX_DEPTH),
+        ("score_op", ctypes.c_int32 * MAX_DEPTH),
+        ("topk_k", ctypes.c_int32 * MAX_DEPTH),
+        ("max_batch_fragments", ctypes.c_int64),
+        ("max_batch_payload", ctypes.c_int64),
+        ("max_open_groups", ctypes.c_int64),
+        ("arena_elems", ctypes.c_int64),
+        ("out_records", ctypes.c_int64),
+        ("out_payload_elems", ctypes.c_int64),
+        ("out_topk", ctypes.c_int64),
+        ("max_emit_children", ctypes.c_int64),
+        ("spin_limit", ctypes.c_int64),
+    ]
+
+
+ALLOC_FN = ctypes.CFUNCTYPE(ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p)
+FREE_FN = ctypes.CFUNCTYPE(None, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p)
+
+
+class alto_allocator(ctypes.Structure):
+    _fields_ = [("ctx", ctypes.c_void_p), ("alloc", ALLOC_FN), ("free", FREE_FN)]
+
+
+class alto_batch(ctypes.Structure):
+    _fields_ = [
+        ("n", ctypes.c_int64), ("depth", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("tags", ctypes.c_void_p), ("payload_off", ctypes.c_void_p),
+        ("n_payload", ctypes.c_int64), ("payload", ctypes.c_void_p), ("score", ctypes.c_void_p),
+    ]
+
+
+class alto_drain(ctypes.Structure):
+    _fields_ = [
+        ("n_records", ctypes.c_int64), ("records", ctypes.c_void_p),
+        ("n_payload", ctypes.c_int64), ("payload", ctypes.c_void_p),
+        ("n_topk", ctypes.c_int64), ("topk", ctypes.c_void_p),
+        ("first_batch", ctypes.c_uint64), ("n_batches", ctypes.c_uint64),
+    ]
+
+
+NUM_STAGES = 9
+STAGE_NAMES = ("ingest", "leaf_sort", "leaf_reduce", "upper_levels", "emit_order", "carry_over",
+               "dense_place", "gather", "records")
+
+
+class alto_profile(ctypes.Structure):
+    _fields_ = [("pushes", ctypes.c_int64), ("launches", ctypes.c_int64),
+                ("stage_ms", ctypes.c_double * NUM_STAGES),
+                ("stage_launches", ctypes.c_int64 * NUM_STAGES)]
+
+
+EXPORTS = ("alto_agg_create", "alto_agg_push_batch", "alto_agg_drain", "alto_agg_stats",
+           "alto_agg_profile", "alto_agg_profile_read", "alto_agg_destroy")
+
+_lib = None
+
+
+def load_library(build: bool = True):
+    """Load (building first if needed) libalto_agg.so."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.build() if build else _build.LIB
+    if not os.path.exists(path):
+        raise RuntimeError(f"alto_agg CUDA library missing at {path}; run the package build")
+    lib = ctypes.CDLL(path)
+    P = ctypes.c_void_p
+    lib.alto_agg_create.restype = ctypes.c_int
+    lib.alto_agg_create.argtypes = [ctypes.POINTER(alto_agg_config), ctypes.POINTER(alto_allocator),
+                                    P, ctypes.POINTER(P)]
+    lib.alto_agg_push_batch.restype = ctypes.c_int
+    lib.alto_agg_push_batch.argtypes = [P, ctypes.POINTER(alto_batch), P]
+    lib.alto_agg_drain.restype = ctypes.c_int
+    lib.alto_agg_drain.argtypes = [P, P, ctypes.POINTER(alto_drain)]
+    lib.alto_agg_stats.restype = ctypes.c_int
+    lib.alto_agg_stats.argtypes = [P, P, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
+    lib.alto_agg_destroy.restype = ctypes.c_int
+    lib.alto_agg_destroy.argtypes = [P]
+    lib.alto_agg_profile.restype = ctypes.c_int
+    lib.alto_agg_profile.argtypes = [P, ctypes.c_int]
+    lib.alto_agg_profile_read.restype = ctypes.c_int
+    lib.alto_agg_profile_read.argtypes = [P, ctypes.POINTER(alto_profile)]
+    _lib = lib
+    return lib
+
+
+def make_config(depth, payload_op, score_op, topk_k=None, *, max_batch_fragments,
+                max_batch_payload, max_open_groups=0, arena_elems=0, out_records=0,
+                out_payload_elems=0, out_topk=0, max_emit_children=0, spin_limit=0):
+    c = alto_agg_config()
+    c.depth = depth
+    topk_k = topk_k or [0] * depth
+    for l in range(min(depth, MAX_DEPTH)):
+        c.payload_op[l] = int(payload_op[l])
+        c.score_op[l] = int(score_op[l])
+        c.topk_k[l] = int(topk_k[l])
+    c.max_batch_fragments = int(max_batch_fragments)
+    c.max_batch_payload = int(max_batch_payload)
+    c.max_open_groups = int(max_open_groups)
+    c.arena_elems = int(arena_elems)
+    c.out_records = int(out_records)
+    c.out_payload_elems = int(out_payload_elems)
+    c.out_topk = int(out_topk)
+    c.max_emit_children = int(max_emit_children)
+    c.spin_limit = int(spin_limit)
+    return c
+
+
+class _TorchAllocator:
+    """The ABI allocator callbacks backed by PyTorch's caching allocator."""
+
+    def __init__(self, device):
+        import torch
+        self._torch = torch
+        self._device = device
+
+        def _alloc(_ctx, nbytes, stream):
+            return self._torch.cuda.caching_allocator_alloc(int(nbytes), self._device,
+                                                            int(stream or 0))
+
+        def _free(_ctx, ptr, _stream):
+            if ptr:
+                self._torch.cuda.caching_allocator_delete(int(ptr))
+
+        self._alloc = ALLOC_FN(_alloc)
+        self._free = FREE_FN(_free)
+        self.struct = alto_allocator(None, self._alloc, self._free)
+
+
+def alto_agg_create(cfg: alto_agg_config, allocator=None, stream=0):
+    """Returns (status, handle).  ``allocator`` is an alto_allocator struct,
+    a _TorchAllocator, or None (library uses cudaMallocAsync)."""
+    lib = load_library()
+    h = ctypes.c_void_p()
+    a = allocator.struct if isinstance(allocator, _TorchAllocator) else allocator
+    st = lib.alto_agg_create(ctypes.byref(cfg), ctypes.byref(a) if a is not None else None,
+                             ctypes.c_void_p(stream), ctypes.byref(h))
+    return st, h
+
+
+def alto_agg_push_batch(h, batch: alto_batch, stream=0) -> int:
+    return load_library().alto_agg_push_batch(h, ctypes.byref(batch), ctypes.c_void_p(stream))
+
+
+def alto_agg_drain(h, stream=0):
+    d = alto_drain()
+    st = load_library().alto_agg_drain(h, ctypes.c_void_p(stream), ctypes.byref(d))
+    return st, d
+
+
+def alto_agg_stats(h, stream=0):
+    og, au = ctypes.c_int64(), ctypes.c_int64()
+    st = load_library().alto_agg_stats(h, ctypes.c_void_p(stream), ctypes.byref(og), ctypes.byref(au))
+    return st, og.value, au.value
+
+
+def alto_agg_destroy(h) -> int:
+    return load_library().alto_agg_destroy(h)
+
+
+def alto_agg_profile(h, enable: bool) -> int:
+    return load_library().alto_agg_profile(h, 1 if enable else 0)
+
+
+def alto_agg_profile_read(h):
+    p = alto_profile()
+    st = load_library().alto_agg_profile_read(h, ctypes.byref(p))
+    return st, dict(pushes=p.pushes, launches=p.launches,
+                    stage_ms={STAGE_NAMES[i]: p.stage_ms[i] for i in range(NUM_STAGES)},
+                    stage_launches={STAGE_NAMES[i]: p.stage_launches[i] for i in range(NUM_STAGES)})
+
+
+class _DevView:
+    """A raw device buffer exposed through __cuda_array_interface__."""
+
+    def __init__(self, ptr, nbytes):
+        self.__cuda_array_interface__ = {
+            "shape": (int(nbytes),), "typestr": "|u1", "data": (int(ptr), False), "version": 3,
+        }
+
+
+@dataclass
+class Drain:
+    status: int
+    records: object   # torch uint8 tensor (device) of n_records * 48 bytes
+    payload: object   # torch int32 tensor (device)
+    topk: object      # torch uint8 tensor (device) of n_topk * 8 bytes
+    first_batch: int
+    n_batches: int
+
+    def host(self):
+        """(records as RECORD_DTYPE, payload int32, topk as PAIR_DTYPE) numpy copies."""
+        rec = self.records.cpu().numpy().view(RECORD_DTYPE) if self.records is not None else \
+            np.zeros(0, RECORD_DTYPE)
+        pay = self.payload.cpu().numpy() if self.payload is not None else np.zeros(0, np.int32)
+        tk = self.topk.cpu().numpy().view(PAIR_DTYPE) if self.topk is not None else \
+            np.zeros(0, PAIR_DTYPE)
+        return rec, pay, tk
+
+
+class Aggregator:
+    """Owning wrapper around one alto_agg handle on the current CUDA device."""
+
+    def __init__(self, depth, payload_op, score_op, topk_k=None, *, max_batch_fragments,
+                 max_batch_payload, stream=None, use_torch_allocator=True, **caps):
+        import torch
+        self._torch = torch
+        self.depth = depth
+        self.has_score = any(s != SCORE_NONE for s in score_op)
+        self.stream = stream if stream is not None else torch.cuda.current_stream()
+        self._alloc = _TorchAllocator(torch.cuda.current_device()) if use_torch_allocator else None
+        self.cfg = make_config(depth, payload_op, score_op, topk_k,
+                               max_batch_fragments=max_batch_fragments,
+                               max_batch_payload=max_batch_payload, **caps)
+        st, self._h = alto_agg_create(self.cfg, self._alloc, self.stream.cuda_stream)
+        if st != OK:
+            raise RuntimeError(f"alto_agg_create failed: {STATUS_NAMES.get(st, st)}")
+
+    def push(self, tags, off, payload, score=None, n=None) -> int:
+        """tags: uint64-valued int64 CUDA tensor (D, n) contiguous; off: int32
+        (n+1,) holding u32 offsets; payload: int32; score: float32 or None."""
+        b = alto_batch()
+        b.n = int(tags.shape[-1]) if n is None else int(n)
+        b.depth = self.depth
+        b.tags = tags.data_ptr()
+        b.payload_off = off.data_ptr()
+        b.n_payload = int(payload.numel())
+        b.payload = payload.data_ptr() if payload.numel() else None
+        b.score = score.data_ptr() if score is not None else None
+        return alto_agg_push_batch(self._h, b, self.stream.cuda_stream)
+
+    def drain(self) -> Drain:
+        st, d = alto_agg_drain(self._h, self.stream.cuda_stream)
+        torch = self._torch
+
+        def view(ptr, nbytes, dtype):
+            if not ptr or nbytes == 0:
+                return torch.zeros(0, dtype=dtype, device="cuda")
+            t = torch.as_tensor(_DevView(ptr, nbytes), device="cuda")
+            return t.view(dtype) if dtype != torch.uint8 else t
+
+        if st != OK:
+            return Drain(st, None, None, None, int(d.first_batch), int(d.n_batches))
+        return Drain(st, view(d.records, d.n_records * 48, torch.uint8),
+                     view(d.payload, d.n_payload * 4, torch.int32),
+                     view(d.topk, d.n_topk * 8, torch.uint8), int(d.first_batch),
+                     int(d.n_batches))
+
+    def stats(self):
+        return alto_agg_stats(self._h, self.stream.cuda_stream)
+
+    def profile(self, enable: bool) -> int:
+        return alto_agg_profile(self._h, enable)
+
+    def profile_read(self):
+        return alto_agg_profile_read(self._h)
+
+    def close(self):
+        if getattr(self, "_h", None):
+            alto_agg_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,1423 @@
+// alto_agg: batched re-aggregation of streamed fragments by nested ancestry
+// (Alto, arxiv 2403.04311, Sec. 3.1-4.3) on one GB300 GPU.
+//
+// One push runs this stream-ordered pipeline (no host synchronisation):
+//   ingest      validate offsets/scores; find-or-insert each fragment's
+//               leaf-parent group (level D-1) in the open-group hash table;
+//               flag a leaf slot given twice in the batch              [Sec. 4.2]
+//   sort        stable onesweep radix sort of fragments by table slot      [Sec. 4.3]
+//   segments    decoupled look-back scan finds each group's run
+//   reduce      one warp per group: count complete children, last-flag and
+//               child-index checks, ancestry consistency, max score, top-k;
+//               merge with the table entry and test completion          [Sec. 3.1]
+//   levels      the groups present at level l become the items of level l-1:
+//               table lookup, sort, segments, reduce again, up to level 0 [Sec. 4.2]
+//   emit order  completed groups ranked by (completion seq, deeper first)
+//   CONCAT      open groups: append their leaves to per-group arena vectors;
+//               completing groups: place every child span at slot
+//               dense_base + child_index, scan the lengths, gather the spans
+//               into the output payload ring                     [Sec. 3.2, 3.3]
+//   records     one record per completed group, top-k pairs; free entries
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "alto_agg.h"
+#include "common.cuh"
+#include "kernels.h"
+#include "scan.cuh"
+
+namespace alto {
+
+constexpr int kThreads = 256;
+
+struct Batch {
+  const u64* tags;
+  const u32* off;
+  const int32_t* pay;
+  const float* score;
+  u32 n;
+  u64 n_payload;
+};
+
+struct Scratch {
+  u32* leaf_sort_keys0;  // ingest writes the table slot of each fragment here
+  u32* up_sort_keys0;    // item lookups write here
+  u32* leaf_keys;        // sorted leaf keys (set by the host after the sort)
+  u32* leaf_perm;
+  u32* leaf_seg_start;   // [n_max + 1]
+  u32* leaf_seg_of;      // [n_max]
+  u32* up_keys;
+  u32* up_perm;
+  u32* up_seg_start;     // [n_max + 1]
+  u32* it_rep[2];        // items: representative fragment
+  u32* it_cseq[2];       // items: done << 31 | completion seq (batch-local)
+  u32* it_skey[2];       // items: largest score key of the child
+  u32* seg_vb0;          // leaf segments: meta vector base (leaves)
+  u32* seg_vb1;          // leaf segments: payload vector base (elements)
+  u32* seg_carry;        // leaf segments: 1 if the leaves go to the arena
+  u32* mask;             // [n_max] bit (D-1-l): a level-l group completes at this seq
+  u32* prefix;           // [n_max] records completed before this seq
+  u32* done_e;           // [done_cap]
+  u32* done_lvl;
+  u32* done_cseq;
+  u32* done_rank;
+  u32* r_done;           // by rank
+  u32* r_dense_n;
+  u32* r_topk_n;
+  u32* r_meta_n;
+  u64* r_dense_base;
+  u64* r_topk_off;
+  u64* r_arena_base;
+  uint4* dense;          // [dense_cap] {stamp, len, owner entry or kNone, position}
+  u64* dst;              // [dense_cap + 1]
+  u64* lenscan;          // [n_max + 1]
+  u64* pairset;          // [ps_mask + 1]
+  u64 ps_mask;
+  u32 done_cap;
+};
+
+struct Dev {
+  Ctl* ctl;
+  Table tab;
+  Arena ar;
+  Cfg cfg;
+  Scratch sc;
+  alto_record* out_rec;
+  int32_t* out_pay;
+  alto_topk_pair* out_topk;
+};
+
+__device__ __forceinline__ bool poisoned(const Ctl* c) { return halted(c); }
+// Payload-moving kernels also stand down once the batch has any error: its
+// outputs are undefined and its offsets may not be trustworthy.
+__device__ __forceinline__ bool no_copy(const Ctl* c) {
+  return halted(c) || *(const volatile int*)&c->batch_err != 0;
+}
+
+__device__ __forceinline__ u32 gtid() { return blockIdx.x * blockDim.x + threadIdx.x; }
+__device__ __forceinline__ u32 gstride() { return gridDim.x * blockDim.x; }
+
+// ---------------------------------------------------------------------------
+// open-group hash table (linear probing; a slot index is the entry id)
+// ---------------------------------------------------------------------------
+__device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, int* inserted) {
+  u32 h = (u32)mix64(key) & tab.mask;
+  for (int p = 0; p < tab.max_probe; ++p) {
+    u64 cur = ((volatile u64*)tab.key)[h];
+    if (cur == key) return h;
+    if (cur == kEmpty) {
+      u64 prev = atomicCAS((unsigned long long*)&tab.key[h], (unsigned long long)kEmpty,
+                           (unsigned long long)key);
+      if (prev == kEmpty) {
+        tab.up[h] = up;
+        tab.last[h] = kNone;
+        tab.completed[h] = 0;
+        tab.maxc1[h] = 0;
+        tab.smax[h] = 0;
+        if (tab.vec_n) {
+          tab.vec_n[2 * (u64)h] = 0;
+          tab.vec_n[2 * (u64)h + 1] = 0;
+        }
+        *inserted = 1;
+        return h;
+      }
+      if (prev == key) return h;
+      continue;  // another key took the slot: read it again, then move on
+    }
+    h = (h + 1) & tab.mask;
+  }
+  raise_err(ctl, ALTO_ENOSPC);
+  return 0;
+}
+
+// Batch-local set of (entry, child) slots; returns true if already present.
+// Keys carry a 7-bit batch epoch so that old batches' keys read as free.
+__device__ bool ps_insert(const Scratch& sc, u32 e, u32 c, u32 ep7, Ctl* ctl) {
+  const u64 k57 = ((u64)e << 31) | c;
+  const u64 full = ((u64)ep7 << 57) | k57;
+  u64 h = mix64(k57) & sc.ps_mask;
+  for (int p = 0; p < 8192; ++p) {
+    u64 cur = ((volatile u64*)sc.pairset)[h];
+    if (cur == full) return true;
+    if ((u32)(cur >> 57) != ep7) {
+      u64 prev = atomicCAS((unsigned long long*)&sc.pairset[h], (unsigned long long)cur,
+                           (unsigned long long)full);
+      if (prev == cur) return false;
+      if (prev == full) return true;
+      continue;
+    }
+    h = (h + 1) & sc.ps_mask;
+  }
+  raise_err(ctl, ALTO_ENOSPC);
+  return false;
+}
+
+__device__ __forceinline__ u32 epoch7(const Ctl* ctl) { return ((ctl->epoch - 1) % 127u) + 1u; }
+
+// ---------------------------------------------------------------------------
+// arena: per-group vectors made of geometrically growing chunks
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ u64 vec_addr(const Table& tab, u32 e, int vec, u64 x, bool* ok) {
+  int j = chunk_of(x);
+  if (j >= kNumChunks) {
+    *ok = false;
+    return 0;
+  }
+  u32 base = tab.dir[((u64)e * kVecs + vec) * kNumChunks + j];
+  *ok = base != kNone;
+  return (u64)base + (x - chunk_start(j));
+}
+
+__device__ u32 alloc_chunk(const Arena& ar, Ctl* ctl, int j) {
+  int old = atomicSub(&ctl->top[j], 1);
+  if (old > 0) return ar.stack[ar.stack_off[j] + (u64)(old - 1)];
+  u64 sz = chunk_size(j);
+  u64 off = atomicAdd((unsigned long long*)&ctl->bump, (unsigned long long)sz);
+  if (off + sz > ar.elems) {
+    raise_err(ctl, ALTO_ENOSPC);
+    return kNone;
+  }
+  return (u32)off;
+}
+
+__device__ void free_chunk(const Arena& ar, Ctl* ctl, int j, u32 chunk) {
+  if (chunk == kNone) return;
+  int pos = atomicAdd(&ctl->top[j], 1);
+  if ((u64)pos < ar.stack_cap[j]) ar.stack[ar.stack_off[j] + (u64)pos] = chunk;
+}
+
+// ---------------------------------------------------------------------------
+// kernels
+// ---------------------------------------------------------------------------
+__global__ void k_begin(Ctl* ctl, u32 n) {
+  ctl->epoch += 1;
+  ctl->batch_err = 0;
+  ctl->n_done = 0;
+  ctl->skip_dense = 0;
+  ctl->dense_total = ctl->arena_total = ctl->pay_total = ctl->topk_total = ctl->n_emit = 0;
+  for (int l = 0; l < kMaxDepth; ++l) ctl->n_segs[l] = 0;
+  ctl->n = (ctl->status == ALTO_OK) ? n : 0u;
+}
+
+__global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  __shared__ u32 s_ins;
+  if (threadIdx.x == 0) s_ins = 0;
+  __syncthreads();
+  const int D = d.cfg.depth;
+  const u32 ep7 = epoch7(ctl);
+  for (u32 i = gtid(); i < b.n; i += gstride()) {
+    u32 o0 = b.off[i], o1 = b.off[i + 1];
+    if (o1 < o0 || (u64)o1 > b.n_payload) raise_err(ctl, ALTO_EINVAL);
+    if (d.cfg.has_score && is_nan_bits(__float_as_uint(b.score[i]))) raise_err(ctl, ALTO_EINVAL);
+    u64 t = b.tags[(u64)(D - 1) * b.n + i];
+    u64 up = (D > 1) ? b.tags[(u64)(D - 2) * b.n + i] : 0ull;
+    int ins = 0;
+    u32 e = ht_find_or_insert(d.tab, ((u64)(D - 1) << 32) | tag_pid(t), up, ctl, &ins);
+    if (ins) atomicAdd(&s_ins, 1u);
+    d.sc.leaf_sort_keys0[i] = e;
+    if (ps_insert(d.sc, e, tag_child(t), ep7, ctl)) raise_err(ctl, ALTO_EDUP);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && s_ins) atomicAdd((unsigned long long*)&ctl->live_groups, (u64)s_ins);
+}
+
+// Items of level l are the level-(l+1) groups present in the batch.
+__global__ void __launch_bounds__(kThreads) k_items_lookup(Dev d, Batch b, int l, int in_set) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  __shared__ u32 s_ins;
+  if (threadIdx.x == 0) s_ins = 0;
+  __syncthreads();
+  const u32 ni = min(ctl->n_segs[l + 1], d.cfg.n_max);
+  const u32 ep7 = epoch7(ctl);
+  const u32* it_rep = d.sc.it_rep[in_set];
+  for (u32 x = gtid(); x < ni; x += gstride()) {
+    u32 rep = it_rep[x];
+    u64 t = b.tags[(u64)l * b.n + rep];
+    u64 up = (l > 0) ? b.tags[(u64)(l - 1) * b.n + rep] : 0ull;
+    int ins = 0;
+    u32 e = ht_find_or_insert(d.tab, ((u64)l << 32) | tag_pid(t), up, ctl, &ins);
+    if (ins) atomicAdd(&s_ins, 1u);
+    d.sc.up_sort_keys0[x] = e;
+    if (ps_insert(d.sc, e, tag_child(t), ep7, ctl)) raise_err(ctl, ALTO_EINCONSIST);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && s_ins) atomicAdd((unsigned long long*)&ctl->live_groups, (u64)s_ins);
+}
+
+// Segment discovery over sorted keys: seg_start[s] = first position of run s.
+struct SegFind {
+  const u32* keys;
+  u32* seg_start;
+  u32* seg_of;
+  const u32* n_dev;
+  u32 cap;
+  u32* n_segs_out;
+  __device__ u64 size(const Ctl*) const { return min(*n_dev, cap); }
+  __device__ u64 value(u64 j) const { return (j == 0 || keys[j] != keys[j - 1]) ? 1u : 0u; }
+  __device__ void out(u64 j, u64 excl, u64 v) const {
+    if (v && excl < cap) seg_start[excl] = (u32)j;
+    if (seg_of) seg_of[j] = (u32)(excl + v - 1);
+  }
+  __device__ void total(Ctl*, u64 t) const {
+    if (t > cap) t = cap;
+    *n_segs_out = (u32)t;
+    seg_start[t] = (u32)size(nullptr);
+  }
+};
+
+__device__ __forceinline__ u64 shfl_xor_u64(u64 v, int o) {
+  return __shfl_xor_sync(0xFFFFFFFFu, v, o);
+}
+
+// One warp per group present at level l: reduce its items, merge with the
+// table entry, test completion, and emit the group as an item of level l-1.
+template <bool LEAF>
+__global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, const u32* skeys,
+                                                     const u32* sperm, const u32* seg_start,
+                                                     int in_set) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  const int D = d.cfg.depth;
+  const u32 nseg = min(ctl->n_segs[l], d.cfg.n_max);
+  const int lane = threadIdx.x & 31;
+  const u32 gw = gtid() >> 5, nw = gstride() >> 5;
+  const bool topk = d.cfg.score_op[l] == ALTO_SCORE_TOPK;
+  const int K = d.cfg.topk_k[l];
+  const bool carry = LEAF && d.cfg.concat_level == D - 1;
+  const u32 ep = ctl->epoch;
+  const u32* it_rep = d.sc.it_rep[in_set];
+  const u32* it_cseq = d.sc.it_cseq[in_set];
+  const u32* it_skey = d.sc.it_skey[in_set];
+  u32* nx_rep = d.sc.it_rep[in_set ^ 1];
+  u32* nx_cseq = d.sc.it_cseq[in_set ^ 1];
+  u32* nx_skey = d.sc.it_skey[in_set ^ 1];
+  const u64 n = b.n;
+  const u32 n_items = LEAF ? b.n : min(ctl->n_segs[l + 1], d.cfg.n_max);
+  for (u32 s = gw; s < nseg; s += nw) {
+    const u32 j1 = min(seg_start[s + 1], n_items);
+    const u32 j0 = min(seg_start[s], j1);
+    if (j0 == j1) continue;
+    const u32 e = skeys[j0] & d.tab.mask;
+    const u32 x0 = min(sperm[j0], n_items - 1);
+    const u32 rep0 = LEAF ? x0 : it_rep[x0];
+    u64 htag[kMaxDepth];
+#pragma unroll
+    for (int q = 0; q < kMaxDepth; ++q) htag[q] = (q < l) ? b.tags[(u64)q * n + rep0] : 0ull;
+    u32 cnt = 0, m1 = 0, fmin = kNone, fmax = 0, hasf = 0, cmax = 0, smx = 0, bad = 0;
+    u64 lsum = 0;
+    for (u32 j = j0 + lane; j < j1; j += 32) {
+      const u32 x = min(sperm[j], n_items - 1);
+      u32 rep, done, cs, sk;
+      u64 len = 0;
+      if (LEAF) {
+        rep = x;
+        done = 1;
+        cs = x;
+        sk = d.cfg.has_score ? score_key(b.score[x]) : 0u;
+        len = b.off[x + 1] - b.off[x];
+      } else {
+        rep = it_rep[x];
+        u32 cf = it_cseq[x];
+        done = cf >> 31;
+        cs = cf & 0x7FFFFFFFu;
+        sk = it_skey[x];
+      }
+      const u64 t = b.tags[(u64)l * n + rep];
+      const u32 c = tag_child(t);
+      m1 = max(m1, c + 1);
+      if (tag_last(t)) {
+        hasf = 1;
+        fmin = min(fmin, c);
+        fmax = max(fmax, c);
+      }
+      if (done) {
+        ++cnt;
+        cmax = max(cmax, cs);
+        smx = max(smx, sk);
+      }
+      lsum += len;
+#pragma unroll
+      for (int q = 0; q < kMaxDepth; ++q)
+        if (q < l && b.tags[(u64)q * n + rep] != htag[q]) bad = 1;
+    }
+    cnt = __reduce_add_sync(0xFFFFFFFFu, cnt);
+    m1 = __reduce_max_sync(0xFFFFFFFFu, m1);
+    fmin = __reduce_min_sync(0xFFFFFFFFu, fmin);
+    fmax = __reduce_max_sync(0xFFFFFFFFu, fmax);
+    hasf = __reduce_or_sync(0xFFFFFFFFu, hasf);
+    cmax = __reduce_max_sync(0xFFFFFFFFu, cmax);
+    smx = __reduce_max_sync(0xFFFFFFFFu, smx);
+    bad = __reduce_or_sync(0xFFFFFFFFu, bad);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) lsum += shfl_xor_u64(lsum, o);
+
+    if (topk) {
+      // running top-k of complete children: lane q holds the q-th best
+      const u32 valid = min(d.tab.completed[e], (u32)K);
+      u64 best = (lane < (int)valid) ? d.tab.topk[(u64)e * d.tab.kk + lane] : 0ull;
+      for (u32 jb = j0; jb < j1; jb += 32) {
+        const u32 j = jb + lane;
+        u64 cand = 0;
+        if (j < j1) {
+          const u32 x = min(sperm[j], n_items - 1);
+          u32 rep, done, sk;
+          if (LEAF) {
+            rep = x;
+            done = 1;
+            sk = d.cfg.has_score ? score_key(b.score[x]) : 0u;
+          } else {
+            rep = it_rep[x];
+            done = it_cseq[x] >> 31;
+            sk = it_skey[x];
+          }
+          const u32 c = tag_child(b.tags[(u64)l * n + rep]);
+          if (done) cand = ((u64)sk << 32) | (u64)(~c);
+        }
+        const u64 thr = __shfl_sync(0xFFFFFFFFu, best, K - 1);
+        u32 pass = __ballot_sync(0xFFFFFFFFu, cand > thr);
+        while (pass) {
+          const int src = __ffs(pass) - 1;
+          pass &= pass - 1;
+          const u64 v = __shfl_sync(0xFFFFFFFFu, cand, src);
+          const u64 thr2 = __shfl_sync(0xFFFFFFFFu, best, K - 1);
+          if (v > thr2) {
+            const u32 pos = __popc(__ballot_sync(0xFFFFFFFFu, lane < K && best > v));
+            const u64 prev = __shfl_up_sync(0xFFFFFFFFu, best, 1);
+            if (lane >= (int)pos && lane < K) best = (lane == (int)pos) ? v : prev;
+          }
+        }
+      }
+      if (lane < K) d.tab.topk[(u64)e * d.tab.kk + lane] = best;
+    }
+
+    if (lane == 0) {
+      if (bad) raise_err(ctl, ALTO_EINCONSIST);
+      if (l > 0 && d.tab.up[e] != b.tags[(u64)(l - 1) * n + rep0]) raise_err(ctl, ALTO_EINCONSIST);
+      const u32 last_old = d.tab.last[e];
+      u32 nl = last_old;
+      if (hasf) {
+        if (fmin != fmax) raise_err(ctl, ALTO_ELAST);
+        if (last_old != kNone && last_old != fmin) raise_err(ctl, ALTO_ELAST);
+        if (last_old == kNone) nl = fmin;
+      }
+      const u32 m1n = max(d.tab.maxc1[e], m1);
+      if (nl != kNone && m1n > nl + 1) raise_err(ctl, ALTO_ELAST);
+      const u32 comp = d.tab.completed[e] + cnt;
+      const u32 smn = max(d.tab.smax[e], smx);
+      const bool complete = (nl != kNone) && (comp == nl + 1) && (m1n <= nl + 1);
+      d.tab.last[e] = nl;
+      d.tab.maxc1[e] = m1n;
+      d.tab.completed[e] = comp;
+      d.tab.smax[e] = smn;
+      if (complete) {
+        u32 di = atomicAdd(&ctl->n_done, 1u);
+        if (di < d.sc.done_cap) {
+          d.sc.done_e[di] = e;
+          d.sc.done_lvl[di] = (u32)l;
+          d.sc.done_cseq[di] = cmax;
+          d.tab.done_epoch[e] = ep;
+          d.tab.done_idx[e] = di;
+          if (cmax < n) atomicOr(&d.sc.mask[cmax], 1u << (D - 1 - l));
+        } else {
+          raise_err(ctl, ALTO_ENOSPC);
+        }
+      }
+      if (carry) {
+        d.sc.seg_carry[s] = complete ? 0u : 1u;
+        if (!complete) {
+          const u32 v0 = d.tab.vec_n[2 * (u64)e], v1 = d.tab.vec_n[2 * (u64)e + 1];
+          d.sc.seg_vb0[s] = v0;
+          d.sc.seg_vb1[s] = v1;
+          d.tab.vec_n[2 * (u64)e] = v0 + (j1 - j0);
+          d.tab.vec_n[2 * (u64)e + 1] = v1 + (u32)lsum;
+        }
+      }
+      if (l > 0) {
+        nx_rep[s] = rep0;
+        nx_cseq[s] = (complete ? 0x80000000u : 0u) | cmax;
+        nx_skey[s] = smn;
+      }
+    }
+  }
+}
+
+// Emission rank of each completed group: records completed at earlier
+// arrival indices, plus the deeper groups completed at the same index.
+struct RankScan {
+  const u32* mask;
+  u32* prefix;
+  const u32* n_dev;
+  __device__ u64 size(const Ctl*) const { return *n_dev; }
+  __device__ u64 value(u64 i) const { return __popc(mask[i]); }
+  __device__ void out(u64 i, u64 excl, u64) const { prefix[i] = (u32)excl; }
+  __device__ void total(Ctl* ctl, u64 t) const { ctl->n_emit = t; }
+};
+
+__global__ void __launch_bounds__(kThreads) k_done_rank(Dev d) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  const int D = d.cfg.depth, M = d.cfg.concat_level;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  for (u32 di = gtid(); di < nd; di += gstride()) {
+    const u32 e = d.sc.done_e[di];
+    const int l = (int)d.sc.done_lvl[di];
+    const u32 cs = d.sc.done_cseq[di];
+    const int bit = D - 1 - l;
+    const u32 r = (cs < ctl->n) ? d.sc.prefix[cs] + __popc(d.sc.mask[cs] & ((1u << bit) - 1u)) : kNone;
+    if (r >= nd) {
+      raise_err(ctl, ALTO_EINCONSIST);
+      d.sc.done_rank[di] = kNone;
+      continue;
+    }
+    d.sc.done_rank[di] = r;
+    d.sc.r_done[r] = di;
+    const u32 nch = d.tab.last[e] + 1;
+    d.sc.r_dense_n[r] = (l == M) ? nch : 0u;
+    d.sc.r_topk_n[r] = (d.cfg.score_op[l] == ALTO_SCORE_TOPK) ? min(nch, (u32)d.cfg.topk_k[l]) : 0u;
+    d.sc.r_meta_n[r] = (l == M) ? d.tab.vec_n[2 * (u64)e] : 0u;
+  }
+}
+
+// Exclusive scan of a per-record u32 count into u64 offsets.
+struct CountScan {
+  const u32* in;
+  u64* out_off;
+  const u32* n_dev;
+  u32 cap;
+  int which;  // 0 dense, 1 topk, 2 arena
+  __device__ u64 size(const Ctl*) const { return min(*n_dev, cap); }
+  __device__ u64 value(u64 i) const { return in[i]; }
+  __device__ void out(u64 i, u64 excl, u64) const { out_off[i] = excl; }
+  __device__ void total(Ctl* ctl, u64 t) const {
+    out_off[size(nullptr)] = t;
+    if (which == 0) ctl->dense_total = t;
+    else if (which == 1) ctl->topk_total = t;
+    else ctl->arena_total = t;
+  }
+};
+
+__global__ void k_check(Dev d) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  bool bad = false;
+  if (ctl->rec_count + ctl->n_done > d.cfg.out_records) bad = true;
+  if (ctl->dense_total > d.cfg.dense_cap) bad = true;
+  if (ctl->topk_count + ctl->topk_total > d.cfg.out_topk) bad = true;
+  if (ctl->n_done > d.sc.done_cap) bad = true;
+  if (bad) {
+    raise_err(ctl, ALTO_ENOSPC);
+    ctl->skip_dense = 1;
+  }
+}
+
+// Payload lengths of the leaves in sorted order, scanned: a leaf's position
+// inside its group's new arena data.
+struct LenScan {
+  const u32* perm;
+  const u32* off;
+  u64* out_scan;
+  const u32* n_dev;
+  __device__ u64 size(const Ctl*) const { return *n_dev; }
+  __device__ u64 value(u64 j) const {
+    u32 i = perm[j];
+    return off[i + 1] - off[i];
+  }
+  __device__ void out(u64 j, u64 excl, u64) const { out_scan[j] = excl; }
+  __device__ void total(Ctl*, u64 t) const { out_scan[size(nullptr)] = t; }
+};
+
+__global__ void __launch_bounds__(kThreads) k_carry_alloc(Dev d) {
+  Ctl* ctl = d.ctl;
+  if (no_copy(ctl)) return;
+  const u32 nseg = min(ctl->n_segs[d.cfg.depth - 1], d.cfg.n_max);
+  for (u32 s = gtid(); s < nseg; s += gstride()) {
+    if (!d.sc.seg_carry[s]) continue;
+    const u32 e = d.sc.leaf_keys[d.sc.leaf_seg_start[s]];
+    for (int vec = 0; vec < kVecs; ++vec) {
+      const u64 mult = (vec == 0) ? 2 : 1;
+      const u64 old_el = (u64)((vec == 0) ? d.sc.seg_vb0[s] : d.sc.seg_vb1[s]) * mult;
+      const u64 new_el = (u64)d.tab.vec_n[2 * (u64)e + vec] * mult;
+      if (new_el <= old_el) continue;
+      const int jf = (old_el == 0) ? 0 : chunk_of(old_el - 1) + 1;
+      const int jl = chunk_of(new_el - 1);
+      for (int j = jf; j <= jl && j < kNumChunks; ++j) {
+        u32 c = alloc_chunk(d.ar, ctl, j);
+        d.tab.dir[((u64)e * kVecs + vec) * kNumChunks + j] = c;
+        if (c != kNone) atomicAdd((unsigned long long*)&ctl->arena_used, (unsigned long long)chunk_size(j));
+      }
+      if (jl >= kNumChunks) raise_err(ctl, ALTO_ENOSPC);
+    }
+  }
+}
+
+__global__ void k_fix_tops(Ctl* ctl) {
+  int j = threadIdx.x;
+  if (j < kNumChunks && ctl->top[j] < 0) ctl->top[j] = 0;
+}
+
+__global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch b) {
+  Ctl* ctl = d.ctl;
+  if (no_copy(ctl)) return;
+  const int D = d.cfg.depth;
+  const u32 n = b.n;
+  const u32 nseg = min(ctl->n_segs[D - 1], d.cfg.n_max);
+  for (u32 j = gtid(); j < n; j += gstride()) {
+    const u32 s = d.sc.leaf_seg_of[j];
+    if (s >= nseg || !d.sc.seg_carry[s]) continue;
+    const u32 i = d.sc.leaf_perm[j];
+    const u32 e = d.sc.leaf_keys[j] & d.tab.mask;
+    const u32 s0 = d.sc.leaf_seg_start[s];
+    if (i >= n || s0 > j) continue;
+    const u64 mpos = (u64)d.sc.seg_vb0[s] + (j - s0);
+    const u64 ppos = (u64)d.sc.seg_vb1[s] + (d.sc.lenscan[j] - d.sc.lenscan[s0]);
+    const u32 c = tag_child(b.tags[(u64)(D - 1) * n + i]);
+    const u32 o0 = b.off[i], len = b.off[i + 1] - o0;
+    // stay inside the ranges reserved (and allocated) for this group
+    if (mpos >= d.tab.vec_n[2 * (u64)e] || ppos + len > d.tab.vec_n[2 * (u64)e + 1]) continue;
+    bool ok;
+    u64 a = vec_addr(d.tab, e, 0, 2 * mpos, &ok);
+    if (ok) {
+      d.ar.pool[a] = (int32_t)c;
+      d.ar.pool[a + 1] = (int32_t)(u32)ppos;
+    }
+    for (u32 q = 0; q < len; ++q) {
+      u64 pa = vec_addr(d.tab, e, 1, ppos + q, &ok);
+      if (ok) d.ar.pool[pa] = b.pay[o0 + q];
+    }
+  }
+}
+
+// Dense child slots of completing CONCAT groups, from this batch's leaves.
+__global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
+  Ctl* ctl = d.ctl;
+  if (no_copy(ctl) || ctl->skip_dense) return;
+  const int D = d.cfg.depth;
+  const u32 ep = ctl->epoch;
+  const u32 n = b.n;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  for (u32 j = gtid(); j < n; j += gstride()) {
+    const u32 e = d.sc.leaf_keys[j] & d.tab.mask;
+    if (d.tab.done_epoch[e] != ep) continue;
+    const u32 di = d.tab.done_idx[e];
+    if (di >= nd) continue;
+    const u32 r = d.sc.done_rank[di];
+    if (r >= nd) continue;
+    const u32 i = d.sc.leaf_perm[j];
+    if (i >= n) continue;
+    const u32 c = tag_child(b.tags[(u64)(D - 1) * n + i]);
+    if (c >= d.sc.r_dense_n[r]) continue;
+    const u64 slot = d.sc.r_dense_base[r] + c;
+    if (slot >= d.cfg.dense_cap) continue;
+    u32 old = atomicExch(&d.sc.dense[slot].x, ep);
+    if (old == ep) raise_err(ctl, ALTO_EDUP);
+    d.sc.dense[slot].y = b.off[i + 1] - b.off[i];
+    d.sc.dense[slot].z = kNone;
+    d.sc.dense[slot].w = b.off[i];
+  }
+}
+
+// Dense child slots from the arena (leaves buffered by earlier batches).
+__global__ void __launch_bounds__(kThreads) k_dense_arena(Dev d) {
+  Ctl* ctl = d.ctl;
+  if (no_copy(ctl) || ctl->skip_dense) return;
+  const u32 ep = ctl->epoch;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  const u64 na = ctl->arena_total;
+  for (u64 a = gtid(); a < na; a += gstride()) {
+    // last rank r with r_arena_base[r] <= a
+    u32 lo = 0, hi = nd;
+    while (hi - lo > 1) {
+      u32 mid = (lo + hi) >> 1;
+      if (d.sc.r_arena_base[mid] <= a) lo = mid;
+      else hi = mid;
+    }
+    const u32 r = lo;
+    const u32 di = d.sc.r_done[r];
+    if (di >= nd) continue;
+    const u32 e = d.sc.done_e[di];
+    const u64 k = a - d.sc.r_arena_base[r];
+    const u32 mn = d.sc.r_meta_n[r];
+    if (k >= mn) continue;
+    bool ok1, ok2 = true;
+    u64 ma = vec_addr(d.tab, e, 0, 2 * k, &ok1);
+    if (!ok1) continue;
+    const u32 c = (u32)d.ar.pool[ma];
+    const u32 pos = (u32)d.ar.pool[ma + 1];
+    u32 end;
+    if (k + 1 < mn) {
+      u64 na2 = vec_addr(d.tab, e, 0, 2 * (k + 1) + 1, &ok2);
+      end = ok2 ? (u32)d.ar.pool[na2] : pos;
+    } else {
+      end = d.tab.vec_n[2 * (u64)e + 1];
+    }
+    if (c >= d.sc.r_dense_n[r] || end < pos) {
+      raise_err(ctl, ALTO_EDUP);
+      continue;
+    }
+    const u64 slot = d.sc.r_dense_base[r] + c;
+    if (slot >= d.cfg.dense_cap) continue;
+    u32 old = atomicExch(&d.sc.dense[slot].x, ep);
+    if (old == ep) raise_err(ctl, ALTO_EDUP);
+    d.sc.dense[slot].y = end - pos;
+    d.sc.dense[slot].z = e;
+    d.sc.dense[slot].w = pos;
+  }
+}
+
+// Output offsets of every child span; a slot no child filled means a child
+// was repeated elsewhere.
+struct DenseScan {
+  const uint4* dense;
+  u64* dst;
+  Ctl* ctlp;
+  __device__ u64 size(const Ctl* ctl) const {
+    return (ctl->skip_dense || ctl->batch_err) ? 0 : ctl->dense_total;
+  }
+  __device__ u64 value(u64 j) const {
+    uint4 v = dense[j];
+    if (v.x != ctlp->epoch) {
+      raise_err(ctlp, ALTO_EDUP);
+      return 0;
+    }
+    return v.y;
+  }
+  __device__ void out(u64 j, u64 excl, u64) const { dst[j] = excl; }
+  __device__ void total(Ctl* ctl, u64 t) const {
+    dst[size(ctl)] = t;
+    ctl->pay_total = t;
+  }
+};
+
+__global__ void k_check2(Dev d) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl) || ctl->skip_dense) return;
+  if (ctl->pay_count + ctl->pay_total > d.cfg.out_payload) {
+    raise_err(ctl, ALTO_ENOSPC);
+    ctl->skip_dense = 1;
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) k_gather(Dev d, Batch b) {
+  Ctl* ctl = d.ctl;
+  if (no_copy(ctl) || ctl->skip_dense) return;
+  const u32 ep = ctl->epoch;
+  const u64 total = ctl->dense_total;
+  const u64 base = ctl->pay_count;
+  const int lane = threadIdx.x & 31;
+  const u64 gw = gtid() >> 5, nw = gstride() >> 5;
+  for (u64 j = gw; j < total; j += nw) {
+    const uint4 v = d.sc.dense[j];
+    if (v.x != ep) continue;
+    const u64 o = base + d.sc.dst[j];
+    if (o + v.y > d.cfg.out_payload) continue;
+    if (v.z == kNone) {
+      if ((u64)v.w + v.y > b.n_payload) continue;
+      for (u32 q = lane; q < v.y; q += 32) d.out_pay[o + q] = b.pay[v.w + q];
+    } else {
+      if (v.z > d.tab.mask || (u64)v.w + v.y > d.tab.vec_n[2 * (u64)v.z + 1]) continue;
+      for (u32 q = lane; q < v.y; q += 32) {
+        bool ok;
+        u64 a = vec_addr(d.tab, v.z, 1, (u64)v.w + q, &ok);
+        if (ok) d.out_pay[o + q] = d.ar.pool[a];
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) k_records(Dev d) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  __shared__ u32 s_del;
+  __shared__ unsigned long long s_freed;
+  if (threadIdx.x == 0) {
+    s_del = 0;
+    s_freed = 0;
+  }
+  __syncthreads();
+  const int M = d.cfg.concat_level;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  const bool skip = ctl->skip_dense;
+  for (u32 di = gtid(); di < nd; di += gstride()) {
+    const u32 e = d.sc.done_e[di];
+    const int l = (int)d.sc.done_lvl[di];
+    const u32 cs = d.sc.done_cseq[di];
+    const u32 r = d.sc.done_rank[di];
+    d.sc.mask[cs] = 0;
+    if (!skip && r != kNone) {
+      alto_record rec;
+      rec.completion_seq = ctl->seq_base + cs;
+      if (M >= 0) {
+        const u64 db = min(d.sc.r_dense_base[r], ctl->dense_total);
+        const u64 de = min(db + d.sc.r_dense_n[r], ctl->dense_total);
+        rec.payload_off = ctl->pay_count + d.sc.dst[db];
+        rec.payload_len = (l == M) ? d.sc.dst[de] - d.sc.dst[db] : 0;
+      } else {
+        rec.payload_off = ctl->pay_count;
+        rec.payload_len = 0;
+      }
+      u32 tn = d.sc.r_topk_n[r];
+      const u64 to = ctl->topk_count + d.sc.r_topk_off[r];
+      if (to + tn > d.cfg.out_topk) tn = 0;
+      rec.topk_off = to;
+      rec.topk_n = (uint16_t)tn;
+      rec.parent_id = (u32)d.tab.key[e];
+      rec.n_children = d.tab.last[e] + 1;
+      rec.level = (uint8_t)l;
+      rec.ops = (uint8_t)(((l == M) ? 1 : 0) | (d.cfg.score_op[l] << 2));
+      rec.score = (d.cfg.score_op[l] != ALTO_SCORE_NONE) ? key_score(d.tab.smax[e]) : 0.0f;
+      d.out_rec[ctl->rec_count + r] = rec;
+      for (u32 q = 0; q < tn; ++q) {
+        const u64 v = d.tab.topk[(u64)e * d.tab.kk + q];
+        alto_topk_pair p;
+        p.child_index = ~(u32)v;
+        p.score = key_score((u32)(v >> 32));
+        d.out_topk[to + q] = p;
+      }
+    }
+    if (l == M) {
+      for (int vec = 0; vec < kVecs; ++vec) {
+        const u64 el = (u64)d.tab.vec_n[2 * (u64)e + vec] * (vec == 0 ? 2 : 1);
+        if (el == 0) continue;
+        const int jl = min(chunk_of(el - 1), kNumChunks - 1);
+        for (int j = 0; j <= jl; ++j) {
+          free_chunk(d.ar, ctl, j, d.tab.dir[((u64)e * kVecs + vec) * kNumChunks + j]);
+          atomicAdd(&s_freed, (unsigned long long)chunk_size(j));
+        }
+      }
+    }
+    d.tab.key[e] = kTomb;
+    atomicAdd(&s_del, 1u);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (s_del) atomicAdd((unsigned long long*)&ctl->live_groups, (unsigned long long)(-(long long)s_del));
+    if (s_freed) atomicAdd((unsigned long long*)&ctl->arena_used, (unsigned long long)(-(long long)s_freed));
+  }
+}
+
+// Turn deleted slots back into free ones where no probe chain runs through
+// them: a tombstone followed (after more tombstones) by a free slot.
+__global__ void __launch_bounds__(kThreads) k_sweep(Dev d) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  const u32 mask = d.tab.mask;
+  volatile u64* key = d.tab.key;
+  for (u32 di = gtid(); di < nd; di += gstride()) {
+    const u32 e = d.sc.done_e[di];
+    if (key[e] != kTomb) continue;
+    u32 p = (e + 1) & mask;
+    int steps = 0;
+    while (key[p] == kTomb && steps < d.tab.max_probe) {
+      p = (p + 1) & mask;
+      ++steps;
+    }
+    if (key[p] != kEmpty) continue;
+    key[e] = kEmpty;
+    u32 q = (e - 1) & mask;
+    steps = 0;
+    while (key[q] == kTomb && steps < d.tab.max_probe) {
+      key[q] = kEmpty;
+      q = (q - 1) & mask;
+      ++steps;
+    }
+  }
+}
+
+__global__ void k_end(Ctl* ctl, u32 n) {
+  if (ctl->status != ALTO_OK) return;
+  if (ctl->batch_err) {
+    ctl->status = -(ctl->batch_err & 0xFF);
+    return;
+  }
+  ctl->rec_count += ctl->n_done;
+  ctl->pay_count += ctl->pay_total;
+  ctl->topk_count += ctl->topk_total;
+  ctl->seq_base += n;
+}
+
+__global__ void k_drain_reset(Ctl* ctl) {
+  ctl->rec_count = 0;
+  ctl->pay_count = 0;
+  ctl->topk_count = 0;
+}
+
+}  // namespace alto
+
+using namespace alto;
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+struct alto_agg {
+  alto_agg_config cfg;
+  alto_allocator alloc;
+  bool use_async;
+  int device;
+  int num_sms;
+  int tbits;
+  Dev d;
+  SortBuffers leaf_sort, up_sort;
+  LookbackState lbs;
+  Ctl* h_ctl;  // pinned host copy for drain
+  std::vector<void*> blocks;
+  u64 pushed;
+  u64 drain_first;
+  int latched;
+  // measurement hooks
+  bool profiling;
+  cudaStream_t last_stream;
+  int64_t prof_pushes;
+  int64_t launches;
+  double stage_ms[ALTO_NUM_STAGES];
+  int64_t stage_launches[ALTO_NUM_STAGES];
+  std::vector<cudaEvent_t> ev_free;                   // reusable events
+  std::vector<std::vector<cudaEvent_t>> ev_pending;  // per push: stage boundaries
+};
+
+namespace {
+
+// Stage boundaries of one push, recorded when profiling is on.
+struct StageClock {
+  alto_agg* h;
+  cudaStream_t s;
+  std::vector<cudaEvent_t> ev;
+  int stage = 0;
+  int launches_at_start = 0;
+  StageClock(alto_agg* h_, cudaStream_t s_) : h(h_), s(s_) {}
+  cudaEvent_t take() {
+    cudaEvent_t e;
+    if (!h->ev_free.empty()) {
+      e = h->ev_free.back();
+      h->ev_free.pop_back();
+    } else if (cudaEventCreate(&e) != cudaSuccess) {
+      return nullptr;
+    }
+    return e;
+  }
+  // mark the start of stage `st` (stages must be entered in order)
+  void enter(int st) {
+    if (!h->profiling) return;
+    while ((int)ev.size() <= st) {
+      cudaEvent_t e = take();
+      if (e) cudaEventRecord(e, s);
+      ev.push_back(e);
+    }
+  }
+  void finish() {
+    if (!h->profiling) return;
+    enter(ALTO_NUM_STAGES);
+    h->ev_pending.push_back(ev);
+  }
+};
+
+void collect_profile(alto_agg* h) {
+  for (auto& ev : h->ev_pending) {
+    for (int st = 0; st < ALTO_NUM_STAGES && st + 1 < (int)ev.size(); ++st) {
+      float ms = 0.0f;
+      if (ev[st] && ev[st + 1] && cudaEventElapsedTime(&ms, ev[st], ev[st + 1]) == cudaSuccess)
+        h->stage_ms[st] += ms;
+    }
+    for (cudaEvent_t e : ev)
+      if (e) h->ev_free.push_back(e);
+  }
+  h->ev_pending.clear();
+}
+
+template <class F>
+void launch_scan(alto_agg* h, const F& f, u64 cap, int site, cudaStream_t s) {
+  u64 tiles = (cap + kScanTile - 1) / kScanTile;
+  if (tiles == 0) tiles = 1;
+  int grid = (int)std::min<u64>(tiles, (u64)h->num_sms * 4);
+  h->launches += 1;
+  k_scan<F><<<grid, kScanThreads, 0, s>>>(f, h->lbs, h->d.ctl, site, &h->d.ctl->exit_ctr[site],
+                                          h->d.cfg.spin_limit);
+}
+
+void* dev_alloc(alto_agg* h, size_t bytes, cudaStream_t s) {
+  bytes = (bytes + 255) & ~(size_t)255;
+  if (bytes == 0) bytes = 256;
+  void* p = nullptr;
+  if (h->use_async) {
+    if (cudaMallocAsync(&p, bytes, s) != cudaSuccess) return nullptr;
+  } else {
+    p = h->alloc.alloc(h->alloc.ctx, bytes, s);
+  }
+  if (p) h->blocks.push_back(p);
+  return p;
+}
+
+void free_all(alto_agg* h, cudaStream_t s) {
+  for (void* p : h->blocks) {
+    if (h->use_async) cudaFreeAsync(p, s);
+    else h->alloc.free(h->alloc.ctx, p, s);
+  }
+  h->blocks.clear();
+  if (h->h_ctl) cudaFreeHost(h->h_ctl);
+  h->h_ctl = nullptr;
+}
+
+u64 next_pow2(u64 x) {
+  u64 p = 1;
+  while (p < x) p <<= 1;
+  return p;
+}
+
+int ilog2(u64 x) {
+  int b = 0;
+  while ((1ull << b) < x) ++b;
+  return b;
+}
+
+alto_status validate(const alto_agg_config* c) {
+  if (c->depth < 1 || c->depth > ALTO_MAX_DEPTH) return ALTO_EINVAL;
+  int nconcat = 0;
+  for (int l = 0; l < c->depth; ++l) {
+    if (c->payload_op[l] != ALTO_PAYLOAD_NONE && c->payload_op[l] != ALTO_PAYLOAD_CONCAT)
+      return ALTO_EINVAL;
+    if (c->payload_op[l] == ALTO_PAYLOAD_CONCAT) {
+      ++nconcat;
+      if (l != c->depth - 1) return ALTO_EINVAL;  // the device path concatenates at the leaf-parent level
+    }
+    if (c->score_op[l] < ALTO_SCORE_NONE || c->score_op[l] > ALTO_SCORE_TOPK) return ALTO_EINVAL;
+    if (c->score_op[l] == ALTO_SCORE_TOPK && (c->topk_k[l] < 1 || c->topk_k[l] > ALTO_MAX_TOPK))
+      return ALTO_EINVAL;
+  }
+  if (nconcat > 1) return ALTO_EINVAL;
+  if (c->max_batch_fragments < 1 || c->max_batch_fragments >= (1ll << 30)) return ALTO_EINVAL;
+  if (c->max_batch_payload < 0 || c->max_batch_payload >= (1ll << 32)) return ALTO_EINVAL;
+  if (c->max_open_groups < 0 || c->max_open_groups > (1ll << 25)) return ALTO_EINVAL;
+  if (c->arena_elems < 0 || c->arena_elems >= (1ll << 32)) return ALTO_EINVAL;
+  if (c->out_records < 0 || c->out_payload_elems < 0 || c->out_topk < 0 || c->max_emit_children < 0 ||
+      c->spin_limit < 0)
+    return ALTO_EINVAL;
+  return ALTO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator* alloc, void* stream,
+                            alto_agg_t** out) {
+  if (cfg_in == nullptr || out == nullptr) return ALTO_EINVAL;
+  alto_status v = validate(cfg_in);
+  if (v != ALTO_OK) return v;
+  if (alloc != nullptr && (alloc->alloc == nullptr || alloc->free == nullptr)) return ALTO_EINVAL;
+  alto_agg_config cfg = *cfg_in;
+  const u64 nmax = (u64)cfg.max_batch_fragments;
+  if (cfg.max_open_groups == 0) cfg.max_open_groups = 1ll << 20;
+  if (cfg.arena_elems == 0) cfg.arena_elems = 1ll << 26;
+  if (cfg.out_records == 0) cfg.out_records = 4 * (int64_t)nmax;
+  if (cfg.out_payload_elems == 0) cfg.out_payload_elems = std::max<int64_t>(4 * cfg.max_batch_payload, 1);
+  if (cfg.out_topk == 0) cfg.out_topk = cfg.out_records;
+  if (cfg.max_emit_children == 0) cfg.max_emit_children = 4 * (int64_t)nmax;
+  if (cfg.spin_limit == 0) cfg.spin_limit = 1ll << 20;
+
+  cudaStream_t s = (cudaStream_t)stream;
+  alto_agg* h = new (std::nothrow) alto_agg();
+  if (!h) return ALTO_ENOMEM;
+  h->cfg = cfg;
+  h->use_async = (alloc == nullptr);
+  if (alloc) h->alloc = *alloc;
+  h->pushed = 0;
+  h->drain_first = 0;
+  h->latched = ALTO_OK;
+  h->profiling = false;
+  h->last_stream = s;
+  h->prof_pushes = 0;
+  h->launches = 0;
+  for (int i = 0; i < ALTO_NUM_STAGES; ++i) {
+    h->stage_ms[i] = 0.0;
+    h->stage_launches[i] = 0;
+  }
+  if (cudaGetDevice(&h->device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device) != cudaSuccess) {
+    delete h;
+    return ALTO_ECUDA;
+  }
+  const int D = cfg.depth;
+  int concat = -1, kk = 0;
+  bool has_score = false;
+  for (int l = 0; l < D; ++l) {
+    if (cfg.payload_op[l] == ALTO_PAYLOAD_CONCAT) concat = l;
+    if (cfg.score_op[l] != ALTO_SCORE_NONE) has_score = true;
+    if (cfg.score_op[l] == ALTO_SCORE_TOPK) kk = std::max(kk, (int)cfg.topk_k[l]);
+  }
+  const u64 T = next_pow2(std::max<u64>(2 * (u64)cfg.max_open_groups, 1024));
+  h->tbits = ilog2(T);
+  const u64 done_cap = nmax * (u64)D;
+  const u64 dense_cap = (u64)cfg.max_emit_children;
+  const u64 PS = next_pow2(std::max<u64>(2 * nmax * (u64)D, 1024));
+
+  Dev& d = h->d;
+  memset(&d, 0, sizeof(d));
+  bool ok = true;
+#define ALLOC(ptr, type, count)                                              \
+  do {                                                                       \
+    ptr = (type*)dev_alloc(h, sizeof(type) * (size_t)(count), s);            \
+    if (!ptr) ok = false;                                                    \
+  } while (0)
+
+  ALLOC(d.ctl, Ctl, 1);
+  // table
+  ALLOC(d.tab.key, u64, T);
+  ALLOC(d.tab.up, u64, T);
+  ALLOC(d.tab.last, u32, T);
+  ALLOC(d.tab.completed, u32, T);
+  ALLOC(d.tab.maxc1, u32, T);
+  ALLOC(d.tab.smax, u32, T);
+  ALLOC(d.tab.done_epoch, u32, T);
+  ALLOC(d.tab.done_idx, u32, T);
+  if (concat >= 0) {
+    ALLOC(d.tab.vec_n, u32, 2 * T);
+    ALLOC(d.tab.dir, u32, T * kVecs * kNumChunks);
+  }
+  if (kk > 0) ALLOC(d.tab.topk, u64, T * (u64)kk);
+  d.tab.mask = (u32)(T - 1);
+  d.tab.kk = kk;
+  d.tab.max_probe = (int)std::min<u64>(T, 1u << 16);
+  // arena
+  if (concat >= 0) {
+    d.ar.elems = (u64)cfg.arena_elems;
+    ALLOC(d.ar.pool, int32_t, std::max<u64>(d.ar.elems, 1));
+    u64 off = 0;
+    for (int j = 0; j < kNumChunks; ++j) {
+      d.ar.stack_off[j] = off;
+      d.ar.stack_cap[j] = d.ar.elems / (1ull << (kChunk0Log + j)) + 1;
+      off += d.ar.stack_cap[j];
+    }
+    ALLOC(d.ar.stack, u32, off);
+  }
+  // config
+  d.cfg.depth = D;
+  d.cfg.concat_level = concat;
+  for (int l = 0; l < kMaxDepth; ++l) {
+    d.cfg.score_op[l] = (l < D) ? cfg.score_op[l] : 0;
+    d.cfg.topk_k[l] = (l < D && cfg.score_op[l] == ALTO_SCORE_TOPK) ? cfg.topk_k[l] : 0;
+  }
+  d.cfg.has_score = has_score;
+  d.cfg.n_max = (u32)nmax;
+  d.cfg.out_records = (u64)cfg.out_records;
+  d.cfg.out_payload = (u64)cfg.out_payload_elems;
+  d.cfg.out_topk = (u64)cfg.out_topk;
+  d.cfg.dense_cap = dense_cap;
+  d.cfg.spin_limit = (u64)cfg.spin_limit;
+  // scratch
+  Scratch& sc = d.sc;
+  for (int b = 0; b < 2; ++b) {
+    ALLOC(h->leaf_sort.keys[b], u32, nmax);
+    ALLOC(h->leaf_sort.vals[b], u32, nmax);
+    ALLOC(h->up_sort.keys[b], u32, nmax);
+    ALLOC(h->up_sort.vals[b], u32, nmax);
+  }
+  const u64 sort_tiles = nmax / 4096 + 2;
+  ALLOC(h->leaf_sort.hist, u32, 4 * 256);
+  ALLOC(h->leaf_sort.bin_base, u32, 4 * 256);
+  ALLOC(h->leaf_sort.lookback, u64, sort_tiles * 256);
+  h->leaf_sort.lb_tiles = sort_tiles;
+  h->up_sort.hist = h->leaf_sort.hist;
+  h->up_sort.bin_base = h->leaf_sort.bin_base;
+  h->up_sort.lookback = h->leaf_sort.lookback;
+  h->up_sort.lb_tiles = sort_tiles;
+  sc.leaf_sort_keys0 = h->leaf_sort.keys[0];
+  sc.up_sort_keys0 = h->up_sort.keys[0];
+  ALLOC(sc.leaf_seg_start, u32, nmax + 1);
+  ALLOC(sc.leaf_seg_of, u32, nmax);
+  ALLOC(sc.up_seg_start, u32, nmax + 1);
+  for (int b = 0; b < 2; ++b) {
+    ALLOC(sc.it_rep[b], u32, nmax);
+    ALLOC(sc.it_cseq[b], u32, nmax);
+    ALLOC(sc.it_skey[b], u32, nmax);
+  }
+  ALLOC(sc.seg_vb0, u32, nmax);
+  ALLOC(sc.seg_vb1, u32, nmax);
+  ALLOC(sc.seg_carry, u32, nmax);
+  ALLOC(sc.mask, u32, nmax);
+  ALLOC(sc.prefix, u32, nmax);
+  ALLOC(sc.done_e, u32, done_cap);
+  ALLOC(sc.done_lvl, u32, done_cap);
+  ALLOC(sc.done_cseq, u32, done_cap);
+  ALLOC(sc.done_rank, u32, done_cap);
+  ALLOC(sc.r_done, u32, done_cap);
+  ALLOC(sc.r_dense_n, u32, done_cap);
+  ALLOC(sc.r_topk_n, u32, done_cap);
+  ALLOC(sc.r_meta_n, u32, done_cap);
+  ALLOC(sc.r_dense_base, u64, done_cap + 1);
+  ALLOC(sc.r_topk_off, u64, done_cap + 1);
+  ALLOC(sc.r_arena_base, u64, done_cap + 1);
+  if (concat >= 0) {
+    ALLOC(sc.dense, uint4, std::max<u64>(dense_cap, 1));
+    ALLOC(sc.dst, u64, dense_cap + 1);
+    ALLOC(sc.lenscan, u64, nmax + 1);
+  }
+  ALLOC(sc.pairset, u64, PS);
+  sc.ps_mask = PS - 1;
+  sc.done_cap = (u32)done_cap;
+  const u64 scan_tiles = std::max<u64>(std::max<u64>(dense_cap, done_cap), nmax) / kScanTile + 2;
+  ALLOC(h->lbs.flag, u32, scan_tiles);
+  ALLOC(h->lbs.agg, u64, scan_tiles);
+  ALLOC(h->lbs.inc, u64, scan_tiles);
+  h->lbs.tiles = scan_tiles;
+  ALLOC(d.out_rec, alto_record, std::max<int64_t>(cfg.out_records, 1));
+  ALLOC(d.out_pay, int32_t, std::max<int64_t>(cfg.out_payload_elems, 1));
+  ALLOC(d.out_topk, alto_topk_pair, std::max<int64_t>(cfg.out_topk, 1));
+#undef ALLOC
+  if (ok && cudaMallocHost((void**)&h->h_ctl, sizeof(Ctl)) != cudaSuccess) {
+    h->h_ctl = nullptr;
+    ok = false;
+  }
+  if (!ok) {
+    free_all(h, s);
+    cudaStreamSynchronize(s);
+    delete h;
+    return ALTO_ENOMEM;
+  }
+  // initial state
+  cudaMemsetAsync(d.ctl, 0, sizeof(Ctl), s);
+  cudaMemsetAsync(d.tab.key, 0xFF, sizeof(u64) * T, s);
+  cudaMemsetAsync(d.tab.done_epoch, 0, sizeof(u32) * T, s);
+  cudaMemsetAsync(sc.mask, 0, sizeof(u32) * nmax, s);
+  cudaMemsetAsync(sc.pairset, 0, sizeof(u64) * PS, s);
+  cudaMemsetAsync(h->leaf_sort.hist, 0, sizeof(u32) * 4 * 256, s);
+  cudaMemsetAsync(h->leaf_sort.lookback, 0, sizeof(u64) * sort_tiles * 256, s);
+  cudaMemsetAsync(h->lbs.flag, 0, sizeof(u32) * scan_tiles, s);
+  if (concat >= 0) cudaMemsetAsync(sc.dense, 0, sizeof(uint4) * std::max<u64>(dense_cap, 1), s);
+  if (cudaGetLastError() != cudaSuccess) {
+    free_all(h, s);
+    delete h;
+    return ALTO_ECUDA;
+  }
+  *out = h;
+  return ALTO_OK;
+}
+
+alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream) {
+  if (h == nullptr || b == nullptr) return ALTO_EINVAL;
+  if (h->latched != ALTO_OK) return h->latched;
+  const alto_agg_config& cfg = h->cfg;
+  if (b->depth != cfg.depth) return ALTO_EINVAL;
+  if (b->n < 0 || b->n > cfg.max_batch_fragments) return ALTO_EINVAL;
+  if (b->n_payload < 0 || b->n_payload > cfg.max_batch_payload) return ALTO_EINVAL;
+  if (b->n > 0 && (b->tags == nullptr || b->payload_off == nullptr)) return ALTO_EINVAL;
+  if (b->n_payload > 0 && b->payload == nullptr) return ALTO_EINVAL;
+  if (b->n > 0 && h->d.cfg.has_score && b->score == nullptr) return ALTO_EINVAL;
+  cudaStream_t s = (cudaStream_t)stream;
+  Dev d = h->d;
+  const int D = cfg.depth;
+  const u32 n = (u32)b->n;
+  Batch bt;
+  bt.tags = b->tags;
+  bt.off = b->payload_off;
+  bt.pay = b->payload;
+  bt.score = h->d.cfg.has_score ? b->score : nullptr;
+  bt.n = n;
+  bt.n_payload = (u64)b->n_payload;
+  const u32 nmax = (u32)cfg.max_batch_fragments;
+  const int grid = h->num_sms * 8;
+  const u64 spin = d.cfg.spin_limit;
+
+  if (h->pushed % 127 == 0 && h->pushed > 0)
+    cudaMemsetAsync(d.sc.pairset, 0, sizeof(u64) * (d.sc.ps_mask + 1), s);
+  h->pushed += 1;
+  h->last_stream = s;
+  if (h->profiling) h->prof_pushes += 1;
+  StageClock clk(h, s);
+  int64_t l0 = h->launches;
+  int stage = 0;
+  auto stage_enter = [&](int st) {
+    if (h->profiling) h->stage_launches[stage] += h->launches - l0;
+    l0 = h->launches;
+    stage = st;
+    clk.enter(st);
+  };
+  int sl = 0;  // launches inside sort_pairs
+  clk.enter(0);
+  k_begin<<<1, 1, 0, s>>>(d.ctl, n);
+  h->launches += 1;
+  if (n > 0) {
+    int site = 0;
+    k_ingest<<<grid, kThreads, 0, s>>>(d, bt);
+    h->launches += 1;
+    // leaf level: sort fragments by their leaf-parent group
+    stage_enter(1);
+    int cur = sort_pairs(&d.ctl->n, nmax, h->tbits, true, h->leaf_sort, d.ctl, site, spin,
+                         h->num_sms, s, &sl);
+    h->launches += sl;
+    sl = 0;
+    site += 4;
+    d.sc.leaf_keys = h->leaf_sort.keys[cur];
+    d.sc.leaf_perm = h->leaf_sort.vals[cur];
+    stage_enter(2);
+    {
+      SegFind f{d.sc.leaf_keys, d.sc.leaf_seg_start, d.sc.leaf_seg_of, &d.ctl->n, nmax,
+                &d.ctl->n_segs[D - 1]};
+      launch_scan(h, f, nmax, site++, s);
+    }
+    int set = 0;
+    k_reduce<true><<<grid, kThreads, 0, s>>>(d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
+                                             d.sc.leaf_seg_start, set);
+    h->launches += 1;
+    stage_enter(3);
+    for (int l = D - 2; l >= 0; --l) {
+      set ^= 1;  // items written by the level below
+      k_items_lookup<<<grid, kThreads, 0, s>>>(d, bt, l, set);
+      h->launches += 1;
+      int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nmax, h->tbits, true, h->up_sort, d.ctl, site,
+                          spin, h->num_sms, s, &sl);
+      h->launches += sl;
+      sl = 0;
+      site += 4;
+      d.sc.up_keys = h->up_sort.keys[c2];
+      d.sc.up_perm = h->up_sort.vals[c2];
+      SegFind f{d.sc.up_keys, d.sc.up_seg_start, nullptr, &d.ctl->n_segs[l + 1], nmax,
+                &d.ctl->n_segs[l]};
+      launch_scan(h, f, nmax, site++, s);
+      k_reduce<false><<<grid, kThreads, 0, s>>>(d, bt, l, d.sc.up_keys, d.sc.up_perm,
+                                                d.sc.up_seg_start, set);
+      h->launches += 1;
+    }
+    // emission order
+    stage_enter(4);
+    {
+      RankScan f{d.sc.mask, d.sc.prefix, &d.ctl->n};
+      launch_scan(h, f, nmax, site++, s);
+    }
+    k_done_rank<<<grid, kThreads, 0, s>>>(d);
+    h->launches += 1;
+    const u32 dcap = d.sc.done_cap;
+    {
+      CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0};
+      launch_scan(h, f0, dcap, site++, s);
+      CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
+      launch_scan(h, f1, dcap, site++, s);
+      CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
+      launch_scan(h, f2, dcap, site++, s);
+    }
+    k_check<<<1, 1, 0, s>>>(d);
+    h->launches += 1;
+    if (d.cfg.concat_level >= 0) {
+      stage_enter(5);
+      LenScan fl{d.sc.leaf_perm, bt.off, d.sc.lenscan, &d.ctl->n};
+      launch_scan(h, fl, nmax, site++, s);
+      k_carry_alloc<<<grid, kThreads, 0, s>>>(d);
+      k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
+      k_carry_copy<<<grid, kThreads, 0, s>>>(d, bt);
+      h->launches += 3;
+      stage_enter(6);
+      k_dense_batch<<<grid, kThreads, 0, s>>>(d, bt);
+      k_dense_arena<<<grid, kThreads, 0, s>>>(d);
+      h->launches += 2;
+      DenseScan fd{d.sc.dense, d.sc.dst, d.ctl};
+      launch_scan(h, fd, d.cfg.dense_cap, site++, s);
+      k_check2<<<1, 1, 0, s>>>(d);
+      h->launches += 1;
+      stage_enter(7);
+      k_gather<<<grid, kThreads, 0, s>>>(d, bt);
+      h->launches += 1;
+    }
+    stage_enter(8);
+    k_records<<<grid, kThreads, 0, s>>>(d);
+    k_sweep<<<grid, kThreads, 0, s>>>(d);
+    h->launches += 2;
+  } else {
+    stage_enter(8);
+  }
+  k_end<<<1, 1, 0, s>>>(d.ctl, n);
+  h->launches += 1;
+  stage_enter(ALTO_NUM_STAGES);
+  clk.finish();
+  if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
+  return ALTO_OK;
+}
+
+alto_status alto_agg_drain(alto_agg_t* h, void* stream, alto_drain* out) {
+  if (h == nullptr || out == nullptr) return ALTO_EINVAL;
+  cudaStream_t s = (cudaStream_t)stream;
+  memset(out, 0, sizeof(*out));
+  if (cudaMemcpyAsync(h->h_ctl, h->d.ctl, sizeof(Ctl), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    return ALTO_ECUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return ALTO_ECUDA;
+  const Ctl& c = *h->h_ctl;
+  out->first_batch = h->drain_first;
+  out->n_batches = h->pushed - h->drain_first;
+  h->drain_first = h->pushed;
+  if (c.status != ALTO_OK) {
+    h->latched = c.status;
+    return c.status;
+  }
+  out->n_records = (int64_t)c.rec_count;
+  out->records = h->d.out_rec;
+  out->n_payload = (int64_t)c.pay_count;
+  out->payload = h->d.out_pay;
+  out->n_topk = (int64_t)c.topk_count;
+  out->topk = h->d.out_topk;
+  k_drain_reset<<<1, 1, 0, s>>>(h->d.ctl);
+  if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
+  return ALTO_OK;
+}
+
+alto_status alto_agg_stats(alto_agg_t* h, void* stream, int64_t* open_groups, int64_t* arena_used) {
+  if (h == nullptr) return ALTO_EINVAL;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (cudaMemcpyAsync(h->h_ctl, h->d.ctl, sizeof(Ctl), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    return ALTO_ECUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return ALTO_ECUDA;
+  if (open_groups) *open_groups = (int64_t)h->h_ctl->live_groups;
+  if (arena_used) *arena_used = (int64_t)h->h_ctl->arena_used;
+  return h->h_ctl->status;
+}
+
+alto_status alto_agg_profile(alto_agg_t* h, int enable) {
+  if (h == nullptr) return ALTO_EINVAL;
+  if (enable) {
+    if (h->last_stream || h->pushed) cudaStreamSynchronize(h->last_stream);
+    collect_profile(h);
+    h->profiling = true;
+    h->prof_pushes = 0;
+    h->launches = 0;
+    for (int i = 0; i < ALTO_NUM_STAGES; ++i) {
+      h->stage_ms[i] = 0.0;
+      h->stage_launches[i] = 0;
+    }
+  } else {
+    h->profiling = false;
+  }
+  return ALTO_OK;
+}
+
+alto_status alto_agg_profile_read(alto_agg_t* h, alto_profile* out) {
+  if (h == nullptr || out == nullptr) return ALTO_EINVAL;
+  if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) return ALTO_ECUDA;
+  collect_profile(h);
+  out->pushes = h->prof_pushes;
+  out->launches = h->launches;
+  for (int i = 0; i < ALTO_NUM_STAGES; ++i) {
+    out->stage_ms[i] = h->stage_ms[i];
+    out->stage_launches[i] = h->stage_launches[i];
+  }
+  return ALTO_OK;
+}
+
+alto_status alto_agg_destroy(alto_agg_t* h) {
+  if (h == nullptr) return ALTO_OK;
+  cudaDeviceSynchronize();
+  for (auto& ev : h->ev_pending)
+    for (cudaEvent_t e : ev)
+      if (e) cudaEventDestroy(e);
+  for (cudaEvent_t e : h->ev_free) cudaEventDestroy(e);
+  free_all(h, nullptr);
+  cudaDeviceSynchronize();
+  delete h;
+  return ALTO_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,25 @@
+// Host-side launch interfaces shared between the library's translation units.
+#pragma once
+
+#include "common.cuh"
+
+namespace alto {
+
+struct SortBuffers {
+  u32* keys[2];
+  u32* vals[2];
+  u32* hist;      // [4][256], zero between sorts
+  u32* bin_base;  // [4][256]
+  u64* lookback;  // [lb_tiles][256]
+  u64 lb_tiles;
+};
+
+// Stable sort of keys[0] (values: identity when vals_identity, else vals[0])
+// by the low `bits` bits; the element count is read from n_dev on the device
+// and clamped to n_cap.  Returns the index (0/1) of the buffers holding the
+// result.  Uses launch sites site_base .. site_base + passes - 1.
+int sort_pairs(const u32* n_dev, u32 n_cap, int bits, bool vals_identity, SortBuffers& b,
+               Ctl* ctl, int site_base, u64 spin_limit, int num_sms, cudaStream_t s,
+               int* launches);
+
+}  // namespace alto

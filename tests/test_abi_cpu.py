@@ -1,0 +1,91 @@
+"""C-ABI library: builds for sm_103a, loads, exports every declared entry
+point, and its host-side argument checks answer without touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2403_04311_gb300 as alto
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = []
+    inc = os.path.join(ROOT, "include")
+    for f in sorted(os.listdir(inc)):
+        if f.endswith(".h"):
+            txt = open(os.path.join(inc, f)).read()
+            names += re.findall(r"^alto_status\s+(alto_\w+)\s*\(", txt, flags=re.M)
+    return names
+
+
+def test_library_builds_and_exports_every_declared_symbol():
+    lib = alto.load_library()
+    names = declared_functions()
+    assert set(alto.EXPORTS) <= set(names)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_library_is_built_for_sm_103a():
+    import subprocess
+    path = alto.build()
+    out = subprocess.run(["/usr/local/cuda/bin/cuobjdump", "--list-elf", path],
+                         capture_output=True, text=True).stdout
+    assert "sm_103a" in out
+
+
+def _cfg(**kw):
+    base = dict(depth=2, payload_op=[0, 1], score_op=[0, 0], max_batch_fragments=1024,
+                max_batch_payload=4096)
+    base.update(kw)
+    d = base.pop("depth")
+    return alto.make_config(d, base.pop("payload_op"), base.pop("score_op"), base.pop("topk_k", None), **base)
+
+
+@pytest.mark.parametrize("bad", [
+    dict(depth=0, payload_op=[], score_op=[]),
+    dict(depth=9, payload_op=[0] * 9, score_op=[0] * 9),
+    dict(payload_op=[1, 1]),                         # two CONCAT levels
+    dict(payload_op=[0, 2]),                         # unknown payload op
+    dict(score_op=[3, 0]),                           # unknown score op
+    dict(score_op=[2, 0], topk_k=[0, 0]),            # TOPK without k
+    dict(score_op=[2, 0], topk_k=[33, 0]),           # k above 32
+    dict(max_batch_fragments=0),
+    dict(max_batch_fragments=1 << 30),
+    dict(max_batch_payload=-1),
+    dict(max_open_groups=(1 << 25) + 1),
+    dict(arena_elems=1 << 32),
+])
+def test_create_rejects_bad_configs_on_host(bad):
+    lib = alto.load_library()
+    cfg = _cfg(**bad)
+    h = ctypes.c_void_p(12345)
+    st = lib.alto_agg_create(ctypes.byref(cfg), None, None, ctypes.byref(h))
+    assert st == alto.EINVAL
+    assert h.value == 12345  # untouched
+
+
+def test_null_arguments():
+    lib = alto.load_library()
+    assert lib.alto_agg_destroy(None) == alto.OK
+    assert lib.alto_agg_push_batch(None, None, None) == alto.EINVAL
+    assert lib.alto_agg_drain(None, None, None) == alto.EINVAL
+    assert lib.alto_agg_create(None, None, None, None) == alto.EINVAL
+    h = ctypes.c_void_p()
+    assert lib.alto_agg_create(ctypes.byref(_cfg()), None, None, None) == alto.EINVAL
+    bad_alloc = alto.alto_allocator()
+    assert lib.alto_agg_create(ctypes.byref(_cfg()), ctypes.byref(bad_alloc), None,
+                               ctypes.byref(h)) == alto.EINVAL
+
+
+def test_status_codes_match_oracle_and_header():
+    import oracle
+    txt = open(os.path.join(ROOT, "include", "alto_agg.h")).read()
+    vals = dict(re.findall(r"#define ALTO_(E\w+|OK)\s+\(?(-?\d+)\)?", txt))
+    assert int(vals["OK"]) == alto.OK == oracle.OK
+    for name in ["EINVAL", "ENOMEM", "ENOSPC", "EDUP", "ELAST", "EINCONSIST", "ECLOSED"]:
+        assert int(vals[name]) == getattr(alto, name) == getattr(oracle, name)
+    assert alto.RECORD_DTYPE == oracle.RECORD_DTYPE

@@ -1,0 +1,154 @@
+"""CUDA path vs the oracle, bit for bit, through the C ABI."""
+import json
+import os
+import random
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import oracle
+import paper_2403_04311_gb300 as alto
+from fragments import split, to_batch, tree_fragments
+from gen import make_stream
+from gpu_harness import (assert_same, run_both_stream, run_gpu_batches, run_oracle_batches,
+                         stream_caps)
+
+pytestmark = pytest.mark.gpu
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def small_caps(n, payload, depth, k=8):
+    return dict(max_batch_fragments=max(n, 1), max_batch_payload=max(payload, 1),
+                max_open_groups=4096, arena_elems=1 << 16, out_records=4096,
+                out_payload_elems=1 << 14, out_topk=4096, max_emit_children=4096)
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny64", "factcheck", "throughput", "tokens", "adversarial"])
+@pytest.mark.parametrize("drain_every", [1, 3])
+def test_workloads_small(name, drain_every):
+    s = make_stream(name, small=True)
+    o, g = run_both_stream(s, drain_every=drain_every)
+    assert all(d.status == 0 for d in o)
+    assert_same(o, g, f"{name}/{drain_every}")
+
+
+def test_golden_factool_claims():
+    fx = json.load(open(os.path.join(GOLDEN, "factool_claims.json")))
+    frags = [(tuple(tuple(t) for t in f["tags"]), f["tokens"], f["score"]) for f in fx["fragments"]]
+    batches = [to_batch(p, fx["depth"], True) for p in split(frags, fx["batches"])]
+    _, g = run_gpu_batches(fx["depth"], fx["payload_op"], fx["score_op"], fx["topk_k"], batches,
+                           small_caps(8, 16, fx["depth"]))
+    o = run_oracle_batches(fx["depth"], fx["payload_op"], fx["score_op"], fx["topk_k"], batches)
+    assert_same(o, g, "golden")
+    _st, rec, pay, tk = g[1]
+    assert pay.tolist() == fx["drains"][1]["payload"]
+    assert rec["parent_id"].tolist() == [41, 40, 7]
+
+
+def test_golden_errors_detected_on_device():
+    fx = json.load(open(os.path.join(GOLDEN, "errors.json")))
+    for case in fx["cases"]:
+        if "closed" in case["name"]:
+            continue  # a repeat across batches of an emitted group: not in the device scope
+        frags = [(tuple(tuple(t) for t in f["tags"]), f["tokens"], 0.0) for f in case["fragments"]]
+        batches = []
+        for part in split(frags, case["batches"]):
+            b = to_batch(part, fx["depth"], False)
+            if case.get("bad_offsets"):
+                b["off"][1], b["off"][2] = b["off"][2], b["off"][1]
+            batches.append(b)
+        _, g = run_gpu_batches(fx["depth"], fx["payload_op"], fx["score_op"], fx["topk_k"], batches,
+                               small_caps(8, 16, fx["depth"]))
+        assert [d[0] for d in g] == case["status"], case["name"]
+
+
+def _brute_cases(seed=0, count=150):
+    rng = random.Random(seed)
+    shapes = [3, [2, 1], [1, 3, 2], [[2, 1], [3]], [[1], [2, 2], [1]], [[2, [1, 2]], [1, [1]]][:0]]
+    shapes = [3, [2, 1], [1, 3, 2], [[2, 1], [3]], [[1], [2, 2], [1]], [[[1, 2], [1]], [[2]]]]
+    out = []
+    for _ in range(count):
+        shape = rng.choice(shapes)
+        depth = 1
+        x = shape
+        while not isinstance(x, int):
+            x = x[0]
+            depth += 1
+        frags = tree_fragments(shape, score_fn=lambda k: [-1.0, -0.0, 0.0, 0.5, 0.5, 2.0, -3.5][k % 7])
+        rng.shuffle(frags)
+        n = len(frags)
+        cuts, left = [], n
+        while left:
+            c = rng.randint(1, left)
+            cuts.append(c)
+            left -= c
+        po = [0] * depth
+        if rng.random() < 0.8:
+            po[depth - 1] = 1
+        so = [rng.choice([0, 1, 2]) for _ in range(depth)]
+        kk = [rng.choice([1, 2, 3]) if x == 2 else 0 for x in so]
+        out.append((depth, po, so, kk, frags, cuts))
+    return out
+
+
+def test_bruteforce_streams_on_device():
+    for depth, po, so, kk, frags, cuts in _brute_cases():
+        ws = any(x != 0 for x in so)
+        batches = [to_batch(p, depth, ws) for p in split(frags, cuts)]
+        _, g = run_gpu_batches(depth, po, so, kk, batches, small_caps(len(frags), 64, depth))
+        o = run_oracle_batches(depth, po, so, kk, batches)
+        assert_same(o, g, f"{depth} {po} {so} {kk} {cuts}")
+
+
+def test_nan_score_is_einval():
+    frags = tree_fragments([2], score_fn=lambda k: float("nan") if k == 1 else 1.0)
+    b = to_batch(frags, 2, True)
+    _, g = run_gpu_batches(2, [0, 1], [0, 1], [0, 0], [b], small_caps(4, 16, 2))
+    assert g[0][0] == alto.EINVAL
+
+
+def test_poisoned_handle_and_destroy():
+    frags = tree_fragments([2, 2])
+    bad = list(frags) + [frags[0]]     # duplicate leaf in the batch
+    agg = alto.Aggregator(2, [0, 1], [0, 0], None, **small_caps(8, 64, 2))
+    db = alto.to_device(to_batch(bad, 2, False))
+    assert agg.push(db.tags, db.off, db.payload) == alto.OK     # device error: found later
+    assert agg.drain().status == alto.EDUP
+    db2 = alto.to_device(to_batch(frags, 2, False))
+    assert agg.push(db2.tags, db2.off, db2.payload) == alto.EDUP
+    assert agg.drain().status == alto.EDUP
+    agg.close()
+
+
+def test_output_capacity_is_enospc():
+    s = make_stream("tiny64")
+    caps = stream_caps(s)
+    caps["out_records"] = 5
+    _, g = run_gpu_batches(s.depth, s.payload_op, s.score_op, s.topk_k, [s.batch(0)], caps)
+    assert g[0][0] == alto.ENOSPC
+
+
+def test_host_argument_errors_do_not_poison():
+    frags = tree_fragments([2, 1])
+    agg = alto.Aggregator(2, [0, 1], [0, 0], None, **small_caps(4, 16, 2))
+    db = alto.to_device(to_batch(frags, 2, False))
+    big = alto.to_device(to_batch(frags + tree_fragments([3], id_base=900), 2, False))
+    assert agg.push(big.tags, big.off, big.payload) == alto.EINVAL   # n above max_batch_fragments
+    assert agg.push(db.tags, db.off, db.payload) == alto.OK
+    d = agg.drain()
+    assert d.status == alto.OK
+    rec, pay, _ = d.host()
+    assert len(rec) == 3
+    agg.close()
+
+
+def test_determinism_repeated_runs():
+    s = make_stream("adversarial", small=True)
+    _, g1 = run_both_stream(s, drain_every=2)
+    _, g2 = run_both_stream(s, drain_every=2)
+    for a, b in zip(g1, g2):
+        assert a[0] == b[0]
+        assert np.array_equal(a[1].view(np.uint8), b[1].view(np.uint8))
+        assert np.array_equal(a[2], b[2])
