@@ -59,7 +59,8 @@ struct Scratch {
   u32* it_skey[2];       // items: largest score key of the child
   u32* seg_vb0;          // leaf segments: meta vector base (leaves)
   u32* seg_vb1;          // leaf segments: payload vector base (elements)
-  u32* seg_carry;        // leaf segments: 1 if the leaves go to the arena
+  u32* seg_carry;        // leaf segments: 1 to the arena, 2 placed densely
+  u32* leaf_pos;         // [n_max] sorted leaf j: payload offset inside its segment
   u32* mask;             // [n_max] bit (D-1-l): a level-l group completes at this seq
   u32* prefix;           // [n_max] records completed before this seq
   u32* done_e;           // [done_cap]
@@ -105,7 +106,8 @@ __device__ __forceinline__ u32 gstride() { return gridDim.x * blockDim.x; }
 // ---------------------------------------------------------------------------
 // open-group hash table (linear probing; a slot index is the entry id)
 // ---------------------------------------------------------------------------
-__device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, int* inserted) {
+__device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, int* inserted,
+                                  const u64* tags = nullptr, u64 n = 0, u32 rep = 0, int l = 0) {
   u32 h = (u32)mix64(key) & tab.mask;
   for (int p = 0; p < tab.max_probe; ++p) {
     u64 cur = ((volatile u64*)tab.key)[h];
@@ -123,6 +125,16 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
           tab.vec_n[2 * (u64)h] = 0;
           tab.vec_n[2 * (u64)h + 1] = 0;
         }
+        if (tags) {
+          for (int q = 0; q < l; ++q) tab.chain[(u64)h * tab.chain_len + q] = tags[(u64)q * n + rep];
+        }
+        tab.touch[h] = 0;
+        tab.acc_cnt[h] = 0;
+        tab.acc_m1[h] = 0;
+        tab.acc_fmin[h] = kNone;
+        tab.acc_fmax1[h] = 0;
+        tab.acc_cs1[h] = 0;
+        tab.acc_smx[h] = 0;
         *inserted = 1;
         return h;
       }
@@ -219,7 +231,8 @@ __global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
     u64 t = b.tags[(u64)(D - 1) * b.n + i];
     u64 up = (D > 1) ? b.tags[(u64)(D - 2) * b.n + i] : 0ull;
     int ins = 0;
-    u32 e = ht_find_or_insert(d.tab, ((u64)(D - 1) << 32) | tag_pid(t), up, ctl, &ins);
+    u32 e = ht_find_or_insert(d.tab, ((u64)(D - 1) << 32) | tag_pid(t), up, ctl, &ins, b.tags,
+                              b.n, i, D - 1);
     if (ins) atomicAdd(&s_ins, 1u);
     d.sc.leaf_sort_keys0[i] = e;
     if (ps_insert(d.sc, e, tag_child(t), ep7, ctl)) raise_err(ctl, ALTO_EDUP);
@@ -243,7 +256,7 @@ __global__ void __launch_bounds__(kThreads) k_items_lookup(Dev d, Batch b, int l
     u64 t = b.tags[(u64)l * b.n + rep];
     u64 up = (l > 0) ? b.tags[(u64)(l - 1) * b.n + rep] : 0ull;
     int ins = 0;
-    u32 e = ht_find_or_insert(d.tab, ((u64)l << 32) | tag_pid(t), up, ctl, &ins);
+    u32 e = ht_find_or_insert(d.tab, ((u64)l << 32) | tag_pid(t), up, ctl, &ins, b.tags, b.n, rep, l);
     if (ins) atomicAdd(&s_ins, 1u);
     d.sc.up_sort_keys0[x] = e;
     if (ps_insert(d.sc, e, tag_child(t), ep7, ctl)) raise_err(ctl, ALTO_EINCONSIST);
@@ -313,40 +326,55 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
     for (int q = 0; q < kMaxDepth; ++q) htag[q] = (q < l) ? b.tags[(u64)q * n + rep0] : 0ull;
     u32 cnt = 0, m1 = 0, fmin = kNone, fmax = 0, hasf = 0, cmax = 0, smx = 0, bad = 0;
     u64 lsum = 0;
-    for (u32 j = j0 + lane; j < j1; j += 32) {
-      const u32 x = min(sperm[j], n_items - 1);
-      u32 rep, done, cs, sk;
-      u64 len = 0;
-      if (LEAF) {
-        rep = x;
-        done = 1;
-        cs = x;
-        sk = d.cfg.has_score ? score_key(b.score[x]) : 0u;
-        len = b.off[x + 1] - b.off[x];
-      } else {
-        rep = it_rep[x];
-        u32 cf = it_cseq[x];
-        done = cf >> 31;
-        cs = cf & 0x7FFFFFFFu;
-        sk = it_skey[x];
-      }
-      const u64 t = b.tags[(u64)l * n + rep];
-      const u32 c = tag_child(t);
-      m1 = max(m1, c + 1);
-      if (tag_last(t)) {
-        hasf = 1;
-        fmin = min(fmin, c);
-        fmax = max(fmax, c);
-      }
-      if (done) {
-        ++cnt;
-        cmax = max(cmax, cs);
-        smx = max(smx, sk);
-      }
-      lsum += len;
+    u32 running = 0;  // payload elements of the segment's earlier leaves (leaf level)
+    for (u32 jb = j0; jb < j1; jb += 32) {
+      const u32 j = jb + lane;
+      const bool valid = j < j1;
+      u32 len = 0;
+      if (valid) {
+        const u32 x = min(sperm[j], n_items - 1);
+        u32 rep, done, cs, sk;
+        if (LEAF) {
+          rep = x;
+          done = 1;
+          cs = x;
+          sk = d.cfg.has_score ? score_key(b.score[x]) : 0u;
+          len = b.off[x + 1] - b.off[x];
+        } else {
+          rep = it_rep[x];
+          u32 cf = it_cseq[x];
+          done = cf >> 31;
+          cs = cf & 0x7FFFFFFFu;
+          sk = it_skey[x];
+        }
+        const u64 t = b.tags[(u64)l * n + rep];
+        const u32 c = tag_child(t);
+        m1 = max(m1, c + 1);
+        if (tag_last(t)) {
+          hasf = 1;
+          fmin = min(fmin, c);
+          fmax = max(fmax, c);
+        }
+        if (done) {
+          ++cnt;
+          cmax = max(cmax, cs);
+          smx = max(smx, sk);
+        }
+        lsum += len;
 #pragma unroll
-      for (int q = 0; q < kMaxDepth; ++q)
-        if (q < l && b.tags[(u64)q * n + rep] != htag[q]) bad = 1;
+        for (int q = 0; q < kMaxDepth; ++q)
+          if (q < l && b.tags[(u64)q * n + rep] != htag[q]) bad = 1;
+      }
+      if (LEAF) {
+        u32 incl = len;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        if (valid) d.sc.leaf_pos[j] = running + incl - len;
+        running += __shfl_sync(0xFFFFFFFFu, incl, 31);
+      }
     }
     cnt = __reduce_add_sync(0xFFFFFFFFu, cnt);
     m1 = __reduce_max_sync(0xFFFFFFFFu, m1);
@@ -431,7 +459,7 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
         }
       }
       if (carry) {
-        d.sc.seg_carry[s] = complete ? 0u : 1u;
+        d.sc.seg_carry[s] = complete ? 2u : 1u;  // 1: to the arena, 2: placed densely
         if (!complete) {
           const u32 v0 = d.tab.vec_n[2 * (u64)e], v1 = d.tab.vec_n[2 * (u64)e + 1];
           d.sc.seg_vb0[s] = v0;
@@ -445,6 +473,131 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
         nx_cseq[s] = (complete ? 0x80000000u : 0u) | cmax;
         nx_skey[s] = smn;
       }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// upper levels without TOPK: hash-table entries accumulate the batch's items
+// with warp-aggregated atomics; the touched entries are then finalised.
+// ---------------------------------------------------------------------------
+// Items of level l: check ancestry against the entry and accumulate.
+__global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int l, int in_set) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  const u32 ni = min(ctl->n_segs[l + 1], d.cfg.n_max);
+  const u32 ep = ctl->epoch;
+  const u32* it_rep = d.sc.it_rep[in_set];
+  const u32* it_cseq = d.sc.it_cseq[in_set];
+  const u32* it_skey = d.sc.it_skey[in_set];
+  u32* list = d.sc.up_seg_start;  // touched entries of this level
+  const u64 n = b.n;
+  const u32 end = (ni + 31) & ~31u;
+  for (u32 x = gtid(); x < end; x += gstride()) {
+    const bool valid = x < ni;
+    u32 e = 0, rep = 0, c = 0, f = 0, done = 0, cs = 0, sk = 0;
+    if (valid) {
+      e = d.sc.up_sort_keys0[x] & d.tab.mask;
+      rep = it_rep[x];
+      const u64 t = b.tags[(u64)l * n + rep];
+      c = tag_child(t);
+      f = tag_last(t);
+      const u32 cf = it_cseq[x];
+      done = cf >> 31;
+      cs = cf & 0x7FFFFFFFu;
+      sk = it_skey[x];
+      bool bad = false;
+      for (int q = 0; q < l; ++q)
+        if (b.tags[(u64)q * n + rep] != d.tab.chain[(u64)e * d.tab.chain_len + q]) bad = true;
+      if (bad) raise_err(ctl, ALTO_EINCONSIST);
+      if (atomicExch(&d.tab.touch[e], ep) != ep) {
+        const u32 pos = atomicAdd(&ctl->n_segs[l], 1u);
+        if (pos < d.cfg.n_max) list[pos] = e;
+        d.tab.acc_rep[e] = rep;
+      }
+    }
+    // lanes past the end form their own group; the whole warp takes part
+    const u32 key = valid ? e : kNone;
+    {
+      const u32 peers = __match_any_sync(0xFFFFFFFFu, key);
+      const int leader = __ffs(peers) - 1;
+      const u32 cnt = __reduce_add_sync(peers, done);
+      const u32 m1 = __reduce_max_sync(peers, valid ? c + 1 : 0u);
+      const u32 fmin = __reduce_min_sync(peers, (valid && f) ? c : kNone);
+      const u32 fmax1 = __reduce_max_sync(peers, (valid && f) ? c + 1 : 0u);
+      const u32 cs1 = __reduce_max_sync(peers, (valid && done) ? cs + 1 : 0u);
+      const u32 smx = __reduce_max_sync(peers, (valid && done) ? sk : 0u);
+      if (valid && (int)(threadIdx.x & 31) == leader) {
+        if (cnt) atomicAdd(&d.tab.acc_cnt[e], cnt);
+        if (m1) atomicMax(&d.tab.acc_m1[e], m1);
+        if (fmin != kNone) atomicMin(&d.tab.acc_fmin[e], fmin);
+        if (fmax1) atomicMax(&d.tab.acc_fmax1[e], fmax1);
+        if (cs1) atomicMax(&d.tab.acc_cs1[e], cs1);
+        if (smx) atomicMax(&d.tab.acc_smx[e], smx);
+      }
+    }
+  }
+}
+
+// One thread per touched entry: merge, test completion, emit the next items.
+__global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l, int in_set) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  const int D = d.cfg.depth;
+  const u32 nt = min(ctl->n_segs[l], d.cfg.n_max);
+  const u32 ep = ctl->epoch;
+  const u32* list = d.sc.up_seg_start;
+  u32* nx_rep = d.sc.it_rep[in_set ^ 1];
+  u32* nx_cseq = d.sc.it_cseq[in_set ^ 1];
+  u32* nx_skey = d.sc.it_skey[in_set ^ 1];
+  const u64 n = b.n;
+  for (u32 s = gtid(); s < nt; s += gstride()) {
+    const u32 e = list[s] & d.tab.mask;
+    const u32 cnt = d.tab.acc_cnt[e], m1 = d.tab.acc_m1[e], fmin = d.tab.acc_fmin[e];
+    const u32 fmax1 = d.tab.acc_fmax1[e], cs1 = d.tab.acc_cs1[e], smx = d.tab.acc_smx[e];
+    const u32 rep = d.tab.acc_rep[e];
+    // reset the accumulators for the next batch
+    d.tab.acc_cnt[e] = 0;
+    d.tab.acc_m1[e] = 0;
+    d.tab.acc_fmin[e] = kNone;
+    d.tab.acc_fmax1[e] = 0;
+    d.tab.acc_cs1[e] = 0;
+    d.tab.acc_smx[e] = 0;
+    if (l > 0 && d.tab.up[e] != b.tags[(u64)(l - 1) * n + rep]) raise_err(ctl, ALTO_EINCONSIST);
+    const u32 last_old = d.tab.last[e];
+    u32 nl = last_old;
+    if (fmax1) {
+      if (fmin + 1 != fmax1) raise_err(ctl, ALTO_ELAST);
+      if (last_old != kNone && last_old != fmin) raise_err(ctl, ALTO_ELAST);
+      if (last_old == kNone) nl = fmin;
+    }
+    const u32 m1n = max(d.tab.maxc1[e], m1);
+    if (nl != kNone && m1n > nl + 1) raise_err(ctl, ALTO_ELAST);
+    const u32 comp = d.tab.completed[e] + cnt;
+    const u32 smn = max(d.tab.smax[e], smx);
+    const bool complete = (nl != kNone) && (comp == nl + 1) && (m1n <= nl + 1);
+    d.tab.last[e] = nl;
+    d.tab.maxc1[e] = m1n;
+    d.tab.completed[e] = comp;
+    d.tab.smax[e] = smn;
+    const u32 cmax = cs1 ? cs1 - 1 : 0;
+    if (complete) {
+      u32 di = atomicAdd(&ctl->n_done, 1u);
+      if (di < d.sc.done_cap) {
+        d.sc.done_e[di] = e;
+        d.sc.done_lvl[di] = (u32)l;
+        d.sc.done_cseq[di] = cmax;
+        d.tab.done_epoch[e] = ep;
+        d.tab.done_idx[e] = di;
+        if (cmax < n) atomicOr(&d.sc.mask[cmax], 1u << (D - 1 - l));
+      } else {
+        raise_err(ctl, ALTO_ENOSPC);
+      }
+    }
+    if (l > 0) {
+      nx_rep[s] = rep;
+      nx_cseq[s] = (complete ? 0x80000000u : 0u) | cmax;
+      nx_skey[s] = smn;
     }
   }
 }
@@ -534,27 +687,88 @@ struct LenScan {
   __device__ void total(Ctl*, u64 t) const { out_scan[size(nullptr)] = t; }
 };
 
+// Chunks for the arena ranges reserved by this batch's open CONCAT groups.
+// A block counts its requests per size class in shared memory and takes them
+// from the class's free stack (or the bump allocator) with one atomic each.
+constexpr int kMaxReq = 8;
+
 __global__ void __launch_bounds__(kThreads) k_carry_alloc(Dev d) {
   Ctl* ctl = d.ctl;
   if (no_copy(ctl)) return;
+  __shared__ u32 s_cnt[kNumChunks];
+  __shared__ int s_old[kNumChunks];
+  __shared__ u32 s_avail[kNumChunks];
+  __shared__ u64 s_bump[kNumChunks];
+  __shared__ unsigned long long s_used;
   const u32 nseg = min(ctl->n_segs[d.cfg.depth - 1], d.cfg.n_max);
-  for (u32 s = gtid(); s < nseg; s += gstride()) {
-    if (!d.sc.seg_carry[s]) continue;
-    const u32 e = d.sc.leaf_keys[d.sc.leaf_seg_start[s]];
-    for (int vec = 0; vec < kVecs; ++vec) {
-      const u64 mult = (vec == 0) ? 2 : 1;
-      const u64 old_el = (u64)((vec == 0) ? d.sc.seg_vb0[s] : d.sc.seg_vb1[s]) * mult;
-      const u64 new_el = (u64)d.tab.vec_n[2 * (u64)e + vec] * mult;
-      if (new_el <= old_el) continue;
-      const int jf = (old_el == 0) ? 0 : chunk_of(old_el - 1) + 1;
-      const int jl = chunk_of(new_el - 1);
-      for (int j = jf; j <= jl && j < kNumChunks; ++j) {
-        u32 c = alloc_chunk(d.ar, ctl, j);
-        d.tab.dir[((u64)e * kVecs + vec) * kNumChunks + j] = c;
-        if (c != kNone) atomicAdd((unsigned long long*)&ctl->arena_used, (unsigned long long)chunk_size(j));
+  for (u32 base = blockIdx.x * blockDim.x; base < nseg; base += gridDim.x * blockDim.x) {
+    if (threadIdx.x < kNumChunks) s_cnt[threadIdx.x] = 0;
+    if (threadIdx.x == 0) s_used = 0;
+    __syncthreads();
+    const u32 s = base + threadIdx.x;
+    u32 e = 0;
+    int nreq = 0;
+    uint8_t rvec[kMaxReq], rj[kMaxReq];
+    u32 rr[kMaxReq];
+    if (s < nseg && d.sc.seg_carry[s] == 1u) {
+      e = d.sc.leaf_keys[d.sc.leaf_seg_start[s]] & d.tab.mask;
+      for (int vec = 0; vec < kVecs; ++vec) {
+        const u64 mult = (vec == 0) ? 2 : 1;
+        const u64 old_el = (u64)((vec == 0) ? d.sc.seg_vb0[s] : d.sc.seg_vb1[s]) * mult;
+        const u64 new_el = (u64)d.tab.vec_n[2 * (u64)e + vec] * mult;
+        if (new_el <= old_el) continue;
+        const int jf = (old_el == 0) ? 0 : chunk_of(old_el - 1) + 1;
+        const int jl = chunk_of(new_el - 1);
+        if (jl >= kNumChunks) raise_err(ctl, ALTO_ENOSPC);
+        for (int j = jf; j <= jl && j < kNumChunks; ++j) {
+          if (nreq < kMaxReq) {
+            rvec[nreq] = (uint8_t)vec;
+            rj[nreq] = (uint8_t)j;
+            rr[nreq] = atomicAdd(&s_cnt[j], 1u);
+            ++nreq;
+          } else {  // rare: a vector grew by many classes at once
+            u32 c = alloc_chunk(d.ar, ctl, j);
+            d.tab.dir[((u64)e * kVecs + vec) * kNumChunks + j] = c;
+            if (c != kNone) atomicAdd(&s_used, (unsigned long long)chunk_size(j));
+          }
+        }
       }
-      if (jl >= kNumChunks) raise_err(ctl, ALTO_ENOSPC);
     }
+    __syncthreads();
+    if (threadIdx.x < kNumChunks) {
+      const int j = threadIdx.x;
+      const u32 cnt = s_cnt[j];
+      if (cnt) {
+        const int old = atomicSub(&ctl->top[j], (int)cnt);
+        const u32 avail = (old <= 0) ? 0u : min((u32)old, cnt);
+        s_old[j] = old;
+        s_avail[j] = avail;
+        if (cnt > avail)
+          s_bump[j] = atomicAdd((unsigned long long*)&ctl->bump,
+                                (unsigned long long)((cnt - avail) * chunk_size(j)));
+      }
+    }
+    __syncthreads();
+    for (int q = 0; q < nreq; ++q) {
+      const int j = rj[q];
+      const u32 r = rr[q];
+      u32 c;
+      if (r < s_avail[j]) {
+        c = d.ar.stack[d.ar.stack_off[j] + (u64)(s_old[j] - 1 - (int)r)];
+      } else {
+        const u64 o = s_bump[j] + (u64)(r - s_avail[j]) * chunk_size(j);
+        if (o + chunk_size(j) > d.ar.elems) {
+          raise_err(ctl, ALTO_ENOSPC);
+          c = kNone;
+        } else {
+          c = (u32)o;
+        }
+      }
+      d.tab.dir[((u64)e * kVecs + rvec[q]) * kNumChunks + j] = c;
+      if (c != kNone) atomicAdd(&s_used, (unsigned long long)chunk_size(j));
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && s_used) atomicAdd((unsigned long long*)&ctl->arena_used, s_used);
   }
 }
 
@@ -563,34 +777,43 @@ __global__ void k_fix_tops(Ctl* ctl) {
   if (j < kNumChunks && ctl->top[j] < 0) ctl->top[j] = 0;
 }
 
+// Append the leaves of open CONCAT groups to their arena vectors: eight lanes
+// per leaf, over the sorted leaves.  A leaf's vector position is its group's
+// reserved base plus its offset inside the segment (written by the reduce).
 __global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch b) {
   Ctl* ctl = d.ctl;
   if (no_copy(ctl)) return;
   const int D = d.cfg.depth;
-  const u32 n = b.n;
+  const u64 n = b.n;
   const u32 nseg = min(ctl->n_segs[D - 1], d.cfg.n_max);
-  for (u32 j = gtid(); j < n; j += gstride()) {
+  const u32 sub = threadIdx.x & 7;
+  const u32 g0 = gtid() >> 3, ng = gstride() >> 3;
+  for (u32 j = g0; j < b.n; j += ng) {
     const u32 s = d.sc.leaf_seg_of[j];
-    if (s >= nseg || !d.sc.seg_carry[s]) continue;
+    if (s >= nseg || d.sc.seg_carry[s] != 1u) continue;
     const u32 i = d.sc.leaf_perm[j];
+    if (i >= b.n) continue;
     const u32 e = d.sc.leaf_keys[j] & d.tab.mask;
     const u32 s0 = d.sc.leaf_seg_start[s];
-    if (i >= n || s0 > j) continue;
+    if (s0 > j) continue;
+    const u32 o0 = b.off[i];
+    const u32 len = b.off[i + 1] - o0;
     const u64 mpos = (u64)d.sc.seg_vb0[s] + (j - s0);
-    const u64 ppos = (u64)d.sc.seg_vb1[s] + (d.sc.lenscan[j] - d.sc.lenscan[s0]);
-    const u32 c = tag_child(b.tags[(u64)(D - 1) * n + i]);
-    const u32 o0 = b.off[i], len = b.off[i + 1] - o0;
-    // stay inside the ranges reserved (and allocated) for this group
-    if (mpos >= d.tab.vec_n[2 * (u64)e] || ppos + len > d.tab.vec_n[2 * (u64)e + 1]) continue;
+    const u64 ppos = (u64)d.sc.seg_vb1[s] + d.sc.leaf_pos[j];
+    if (mpos >= d.tab.vec_n[2 * (u64)e] || ppos + len > d.tab.vec_n[2 * (u64)e + 1] ||
+        (u64)o0 + len > b.n_payload)
+      continue;
     bool ok;
-    u64 a = vec_addr(d.tab, e, 0, 2 * mpos, &ok);
-    if (ok) {
-      d.ar.pool[a] = (int32_t)c;
-      d.ar.pool[a + 1] = (int32_t)(u32)ppos;
+    if (sub == 0) {
+      const u64 a = vec_addr(d.tab, e, 0, 2 * mpos, &ok);
+      if (ok) {
+        d.ar.pool[a] = (int32_t)tag_child(b.tags[(u64)(D - 1) * n + i]);
+        d.ar.pool[a + 1] = (int32_t)(u32)ppos;
+      }
     }
-    for (u32 q = 0; q < len; ++q) {
-      u64 pa = vec_addr(d.tab, e, 1, ppos + q, &ok);
-      if (ok) d.ar.pool[pa] = b.pay[o0 + q];
+    for (u32 k = sub; k < len; k += 8) {
+      const u64 a = vec_addr(d.tab, e, 1, ppos + k, &ok);
+      if (ok) d.ar.pool[a] = b.pay[o0 + k];
     }
   }
 }
@@ -601,26 +824,29 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
   if (no_copy(ctl) || ctl->skip_dense) return;
   const int D = d.cfg.depth;
   const u32 ep = ctl->epoch;
-  const u32 n = b.n;
+  const u64 n = b.n;
   const u32 nd = min(ctl->n_done, d.sc.done_cap);
-  for (u32 j = gtid(); j < n; j += gstride()) {
+  const u32 nseg = min(ctl->n_segs[D - 1], d.cfg.n_max);
+  for (u32 j = gtid(); j < b.n; j += gstride()) {
+    const u32 s = d.sc.leaf_seg_of[j];
+    if (s >= nseg || d.sc.seg_carry[s] != 2u) continue;
     const u32 e = d.sc.leaf_keys[j] & d.tab.mask;
-    if (d.tab.done_epoch[e] != ep) continue;
+    const u32 i = d.sc.leaf_perm[j];
+    if (i >= b.n || d.tab.done_epoch[e] != ep) continue;
     const u32 di = d.tab.done_idx[e];
     if (di >= nd) continue;
     const u32 r = d.sc.done_rank[di];
     if (r >= nd) continue;
-    const u32 i = d.sc.leaf_perm[j];
-    if (i >= n) continue;
     const u32 c = tag_child(b.tags[(u64)(D - 1) * n + i]);
     if (c >= d.sc.r_dense_n[r]) continue;
     const u64 slot = d.sc.r_dense_base[r] + c;
     if (slot >= d.cfg.dense_cap) continue;
-    u32 old = atomicExch(&d.sc.dense[slot].x, ep);
+    const u32 old = atomicExch(&d.sc.dense[slot].x, ep);
     if (old == ep) raise_err(ctl, ALTO_EDUP);
-    d.sc.dense[slot].y = b.off[i + 1] - b.off[i];
+    const u32 o0 = b.off[i];
+    d.sc.dense[slot].y = b.off[i + 1] - o0;
     d.sc.dense[slot].z = kNone;
-    d.sc.dense[slot].w = b.off[i];
+    d.sc.dense[slot].w = o0;
   }
 }
 
@@ -705,29 +931,73 @@ __global__ void k_check2(Dev d) {
   }
 }
 
+// Copy every child span into the output payload ring.  A warp takes 32
+// consecutive dense slots -- one contiguous output range -- reads their
+// headers in one go, then copies four spans per round with all loads issued
+// before the stores.  Spans longer than 32 elements finish in a second loop.
+__device__ __forceinline__ int32_t span_load(const Dev& d, const Batch& b, u32 owner, u32 pos,
+                                             u32 k) {
+  if (owner == kNone) return b.pay[(u64)pos + k];
+  bool ok;
+  const u64 a = vec_addr(d.tab, owner, 1, (u64)pos + k, &ok);
+  return ok ? d.ar.pool[a] : 0;
+}
+
 __global__ void __launch_bounds__(kThreads) k_gather(Dev d, Batch b) {
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
   const u32 ep = ctl->epoch;
   const u64 total = ctl->dense_total;
   const u64 base = ctl->pay_count;
+  const u64 cap = d.cfg.out_payload;
   const int lane = threadIdx.x & 31;
   const u64 gw = gtid() >> 5, nw = gstride() >> 5;
-  for (u64 j = gw; j < total; j += nw) {
-    const uint4 v = d.sc.dense[j];
-    if (v.x != ep) continue;
-    const u64 o = base + d.sc.dst[j];
-    if (o + v.y > d.cfg.out_payload) continue;
-    if (v.z == kNone) {
-      if ((u64)v.w + v.y > b.n_payload) continue;
-      for (u32 q = lane; q < v.y; q += 32) d.out_pay[o + q] = b.pay[v.w + q];
-    } else {
-      if (v.z > d.tab.mask || (u64)v.w + v.y > d.tab.vec_n[2 * (u64)v.z + 1]) continue;
-      for (u32 q = lane; q < v.y; q += 32) {
-        bool ok;
-        u64 a = vec_addr(d.tab, v.z, 1, (u64)v.w + q, &ok);
-        if (ok) d.out_pay[o + q] = d.ar.pool[a];
+  int32_t* __restrict__ out = d.out_pay;
+  for (u64 jb = gw * 32; jb < total; jb += nw * 32) {
+    // this lane's slot header; an unusable slot copies nothing
+    const u64 j = jb + lane;
+    u32 len = 0, owner = kNone, pos = 0;
+    u64 o = 0;
+    if (j < total) {
+      const uint4 v = d.sc.dense[j];
+      o = base + d.sc.dst[j];
+      bool good = v.x == ep && o + v.y <= cap;
+      if (good && v.z == kNone) good = (u64)v.w + v.y <= b.n_payload;
+      if (good && v.z != kNone)
+        good = v.z <= d.tab.mask && (u64)v.w + v.y <= d.tab.vec_n[2 * (u64)v.z + 1];
+      if (good) {
+        len = v.y;
+        owner = v.z;
+        pos = v.w;
       }
+    }
+    const u32 cnt = (total - jb < 32) ? (u32)(total - jb) : 32u;
+    for (u32 k0 = 0; k0 < cnt; k0 += 4) {
+      int32_t val[4];
+      u32 L[4];
+      u64 O[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int src = (k0 + u < 31u) ? (int)(k0 + u) : 31;
+        L[u] = __shfl_sync(0xFFFFFFFFu, len, src);
+        const u32 ow = __shfl_sync(0xFFFFFFFFu, owner, src);
+        const u32 ps = __shfl_sync(0xFFFFFFFFu, pos, src);
+        O[u] = __shfl_sync(0xFFFFFFFFu, o, src);
+        if (k0 + u >= cnt) L[u] = 0;
+        val[u] = ((u32)lane < L[u]) ? span_load(d, b, ow, ps, lane) : 0;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if ((u32)lane < L[u]) out[O[u] + lane] = val[u];
+    }
+    // the remainder of long spans
+    for (u32 k = 0; k < cnt; ++k) {
+      const u32 Lk = __shfl_sync(0xFFFFFFFFu, len, k);
+      if (Lk <= 32) continue;
+      const u32 ow = __shfl_sync(0xFFFFFFFFu, owner, k);
+      const u32 ps = __shfl_sync(0xFFFFFFFFu, pos, k);
+      const u64 Ok = __shfl_sync(0xFFFFFFFFu, o, k);
+      for (u32 q = 32 + lane; q < Lk; q += 32) out[Ok + q] = span_load(d, b, ow, ps, q);
     }
   }
 }
@@ -1082,6 +1352,16 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     ALLOC(d.tab.dir, u32, T * kVecs * kNumChunks);
   }
   if (kk > 0) ALLOC(d.tab.topk, u64, T * (u64)kk);
+  d.tab.chain_len = std::max(D - 1, 1);
+  ALLOC(d.tab.chain, u64, T * (u64)d.tab.chain_len);
+  ALLOC(d.tab.touch, u32, T);
+  ALLOC(d.tab.acc_cnt, u32, T);
+  ALLOC(d.tab.acc_m1, u32, T);
+  ALLOC(d.tab.acc_fmin, u32, T);
+  ALLOC(d.tab.acc_fmax1, u32, T);
+  ALLOC(d.tab.acc_cs1, u32, T);
+  ALLOC(d.tab.acc_smx, u32, T);
+  ALLOC(d.tab.acc_rep, u32, T);
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
   d.tab.max_probe = (int)std::min<u64>(T, 1u << 16);
@@ -1141,6 +1421,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(sc.seg_vb0, u32, nmax);
   ALLOC(sc.seg_vb1, u32, nmax);
   ALLOC(sc.seg_carry, u32, nmax);
+  ALLOC(sc.leaf_pos, u32, nmax);
   ALLOC(sc.mask, u32, nmax);
   ALLOC(sc.prefix, u32, nmax);
   ALLOC(sc.done_e, u32, done_cap);
@@ -1271,6 +1552,12 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
       set ^= 1;  // items written by the level below
       k_items_lookup<<<grid, kThreads, 0, s>>>(d, bt, l, set);
       h->launches += 1;
+      if (d.cfg.score_op[l] != ALTO_SCORE_TOPK) {
+        k_up_accumulate<<<grid, kThreads, 0, s>>>(d, bt, l, set);
+        k_up_finalize<<<grid, kThreads, 0, s>>>(d, bt, l, set);
+        h->launches += 2;
+        continue;
+      }
       int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nmax, h->tbits, true, h->up_sort, d.ctl, site,
                           spin, h->num_sms, s, &sl);
       h->launches += sl;
@@ -1306,8 +1593,6 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
     h->launches += 1;
     if (d.cfg.concat_level >= 0) {
       stage_enter(5);
-      LenScan fl{d.sc.leaf_perm, bt.off, d.sc.lenscan, &d.ctl->n};
-      launch_scan(h, fl, nmax, site++, s);
       k_carry_alloc<<<grid, kThreads, 0, s>>>(d);
       k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
       k_carry_copy<<<grid, kThreads, 0, s>>>(d, bt);

@@ -140,6 +140,17 @@ struct Table {
   u32* vec_n;      // [T][2] CONCAT level: leaves in meta vector, elements in payload vector
   u32* dir;        // [T][2][kNumChunks] CONCAT level: chunk offsets in the arena
   u64* topk;       // [T][kk] TOPK levels: best (score_key << 32 | ~child) first
+  u64* chain;      // [T][D-1] tags 0..l-1 of the group's first fragment (ancestry)
+  // per-batch accumulators of the atomic upper-level path (zero between batches)
+  u32* touch;      // [T] epoch of the batch that last touched the entry
+  u32* acc_cnt;    // [T] complete children in this batch
+  u32* acc_m1;     // [T] largest child index + 1 in this batch
+  u32* acc_fmin;   // [T] smallest flagged child index (kNone = none)
+  u32* acc_fmax1;  // [T] largest flagged child index + 1 (0 = none)
+  u32* acc_cs1;    // [T] largest completion seq + 1 of complete children
+  u32* acc_smx;    // [T] largest score key of complete children
+  u32* acc_rep;    // [T] a representative fragment
+  int chain_len;   // D - 1
   u32 mask;        // T - 1
   int kk;          // stride of topk (largest k over levels)
   int max_probe;

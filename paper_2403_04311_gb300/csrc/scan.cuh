@@ -58,98 +58,124 @@ __device__ __forceinline__ void lb_publish(LookbackState st, u32 tile, u32 es, u
   *fp = (es << 2) | kind;
 }
 
-// Sum of everything before `tile`; serial walk by one thread.
-__device__ __forceinline__ u64 lb_walk(LookbackState st, u32 tile, u32 es, Ctl* ctl, u64 spin_limit) {
+// Sum of everything before `tile`, found by warp 0: each lane reads one
+// predecessor of a 32-tile window; the nearest inclusive prefix ends the walk.
+__device__ __forceinline__ u64 lb_walk_warp(LookbackState st, u32 tile, u32 es, Ctl* ctl,
+                                            u64 spin_limit) {
+  const int lane = threadIdx.x & 31;
   u64 excl = 0;
-  long long pred = (long long)tile - 1;
+  long long top = (long long)tile - 1;
   u64 spins = 0;
-  while (pred >= 0) {
-    volatile u32* fp = st.flag + pred;
-    u32 f = *fp;
-    if ((f >> 2) != es || (f & 3u) == 0) {
+  while (top >= 0) {
+    const long long p = top - lane;
+    u32 f = 0;
+    bool ready = true;
+    if (p >= 0) {
+      f = *((volatile u32*)st.flag + p);
+      ready = ((f >> 2) == es) && ((f & 3u) != 0);
+    }
+    if (!__all_sync(0xFFFFFFFFu, ready)) {
       if (++spins > spin_limit || *(volatile int*)&ctl->abort) {
-        raise_timeout(ctl);
+        if (lane == 0) raise_timeout(ctl);
         break;
       }
       continue;
     }
     __threadfence();
-    const bool inclusive = (f & 3u) == 2u;
-    volatile u64* vp = (inclusive ? st.inc : st.agg) + pred;
-    excl += *vp;
-    if (inclusive) break;
-    --pred;
+    const bool inc = (p < 0) || ((f & 3u) == 2u);
+    const u32 inc_mask = __ballot_sync(0xFFFFFFFFu, inc);
+    const int stop = inc_mask ? __ffs(inc_mask) - 1 : 32;  // nearest inclusive predecessor
+    u64 v = 0;
+    if (p >= 0 && lane <= stop) v = *((volatile u64*)((lane == stop) ? st.inc : st.agg) + p);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    excl += v;
+    if (inc_mask) break;
+    top -= 32;
   }
   return excl;
 }
 
+// Tile = kScanItems rows of kScanThreads consecutive elements; thread t owns
+// column t, so every value()/out() call is coalesced across the warp.
 template <class F>
 __global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ctl* ctl, int site,
                                                        u32* exit_ctr, u64 spin_limit) {
   __shared__ u32 s_tile;
-  __shared__ u64 s_warp[kWarps];
+  __shared__ u64 s_w[kScanItems][kWarps];
   __shared__ u64 s_excl;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const u64 n = halted(ctl) ? 0 : f.size(ctl);
   u64 ntiles = (n + kScanTile - 1) / kScanTile;
   if (ntiles == 0) ntiles = 1;
-  if (ntiles > st.tiles) {  // capacity guard; the size itself is checked by the producer
-    ntiles = st.tiles;
-  }
+  if (ntiles > st.tiles) ntiles = st.tiles;
   const u32 es = epoch_site(ctl, site);
   for (;;) {
-    if (threadIdx.x == 0) s_tile = take_tile(ctl, site);
+    if (t == 0) s_tile = take_tile(ctl, site);
     __syncthreads();
     const u32 tile = s_tile;
-    __syncthreads();
     if (tile >= ntiles) break;
-    const u64 base = (u64)tile * kScanTile + (u64)threadIdx.x * kScanItems;
-    u64 v[kScanItems];
-    u64 sum = 0;
+    const u64 base = (u64)tile * kScanTile;
+    u64 v[kScanItems], x[kScanItems];
 #pragma unroll
     for (int k = 0; k < kScanItems; ++k) {
-      u64 i = base + k;
+      const u64 i = base + (u64)k * kScanThreads + t;
       v[k] = (i < n) ? f.value(i) : 0;
-      sum += v[k];
+      x[k] = v[k];
     }
-    u64 x = sum;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      u64 y = __shfl_up_sync(0xFFFFFFFFu, x, o);
-      if (lane >= o) x += y;
-    }
-    if (lane == 31) s_warp[warp] = x;
-    __syncthreads();
-    u64 wpre = 0, agg = 0;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
-      u64 t = s_warp[w];
-      if (w < warp) wpre += t;
-      agg += t;
-    }
-    if (threadIdx.x == 0) {
-      u64 excl = 0;
-      if (tile == 0) {
-        lb_publish(st, tile, es, 2u, agg);
-      } else {
-        lb_publish(st, tile, es, 1u, agg);
-        excl = lb_walk(st, tile, es, ctl, spin_limit);
-        lb_publish(st, tile, es, 2u, excl + agg);
+      for (int k = 0; k < kScanItems; ++k) {
+        const u64 y = __shfl_up_sync(0xFFFFFFFFu, x[k], o);
+        if (lane >= o) x[k] += y;
       }
-      s_excl = excl;
-      if (tile == ntiles - 1) f.total(ctl, excl + agg);
+    }
+    if (lane == 31) {
+#pragma unroll
+      for (int k = 0; k < kScanItems; ++k) s_w[k][warp] = x[k];
     }
     __syncthreads();
-    u64 run = s_excl + wpre + (x - sum);
+    // row totals and this warp's offset inside each row
+    u64 row_pre = 0, agg = 0;
+    u64 off[kScanItems];
 #pragma unroll
     for (int k = 0; k < kScanItems; ++k) {
-      u64 i = base + k;
-      if (i < n) f.out(i, run, v[k]);
-      run += v[k];
+      u64 rt = 0, wp = 0;
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) {
+        const u64 c = s_w[k][w];
+        if (w < warp) wp += c;
+        rt += c;
+      }
+      off[k] = row_pre + wp;
+      row_pre += rt;
+    }
+    agg = row_pre;
+    if (warp == 0) {
+      u64 excl = 0;
+      if (tile == 0) {
+        if (lane == 0) lb_publish(st, tile, es, 2u, agg);
+      } else {
+        if (lane == 0) lb_publish(st, tile, es, 1u, agg);
+        excl = lb_walk_warp(st, tile, es, ctl, spin_limit);
+        if (lane == 0) lb_publish(st, tile, es, 2u, excl + agg);
+      }
+      if (lane == 0) {
+        s_excl = excl;
+        if (tile == ntiles - 1) f.total(ctl, excl + agg);
+      }
+    }
+    __syncthreads();
+    const u64 ex0 = s_excl;
+#pragma unroll
+    for (int k = 0; k < kScanItems; ++k) {
+      const u64 i = base + (u64)k * kScanThreads + t;
+      if (i < n) f.out(i, ex0 + off[k] + x[k] - v[k], v[k]);
     }
     __syncthreads();
   }
-  if (threadIdx.x == 0) finish_ctas(ctl, site, exit_ctr);
+  if (t == 0) finish_ctas(ctl, site, exit_ctr);
 }
 
 }  // namespace alto
