@@ -135,6 +135,8 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
         tab.acc_fmax1[h] = 0;
         tab.acc_cs1[h] = 0;
         tab.acc_smx[h] = 0;
+        tab.acc_len[h] = 0;
+        tab.carry_epoch[h] = 0;
         *inserted = 1;
         return h;
       }
@@ -539,14 +541,77 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
   }
 }
 
+// Leaf level without TOPK: every fragment, in arrival order (coalesced),
+// checks its ancestry against its group's entry and adds itself to the
+// entry's batch accumulators (warp-aggregated over lanes of the same group).
+__global__ void __launch_bounds__(kThreads) k_leaf_accumulate(Dev d, Batch b) {
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  const int D = d.cfg.depth;
+  const int L = D - 1;
+  const u64 n = b.n;
+  const bool scores = d.cfg.has_score;
+  u32* list = d.sc.leaf_seg_start;  // touched leaf-parent entries
+  const u32 end = (b.n + 31) & ~31u;
+  for (u32 i = gtid(); i < end; i += gstride()) {
+    const bool valid = i < b.n;
+    u32 e = 0, c = 0, f = 0, len = 0, sk = 0;
+    if (valid) {
+      e = d.sc.leaf_sort_keys0[i] & d.tab.mask;
+      const u64 t = b.tags[(u64)L * n + i];
+      c = tag_child(t);
+      f = tag_last(t);
+      len = b.off[i + 1] - b.off[i];
+      if (scores) sk = score_key(b.score[i]);
+      bool bad = false;
+      for (int q = 0; q < L; ++q)
+        if (b.tags[(u64)q * n + i] != d.tab.chain[(u64)e * d.tab.chain_len + q]) bad = true;
+      if (bad) raise_err(ctl, ALTO_EINCONSIST);
+    }
+    const u32 key = valid ? e : kNone;
+    const u32 peers = __match_any_sync(0xFFFFFFFFu, key);
+    const int leader = __ffs(peers) - 1;
+    const u32 cnt = __popc(peers);
+    const u32 m1 = __reduce_max_sync(peers, valid ? c + 1 : 0u);
+    const u32 cs1 = __reduce_max_sync(peers, valid ? i + 1 : 0u);
+    const u32 lsum = __reduce_add_sync(peers, len);
+    const u32 anyf = __reduce_or_sync(peers, f);
+    if (valid && (int)(threadIdx.x & 31) == leader) {
+      const u32 old = atomicAdd(&d.tab.acc_cnt[e], cnt);
+      if (old == 0) {
+        const u32 pos = atomicAdd(&ctl->n_segs[L], 1u);
+        if (pos < d.cfg.n_max) list[pos] = e;
+        d.tab.acc_rep[e] = i;
+      }
+      atomicMax(&d.tab.acc_m1[e], m1);
+      atomicMax(&d.tab.acc_cs1[e], cs1);
+      if (lsum) atomicAdd(&d.tab.acc_len[e], lsum);
+    }
+    if (anyf) {
+      const u32 fmin = __reduce_min_sync(peers, (valid && f) ? c : kNone);
+      const u32 fmax1 = __reduce_max_sync(peers, (valid && f) ? c + 1 : 0u);
+      if (valid && (int)(threadIdx.x & 31) == leader && fmax1) {
+        atomicMin(&d.tab.acc_fmin[e], fmin);
+        atomicMax(&d.tab.acc_fmax1[e], fmax1);
+      }
+    }
+    if (scores) {
+      const u32 smx = __reduce_max_sync(peers, valid ? sk : 0u);
+      if (valid && (int)(threadIdx.x & 31) == leader && smx) atomicMax(&d.tab.acc_smx[e], smx);
+    }
+  }
+}
+
 // One thread per touched entry: merge, test completion, emit the next items.
+template <bool LEAF>
 __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l, int in_set) {
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const int D = d.cfg.depth;
+  const bool carry = LEAF && d.cfg.concat_level == D - 1;
   const u32 nt = min(ctl->n_segs[l], d.cfg.n_max);
   const u32 ep = ctl->epoch;
-  const u32* list = d.sc.up_seg_start;
+  const u32* list = LEAF ? d.sc.leaf_seg_start : d.sc.up_seg_start;
   u32* nx_rep = d.sc.it_rep[in_set ^ 1];
   u32* nx_cseq = d.sc.it_cseq[in_set ^ 1];
   u32* nx_skey = d.sc.it_skey[in_set ^ 1];
@@ -556,7 +621,9 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
     const u32 cnt = d.tab.acc_cnt[e], m1 = d.tab.acc_m1[e], fmin = d.tab.acc_fmin[e];
     const u32 fmax1 = d.tab.acc_fmax1[e], cs1 = d.tab.acc_cs1[e], smx = d.tab.acc_smx[e];
     const u32 rep = d.tab.acc_rep[e];
+    const u32 blen = LEAF ? d.tab.acc_len[e] : 0u;
     // reset the accumulators for the next batch
+    if (LEAF) d.tab.acc_len[e] = 0;
     d.tab.acc_cnt[e] = 0;
     d.tab.acc_m1[e] = 0;
     d.tab.acc_fmin[e] = kNone;
@@ -581,6 +648,14 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
     d.tab.completed[e] = comp;
     d.tab.smax[e] = smn;
     const u32 cmax = cs1 ? cs1 - 1 : 0;
+    if (carry && !complete) {
+      // reserve this batch's leaves at the end of the group's arena vectors
+      const u32 v0 = d.tab.vec_n[2 * (u64)e], v1 = d.tab.vec_n[2 * (u64)e + 1];
+      d.tab.cur[e] = ((u64)v0 << 40) | v1;
+      d.tab.vec_n[2 * (u64)e] = v0 + cnt;
+      d.tab.vec_n[2 * (u64)e + 1] = v1 + blen;
+      d.tab.carry_epoch[e] = ep;
+    }
     if (complete) {
       u32 di = atomicAdd(&ctl->n_done, 1u);
       if (di < d.sc.done_cap) {
@@ -692,9 +767,11 @@ struct LenScan {
 // from the class's free stack (or the bump allocator) with one atomic each.
 constexpr int kMaxReq = 8;
 
+template <bool ATOMIC>
 __global__ void __launch_bounds__(kThreads) k_carry_alloc(Dev d) {
   Ctl* ctl = d.ctl;
   if (no_copy(ctl)) return;
+  const u32 ep = ctl->epoch;
   __shared__ u32 s_cnt[kNumChunks];
   __shared__ int s_old[kNumChunks];
   __shared__ u32 s_avail[kNumChunks];
@@ -710,11 +787,28 @@ __global__ void __launch_bounds__(kThreads) k_carry_alloc(Dev d) {
     int nreq = 0;
     uint8_t rvec[kMaxReq], rj[kMaxReq];
     u32 rr[kMaxReq];
-    if (s < nseg && d.sc.seg_carry[s] == 1u) {
-      e = d.sc.leaf_keys[d.sc.leaf_seg_start[s]] & d.tab.mask;
+    bool want = false;
+    u64 old0 = 0, old1 = 0;
+    if (s < nseg) {
+      if (ATOMIC) {
+        e = d.sc.leaf_seg_start[s] & d.tab.mask;
+        want = d.tab.carry_epoch[e] == ep;
+        if (want) {
+          const u64 cu = d.tab.cur[e];
+          old0 = cu >> 40;
+          old1 = cu & ((1ull << 40) - 1);
+        }
+      } else if (d.sc.seg_carry[s] == 1u) {
+        e = d.sc.leaf_keys[d.sc.leaf_seg_start[s]] & d.tab.mask;
+        want = true;
+        old0 = d.sc.seg_vb0[s];
+        old1 = d.sc.seg_vb1[s];
+      }
+    }
+    if (want) {
       for (int vec = 0; vec < kVecs; ++vec) {
         const u64 mult = (vec == 0) ? 2 : 1;
-        const u64 old_el = (u64)((vec == 0) ? d.sc.seg_vb0[s] : d.sc.seg_vb1[s]) * mult;
+        const u64 old_el = ((vec == 0) ? old0 : old1) * mult;
         const u64 new_el = (u64)d.tab.vec_n[2 * (u64)e + vec] * mult;
         if (new_el <= old_el) continue;
         const int jf = (old_el == 0) ? 0 : chunk_of(old_el - 1) + 1;
@@ -847,6 +941,73 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
     d.sc.dense[slot].y = b.off[i + 1] - o0;
     d.sc.dense[slot].z = kNone;
     d.sc.dense[slot].w = o0;
+  }
+}
+
+// Leaf level without TOPK, per fragment in arrival order, eight lanes each:
+// a fragment of a group left open takes its arena position from the group's
+// cursor (one 64-bit atomic: leaf index and payload offset together) and is
+// copied there; a fragment of a group completed by this batch is placed at
+// its dense child slot.
+__global__ void __launch_bounds__(kThreads) k_leaf_place(Dev d, Batch b) {
+  Ctl* ctl = d.ctl;
+  if (no_copy(ctl)) return;
+  const int D = d.cfg.depth;
+  const u32 ep = ctl->epoch;
+  const u64 n = b.n;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  const bool dense_ok = !ctl->skip_dense;
+  const u32 sub = threadIdx.x & 7;
+  const u32 g0 = gtid() >> 3, ng = gstride() >> 3;
+  const u32 end = (b.n + 3) & ~3u;  // four groups per warp: keep warps converged
+  for (u32 i = g0; i < end; i += ng) {
+    const bool valid = i < b.n;
+    u32 e = 0, mode = 0;  // 1 arena, 2 dense
+    if (valid) {
+      e = d.sc.leaf_sort_keys0[i] & d.tab.mask;
+      if (d.tab.carry_epoch[e] == ep) mode = 1;
+      else if (dense_ok && d.tab.done_epoch[e] == ep) mode = 2;
+    }
+    u32 o0 = 0, len = 0, c = 0;
+    if (mode) {
+      o0 = b.off[i];
+      len = b.off[i + 1] - o0;
+      c = tag_child(b.tags[(u64)(D - 1) * n + i]);
+    }
+    u64 old = 0;
+    if (mode == 1 && sub == 0) old = atomicAdd((unsigned long long*)&d.tab.cur[e], (1ull << 40) | len);
+    old = __shfl_sync(0xFFFFFFFFu, old, 0, 8);
+    if (mode == 1) {
+      const u64 mpos = old >> 40, ppos = old & ((1ull << 40) - 1);
+      if (mpos < d.tab.vec_n[2 * (u64)e] && ppos + len <= d.tab.vec_n[2 * (u64)e + 1] &&
+          (u64)o0 + len <= b.n_payload) {
+        bool ok;
+        if (sub == 0) {
+          const u64 a = vec_addr(d.tab, e, 0, 2 * mpos, &ok);
+          if (ok) {
+            d.ar.pool[a] = (int32_t)c;
+            d.ar.pool[a + 1] = (int32_t)(u32)ppos;
+          }
+        }
+        for (u32 k = sub; k < len; k += 8) {
+          const u64 a = vec_addr(d.tab, e, 1, ppos + k, &ok);
+          if (ok) d.ar.pool[a] = b.pay[o0 + k];
+        }
+      }
+    } else if (mode == 2 && sub == 0) {
+      const u32 di = d.tab.done_idx[e];
+      const u32 r = (di < nd) ? d.sc.done_rank[di] : kNone;
+      if (r < nd && c < d.sc.r_dense_n[r]) {
+        const u64 slot = d.sc.r_dense_base[r] + c;
+        if (slot < d.cfg.dense_cap) {
+          const u32 prev = atomicExch(&d.sc.dense[slot].x, ep);
+          if (prev == ep) raise_err(ctl, ALTO_EDUP);
+          d.sc.dense[slot].y = len;
+          d.sc.dense[slot].z = kNone;
+          d.sc.dense[slot].w = o0;
+        }
+      }
+    }
   }
 }
 
@@ -1362,6 +1523,9 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(d.tab.acc_cs1, u32, T);
   ALLOC(d.tab.acc_smx, u32, T);
   ALLOC(d.tab.acc_rep, u32, T);
+  ALLOC(d.tab.acc_len, u32, T);
+  ALLOC(d.tab.carry_epoch, u32, T);
+  ALLOC(d.tab.cur, u64, T);
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
   d.tab.max_probe = (int)std::min<u64>(T, 1u << 16);
@@ -1503,7 +1667,8 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
   bt.n = n;
   bt.n_payload = (u64)b->n_payload;
   const u32 nmax = (u32)cfg.max_batch_fragments;
-  const int grid = h->num_sms * 8;
+  const int grid = h->num_sms * 8;          // kernels over fragments or leaves
+  const int sgrid = h->num_sms * 2;         // kernels over groups (fewer items)
   const u64 spin = d.cfg.spin_limit;
 
   if (h->pushed % 127 == 0 && h->pushed > 0)
@@ -1528,33 +1693,43 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
     int site = 0;
     k_ingest<<<grid, kThreads, 0, s>>>(d, bt);
     h->launches += 1;
-    // leaf level: sort fragments by their leaf-parent group
-    stage_enter(1);
-    int cur = sort_pairs(&d.ctl->n, nmax, h->tbits, true, h->leaf_sort, d.ctl, site, spin,
-                         h->num_sms, s, &sl);
-    h->launches += sl;
-    sl = 0;
-    site += 4;
-    d.sc.leaf_keys = h->leaf_sort.keys[cur];
-    d.sc.leaf_perm = h->leaf_sort.vals[cur];
-    stage_enter(2);
-    {
-      SegFind f{d.sc.leaf_keys, d.sc.leaf_seg_start, d.sc.leaf_seg_of, &d.ctl->n, nmax,
-                &d.ctl->n_segs[D - 1]};
-      launch_scan(h, f, nmax, site++, s);
-    }
+    const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK;
     int set = 0;
-    k_reduce<true><<<grid, kThreads, 0, s>>>(d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
-                                             d.sc.leaf_seg_start, set);
-    h->launches += 1;
+    if (leaf_sorted) {
+      // leaf level with TOPK: sort fragments by their leaf-parent group so that
+      // each group's candidates are contiguous for the segmented top-k
+      stage_enter(1);
+      int cur = sort_pairs(&d.ctl->n, nmax, h->tbits, true, h->leaf_sort, d.ctl, site, spin,
+                           h->num_sms, s, &sl);
+      h->launches += sl;
+      sl = 0;
+      d.sc.leaf_keys = h->leaf_sort.keys[cur];
+      d.sc.leaf_perm = h->leaf_sort.vals[cur];
+      stage_enter(2);
+      {
+        SegFind f{d.sc.leaf_keys, d.sc.leaf_seg_start, d.sc.leaf_seg_of, &d.ctl->n, nmax,
+                  &d.ctl->n_segs[D - 1]};
+        launch_scan(h, f, nmax, site + 4, s);
+      }
+      k_reduce<true><<<grid, kThreads, 0, s>>>(d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
+                                               d.sc.leaf_seg_start, set);
+      h->launches += 1;
+    } else {
+      // leaf level without TOPK: accumulate into the table in arrival order
+      stage_enter(2);
+      k_leaf_accumulate<<<grid, kThreads, 0, s>>>(d, bt);
+      k_up_finalize<true><<<sgrid, kThreads, 0, s>>>(d, bt, D - 1, set);
+      h->launches += 2;
+    }
+    site += 5;
     stage_enter(3);
     for (int l = D - 2; l >= 0; --l) {
       set ^= 1;  // items written by the level below
-      k_items_lookup<<<grid, kThreads, 0, s>>>(d, bt, l, set);
+      k_items_lookup<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
       h->launches += 1;
       if (d.cfg.score_op[l] != ALTO_SCORE_TOPK) {
-        k_up_accumulate<<<grid, kThreads, 0, s>>>(d, bt, l, set);
-        k_up_finalize<<<grid, kThreads, 0, s>>>(d, bt, l, set);
+        k_up_accumulate<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+        k_up_finalize<false><<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
         h->launches += 2;
         continue;
       }
@@ -1578,7 +1753,7 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
       RankScan f{d.sc.mask, d.sc.prefix, &d.ctl->n};
       launch_scan(h, f, nmax, site++, s);
     }
-    k_done_rank<<<grid, kThreads, 0, s>>>(d);
+    k_done_rank<<<sgrid, kThreads, 0, s>>>(d);
     h->launches += 1;
     const u32 dcap = d.sc.done_cap;
     {
@@ -1593,14 +1768,20 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
     h->launches += 1;
     if (d.cfg.concat_level >= 0) {
       stage_enter(5);
-      k_carry_alloc<<<grid, kThreads, 0, s>>>(d);
-      k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
-      k_carry_copy<<<grid, kThreads, 0, s>>>(d, bt);
-      h->launches += 3;
-      stage_enter(6);
-      k_dense_batch<<<grid, kThreads, 0, s>>>(d, bt);
-      k_dense_arena<<<grid, kThreads, 0, s>>>(d);
-      h->launches += 2;
+      if (leaf_sorted) {
+        k_carry_alloc<false><<<sgrid, kThreads, 0, s>>>(d);
+        k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
+        k_carry_copy<<<grid, kThreads, 0, s>>>(d, bt);
+        stage_enter(6);
+        k_dense_batch<<<grid, kThreads, 0, s>>>(d, bt);
+      } else {
+        k_carry_alloc<true><<<sgrid, kThreads, 0, s>>>(d);
+        k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
+        stage_enter(6);
+        k_leaf_place<<<grid, kThreads, 0, s>>>(d, bt);
+      }
+      k_dense_arena<<<sgrid, kThreads, 0, s>>>(d);
+      h->launches += 4;
       DenseScan fd{d.sc.dense, d.sc.dst, d.ctl};
       launch_scan(h, fd, d.cfg.dense_cap, site++, s);
       k_check2<<<1, 1, 0, s>>>(d);
@@ -1610,8 +1791,8 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
       h->launches += 1;
     }
     stage_enter(8);
-    k_records<<<grid, kThreads, 0, s>>>(d);
-    k_sweep<<<grid, kThreads, 0, s>>>(d);
+    k_records<<<sgrid, kThreads, 0, s>>>(d);
+    k_sweep<<<sgrid, kThreads, 0, s>>>(d);
     h->launches += 2;
   } else {
     stage_enter(8);

@@ -150,6 +150,9 @@ struct Table {
   u32* acc_cs1;    // [T] largest completion seq + 1 of complete children
   u32* acc_smx;    // [T] largest score key of complete children
   u32* acc_rep;    // [T] a representative fragment
+  u32* acc_len;    // [T] payload elements of this batch's leaves (leaf level)
+  u32* carry_epoch;// [T] epoch in which the entry's leaves go to its arena vectors
+  u64* cur;        // [T] arena cursor: leaves << 40 | payload elements
   int chain_len;   // D - 1
   u32 mask;        // T - 1
   int kk;          // stride of topk (largest k over levels)

@@ -112,12 +112,17 @@ __global__ void __launch_bounds__(kSortThreads) k_onesweep(const u32* n_dev, u32
     const u32 wbase = tile * kSortTile + warp * (kSortItems * 32);
     u32 keys[kSortItems];
     u32 rank[kSortItems];
+    // issue every load of the tile before ranking
+#pragma unroll
+    for (int r = 0; r < kSortItems; ++r) {
+      const u32 idx = wbase + r * 32 + lane;
+      keys[r] = (idx < n) ? __ldcs(kin + idx) : 0u;
+    }
 #pragma unroll
     for (int r = 0; r < kSortItems; ++r) {
       u32 idx = wbase + r * 32 + lane;
       bool valid = idx < n;
-      u32 k = valid ? kin[idx] : 0u;
-      keys[r] = k;
+      u32 k = keys[r];
       u32 d = valid ? ((k >> shift) & 255u) : 256u;
       u32 peers = __match_any_sync(0xFFFFFFFFu, d);
       int leader = __ffs(peers) - 1;
@@ -176,7 +181,7 @@ __global__ void __launch_bounds__(kSortThreads) k_onesweep(const u32* n_dev, u32
         u32 d = (keys[r] >> shift) & 255u;
         u32 p = s_toff[d] + whist[warp][d] + rank[r];
         s_k[p] = keys[r];
-        s_v[p] = vin ? vin[idx] : idx;
+        s_v[p] = vin ? __ldcs(vin + idx) : idx;
       }
     }
     __syncthreads();

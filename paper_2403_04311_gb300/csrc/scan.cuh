@@ -17,8 +17,9 @@
 
 namespace alto {
 
-constexpr int kScanThreads = 256;
+constexpr int kScanThreads = 512;
 constexpr int kScanItems = 8;
+constexpr int kScanWarps = kScanThreads / 32;
 constexpr int kScanTile = kScanThreads * kScanItems;
 
 // A tile's aggregate and its inclusive prefix live in separate arrays: a
@@ -102,7 +103,7 @@ template <class F>
 __global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ctl* ctl, int site,
                                                        u32* exit_ctr, u64 spin_limit) {
   __shared__ u32 s_tile;
-  __shared__ u64 s_w[kScanItems][kWarps];
+  __shared__ u64 s_w[kScanItems][kScanWarps];
   __shared__ u64 s_excl;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const u64 n = halted(ctl) ? 0 : f.size(ctl);
@@ -143,7 +144,7 @@ __global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ct
     for (int k = 0; k < kScanItems; ++k) {
       u64 rt = 0, wp = 0;
 #pragma unroll
-      for (int w = 0; w < kWarps; ++w) {
+      for (int w = 0; w < kScanWarps; ++w) {
         const u64 c = s_w[k][w];
         if (w < warp) wp += c;
         rt += c;
