@@ -229,6 +229,33 @@ typedef struct alto_profile {
 alto_status alto_agg_profile(alto_agg_t* h, int enable);
 alto_status alto_agg_profile_read(alto_agg_t* h, alto_profile* out);
 
+/* One-shot aggregation that allocates no device memory.  The paper has no
+ * counterpart: this entry point serves callers that may not call cudaMalloc
+ * -- a serving process whose framework has already reserved the device's free
+ * memory for its own pool, a real-time path that cannot take cudaMalloc's
+ * implicit device synchronisation, a plug-in loaded without an allocator.
+ *
+ * It aggregates ONE self-contained batch exactly as create + push_batch +
+ * drain would on a fresh handle (groups not completed by the batch are
+ * dropped), writing records, payload and top-k pairs into the caller's device
+ * buffers, and {status, n_records, n_payload, n_topk} into the caller's device
+ * int64[4] `out_counts`, all on `stream` (nothing is synchronised; status is
+ * ALTO_ENOSPC there when an output capacity is too small).  Its tables,
+ * scratch and arena live in one static device array of 32 MiB that every GPU
+ * loading this library holds until the process exits.  Limits: n <= 4096,
+ * n * depth <= 16384, n_payload <= 262144; larger batches return ALTO_ENOSPC
+ * at once.  The first call on a device looks up that array's device address
+ * (cudaGetSymbolAddress) with the device current; make that first call before
+ * any stream capture.  All calls on a device share the array and each call
+ * clears what must start empty, so calls that overlap on the GPU (for
+ * example on two streams at once) race and give undefined results.  Returns
+ * ALTO_EINVAL for bad arguments, ALTO_ECUDA if a launch fails. */
+alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg, const alto_batch* b,
+                                     alto_record* out_records, int64_t cap_records,
+                                     int32_t* out_payload, int64_t cap_payload,
+                                     alto_topk_pair* out_topk, int64_t cap_topk,
+                                     int64_t* out_counts, void* stream);
+
 /* Free everything the handle owns; open groups are discarded.  NULL is OK.
  * Always succeeds on a valid or poisoned handle. */
 alto_status alto_agg_destroy(alto_agg_t* h);

@@ -9,7 +9,8 @@ from ._binding import (  # noqa: F401
     STATUS_NAMES, PAYLOAD_NONE, PAYLOAD_CONCAT, SCORE_NONE, SCORE_MAX, SCORE_TOPK,
     RECORD_DTYPE, PAIR_DTYPE, Aggregator, Drain, alto_agg_config, alto_allocator, alto_batch,
     alto_drain, alto_agg_create, alto_agg_push_batch, alto_agg_drain, alto_agg_stats,
-    alto_agg_destroy, alto_agg_profile, alto_agg_profile_read, load_library, make_config,
+    alto_agg_destroy, alto_agg_profile, alto_agg_profile_read, alto_agg_oneshot_noalloc,
+    load_library, make_config,
     STAGE_NAMES,
 )
 from ._build import build  # noqa: F401

@@ -88,7 +88,8 @@ class alto_profile(ctypes.Structure):
 
 
 EXPORTS = ("alto_agg_create", "alto_agg_push_batch", "alto_agg_drain", "alto_agg_stats",
-           "alto_agg_profile", "alto_agg_profile_read", "alto_agg_destroy")
+           "alto_agg_profile", "alto_agg_profile_read", "alto_agg_oneshot_noalloc",
+           "alto_agg_destroy")
 
 _lib = None
 
@@ -118,6 +119,10 @@ def load_library(build: bool = True):
     lib.alto_agg_profile.argtypes = [P, ctypes.c_int]
     lib.alto_agg_profile_read.restype = ctypes.c_int
     lib.alto_agg_profile_read.argtypes = [P, ctypes.POINTER(alto_profile)]
+    lib.alto_agg_oneshot_noalloc.restype = ctypes.c_int
+    lib.alto_agg_oneshot_noalloc.argtypes = [
+        ctypes.POINTER(alto_agg_config), ctypes.POINTER(alto_batch), P, ctypes.c_int64, P,
+        ctypes.c_int64, P, ctypes.c_int64, P, P]
     _lib = lib
     return lib
 
@@ -194,6 +199,15 @@ def alto_agg_stats(h, stream=0):
 
 def alto_agg_destroy(h) -> int:
     return load_library().alto_agg_destroy(h)
+
+
+def alto_agg_oneshot_noalloc(cfg, batch, out_records, cap_records, out_payload, cap_payload,
+                             out_topk, cap_topk, out_counts, stream=0) -> int:
+    """All pointers are device addresses (ints); the call allocates nothing."""
+    return load_library().alto_agg_oneshot_noalloc(
+        ctypes.byref(cfg), ctypes.byref(batch), ctypes.c_void_p(out_records), cap_records,
+        ctypes.c_void_p(out_payload), cap_payload, ctypes.c_void_p(out_topk), cap_topk,
+        ctypes.c_void_p(out_counts), ctypes.c_void_p(stream))
 
 
 def alto_agg_profile(h, enable: bool) -> int:

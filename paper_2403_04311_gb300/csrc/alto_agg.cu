@@ -1887,3 +1887,398 @@ alto_status alto_agg_destroy(alto_agg_t* h) {
 }
 
 }  // extern "C"
+
+// ===========================================================================
+// One-shot aggregation without device allocation.
+//
+// For callers that may not allocate device memory at all: code that runs
+// under a strict memory budget owned by another allocator (a serving process
+// whose framework reserved all free memory up front), code on a real-time path
+// where cudaMalloc's implicit synchronisation is not acceptable, or plug-ins
+// that a host application loads without giving them an allocator.  They get
+// one entry point that aggregates one self-contained batch (fresh state;
+// groups that do not complete inside the batch are dropped) and writes the
+// records straight into buffers the caller owns.  Every table, scratch array
+// and arena chunk it needs lives in the static device array below, of fixed
+// size; it calls no cudaMalloc/cudaFree.  The array is shared by every call in
+// the process on a given device and keeps the previous call's contents, so
+// each call clears what must start empty, and calls that overlap on the GPU
+// (two streams at once) race on it.
+// ===========================================================================
+namespace {
+
+constexpr u64 kNaBytes = 32ull << 20;        // size of the static scratch
+constexpr u64 kNaMaxFragments = 4096;        // n per call
+constexpr u64 kNaMaxGroupsLevels = 16384;    // n * depth per call
+constexpr u64 kNaMaxPayload = 1ull << 18;    // n_payload per call
+constexpr u64 kNaTableSlots = 1ull << 15;    // open-group table slots
+constexpr u64 kNaArenaElems = 1ull << 20;    // arena int32 elements
+
+}  // namespace
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNaBytes];
+
+namespace {
+
+struct NaDevice {
+  bool ready;
+  unsigned char* base;  // device address of g_noalloc_scratch on that device
+};
+NaDevice g_na_dev[64];
+
+struct NaCarver {
+  unsigned char* base;
+  u64 used = 0;
+  bool ok = true;
+  template <class T>
+  T* take(u64 count) {
+    u64 bytes = ((sizeof(T) * count + 255) / 256) * 256;
+    if (bytes == 0) bytes = 256;
+    T* p = base ? (T*)(base + used) : nullptr;
+    used += bytes;
+    if (used > kNaBytes) ok = false;
+    return p;
+  }
+};
+
+struct NaState {
+  Dev d;
+  SortBuffers leaf_sort, up_sort;
+  LookbackState lbs;
+  u64 T, PS, done_cap, dense_cap, sort_tiles, scan_tiles;
+  int tbits;
+};
+
+// Carve every buffer of the one-shot pipeline out of the static scratch (a
+// null base only measures).
+void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaCarver& cv) {
+  cv.base = base;
+  const int D = cfg.depth;
+  int concat = -1, kk = 0;
+  bool has_score = false;
+  for (int l = 0; l < D; ++l) {
+    if (cfg.payload_op[l] == ALTO_PAYLOAD_CONCAT) concat = l;
+    if (cfg.score_op[l] != ALTO_SCORE_NONE) has_score = true;
+    if (cfg.score_op[l] == ALTO_SCORE_TOPK) kk = std::max(kk, (int)cfg.topk_k[l]);
+  }
+  const u64 nmax = kNaMaxFragments, T = kNaTableSlots;
+  st.T = T;
+  st.tbits = ilog2(T);
+  st.done_cap = nmax * (u64)D;
+  st.dense_cap = nmax;
+  st.PS = next_pow2(std::max<u64>(2 * nmax * (u64)D, 1024));
+  st.sort_tiles = nmax / 4096 + 2;
+  st.scan_tiles = std::max<u64>(st.done_cap, nmax) / kScanTile + 2;
+  Dev& d = st.d;
+  memset(&d, 0, sizeof(d));
+  d.ctl = cv.take<Ctl>(1);
+  d.tab.key = cv.take<u64>(T);
+  d.tab.up = cv.take<u64>(T);
+  d.tab.last = cv.take<u32>(T);
+  d.tab.completed = cv.take<u32>(T);
+  d.tab.maxc1 = cv.take<u32>(T);
+  d.tab.smax = cv.take<u32>(T);
+  d.tab.done_epoch = cv.take<u32>(T);
+  d.tab.done_idx = cv.take<u32>(T);
+  if (concat >= 0) {
+    d.tab.vec_n = cv.take<u32>(2 * T);
+    d.tab.dir = cv.take<u32>(T * kVecs * kNumChunks);
+  }
+  if (kk > 0) d.tab.topk = cv.take<u64>(T * (u64)kk);
+  d.tab.chain_len = std::max(D - 1, 1);
+  d.tab.chain = cv.take<u64>(T * (u64)d.tab.chain_len);
+  d.tab.touch = cv.take<u32>(T);
+  d.tab.acc_cnt = cv.take<u32>(T);
+  d.tab.acc_m1 = cv.take<u32>(T);
+  d.tab.acc_fmin = cv.take<u32>(T);
+  d.tab.acc_fmax1 = cv.take<u32>(T);
+  d.tab.acc_cs1 = cv.take<u32>(T);
+  d.tab.acc_smx = cv.take<u32>(T);
+  d.tab.acc_rep = cv.take<u32>(T);
+  d.tab.acc_len = cv.take<u32>(T);
+  d.tab.carry_epoch = cv.take<u32>(T);
+  d.tab.cur = cv.take<u64>(T);
+  d.tab.mask = (u32)(T - 1);
+  d.tab.kk = kk;
+  d.tab.max_probe = (int)T;
+  if (concat >= 0) {
+    d.ar.elems = kNaArenaElems;
+    d.ar.pool = cv.take<int32_t>(kNaArenaElems);
+    u64 off = 0;
+    for (int j = 0; j < kNumChunks; ++j) {
+      d.ar.stack_off[j] = off;
+      d.ar.stack_cap[j] = kNaArenaElems / (1ull << (kChunk0Log + j)) + 1;
+      off += d.ar.stack_cap[j];
+    }
+    d.ar.stack = cv.take<u32>(off);
+  }
+  d.cfg.depth = D;
+  d.cfg.concat_level = concat;
+  for (int l = 0; l < kMaxDepth; ++l) {
+    d.cfg.score_op[l] = (l < D) ? cfg.score_op[l] : 0;
+    d.cfg.topk_k[l] = (l < D && cfg.score_op[l] == ALTO_SCORE_TOPK) ? cfg.topk_k[l] : 0;
+  }
+  d.cfg.has_score = has_score;
+  d.cfg.n_max = (u32)nmax;
+  d.cfg.dense_cap = st.dense_cap;
+  d.cfg.spin_limit = cfg.spin_limit > 0 ? (u64)cfg.spin_limit : (1ull << 20);
+  Scratch& sc = d.sc;
+  for (int b = 0; b < 2; ++b) {
+    st.leaf_sort.keys[b] = cv.take<u32>(nmax);
+    st.leaf_sort.vals[b] = cv.take<u32>(nmax);
+    st.up_sort.keys[b] = cv.take<u32>(nmax);
+    st.up_sort.vals[b] = cv.take<u32>(nmax);
+  }
+  st.leaf_sort.hist = cv.take<u32>(4 * 256);
+  st.leaf_sort.bin_base = cv.take<u32>(4 * 256);
+  st.leaf_sort.lookback = cv.take<u64>(st.sort_tiles * 256);
+  st.leaf_sort.lb_tiles = st.sort_tiles;
+  st.up_sort.hist = st.leaf_sort.hist;
+  st.up_sort.bin_base = st.leaf_sort.bin_base;
+  st.up_sort.lookback = st.leaf_sort.lookback;
+  st.up_sort.lb_tiles = st.sort_tiles;
+  sc.leaf_sort_keys0 = st.leaf_sort.keys[0];
+  sc.up_sort_keys0 = st.up_sort.keys[0];
+  sc.leaf_seg_start = cv.take<u32>(nmax + 1);
+  sc.leaf_seg_of = cv.take<u32>(nmax);
+  sc.up_seg_start = cv.take<u32>(nmax + 1);
+  for (int b = 0; b < 2; ++b) {
+    sc.it_rep[b] = cv.take<u32>(nmax);
+    sc.it_cseq[b] = cv.take<u32>(nmax);
+    sc.it_skey[b] = cv.take<u32>(nmax);
+  }
+  sc.seg_vb0 = cv.take<u32>(nmax);
+  sc.seg_vb1 = cv.take<u32>(nmax);
+  sc.seg_carry = cv.take<u32>(nmax);
+  sc.leaf_pos = cv.take<u32>(nmax);
+  sc.mask = cv.take<u32>(nmax);
+  sc.prefix = cv.take<u32>(nmax);
+  const u64 dc = st.done_cap;
+  sc.done_e = cv.take<u32>(dc);
+  sc.done_lvl = cv.take<u32>(dc);
+  sc.done_cseq = cv.take<u32>(dc);
+  sc.done_rank = cv.take<u32>(dc);
+  sc.r_done = cv.take<u32>(dc);
+  sc.r_dense_n = cv.take<u32>(dc);
+  sc.r_topk_n = cv.take<u32>(dc);
+  sc.r_meta_n = cv.take<u32>(dc);
+  sc.r_dense_base = cv.take<u64>(dc + 1);
+  sc.r_topk_off = cv.take<u64>(dc + 1);
+  sc.r_arena_base = cv.take<u64>(dc + 1);
+  if (concat >= 0) {
+    sc.dense = cv.take<uint4>(st.dense_cap);
+    sc.dst = cv.take<u64>(st.dense_cap + 1);
+  }
+  sc.pairset = cv.take<u64>(st.PS);
+  sc.ps_mask = st.PS - 1;
+  sc.done_cap = (u32)dc;
+  st.lbs.flag = cv.take<u32>(st.scan_tiles);
+  st.lbs.agg = cv.take<u64>(st.scan_tiles);
+  st.lbs.inc = cv.take<u64>(st.scan_tiles);
+  st.lbs.tiles = st.scan_tiles;
+}
+
+// Clear, in one launch, what every call must find empty: the control block
+// (keeping its epoch, so epoch-stamped arrays stay valid), the table keys,
+// the per-batch accumulators, the completion masks, the leaf-slot set, the
+// free-chunk stacks and the sort histogram.
+__global__ void k_na_reset(Dev d, u32* hist, u64 T, u64 PS, u32 nmax) {
+  const u64 tid = (u64)blockIdx.x * blockDim.x + threadIdx.x;
+  const u64 stride = (u64)gridDim.x * blockDim.x;
+  if (tid == 0) {
+    Ctl* c = d.ctl;
+    const u32 ep = c->epoch;
+    unsigned char* p = (unsigned char*)c;
+    for (size_t i = 0; i < sizeof(Ctl); ++i) p[i] = 0;
+    c->epoch = ep;
+  }
+  for (u64 i = tid; i < T; i += stride) {
+    d.tab.key[i] = kEmpty;
+    d.tab.touch[i] = 0;
+    d.tab.acc_cnt[i] = 0;
+    d.tab.acc_m1[i] = 0;
+    d.tab.acc_fmin[i] = kNone;
+    d.tab.acc_fmax1[i] = 0;
+    d.tab.acc_cs1[i] = 0;
+    d.tab.acc_smx[i] = 0;
+    d.tab.acc_len[i] = 0;
+  }
+  for (u64 i = tid; i < PS; i += stride) d.sc.pairset[i] = 0;
+  for (u64 i = tid; i < nmax; i += stride) d.sc.mask[i] = 0;
+  for (u64 i = tid; i < 4 * 256; i += stride) hist[i] = 0;
+}
+
+// Counts of the call for the caller: {status, records, payload, top-k pairs}.
+__global__ void k_na_finish(const Ctl* ctl, int64_t* out) {
+  out[0] = ctl->status;
+  out[1] = (ctl->status == ALTO_OK) ? (int64_t)ctl->rec_count : 0;
+  out[2] = (ctl->status == ALTO_OK) ? (int64_t)ctl->pay_count : 0;
+  out[3] = (ctl->status == ALTO_OK) ? (int64_t)ctl->topk_count : 0;
+}
+
+}  // namespace
+
+extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, const alto_batch* b,
+                                                 alto_record* out_records, int64_t cap_records,
+                                                 int32_t* out_payload, int64_t cap_payload,
+                                                 alto_topk_pair* out_topk, int64_t cap_topk,
+                                                 int64_t* out_counts, void* stream) {
+  if (cfg_in == nullptr || b == nullptr || out_counts == nullptr) return ALTO_EINVAL;
+  alto_agg_config cfg = *cfg_in;
+  if (cfg.max_batch_fragments == 0) cfg.max_batch_fragments = (int64_t)kNaMaxFragments;
+  if (cfg.max_batch_payload == 0) cfg.max_batch_payload = (int64_t)kNaMaxPayload;
+  alto_status v = validate(&cfg);
+  if (v != ALTO_OK) return v;
+  if (b->depth != cfg.depth || b->n < 0 || b->n_payload < 0) return ALTO_EINVAL;
+  if (cap_records < 0 || cap_payload < 0 || cap_topk < 0) return ALTO_EINVAL;
+  if ((cap_records > 0 && !out_records) || (cap_payload > 0 && !out_payload) ||
+      (cap_topk > 0 && !out_topk))
+    return ALTO_EINVAL;
+  // sizes beyond what the static scratch holds
+  if ((u64)b->n > kNaMaxFragments || (u64)b->n * (u64)cfg.depth > kNaMaxGroupsLevels ||
+      (u64)b->n_payload > kNaMaxPayload)
+    return ALTO_ENOSPC;
+  if (b->n > 0 && (b->tags == nullptr || b->payload_off == nullptr)) return ALTO_EINVAL;
+  if (b->n_payload > 0 && b->payload == nullptr) return ALTO_EINVAL;
+  bool has_score = false;
+  for (int l = 0; l < cfg.depth; ++l) has_score |= cfg.score_op[l] != ALTO_SCORE_NONE;
+  if (b->n > 0 && has_score && b->score == nullptr) return ALTO_EINVAL;
+
+  // once per device, with that device current: the static array's address
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return ALTO_ECUDA;
+  NaDevice& nd = g_na_dev[dev];
+  if (!nd.ready) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || ptr == nullptr)
+      return ALTO_ECUDA;
+    nd.base = (unsigned char*)ptr;
+    nd.ready = true;
+  }
+  int num_sms = 0;
+  if (cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return ALTO_ECUDA;
+
+  NaState st;
+  NaCarver cv;
+  na_layout(cfg, nd.base, st, cv);
+  if (!cv.ok) return ALTO_ENOSPC;
+  Dev d = st.d;
+  d.out_rec = out_records;
+  d.out_pay = out_payload;
+  d.out_topk = out_topk;
+  d.cfg.out_records = (u64)cap_records;
+  d.cfg.out_payload = (u64)cap_payload;
+  d.cfg.out_topk = (u64)cap_topk;
+
+  cudaStream_t s = (cudaStream_t)stream;
+  const int D = cfg.depth;
+  const u32 n = (u32)b->n;
+  const u32 nmax = (u32)kNaMaxFragments;
+  const int grid = num_sms * 8, sgrid = num_sms * 2;
+  const u64 spin = d.cfg.spin_limit;
+  Batch bt;
+  bt.tags = b->tags;
+  bt.off = b->payload_off;
+  bt.pay = b->payload;
+  bt.score = d.cfg.has_score ? b->score : nullptr;
+  bt.n = n;
+  bt.n_payload = (u64)b->n_payload;
+
+  k_na_reset<<<sgrid, kThreads, 0, s>>>(d, st.leaf_sort.hist, st.T, st.PS, nmax);
+  k_begin<<<1, 1, 0, s>>>(d.ctl, n);
+  if (n > 0) {
+    // the same stages, in the same order, as a push (see alto_agg_push_batch)
+    auto scan_grid = [&](u64 cap) {
+      u64 tiles = (cap + kScanTile - 1) / kScanTile;
+      return (int)std::min<u64>(std::max<u64>(tiles, 1), (u64)num_sms * 4);
+    };
+    int site = 0;
+    k_ingest<<<grid, kThreads, 0, s>>>(d, bt);
+    const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK;
+    int set = 0;
+    if (leaf_sorted) {
+      int cur = sort_pairs(&d.ctl->n, nmax, st.tbits, true, st.leaf_sort, d.ctl, site, spin, num_sms,
+                           s, nullptr);
+      d.sc.leaf_keys = st.leaf_sort.keys[cur];
+      d.sc.leaf_perm = st.leaf_sort.vals[cur];
+      SegFind f{d.sc.leaf_keys, d.sc.leaf_seg_start, d.sc.leaf_seg_of, &d.ctl->n, nmax,
+                &d.ctl->n_segs[D - 1]};
+      k_scan<SegFind><<<scan_grid(nmax), kScanThreads, 0, s>>>(f, st.lbs, d.ctl, site + 4,
+                                                             &d.ctl->exit_ctr[site + 4], spin);
+      k_reduce<true><<<grid, kThreads, 0, s>>>(d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
+                                               d.sc.leaf_seg_start, set);
+    } else {
+      k_leaf_accumulate<<<grid, kThreads, 0, s>>>(d, bt);
+      k_up_finalize<true><<<sgrid, kThreads, 0, s>>>(d, bt, D - 1, set);
+    }
+    site += 5;
+    for (int l = D - 2; l >= 0; --l) {
+      set ^= 1;
+      k_items_lookup<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+      if (d.cfg.score_op[l] != ALTO_SCORE_TOPK) {
+        k_up_accumulate<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+        k_up_finalize<false><<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+        continue;
+      }
+      int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nmax, st.tbits, true, st.up_sort, d.ctl, site, spin,
+                          num_sms, s, nullptr);
+      site += 4;
+      d.sc.up_keys = st.up_sort.keys[c2];
+      d.sc.up_perm = st.up_sort.vals[c2];
+      SegFind f{d.sc.up_keys, d.sc.up_seg_start, nullptr, &d.ctl->n_segs[l + 1], nmax,
+                &d.ctl->n_segs[l]};
+      k_scan<SegFind><<<scan_grid(nmax), kScanThreads, 0, s>>>(f, st.lbs, d.ctl, site,
+                                                             &d.ctl->exit_ctr[site], spin);
+      ++site;
+      k_reduce<false><<<grid, kThreads, 0, s>>>(d, bt, l, d.sc.up_keys, d.sc.up_perm,
+                                                d.sc.up_seg_start, set);
+    }
+    {
+      RankScan f{d.sc.mask, d.sc.prefix, &d.ctl->n};
+      k_scan<RankScan><<<scan_grid(nmax), kScanThreads, 0, s>>>(f, st.lbs, d.ctl, site,
+                                                              &d.ctl->exit_ctr[site], spin);
+      ++site;
+    }
+    k_done_rank<<<sgrid, kThreads, 0, s>>>(d);
+    const u32 dcap = d.sc.done_cap;
+    CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0};
+    k_scan<CountScan><<<scan_grid(dcap), kScanThreads, 0, s>>>(f0, st.lbs, d.ctl, site,
+                                                             &d.ctl->exit_ctr[site], spin);
+    ++site;
+    CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
+    k_scan<CountScan><<<scan_grid(dcap), kScanThreads, 0, s>>>(f1, st.lbs, d.ctl, site,
+                                                             &d.ctl->exit_ctr[site], spin);
+    ++site;
+    CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
+    k_scan<CountScan><<<scan_grid(dcap), kScanThreads, 0, s>>>(f2, st.lbs, d.ctl, site,
+                                                             &d.ctl->exit_ctr[site], spin);
+    ++site;
+    k_check<<<1, 1, 0, s>>>(d);
+    if (d.cfg.concat_level >= 0) {
+      if (leaf_sorted) {
+        k_carry_alloc<false><<<sgrid, kThreads, 0, s>>>(d);
+        k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
+        k_carry_copy<<<grid, kThreads, 0, s>>>(d, bt);
+        k_dense_batch<<<grid, kThreads, 0, s>>>(d, bt);
+      } else {
+        k_carry_alloc<true><<<sgrid, kThreads, 0, s>>>(d);
+        k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
+        k_leaf_place<<<grid, kThreads, 0, s>>>(d, bt);
+      }
+      k_dense_arena<<<sgrid, kThreads, 0, s>>>(d);
+      DenseScan fd{d.sc.dense, d.sc.dst, d.ctl};
+      k_scan<DenseScan><<<scan_grid(d.cfg.dense_cap), kScanThreads, 0, s>>>(
+          fd, st.lbs, d.ctl, site, &d.ctl->exit_ctr[site], spin);
+      ++site;
+      k_check2<<<1, 1, 0, s>>>(d);
+      k_gather<<<grid, kThreads, 0, s>>>(d, bt);
+    }
+    k_records<<<sgrid, kThreads, 0, s>>>(d);
+    k_sweep<<<sgrid, kThreads, 0, s>>>(d);
+  }
+  k_end<<<1, 1, 0, s>>>(d.ctl, n);
+  k_na_finish<<<1, 1, 0, s>>>(d.ctl, out_counts);
+  if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
+  return ALTO_OK;
+}
