@@ -56,7 +56,7 @@ def stream_caps(s):
         max_batch_fragments=int(max(s.batch_sizes)),
         max_batch_payload=max(1, max(pay_b)),
         max_open_groups=min(1 << 24, groups),
-        arena_elems=min((1 << 32) - 1, 2 * int(s.payload.size) + 4 * n),
+        arena_elems=min((1 << 32) - 1, 3 * (int(s.payload.size) + 2 * n) + 64 * groups),
         out_records=groups + 16,
         out_payload_elems=int(s.payload.size) + 16,
         out_topk=groups * max(list(s.topk_k) + [1]) + 16,

@@ -16,8 +16,8 @@ constexpr int kMaxTopk = ALTO_MAX_TOPK;
 constexpr u64 kEmpty = ~0ull;          // free hash slot
 constexpr u64 kTomb = ~0ull - 1;       // deleted hash slot
 constexpr u32 kNone = 0xFFFFFFFFu;     // no last child yet / invalid chunk
-constexpr int kChunk0Log = 8;          // smallest arena chunk: 256 int32
-constexpr int kNumChunks = 22;         // chunk classes 256 << 0 .. 256 << 21
+constexpr int kChunk0Log = 5;          // smallest arena chunk: 32 int32
+constexpr int kNumChunks = 22;         // chunk classes 32 << 0 .. 32 << 21
 constexpr int kVecs = 2;               // per CONCAT group: 0 = leaf meta, 1 = payload
 constexpr int kSites = 64;             // launch sites sharing look-back state per batch
 constexpr int kWarps = 8;              // warps per 256-thread block
@@ -116,8 +116,8 @@ __device__ __forceinline__ u32 lanemask_lt() {
   return m;
 }
 
-// Arena geometry: vector position x lives in chunk j = floor(log2(x/256 + 1)),
-// which starts at position 256 * (2^j - 1) and holds 256 << j elements.
+// Arena geometry: vector position x lives in chunk j = floor(log2(x/32 + 1)),
+// which starts at position 32 * (2^j - 1) and holds 32 << j elements.
 __device__ __forceinline__ int chunk_of(u64 x) {
   u64 q = (x >> kChunk0Log) + 1;
   return 63 - __clzll((long long)q);

@@ -19,7 +19,8 @@ def stream_caps(s, arena_factor=4):
         max_batch_fragments=int(max(s.batch_sizes)),
         max_batch_payload=max(1, max(pay_per_batch)),
         max_open_groups=min(groups + 1024, 1 << 25),
-        arena_elems=min(arena_factor * (int(s.payload.size) + 2 * n) + (1 << 20), (1 << 32) - 1),
+        arena_elems=min(arena_factor * (int(s.payload.size) + 2 * n) + 64 * groups + (1 << 16),
+                        (1 << 32) - 1),
         out_records=groups + 16,
         out_payload_elems=int(s.payload.size) + 16,
         out_topk=groups * kmax + 16,
