@@ -208,6 +208,8 @@ def main():
     ap.add_argument("--ref-sample", type=float, default=250_000)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--latency-batches", type=int, default=16)
+    ap.add_argument("--max-batches", type=int, default=0,
+                    help="profiling only: push just the first B batches per step")
     args = ap.parse_args()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -240,10 +242,16 @@ def main():
     stream = torch.cuda.current_stream()
     caps = stream_caps(s)
     agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, stream=stream, **caps)
-    batches = [alto.to_device(s.batch(b)) for b in range(s.n_batches)]
+    nb = s.n_batches if args.max_batches <= 0 else min(args.max_batches, s.n_batches)
+    batches = [alto.to_device(s.batch(b)) for b in range(nb)]
     torch.cuda.synchronize()
 
     def step():
+        nonlocal agg
+        if args.max_batches > 0:
+            # a truncated stream leaves groups open: start every step afresh
+            agg.close()
+            agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, stream=stream, **caps)
         for db in batches:
             st = agg.push(db.tags, db.off, db.payload, db.score)
             if st != alto.OK:
@@ -310,6 +318,15 @@ def main():
             traffic = json.load(open(tf)).get(dom_for_roof)
         except Exception:
             traffic = None
+
+    if args.max_batches > 0:
+        # profiling runs stop here: the truncated stream cannot be replayed on
+        # one handle
+        agg.close()
+        if rank == 0:
+            print(json.dumps({"profiling_only": True, "ms_per_step": ms_per_step,
+                              "stage_ms_per_step": {k: v / args.steps for k, v in stage_ms.items()}}))
+        return
 
     # ---- end to end: host buffers through the public API ---------------------
     host = []

@@ -136,6 +136,7 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
         tab.acc_cs1[h] = 0;
         tab.acc_smx[h] = 0;
         tab.acc_len[h] = 0;
+        tab.acc_leaf[h] = make_uint4(0, 0, 0, 0);
         tab.carry_epoch[h] = 0;
         *inserted = 1;
         return h;
@@ -151,6 +152,8 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
 
 // Batch-local set of (entry, child) slots; returns true if already present.
 // Keys carry a 7-bit batch epoch so that old batches' keys read as free.
+// (Placing a group's children in neighbouring slots was tried: the runs it
+// builds lengthen every other probe, and the batch got 4x slower.)
 __device__ bool ps_insert(const Scratch& sc, u32 e, u32 c, u32 ep7, Ctl* ctl) {
   const u64 k57 = ((u64)e << 31) | c;
   const u64 full = ((u64)ep7 << 57) | k57;
@@ -169,6 +172,19 @@ __device__ bool ps_insert(const Scratch& sc, u32 e, u32 c, u32 ep7, Ctl* ctl) {
   }
   raise_err(ctl, ALTO_ENOSPC);
   return false;
+}
+
+__device__ __forceinline__ bool chain_differs(const Table& tab, u32 e, const u64* tags, u64 n, u32 rep,
+                                              int l) {
+  // the chain row is padded to an even length: read it two tags at a time
+  const ulonglong2* row = reinterpret_cast<const ulonglong2*>(tab.chain + (u64)e * tab.chain_len);
+  bool bad = false;
+  for (int q = 0; q < l; q += 2) {
+    const ulonglong2 v = row[q >> 1];
+    if (tags[(u64)q * n + rep] != v.x) bad = true;
+    if (q + 1 < l && tags[(u64)(q + 1) * n + rep] != v.y) bad = true;
+  }
+  return bad;
 }
 
 __device__ __forceinline__ u32 epoch7(const Ctl* ctl) { return ((ctl->epoch - 1) % 127u) + 1u; }
@@ -226,6 +242,7 @@ __global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
   __syncthreads();
   const int D = d.cfg.depth;
   const u32 ep7 = epoch7(ctl);
+  const bool sorted_leaf = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK;
   for (u32 i = gtid(); i < b.n; i += gstride()) {
     u32 o0 = b.off[i], o1 = b.off[i + 1];
     if (o1 < o0 || (u64)o1 > b.n_payload) raise_err(ctl, ALTO_EINVAL);
@@ -237,7 +254,8 @@ __global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
                               b.n, i, D - 1);
     if (ins) atomicAdd(&s_ins, 1u);
     d.sc.leaf_sort_keys0[i] = e;
-    if (ps_insert(d.sc, e, tag_child(t), ep7, ctl)) raise_err(ctl, ALTO_EDUP);
+    // the sorted (TOPK) leaf path checks leaf slots here; the accumulate does otherwise
+    if (sorted_leaf && ps_insert(d.sc, e, tag_child(t), ep7, ctl)) raise_err(ctl, ALTO_EDUP);
   }
   __syncthreads();
   if (threadIdx.x == 0 && s_ins) atomicAdd((unsigned long long*)&ctl->live_groups, (u64)s_ins);
@@ -508,10 +526,7 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
       done = cf >> 31;
       cs = cf & 0x7FFFFFFFu;
       sk = it_skey[x];
-      bool bad = false;
-      for (int q = 0; q < l; ++q)
-        if (b.tags[(u64)q * n + rep] != d.tab.chain[(u64)e * d.tab.chain_len + q]) bad = true;
-      if (bad) raise_err(ctl, ALTO_EINCONSIST);
+      if (chain_differs(d.tab, e, b.tags, n, rep, l)) raise_err(ctl, ALTO_EINCONSIST);
       if (atomicExch(&d.tab.touch[e], ep) != ep) {
         const u32 pos = atomicAdd(&ctl->n_segs[l], 1u);
         if (pos < d.cfg.n_max) list[pos] = e;
@@ -520,8 +535,24 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
     }
     // lanes past the end form their own group; the whole warp takes part
     const u32 key = valid ? e : kNone;
+    const u32 peers0 = __match_any_sync(0xFFFFFFFFu, key);
+    if (__all_sync(0xFFFFFFFFu, peers0 == (1u << (threadIdx.x & 31)))) {
+      if (valid) {
+        if (done) {
+          atomicAdd(&d.tab.acc_cnt[e], 1u);
+          atomicMax(&d.tab.acc_cs1[e], cs + 1);
+          if (sk) atomicMax(&d.tab.acc_smx[e], sk);
+        }
+        atomicMax(&d.tab.acc_m1[e], c + 1);
+        if (f) {
+          atomicMin(&d.tab.acc_fmin[e], c);
+          atomicMax(&d.tab.acc_fmax1[e], c + 1);
+        }
+      }
+      continue;
+    }
     {
-      const u32 peers = __match_any_sync(0xFFFFFFFFu, key);
+      const u32 peers = peers0;
       const int leader = __ffs(peers) - 1;
       const u32 cnt = __reduce_add_sync(peers, done);
       const u32 m1 = __reduce_max_sync(peers, valid ? c + 1 : 0u);
@@ -551,8 +582,10 @@ __global__ void __launch_bounds__(kThreads) k_leaf_accumulate(Dev d, Batch b) {
   const int L = D - 1;
   const u64 n = b.n;
   const bool scores = d.cfg.has_score;
+  const u32 ep7 = epoch7(ctl);
   u32* list = d.sc.leaf_seg_start;  // touched leaf-parent entries
   const u32 end = (b.n + 31) & ~31u;
+  const int lane = threadIdx.x & 31;
   for (u32 i = gtid(); i < end; i += gstride()) {
     const bool valid = i < b.n;
     u32 e = 0, c = 0, f = 0, len = 0, sk = 0;
@@ -563,41 +596,60 @@ __global__ void __launch_bounds__(kThreads) k_leaf_accumulate(Dev d, Batch b) {
       f = tag_last(t);
       len = b.off[i + 1] - b.off[i];
       if (scores) sk = score_key(b.score[i]);
-      bool bad = false;
-      for (int q = 0; q < L; ++q)
-        if (b.tags[(u64)q * n + i] != d.tab.chain[(u64)e * d.tab.chain_len + q]) bad = true;
-      if (bad) raise_err(ctl, ALTO_EINCONSIST);
+      if (chain_differs(d.tab, e, b.tags, n, i, L)) raise_err(ctl, ALTO_EINCONSIST);
+      if (ps_insert(d.sc, e, c, ep7, ctl)) raise_err(ctl, ALTO_EDUP);
     }
     const u32 key = valid ? e : kNone;
     const u32 peers = __match_any_sync(0xFFFFFFFFu, key);
+    if (__all_sync(0xFFFFFFFFu, peers == (1u << lane))) {
+      // every lane its own group (the common case): plain atomics, no reductions
+      if (valid) {
+        uint4* rec = d.tab.acc_leaf + e;
+        const u64 old = atomicAdd((unsigned long long*)&rec->x, (1ull << 40) | len);
+        if (old == 0) {
+          const u32 pos = atomicAdd(&ctl->n_segs[L], 1u);
+          if (pos < d.cfg.n_max) list[pos] = e;
+          d.tab.acc_rep[e] = i;
+        }
+        atomicMax(&rec->z, c + 1);
+        atomicMax(&rec->w, i + 1);
+        if (f) {
+          atomicMin(&d.tab.acc_fmin[e], c);
+          atomicMax(&d.tab.acc_fmax1[e], c + 1);
+        }
+        if (scores) atomicMax(&d.tab.acc_smx[e], sk);
+      }
+      continue;
+    }
     const int leader = __ffs(peers) - 1;
     const u32 cnt = __popc(peers);
     const u32 m1 = __reduce_max_sync(peers, valid ? c + 1 : 0u);
     const u32 cs1 = __reduce_max_sync(peers, valid ? i + 1 : 0u);
     const u32 lsum = __reduce_add_sync(peers, len);
     const u32 anyf = __reduce_or_sync(peers, f);
-    if (valid && (int)(threadIdx.x & 31) == leader) {
-      const u32 old = atomicAdd(&d.tab.acc_cnt[e], cnt);
+    if (valid && lane == leader) {
+      // one returning atomic per group and warp: leaves and payload together
+      uint4* rec = d.tab.acc_leaf + e;
+      const u64 old = atomicAdd((unsigned long long*)&rec->x, ((unsigned long long)cnt << 40) | lsum);
       if (old == 0) {
         const u32 pos = atomicAdd(&ctl->n_segs[L], 1u);
         if (pos < d.cfg.n_max) list[pos] = e;
         d.tab.acc_rep[e] = i;
       }
-      atomicMax(&d.tab.acc_m1[e], m1);
-      atomicMax(&d.tab.acc_cs1[e], cs1);
-      if (lsum) atomicAdd(&d.tab.acc_len[e], lsum);
+      atomicMax(&rec->z, m1);
+      atomicMax(&rec->w, cs1);
     }
     if (anyf) {
       const u32 fmin = __reduce_min_sync(peers, (valid && f) ? c : kNone);
       const u32 fmax1 = __reduce_max_sync(peers, (valid && f) ? c + 1 : 0u);
-      if (valid && (int)(threadIdx.x & 31) == leader && fmax1) {
+      if (valid && lane == leader && fmax1) {
         atomicMin(&d.tab.acc_fmin[e], fmin);
         atomicMax(&d.tab.acc_fmax1[e], fmax1);
       }
     }
     if (scores) {
       const u32 smx = __reduce_max_sync(peers, valid ? sk : 0u);
-      if (valid && (int)(threadIdx.x & 31) == leader && smx) atomicMax(&d.tab.acc_smx[e], smx);
+      if (valid && lane == leader && smx) atomicMax(&d.tab.acc_smx[e], smx);
     }
   }
 }
@@ -611,6 +663,10 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
   const bool carry = LEAF && d.cfg.concat_level == D - 1;
   const u32 nt = min(ctl->n_segs[l], d.cfg.n_max);
   const u32 ep = ctl->epoch;
+  const u32 ep7 = epoch7(ctl);
+  __shared__ u32 s_ins;
+  if (threadIdx.x == 0) s_ins = 0;
+  __syncthreads();
   const u32* list = LEAF ? d.sc.leaf_seg_start : d.sc.up_seg_start;
   u32* nx_rep = d.sc.it_rep[in_set ^ 1];
   u32* nx_cseq = d.sc.it_cseq[in_set ^ 1];
@@ -618,12 +674,25 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
   const u64 n = b.n;
   for (u32 s = gtid(); s < nt; s += gstride()) {
     const u32 e = list[s] & d.tab.mask;
-    const u32 cnt = d.tab.acc_cnt[e], m1 = d.tab.acc_m1[e], fmin = d.tab.acc_fmin[e];
-    const u32 fmax1 = d.tab.acc_fmax1[e], cs1 = d.tab.acc_cs1[e], smx = d.tab.acc_smx[e];
+    u32 cnt, m1, cs1;
+    u32 blen = 0;
+    if (LEAF) {
+      const uint4 a = d.tab.acc_leaf[e];
+      const u64 cl = ((u64)a.y << 32) | a.x;
+      cnt = (u32)(cl >> 40);
+      blen = (u32)(cl & ((1ull << 40) - 1));
+      m1 = a.z;
+      cs1 = a.w;
+      d.tab.acc_leaf[e] = make_uint4(0, 0, 0, 0);
+    } else {
+      cnt = d.tab.acc_cnt[e];
+      m1 = d.tab.acc_m1[e];
+      cs1 = d.tab.acc_cs1[e];
+    }
+    const u32 fmin = d.tab.acc_fmin[e];
+    const u32 fmax1 = d.tab.acc_fmax1[e], smx = d.tab.acc_smx[e];
     const u32 rep = d.tab.acc_rep[e];
-    const u32 blen = LEAF ? d.tab.acc_len[e] : 0u;
     // reset the accumulators for the next batch
-    if (LEAF) d.tab.acc_len[e] = 0;
     d.tab.acc_cnt[e] = 0;
     d.tab.acc_m1[e] = 0;
     d.tab.acc_fmin[e] = kNone;
@@ -673,8 +742,19 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
       nx_rep[s] = rep;
       nx_cseq[s] = (complete ? 0x80000000u : 0u) | cmax;
       nx_skey[s] = smn;
+      // the next level's item is known now: find or insert its parent group
+      const u64 tp = b.tags[(u64)(l - 1) * n + rep];
+      const u64 upp = (l > 1) ? b.tags[(u64)(l - 2) * n + rep] : 0ull;
+      int ins = 0;
+      const u32 e2 = ht_find_or_insert(d.tab, ((u64)(l - 1) << 32) | tag_pid(tp), upp, ctl, &ins,
+                                       b.tags, n, rep, l - 1);
+      if (ins) atomicAdd(&s_ins, 1u);
+      d.sc.up_sort_keys0[s] = e2;
+      if (ps_insert(d.sc, e2, tag_child(tp), ep7, ctl)) raise_err(ctl, ALTO_EINCONSIST);
     }
   }
+  __syncthreads();
+  if (threadIdx.x == 0 && s_ins) atomicAdd((unsigned long long*)&ctl->live_groups, (u64)s_ins);
 }
 
 // Emission rank of each completed group: records completed at earlier
@@ -721,9 +801,20 @@ struct CountScan {
   const u32* n_dev;
   u32 cap;
   int which;  // 0 dense, 1 topk, 2 arena
+  // dense only: also leave each completing group's first slot in its entry
+  const u32* r_done = nullptr;
+  const u32* done_e = nullptr;
+  u64* dbase = nullptr;
+  u32 tmask = 0;
   __device__ u64 size(const Ctl*) const { return min(*n_dev, cap); }
   __device__ u64 value(u64 i) const { return in[i]; }
-  __device__ void out(u64 i, u64 excl, u64) const { out_off[i] = excl; }
+  __device__ void out(u64 i, u64 excl, u64 v) const {
+    out_off[i] = excl;
+    if (dbase && v) {
+      const u32 di = r_done[i];
+      if (di < cap) dbase[done_e[di] & tmask] = excl;
+    }
+  }
   __device__ void total(Ctl* ctl, u64 t) const {
     out_off[size(nullptr)] = t;
     if (which == 0) ctl->dense_total = t;
@@ -955,56 +1046,69 @@ __global__ void __launch_bounds__(kThreads) k_leaf_place(Dev d, Batch b) {
   const int D = d.cfg.depth;
   const u32 ep = ctl->epoch;
   const u64 n = b.n;
-  const u32 nd = min(ctl->n_done, d.sc.done_cap);
   const bool dense_ok = !ctl->skip_dense;
-  const u32 sub = threadIdx.x & 7;
-  const u32 g0 = gtid() >> 3, ng = gstride() >> 3;
-  const u32 end = (b.n + 3) & ~3u;  // four groups per warp: keep warps converged
-  for (u32 i = g0; i < end; i += ng) {
-    const bool valid = i < b.n;
+  const u64 dcap = d.cfg.dense_cap;
+  const int lane = threadIdx.x & 31;
+  const u32 end = (b.n + 31) & ~31u;  // whole warps iterate together
+  for (u32 i = gtid(); i < end; i += gstride()) {
     u32 e = 0, mode = 0;  // 1 arena, 2 dense
-    if (valid) {
-      e = d.sc.leaf_sort_keys0[i] & d.tab.mask;
-      if (d.tab.carry_epoch[e] == ep) mode = 1;
-      else if (dense_ok && d.tab.done_epoch[e] == ep) mode = 2;
-    }
     u32 o0 = 0, len = 0, c = 0;
-    if (mode) {
+    if (i < b.n) {
+      // the fragment's own fields do not depend on its group: load them first
+      e = d.sc.leaf_sort_keys0[i] & d.tab.mask;
       o0 = b.off[i];
       len = b.off[i + 1] - o0;
       c = tag_child(b.tags[(u64)(D - 1) * n + i]);
+      const u32 ce = d.tab.carry_epoch[e], de = d.tab.done_epoch[e];
+      if (ce == ep) mode = 1;
+      else if (dense_ok && de == ep) mode = 2;
     }
-    u64 old = 0;
-    if (mode == 1 && sub == 0) old = atomicAdd((unsigned long long*)&d.tab.cur[e], (1ull << 40) | len);
-    old = __shfl_sync(0xFFFFFFFFu, old, 0, 8);
+    if (mode == 2) {
+      // every child index is below n_children (checked at completion); a
+      // repeated child leaves some other slot unfilled, which the length
+      // scan reports
+      const u64 slot = d.tab.dbase[e] + c;
+      if (slot < dcap) d.sc.dense[slot] = make_uint4(ep, len, kNone, o0);
+    }
+    u64 ppos = 0;
+    bool copy = false;
     if (mode == 1) {
-      const u64 mpos = old >> 40, ppos = old & ((1ull << 40) - 1);
+      const u64 old = atomicAdd((unsigned long long*)&d.tab.cur[e], (1ull << 40) | len);
+      const u64 mpos = old >> 40;
+      ppos = old & ((1ull << 40) - 1);
       if (mpos < d.tab.vec_n[2 * (u64)e] && ppos + len <= d.tab.vec_n[2 * (u64)e + 1] &&
           (u64)o0 + len <= b.n_payload) {
         bool ok;
-        if (sub == 0) {
-          const u64 a = vec_addr(d.tab, e, 0, 2 * mpos, &ok);
-          if (ok) {
-            d.ar.pool[a] = (int32_t)c;
-            d.ar.pool[a + 1] = (int32_t)(u32)ppos;
-          }
+        const u64 a = vec_addr(d.tab, e, 0, 2 * mpos, &ok);
+        if (ok) {
+          d.ar.pool[a] = (int32_t)c;
+          d.ar.pool[a + 1] = (int32_t)(u32)ppos;
         }
-        for (u32 k = sub; k < len; k += 8) {
-          const u64 a = vec_addr(d.tab, e, 1, ppos + k, &ok);
-          if (ok) d.ar.pool[a] = b.pay[o0 + k];
-        }
+        copy = true;
       }
-    } else if (mode == 2 && sub == 0) {
-      const u32 di = d.tab.done_idx[e];
-      const u32 r = (di < nd) ? d.sc.done_rank[di] : kNone;
-      if (r < nd && c < d.sc.r_dense_n[r]) {
-        const u64 slot = d.sc.r_dense_base[r] + c;
-        if (slot < d.cfg.dense_cap) {
-          const u32 prev = atomicExch(&d.sc.dense[slot].x, ep);
-          if (prev == ep) raise_err(ctl, ALTO_EDUP);
-          d.sc.dense[slot].y = len;
-          d.sc.dense[slot].z = kNone;
-          d.sc.dense[slot].w = o0;
+    }
+    // the warp copies the tokens of its arena-bound fragments one after another
+    u32 pending = __ballot_sync(0xFFFFFFFFu, copy);
+    while (pending) {
+      const int src = __ffs(pending) - 1;
+      pending &= pending - 1;
+      const u32 se = __shfl_sync(0xFFFFFFFFu, e, src);
+      const u32 so = __shfl_sync(0xFFFFFFFFu, o0, src);
+      const u32 sl = __shfl_sync(0xFFFFFFFFu, len, src);
+      const u64 sp = __shfl_sync(0xFFFFFFFFu, ppos, src);
+      // positions before the end of the first chunk need no directory lookup
+      const int j1 = chunk_of(sp);
+      const u64 cend = chunk_start(j1) + chunk_size(j1);
+      bool ok1;
+      const u64 a1 = vec_addr(d.tab, se, 1, sp, &ok1);
+      for (u32 k = lane; k < sl; k += 32) {
+        const int32_t v = b.pay[(u64)so + k];
+        if (sp + k < cend) {
+          if (ok1) d.ar.pool[a1 + k] = v;
+        } else {
+          bool ok;
+          const u64 a = vec_addr(d.tab, se, 1, sp + k, &ok);
+          if (ok) d.ar.pool[a] = v;
         }
       }
     }
@@ -1095,7 +1199,7 @@ __global__ void k_check2(Dev d) {
 // Copy every child span into the output payload ring.  A warp takes 32
 // consecutive dense slots -- one contiguous output range -- reads their
 // headers in one go, then copies four spans per round with all loads issued
-// before the stores.  Spans longer than 32 elements finish in a second loop.
+// before the stores.  Spans longer than 64 elements finish in a second loop.
 __device__ __forceinline__ int32_t span_load(const Dev& d, const Batch& b, u32 owner, u32 pos,
                                              u32 k) {
   if (owner == kNone) return b.pay[(u64)pos + k];
@@ -1133,8 +1237,10 @@ __global__ void __launch_bounds__(kThreads) k_gather(Dev d, Batch b) {
       }
     }
     const u32 cnt = (total - jb < 32) ? (u32)(total - jb) : 32u;
+    // four spans per round, two elements per lane per span: all eight loads
+    // are in flight before the first store
     for (u32 k0 = 0; k0 < cnt; k0 += 4) {
-      int32_t val[4];
+      int32_t val[4][2];
       u32 L[4];
       u64 O[4];
 #pragma unroll
@@ -1145,20 +1251,23 @@ __global__ void __launch_bounds__(kThreads) k_gather(Dev d, Batch b) {
         const u32 ps = __shfl_sync(0xFFFFFFFFu, pos, src);
         O[u] = __shfl_sync(0xFFFFFFFFu, o, src);
         if (k0 + u >= cnt) L[u] = 0;
-        val[u] = ((u32)lane < L[u]) ? span_load(d, b, ow, ps, lane) : 0;
+        val[u][0] = ((u32)lane < L[u]) ? span_load(d, b, ow, ps, lane) : 0;
+        val[u][1] = ((u32)lane + 32 < L[u]) ? span_load(d, b, ow, ps, lane + 32) : 0;
       }
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if ((u32)lane < L[u]) out[O[u] + lane] = val[u];
+      for (int u = 0; u < 4; ++u) {
+        if ((u32)lane < L[u]) out[O[u] + lane] = val[u][0];
+        if ((u32)lane + 32 < L[u]) out[O[u] + lane + 32] = val[u][1];
+      }
     }
     // the remainder of long spans
     for (u32 k = 0; k < cnt; ++k) {
       const u32 Lk = __shfl_sync(0xFFFFFFFFu, len, k);
-      if (Lk <= 32) continue;
+      if (Lk <= 64) continue;
       const u32 ow = __shfl_sync(0xFFFFFFFFu, owner, k);
       const u32 ps = __shfl_sync(0xFFFFFFFFu, pos, k);
       const u64 Ok = __shfl_sync(0xFFFFFFFFu, o, k);
-      for (u32 q = 32 + lane; q < Lk; q += 32) out[Ok + q] = span_load(d, b, ow, ps, q);
+      for (u32 q = 64 + lane; q < Lk; q += 32) out[Ok + q] = span_load(d, b, ow, ps, q);
     }
   }
 }
@@ -1168,66 +1277,96 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
   if (poisoned(ctl)) return;
   __shared__ u32 s_del;
   __shared__ unsigned long long s_freed;
+  __shared__ u32 s_cnt[kNumChunks];
+  __shared__ u32 s_rank[kNumChunks];
+  __shared__ int s_base[kNumChunks];
   if (threadIdx.x == 0) {
     s_del = 0;
     s_freed = 0;
   }
-  __syncthreads();
   const int M = d.cfg.concat_level;
   const u32 nd = min(ctl->n_done, d.sc.done_cap);
   const bool skip = ctl->skip_dense;
-  for (u32 di = gtid(); di < nd; di += gstride()) {
-    const u32 e = d.sc.done_e[di];
-    const int l = (int)d.sc.done_lvl[di];
-    const u32 cs = d.sc.done_cseq[di];
-    const u32 r = d.sc.done_rank[di];
-    d.sc.mask[cs] = 0;
-    if (!skip && r != kNone) {
-      alto_record rec;
-      rec.completion_seq = ctl->seq_base + cs;
-      if (M >= 0) {
-        const u64 db = min(d.sc.r_dense_base[r], ctl->dense_total);
-        const u64 de = min(db + d.sc.r_dense_n[r], ctl->dense_total);
-        rec.payload_off = ctl->pay_count + d.sc.dst[db];
-        rec.payload_len = (l == M) ? d.sc.dst[de] - d.sc.dst[db] : 0;
-      } else {
-        rec.payload_off = ctl->pay_count;
-        rec.payload_len = 0;
-      }
-      u32 tn = d.sc.r_topk_n[r];
-      const u64 to = ctl->topk_count + d.sc.r_topk_off[r];
-      if (to + tn > d.cfg.out_topk) tn = 0;
-      rec.topk_off = to;
-      rec.topk_n = (uint16_t)tn;
-      rec.parent_id = (u32)d.tab.key[e];
-      rec.n_children = d.tab.last[e] + 1;
-      rec.level = (uint8_t)l;
-      rec.ops = (uint8_t)(((l == M) ? 1 : 0) | (d.cfg.score_op[l] << 2));
-      rec.score = (d.cfg.score_op[l] != ALTO_SCORE_NONE) ? key_score(d.tab.smax[e]) : 0.0f;
-      d.out_rec[ctl->rec_count + r] = rec;
-      for (u32 q = 0; q < tn; ++q) {
-        const u64 v = d.tab.topk[(u64)e * d.tab.kk + q];
-        alto_topk_pair p;
-        p.child_index = ~(u32)v;
-        p.score = key_score((u32)(v >> 32));
-        d.out_topk[to + q] = p;
-      }
+  for (u32 base = blockIdx.x * blockDim.x; base < nd; base += gridDim.x * blockDim.x) {
+    if (threadIdx.x < kNumChunks) {
+      s_cnt[threadIdx.x] = 0;
+      s_rank[threadIdx.x] = 0;
     }
-    if (l == M) {
+    __syncthreads();
+    const u32 di = base + threadIdx.x;
+    const bool mine = di < nd;
+    u32 e = 0;
+    int l = 0;
+    u64 el[kVecs] = {0, 0};
+    if (mine) {
+      e = d.sc.done_e[di] & d.tab.mask;
+      l = (int)d.sc.done_lvl[di];
+      const u32 cs = d.sc.done_cseq[di];
+      const u32 r = d.sc.done_rank[di];
+      if (cs < d.cfg.n_max) d.sc.mask[cs] = 0;
+      if (!skip && r != kNone) {
+        alto_record rec;
+        rec.completion_seq = ctl->seq_base + cs;
+        if (M >= 0) {
+          const u64 db = min(d.sc.r_dense_base[r], ctl->dense_total);
+          const u64 de = min(db + d.sc.r_dense_n[r], ctl->dense_total);
+          rec.payload_off = ctl->pay_count + d.sc.dst[db];
+          rec.payload_len = (l == M) ? d.sc.dst[de] - d.sc.dst[db] : 0;
+        } else {
+          rec.payload_off = ctl->pay_count;
+          rec.payload_len = 0;
+        }
+        u32 tn = d.sc.r_topk_n[r];
+        const u64 to = ctl->topk_count + d.sc.r_topk_off[r];
+        if (to + tn > d.cfg.out_topk) tn = 0;
+        rec.topk_off = to;
+        rec.topk_n = (uint16_t)tn;
+        rec.parent_id = (u32)d.tab.key[e];
+        rec.n_children = d.tab.last[e] + 1;
+        rec.level = (uint8_t)l;
+        rec.ops = (uint8_t)(((l == M) ? 1 : 0) | (d.cfg.score_op[l] << 2));
+        rec.score = (d.cfg.score_op[l] != ALTO_SCORE_NONE) ? key_score(d.tab.smax[e]) : 0.0f;
+        d.out_rec[ctl->rec_count + r] = rec;
+        for (u32 q = 0; q < tn; ++q) {
+          const u64 v = d.tab.topk[(u64)e * d.tab.kk + q];
+          alto_topk_pair p;
+          p.child_index = ~(u32)v;
+          p.score = key_score((u32)(v >> 32));
+          d.out_topk[to + q] = p;
+        }
+      }
+      if (l == M) {
+        for (int vec = 0; vec < kVecs; ++vec) {
+          el[vec] = (u64)d.tab.vec_n[2 * (u64)e + vec] * (vec == 0 ? 2 : 1);
+          if (el[vec] == 0) continue;
+          const int jl = min(chunk_of(el[vec] - 1), kNumChunks - 1);
+          for (int j = 0; j <= jl; ++j) atomicAdd(&s_cnt[j], 1u);
+        }
+      }
+      d.tab.key[e] = kTomb;
+      atomicAdd(&s_del, 1u);
+    }
+    __syncthreads();
+    // one push per chunk class for the whole block
+    if (threadIdx.x < kNumChunks && s_cnt[threadIdx.x]) {
+      const int j = threadIdx.x;
+      s_base[j] = atomicAdd(&ctl->top[j], (int)s_cnt[j]);
+      atomicAdd(&s_freed, (unsigned long long)s_cnt[j] * chunk_size(j));
+    }
+    __syncthreads();
+    if (mine && l == M) {
       for (int vec = 0; vec < kVecs; ++vec) {
-        const u64 el = (u64)d.tab.vec_n[2 * (u64)e + vec] * (vec == 0 ? 2 : 1);
-        if (el == 0) continue;
-        const int jl = min(chunk_of(el - 1), kNumChunks - 1);
+        if (el[vec] == 0) continue;
+        const int jl = min(chunk_of(el[vec] - 1), kNumChunks - 1);
         for (int j = 0; j <= jl; ++j) {
-          free_chunk(d.ar, ctl, j, d.tab.dir[((u64)e * kVecs + vec) * kNumChunks + j]);
-          atomicAdd(&s_freed, (unsigned long long)chunk_size(j));
+          const u32 chunk = d.tab.dir[((u64)e * kVecs + vec) * kNumChunks + j];
+          const u64 pos = (u64)s_base[j] + atomicAdd(&s_rank[j], 1u);
+          if (chunk != kNone && pos < d.ar.stack_cap[j]) d.ar.stack[d.ar.stack_off[j] + pos] = chunk;
         }
       }
     }
-    d.tab.key[e] = kTomb;
-    atomicAdd(&s_del, 1u);
+    __syncthreads();
   }
-  __syncthreads();
   if (threadIdx.x == 0) {
     if (s_del) atomicAdd((unsigned long long*)&ctl->live_groups, (unsigned long long)(-(long long)s_del));
     if (s_freed) atomicAdd((unsigned long long*)&ctl->arena_used, (unsigned long long)(-(long long)s_freed));
@@ -1513,7 +1652,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     ALLOC(d.tab.dir, u32, T * kVecs * kNumChunks);
   }
   if (kk > 0) ALLOC(d.tab.topk, u64, T * (u64)kk);
-  d.tab.chain_len = std::max(D - 1, 1);
+  d.tab.chain_len = std::max((D - 1 + 1) & ~1, 2);  // even: read as 16-byte pairs
   ALLOC(d.tab.chain, u64, T * (u64)d.tab.chain_len);
   ALLOC(d.tab.touch, u32, T);
   ALLOC(d.tab.acc_cnt, u32, T);
@@ -1526,6 +1665,8 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(d.tab.acc_len, u32, T);
   ALLOC(d.tab.carry_epoch, u32, T);
   ALLOC(d.tab.cur, u64, T);
+  ALLOC(d.tab.acc_leaf, uint4, T);
+  ALLOC(d.tab.dbase, u64, T);
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
   d.tab.max_probe = (int)std::min<u64>(T, 1u << 16);
@@ -1723,16 +1864,22 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
     }
     site += 5;
     stage_enter(3);
+    // an atomic finalize also looks up the parent groups of the items it emits
+    bool looked_up = !leaf_sorted;
     for (int l = D - 2; l >= 0; --l) {
       set ^= 1;  // items written by the level below
-      k_items_lookup<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
-      h->launches += 1;
+      if (!looked_up) {
+        k_items_lookup<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+        h->launches += 1;
+      }
       if (d.cfg.score_op[l] != ALTO_SCORE_TOPK) {
         k_up_accumulate<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
         k_up_finalize<false><<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
         h->launches += 2;
+        looked_up = true;
         continue;
       }
+      looked_up = false;
       int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nmax, h->tbits, true, h->up_sort, d.ctl, site,
                           spin, h->num_sms, s, &sl);
       h->launches += sl;
@@ -1757,7 +1904,8 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
     h->launches += 1;
     const u32 dcap = d.sc.done_cap;
     {
-      CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0};
+      CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0,
+                   d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask};
       launch_scan(h, f0, dcap, site++, s);
       CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
       launch_scan(h, f1, dcap, site++, s);
@@ -1985,7 +2133,7 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
     d.tab.dir = cv.take<u32>(T * kVecs * kNumChunks);
   }
   if (kk > 0) d.tab.topk = cv.take<u64>(T * (u64)kk);
-  d.tab.chain_len = std::max(D - 1, 1);
+  d.tab.chain_len = std::max((D - 1 + 1) & ~1, 2);  // even: read as 16-byte pairs
   d.tab.chain = cv.take<u64>(T * (u64)d.tab.chain_len);
   d.tab.touch = cv.take<u32>(T);
   d.tab.acc_cnt = cv.take<u32>(T);
@@ -1998,6 +2146,8 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   d.tab.acc_len = cv.take<u32>(T);
   d.tab.carry_epoch = cv.take<u32>(T);
   d.tab.cur = cv.take<u64>(T);
+  d.tab.acc_leaf = cv.take<uint4>(T);
+  d.tab.dbase = cv.take<u64>(T);
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
   d.tab.max_probe = (int)T;
@@ -2102,6 +2252,7 @@ __global__ void k_na_reset(Dev d, u32* hist, u64 T, u64 PS, u32 nmax) {
     d.tab.acc_cs1[i] = 0;
     d.tab.acc_smx[i] = 0;
     d.tab.acc_len[i] = 0;
+    d.tab.acc_leaf[i] = make_uint4(0, 0, 0, 0);
   }
   for (u64 i = tid; i < PS; i += stride) d.sc.pairset[i] = 0;
   for (u64 i = tid; i < nmax; i += stride) d.sc.mask[i] = 0;
@@ -2213,14 +2364,17 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
       k_up_finalize<true><<<sgrid, kThreads, 0, s>>>(d, bt, D - 1, set);
     }
     site += 5;
+    bool looked_up = !leaf_sorted;
     for (int l = D - 2; l >= 0; --l) {
       set ^= 1;
-      k_items_lookup<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+      if (!looked_up) k_items_lookup<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
       if (d.cfg.score_op[l] != ALTO_SCORE_TOPK) {
         k_up_accumulate<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
         k_up_finalize<false><<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+        looked_up = true;
         continue;
       }
+      looked_up = false;
       int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nmax, st.tbits, true, st.up_sort, d.ctl, site, spin,
                           num_sms, s, nullptr);
       site += 4;
@@ -2242,7 +2396,8 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
     }
     k_done_rank<<<sgrid, kThreads, 0, s>>>(d);
     const u32 dcap = d.sc.done_cap;
-    CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0};
+    CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0,
+                 d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask};
     k_scan<CountScan><<<scan_grid(dcap), kScanThreads, 0, s>>>(f0, st.lbs, d.ctl, site,
                                                              &d.ctl->exit_ctr[site], spin);
     ++site;
