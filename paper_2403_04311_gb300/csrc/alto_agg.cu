@@ -724,6 +724,7 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
       d.tab.vec_n[2 * (u64)e] = v0 + cnt;
       d.tab.vec_n[2 * (u64)e + 1] = v1 + blen;
       d.tab.carry_epoch[e] = ep;
+      d.tab.bstate[e] = make_uint4(ep, 1u, 0u, 0u);
     }
     if (complete) {
       u32 di = atomicAdd(&ctl->n_done, 1u);
@@ -806,13 +807,20 @@ struct CountScan {
   const u32* done_e = nullptr;
   u64* dbase = nullptr;
   u32 tmask = 0;
+  uint4* bstate = nullptr;
+  const Ctl* ctlp = nullptr;
   __device__ u64 size(const Ctl*) const { return min(*n_dev, cap); }
   __device__ u64 value(u64 i) const { return in[i]; }
   __device__ void out(u64 i, u64 excl, u64 v) const {
     out_off[i] = excl;
     if (dbase && v) {
       const u32 di = r_done[i];
-      if (di < cap) dbase[done_e[di] & tmask] = excl;
+      if (di < cap) {
+        const u32 e = done_e[di] & tmask;
+        dbase[e] = excl;
+        if (bstate && !ctlp->skip_dense)
+          bstate[e] = make_uint4(ctlp->epoch, 2u, (u32)excl, (u32)(excl >> 32));
+      }
     }
   }
   __device__ void total(Ctl* ctl, u64 t) const {
@@ -1053,21 +1061,22 @@ __global__ void __launch_bounds__(kThreads) k_leaf_place(Dev d, Batch b) {
   for (u32 i = gtid(); i < end; i += gstride()) {
     u32 e = 0, mode = 0;  // 1 arena, 2 dense
     u32 o0 = 0, len = 0, c = 0;
+    uint4 bs = make_uint4(0, 0, 0, 0);
     if (i < b.n) {
       // the fragment's own fields do not depend on its group: load them first
       e = d.sc.leaf_sort_keys0[i] & d.tab.mask;
       o0 = b.off[i];
       len = b.off[i + 1] - o0;
       c = tag_child(b.tags[(u64)(D - 1) * n + i]);
-      const u32 ce = d.tab.carry_epoch[e], de = d.tab.done_epoch[e];
-      if (ce == ep) mode = 1;
-      else if (dense_ok && de == ep) mode = 2;
+      bs = d.tab.bstate[e];
+      if (bs.x == ep) mode = bs.y;
+      if (mode == 2 && !dense_ok) mode = 0;
     }
     if (mode == 2) {
       // every child index is below n_children (checked at completion); a
       // repeated child leaves some other slot unfilled, which the length
       // scan reports
-      const u64 slot = d.tab.dbase[e] + c;
+      const u64 slot = (((u64)bs.w << 32) | bs.z) + c;
       if (slot < dcap) d.sc.dense[slot] = make_uint4(ep, len, kNone, o0);
     }
     u64 ppos = 0;
@@ -1502,6 +1511,25 @@ void collect_profile(alto_agg* h) {
   h->ev_pending.clear();
 }
 
+LookbackState lb_region(const LookbackState& lb, int k) {
+  LookbackState r = lb;
+  r.desc += (u64)k * lb.tiles;
+  return r;
+}
+
+template <class F>
+void launch_scan3(const LookbackState& lb, int num_sms, Ctl* ctl, const F& f0, const F& f1,
+                  const F& f2, u64 cap, int site, u64 spin, cudaStream_t s) {
+  u64 tiles = (cap + kScanTile - 1) / kScanTile;
+  if (tiles == 0) tiles = 1;
+  // the record scans run over completed groups (far fewer than fragments):
+  // a small persistent grid, so that hundreds of idle CTAs do not contend on
+  // the tile and exit counters
+  dim3 grid((unsigned)std::min<u64>(tiles, 32), 3);
+  k_scan3<F><<<grid, kScanThreads, 0, s>>>(f0, f1, f2, lb_region(lb, 0), lb_region(lb, 1),
+                                           lb_region(lb, 2), ctl, site, spin);
+}
+
 template <class F>
 void launch_scan(alto_agg* h, const F& f, u64 cap, int site, cudaStream_t s) {
   u64 tiles = (cap + kScanTile - 1) / kScanTile;
@@ -1667,6 +1695,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(d.tab.cur, u64, T);
   ALLOC(d.tab.acc_leaf, uint4, T);
   ALLOC(d.tab.dbase, u64, T);
+  ALLOC(d.tab.bstate, uint4, T);
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
   d.tab.max_probe = (int)std::min<u64>(T, 1u << 16);
@@ -1749,9 +1778,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   sc.ps_mask = PS - 1;
   sc.done_cap = (u32)done_cap;
   const u64 scan_tiles = std::max<u64>(std::max<u64>(dense_cap, done_cap), nmax) / kScanTile + 2;
-  ALLOC(h->lbs.flag, u32, scan_tiles);
-  ALLOC(h->lbs.agg, u64, scan_tiles);
-  ALLOC(h->lbs.inc, u64, scan_tiles);
+  ALLOC(h->lbs.desc, ulonglong2, 3 * scan_tiles);
   h->lbs.tiles = scan_tiles;
   ALLOC(d.out_rec, alto_record, std::max<int64_t>(cfg.out_records, 1));
   ALLOC(d.out_pay, int32_t, std::max<int64_t>(cfg.out_payload_elems, 1));
@@ -1775,7 +1802,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   cudaMemsetAsync(sc.pairset, 0, sizeof(u64) * PS, s);
   cudaMemsetAsync(h->leaf_sort.hist, 0, sizeof(u32) * 4 * 256, s);
   cudaMemsetAsync(h->leaf_sort.lookback, 0, sizeof(u64) * sort_tiles * 256, s);
-  cudaMemsetAsync(h->lbs.flag, 0, sizeof(u32) * scan_tiles, s);
+  cudaMemsetAsync(h->lbs.desc, 0, sizeof(ulonglong2) * 3 * scan_tiles, s);
   if (concat >= 0) cudaMemsetAsync(sc.dense, 0, sizeof(uint4) * std::max<u64>(dense_cap, 1), s);
   if (cudaGetLastError() != cudaSuccess) {
     free_all(h, s);
@@ -1905,12 +1932,12 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
     const u32 dcap = d.sc.done_cap;
     {
       CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0,
-                   d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask};
-      launch_scan(h, f0, dcap, site++, s);
+                   d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask, d.tab.bstate, d.ctl};
       CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
-      launch_scan(h, f1, dcap, site++, s);
       CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
-      launch_scan(h, f2, dcap, site++, s);
+      launch_scan3(h->lbs, h->num_sms, d.ctl, f0, f1, f2, dcap, site, spin, s);
+      h->launches += 1;
+      site += 3;
     }
     k_check<<<1, 1, 0, s>>>(d);
     h->launches += 1;
@@ -2148,6 +2175,7 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   d.tab.cur = cv.take<u64>(T);
   d.tab.acc_leaf = cv.take<uint4>(T);
   d.tab.dbase = cv.take<u64>(T);
+  d.tab.bstate = cv.take<uint4>(T);
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
   d.tab.max_probe = (int)T;
@@ -2222,9 +2250,7 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   sc.pairset = cv.take<u64>(st.PS);
   sc.ps_mask = st.PS - 1;
   sc.done_cap = (u32)dc;
-  st.lbs.flag = cv.take<u32>(st.scan_tiles);
-  st.lbs.agg = cv.take<u64>(st.scan_tiles);
-  st.lbs.inc = cv.take<u64>(st.scan_tiles);
+  st.lbs.desc = cv.take<ulonglong2>(3 * st.scan_tiles);
   st.lbs.tiles = st.scan_tiles;
 }
 
@@ -2397,18 +2423,11 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
     k_done_rank<<<sgrid, kThreads, 0, s>>>(d);
     const u32 dcap = d.sc.done_cap;
     CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0,
-                 d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask};
-    k_scan<CountScan><<<scan_grid(dcap), kScanThreads, 0, s>>>(f0, st.lbs, d.ctl, site,
-                                                             &d.ctl->exit_ctr[site], spin);
-    ++site;
+                 d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask, d.tab.bstate, d.ctl};
     CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
-    k_scan<CountScan><<<scan_grid(dcap), kScanThreads, 0, s>>>(f1, st.lbs, d.ctl, site,
-                                                             &d.ctl->exit_ctr[site], spin);
-    ++site;
     CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
-    k_scan<CountScan><<<scan_grid(dcap), kScanThreads, 0, s>>>(f2, st.lbs, d.ctl, site,
-                                                             &d.ctl->exit_ctr[site], spin);
-    ++site;
+    launch_scan3(st.lbs, num_sms, d.ctl, f0, f1, f2, dcap, site, spin, s);
+    site += 3;
     k_check<<<1, 1, 0, s>>>(d);
     if (d.cfg.concat_level >= 0) {
       if (leaf_sorted) {

@@ -156,6 +156,8 @@ struct Table {
   uint4* acc_leaf; // [T] leaf level, one sector per group: {leaves << 40 | payload
                    //     elements (as u64 in .x/.y), max child + 1, max seq + 1}
   u64* dbase;      // [T] first dense child slot of a group completing this batch
+  uint4* bstate;   // [T] where this batch's leaves go, one load per fragment:
+                   //     {epoch, mode (1 arena, 2 dense), dense base lo, hi}
   int chain_len;   // D - 1
   u32 mask;        // T - 1
   int kk;          // stride of topk (largest k over levels)

@@ -22,14 +22,14 @@ constexpr int kScanItems = 8;
 constexpr int kScanWarps = kScanThreads / 32;
 constexpr int kScanTile = kScanThreads * kScanItems;
 
-// A tile's aggregate and its inclusive prefix live in separate arrays: a
-// reader that saw the "aggregate" flag must never pick up the inclusive value
-// written later into the same place.
+// One 16-byte descriptor per tile, {value, epoch_site << 2 | kind} with kind
+// 1 = the tile's own sum, 2 = the sum of tiles 0..t.  It is written and read
+// with single 16-byte vector accesses, so a reader sees the old or the new
+// descriptor whole -- never a value with the other kind's flag -- and no
+// fence is needed between value and flag.
 struct LookbackState {
-  u32* flag;  // [tiles] epoch_site << 2 | kind (1 aggregate, 2 inclusive)
-  u64* agg;   // [tiles] the tile's own sum
-  u64* inc;   // [tiles] sum of tiles 0..t
-  u64 tiles;  // capacity
+  ulonglong2* desc;  // [tiles]
+  u64 tiles;         // capacity
 };
 
 __device__ __forceinline__ u32 epoch_site(const Ctl* ctl, int site) {
@@ -52,15 +52,23 @@ __device__ __forceinline__ void finish_ctas(Ctl* ctl, int site, u32* exit_ctr) {
 }
 
 __device__ __forceinline__ void lb_publish(LookbackState st, u32 tile, u32 es, u32 kind, u64 v) {
-  volatile u64* vp = (kind == 2u ? st.inc : st.agg) + tile;
-  volatile u32* fp = st.flag + tile;
-  *vp = v;
-  __threadfence();
-  *fp = (es << 2) | kind;
+  const u64 f = (u64)((es << 2) | kind);
+  asm volatile("st.volatile.global.v2.u64 [%0], {%1, %2};" ::"l"(st.desc + tile), "l"(v), "l"(f)
+               : "memory");
 }
 
-// Sum of everything before `tile`, found by warp 0: each lane reads one
-// predecessor of a 32-tile window; the nearest inclusive prefix ends the walk.
+__device__ __forceinline__ ulonglong2 lb_read(LookbackState st, long long tile) {
+  ulonglong2 r;
+  asm volatile("ld.volatile.global.v2.u64 {%0, %1}, [%2];"
+               : "=l"(r.x), "=l"(r.y)
+               : "l"(st.desc + tile)
+               : "memory");
+  return r;
+}
+
+// Sum of everything before `tile`, found by warp 0: each lane reads four
+// predecessors of a 128-tile window (lane l takes tiles top-l, top-l-32, ...);
+// the nearest inclusive prefix ends the walk.
 __device__ __forceinline__ u64 lb_walk_warp(LookbackState st, u32 tile, u32 es, Ctl* ctl,
                                             u64 spin_limit) {
   const int lane = threadIdx.x & 31;
@@ -68,42 +76,70 @@ __device__ __forceinline__ u64 lb_walk_warp(LookbackState st, u32 tile, u32 es, 
   long long top = (long long)tile - 1;
   u64 spins = 0;
   while (top >= 0) {
-    const long long p = top - lane;
-    u32 f = 0;
+    ulonglong2 dsc[4];
     bool ready = true;
-    if (p >= 0) {
-      f = *((volatile u32*)st.flag + p);
-      ready = ((f >> 2) == es) && ((f & 3u) != 0);
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const long long p = top - lane - 32 * r;
+      dsc[r] = make_ulonglong2(0, 0);
+      if (p >= 0) {
+        dsc[r] = lb_read(st, p);
+        const u32 f = (u32)dsc[r].y;
+        ready = ready && ((f >> 2) == es) && ((f & 3u) != 0);
+      }
     }
     if (!__all_sync(0xFFFFFFFFu, ready)) {
       if (++spins > spin_limit || *(volatile int*)&ctl->abort) {
         if (lane == 0) raise_timeout(ctl);
         break;
       }
+      // back off: every waiting warp polls the same few lines of descriptors
+      __nanosleep(64);
       continue;
     }
-    __threadfence();
-    const bool inc = (p < 0) || ((f & 3u) == 2u);
-    const u32 inc_mask = __ballot_sync(0xFFFFFFFFu, inc);
-    const int stop = inc_mask ? __ffs(inc_mask) - 1 : 32;  // nearest inclusive predecessor
+    // nearest inclusive predecessor: smallest distance d = lane + 32 r
+    int stop = 128;
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const long long p = top - lane - 32 * r;
+      const bool inc = (p < 0) || (((u32)dsc[r].y & 3u) == 2u);
+      const u32 m = __ballot_sync(0xFFFFFFFFu, inc);
+      if (m && stop == 128) stop = 32 * r + __ffs(m) - 1;
+    }
     u64 v = 0;
-    if (p >= 0 && lane <= stop) v = *((volatile u64*)((lane == stop) ? st.inc : st.agg) + p);
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const int dist = lane + 32 * r;
+      const long long p = top - dist;
+      if (p >= 0 && dist <= stop) v += dsc[r].x;
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
     excl += v;
-    if (inc_mask) break;
-    top -= 32;
+    if (stop < 128) break;
+    top -= 128;
   }
   return excl;
 }
 
-// Tile = kScanItems rows of kScanThreads consecutive elements; thread t owns
-// column t, so every value()/out() call is coalesced across the warp.
+// A tile's values are read in striped order (coalesced) into shared memory;
+// each thread then owns kScanItems consecutive elements: a serial sum, one
+// warp scan of the thread sums, one pass over the warp sums.  The thread
+// writes its elements' tile-local exclusive prefixes back into shared memory
+// so that the out() calls run in striped order too (coalesced stores).
+// Element values fit in 32 bits (counts, lengths, flags); prefixes are
+// 64-bit, tile-local prefixes 32-bit (a tile whose sum does not fit takes the
+// blocked order instead).  Shared memory is padded by one word per 32 so that
+// both access orders are free of bank conflicts.  The next tile's id is
+// taken while the current one is processed.
+__device__ __forceinline__ u32 scan_pad(u32 p) { return p + (p >> 5); }
+
 template <class F>
-__global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ctl* ctl, int site,
-                                                       u32* exit_ctr, u64 spin_limit) {
-  __shared__ u32 s_tile;
-  __shared__ u64 s_w[kScanItems][kScanWarps];
+__device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl, int site,
+                                          u32* exit_ctr, u64 spin_limit) {
+  __shared__ u32 s_next;
+  __shared__ u32 s_v[kScanTile + kScanTile / 32];
+  __shared__ u64 s_w[kScanWarps];
   __shared__ u64 s_excl;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const u64 n = halted(ctl) ? 0 : f.size(ctl);
@@ -111,48 +147,52 @@ __global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ct
   if (ntiles == 0) ntiles = 1;
   if (ntiles > st.tiles) ntiles = st.tiles;
   const u32 es = epoch_site(ctl, site);
+  if (t == 0) s_next = take_tile(ctl, site);
+  __syncthreads();
   for (;;) {
-    if (t == 0) s_tile = take_tile(ctl, site);
+    const u32 tile = s_next;
     __syncthreads();
-    const u32 tile = s_tile;
     if (tile >= ntiles) break;
+    if (t == 0) s_next = take_tile(ctl, site);  // read after the barriers below
     const u64 base = (u64)tile * kScanTile;
-    u64 v[kScanItems], x[kScanItems];
 #pragma unroll
     for (int k = 0; k < kScanItems; ++k) {
-      const u64 i = base + (u64)k * kScanThreads + t;
-      v[k] = (i < n) ? f.value(i) : 0;
-      x[k] = v[k];
+      const u32 p = (u32)(k * kScanThreads + t);
+      const u64 i = base + p;
+      s_v[scan_pad(p)] = (i < n) ? (u32)f.value(i) : 0u;
     }
+    __syncthreads();
+    u32 w[kScanItems];
+    u64 sum = 0;
+#pragma unroll
+    for (int k = 0; k < kScanItems; ++k) {
+      w[k] = s_v[scan_pad((u32)(t * kScanItems + k))];
+      sum += w[k];
+    }
+    u64 x = sum;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
+      const u64 y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) s_w[warp] = x;
+    __syncthreads();
+    u64 wpre = 0, agg = 0;
+#pragma unroll
+    for (int q = 0; q < kScanWarps; ++q) {
+      const u64 c = s_w[q];
+      if (q < warp) wpre += c;
+      agg += c;
+    }
+    const bool narrow = agg < (1ull << 32);
+    u64 rel = wpre + (x - sum);  // tile-local exclusive prefix of this thread's first element
+    if (narrow) {
 #pragma unroll
       for (int k = 0; k < kScanItems; ++k) {
-        const u64 y = __shfl_up_sync(0xFFFFFFFFu, x[k], o);
-        if (lane >= o) x[k] += y;
+        s_v[scan_pad((u32)(t * kScanItems + k))] = (u32)rel;
+        rel += w[k];
       }
     }
-    if (lane == 31) {
-#pragma unroll
-      for (int k = 0; k < kScanItems; ++k) s_w[k][warp] = x[k];
-    }
-    __syncthreads();
-    // row totals and this warp's offset inside each row
-    u64 row_pre = 0, agg = 0;
-    u64 off[kScanItems];
-#pragma unroll
-    for (int k = 0; k < kScanItems; ++k) {
-      u64 rt = 0, wp = 0;
-#pragma unroll
-      for (int w = 0; w < kScanWarps; ++w) {
-        const u64 c = s_w[k][w];
-        if (w < warp) wp += c;
-        rt += c;
-      }
-      off[k] = row_pre + wp;
-      row_pre += rt;
-    }
-    agg = row_pre;
     if (warp == 0) {
       u64 excl = 0;
       if (tile == 0) {
@@ -169,14 +209,45 @@ __global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ct
     }
     __syncthreads();
     const u64 ex0 = s_excl;
+    if (narrow) {
 #pragma unroll
-    for (int k = 0; k < kScanItems; ++k) {
-      const u64 i = base + (u64)k * kScanThreads + t;
-      if (i < n) f.out(i, ex0 + off[k] + x[k] - v[k], v[k]);
+      for (int k = 0; k < kScanItems; ++k) {
+        const u32 p = (u32)(k * kScanThreads + t);
+        const u64 i = base + p;
+        const u32 r0 = s_v[scan_pad(p)];
+        const u32 r1 = (p + 1 < (u32)kScanTile) ? s_v[scan_pad(p + 1)] : (u32)agg;
+        if (i < n) f.out(i, ex0 + r0, (u64)(r1 - r0));
+      }
+    } else {
+      u64 run = ex0 + wpre + (x - sum);
+      const u64 first = base + (u64)t * kScanItems;
+#pragma unroll
+      for (int k = 0; k < kScanItems; ++k) {
+        if (first + k < n) f.out(first + k, run, w[k]);
+        run += w[k];
+      }
     }
     __syncthreads();
   }
   if (t == 0) finish_ctas(ctl, site, exit_ctr);
+}
+
+template <class F>
+__global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ctl* ctl, int site,
+                                                       u32* exit_ctr, u64 spin_limit) {
+  scan_body(f, st, ctl, site, exit_ctr, spin_limit);
+}
+
+// Three independent scans in one launch: blockIdx.y selects the scan, each
+// with its own launch site (tile and exit counters) and look-back arrays.
+template <class F>
+__global__ void __launch_bounds__(kScanThreads) k_scan3(F f0, F f1, F f2, LookbackState st0,
+                                                        LookbackState st1, LookbackState st2,
+                                                        Ctl* ctl, int site, u64 spin_limit) {
+  const int y = blockIdx.y;
+  const F& f = (y == 0) ? f0 : (y == 1) ? f1 : f2;
+  const LookbackState st = (y == 0) ? st0 : (y == 1) ? st1 : st2;
+  scan_body(f, st, ctl, site + y, &ctl->exit_ctr[site + y], spin_limit);
 }
 
 }  // namespace alto
