@@ -17,6 +17,9 @@
 //               completing groups: place every child span at slot
 //               dense_base + child_index, scan the lengths, gather the spans
 //               into the output payload ring                     [Sec. 3.2, 3.3]
+//               With the CONCAT level M above the leaf parent, a group of a
+//               level between completes into one span of its parent's vectors
+//               (gathered level by level, bottom-up) before level M gathers.
 //   records     one record per completed group, top-k pairs; free entries
 #include <cuda_runtime.h>
 
@@ -74,6 +77,8 @@ struct Scratch {
   u64* r_dense_base;
   u64* r_topk_off;
   u64* r_arena_base;
+  u64* c_dense_base;     // [done_cap + 1] by done index: dense slots of levels M < l
+  u64* c_arena_base;     // [done_cap + 1] by done index: their buffered spans
   uint4* dense;          // [dense_cap] {stamp, len, owner entry or kNone, position}
   u64* dst;              // [dense_cap + 1]
   u64* lenscan;          // [n_max + 1]
@@ -222,6 +227,69 @@ __device__ void free_chunk(const Arena& ar, Ctl* ctl, int j, u32 chunk) {
 }
 
 // ---------------------------------------------------------------------------
+// CONCAT at a level M above the leaf parent.  A group of a level l with
+// M < l <= D-1 that completes becomes one child span of its parent: its
+// concatenation is reserved at the end of the parent's vectors (one 64-bit
+// atomic on the parent's cursor: span index and payload position together)
+// and copied there later in the batch, so that a group of level M finds all
+// its children's concatenations, in any order, in its own vectors.
+// ---------------------------------------------------------------------------
+constexpr u64 kPos40 = (1ull << 40) - 1;
+
+// levels whose completed groups hand a span to their parent
+__device__ __forceinline__ bool chain_level(const Cfg& c, int l) {
+  return c.concat_level >= 0 && l > c.concat_level;
+}
+// levels whose groups receive their children's spans (the leaf parent buffers leaves instead)
+__device__ __forceinline__ bool chain_parent(const Cfg& c, int l) {
+  return c.concat_level >= 0 && l >= c.concat_level && l < c.depth - 1;
+}
+
+// Chunks of every class that starts in [old_el, new_el) of entry e's vector vec.
+__device__ void grow_vec(const Table& tab, const Arena& ar, Ctl* ctl, u32 e, int vec, u64 old_el,
+                         u64 new_el) {
+  if (new_el <= old_el) return;
+  const int jf = (old_el == 0) ? 0 : chunk_of(old_el - 1) + 1;
+  const int jl = chunk_of(new_el - 1);
+  if (jl >= kNumChunks) raise_err(ctl, ALTO_ENOSPC);
+  u64 got = 0;
+  for (int j = jf; j <= jl && j < kNumChunks; ++j) {
+    const u32 c = alloc_chunk(ar, ctl, j);
+    tab.dir[((u64)e * kVecs + vec) * kNumChunks + j] = c;
+    if (c != kNone) got += chunk_size(j);
+  }
+  if (got) atomicAdd((unsigned long long*)&ctl->arena_used, (unsigned long long)got);
+}
+
+// A receiving group takes the spans its children reserved in earlier launches
+// of this batch: chunks for the growth, then the new sizes.
+__device__ void chain_sync(const Table& tab, const Arena& ar, Ctl* ctl, u32 e) {
+  const u64 cu = tab.cur[e];
+  const u64 n0 = cu >> 40, n1 = cu & kPos40;
+  const u32 o0 = tab.vec_n[2 * (u64)e], o1 = tab.vec_n[2 * (u64)e + 1];
+  if (n0 == o0 && n1 == o1) return;
+  // the 24-bit span count and the 32-bit sizes must not wrap
+  if (n0 >= (1ull << 23) || n1 >= (1ull << 32)) {
+    raise_err(ctl, ALTO_ENOSPC);
+    return;
+  }
+  grow_vec(tab, ar, ctl, e, 0, 2 * (u64)o0, 2 * n0);
+  grow_vec(tab, ar, ctl, e, 1, o1, n1);
+  tab.vec_n[2 * (u64)e] = (u32)n0;
+  tab.vec_n[2 * (u64)e + 1] = (u32)n1;
+}
+
+// Completed group e (child c of parent entry P) reserves its `total` elements.
+// A cursor is zeroed when its entry is freed, so a parent inserted in the same
+// launch can take reservations at once.
+__device__ __forceinline__ void chain_reserve(const Table& tab, u32 e, u32 P, u32 c, u64 total) {
+  const u64 old = atomicAdd((unsigned long long*)&tab.cur[P], (unsigned long long)((1ull << 40) | total));
+  tab.par[e] = P;
+  tab.cidx[e] = c;
+  tab.app[e] = old;
+}
+
+// ---------------------------------------------------------------------------
 // kernels
 // ---------------------------------------------------------------------------
 __global__ void k_begin(Ctl* ctl, u32 n) {
@@ -324,7 +392,9 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
   const u32 gw = gtid() >> 5, nw = gstride() >> 5;
   const bool topk = d.cfg.score_op[l] == ALTO_SCORE_TOPK;
   const int K = d.cfg.topk_k[l];
-  const bool carry = LEAF && d.cfg.concat_level == D - 1;
+  const bool carry = LEAF && d.cfg.concat_level >= 0;
+  const bool receives = !LEAF && chain_parent(d.cfg, l);
+  const bool hands_up = chain_level(d.cfg, l);
   const u32 ep = ctl->epoch;
   const u32* it_rep = d.sc.it_rep[in_set];
   const u32* it_cseq = d.sc.it_cseq[in_set];
@@ -447,6 +517,7 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
     }
 
     if (lane == 0) {
+      if (receives) chain_sync(d.tab, d.ar, ctl, e);
       if (bad) raise_err(ctl, ALTO_EINCONSIST);
       if (l > 0 && d.tab.up[e] != b.tags[(u64)(l - 1) * n + rep0]) raise_err(ctl, ALTO_EINCONSIST);
       const u32 last_old = d.tab.last[e];
@@ -487,6 +558,16 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
           d.tab.vec_n[2 * (u64)e] = v0 + (j1 - j0);
           d.tab.vec_n[2 * (u64)e + 1] = v1 + (u32)lsum;
         }
+      }
+      if (hands_up && complete) {
+        const u64 tp = b.tags[(u64)(l - 1) * n + rep0];
+        const u64 upp = (l > 1) ? b.tags[(u64)(l - 2) * n + rep0] : 0ull;
+        int ins = 0;
+        const u32 P = ht_find_or_insert(d.tab, ((u64)(l - 1) << 32) | tag_pid(tp), upp, ctl, &ins,
+                                        b.tags, n, rep0, l - 1);
+        if (ins) atomicAdd((unsigned long long*)&ctl->live_groups, 1ull);
+        const u64 total = (u64)d.tab.vec_n[2 * (u64)e + 1] + (LEAF ? lsum : 0ull);
+        chain_reserve(d.tab, e, P, tag_child(tp), total);
       }
       if (l > 0) {
         nx_rep[s] = rep0;
@@ -660,7 +741,9 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const int D = d.cfg.depth;
-  const bool carry = LEAF && d.cfg.concat_level == D - 1;
+  const bool carry = LEAF && d.cfg.concat_level >= 0;
+  const bool receives = !LEAF && chain_parent(d.cfg, l);
+  const bool hands_up = chain_level(d.cfg, l);
   const u32 nt = min(ctl->n_segs[l], d.cfg.n_max);
   const u32 ep = ctl->epoch;
   const u32 ep7 = epoch7(ctl);
@@ -674,6 +757,7 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
   const u64 n = b.n;
   for (u32 s = gtid(); s < nt; s += gstride()) {
     const u32 e = list[s] & d.tab.mask;
+    if (receives) chain_sync(d.tab, d.ar, ctl, e);
     u32 cnt, m1, cs1;
     u32 blen = 0;
     if (LEAF) {
@@ -752,6 +836,8 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
       if (ins) atomicAdd(&s_ins, 1u);
       d.sc.up_sort_keys0[s] = e2;
       if (ps_insert(d.sc, e2, tag_child(tp), ep7, ctl)) raise_err(ctl, ALTO_EINCONSIST);
+      if (hands_up && complete)
+        chain_reserve(d.tab, e, e2, tag_child(tp), (u64)d.tab.vec_n[2 * (u64)e + 1] + blen);
     }
   }
   __syncthreads();
@@ -831,12 +917,66 @@ struct CountScan {
   }
 };
 
+// Levels M < l: dense slots (which 0) and buffered spans (which 1) of the
+// groups completing in this batch, over the done list; which 2 is empty.
+// Their dense region follows level M's.  The slot scan also leaves each such
+// group's first slot in its entry (and, for a leaf parent, where this batch's
+// leaves go) and writes the group's meta entry {child index, payload
+// position} into its parent's vectors, whose chunks the parent's finalize
+// allocated.
+struct ChainScan {
+  const u32* done_e;
+  const u32* done_lvl;
+  const u32* n_dev;
+  u32 cap;
+  int which;
+  u64* out_off;
+  Table tab;
+  int32_t* arena_pool;
+  Ctl* ctlp;
+  int M, L;
+  __device__ u64 size(const Ctl*) const { return (which == 2) ? 0 : min(*n_dev, cap); }
+  __device__ u64 value(u64 i) const {
+    if ((int)done_lvl[i] <= M) return 0;
+    const u32 e = done_e[i] & tab.mask;
+    return (which == 0) ? (u64)tab.last[e] + 1 : (u64)tab.vec_n[2 * (u64)e];
+  }
+  __device__ void out(u64 i, u64 excl, u64 v) const {
+    if (which == 2) return;
+    const u64 off = (which == 0) ? ctlp->dense_total : 0;
+    out_off[i] = off + excl;
+    if (which != 0 || v == 0) return;
+    const u32 e = done_e[i] & tab.mask;
+    const u64 base = off + excl;
+    tab.dbase[e] = base;
+    if ((int)done_lvl[i] == L)
+      tab.bstate[e] = make_uint4(ctlp->epoch, 2u, (u32)base, (u32)(base >> 32));
+    if (*(const volatile int*)&ctlp->batch_err) return;  // a parent entry may be unusable
+    const u32 P = tab.par[e] & tab.mask;
+    const u64 ap = tab.app[e];
+    const u64 m = ap >> 40;
+    if (m >= tab.vec_n[2 * (u64)P]) return;
+    bool ok;
+    const u64 a = vec_addr(tab, P, 0, 2 * m, &ok);
+    if (!ok) return;
+    arena_pool[a] = (int32_t)tab.cidx[e];
+    arena_pool[a + 1] = (int32_t)(u32)(ap & kPos40);
+  }
+  __device__ void total(Ctl* ctl, u64 t) const {
+    if (which == 2) return;
+    const u64 off = (which == 0) ? ctl->dense_total : 0;
+    out_off[size(ctl)] = off + t;
+    if (which == 0) ctl->chain_total = t;
+    else ctl->chain_arena = t;
+  }
+};
+
 __global__ void k_check(Dev d) {
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   bool bad = false;
   if (ctl->rec_count + ctl->n_done > d.cfg.out_records) bad = true;
-  if (ctl->dense_total > d.cfg.dense_cap) bad = true;
+  if (ctl->dense_total + ctl->chain_total > d.cfg.dense_cap) bad = true;
   if (ctl->topk_count + ctl->topk_total > d.cfg.out_topk) bad = true;
   if (ctl->n_done > d.sc.done_cap) bad = true;
   if (bad) {
@@ -1028,11 +1168,9 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
     if (i >= b.n || d.tab.done_epoch[e] != ep) continue;
     const u32 di = d.tab.done_idx[e];
     if (di >= nd) continue;
-    const u32 r = d.sc.done_rank[di];
-    if (r >= nd) continue;
     const u32 c = tag_child(b.tags[(u64)(D - 1) * n + i]);
-    if (c >= d.sc.r_dense_n[r]) continue;
-    const u64 slot = d.sc.r_dense_base[r] + c;
+    if (c > d.tab.last[e]) continue;
+    const u64 slot = d.tab.dbase[e] + c;  // the group's first slot, from the count scan
     if (slot >= d.cfg.dense_cap) continue;
     const u32 old = atomicExch(&d.sc.dense[slot].x, ep);
     if (old == ep) raise_err(ctl, ALTO_EDUP);
@@ -1124,27 +1262,32 @@ __global__ void __launch_bounds__(kThreads) k_leaf_place(Dev d, Batch b) {
   }
 }
 
-// Dense child slots from the arena (leaves buffered by earlier batches).
+// Dense child slots from the arena: spans buffered by earlier batches (and,
+// above the leaf parent, handed up earlier in this batch).  LEVEL_M: the
+// groups of level M, by emission rank; otherwise the groups of levels M < l,
+// by done index.
+template <bool LEVEL_M>
 __global__ void __launch_bounds__(kThreads) k_dense_arena(Dev d) {
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
   const u32 ep = ctl->epoch;
   const u32 nd = min(ctl->n_done, d.sc.done_cap);
-  const u64 na = ctl->arena_total;
+  const u64 na = LEVEL_M ? ctl->arena_total : ctl->chain_arena;
+  const u64* abase = LEVEL_M ? d.sc.r_arena_base : d.sc.c_arena_base;
   for (u64 a = gtid(); a < na; a += gstride()) {
-    // last rank r with r_arena_base[r] <= a
+    // last index x with abase[x] <= a: the one whose spans contain a
     u32 lo = 0, hi = nd;
     while (hi - lo > 1) {
       u32 mid = (lo + hi) >> 1;
-      if (d.sc.r_arena_base[mid] <= a) lo = mid;
+      if (abase[mid] <= a) lo = mid;
       else hi = mid;
     }
-    const u32 r = lo;
-    const u32 di = d.sc.r_done[r];
+    const u32 di = LEVEL_M ? d.sc.r_done[lo] : lo;
     if (di >= nd) continue;
-    const u32 e = d.sc.done_e[di];
-    const u64 k = a - d.sc.r_arena_base[r];
-    const u32 mn = d.sc.r_meta_n[r];
+    if (!LEVEL_M && (int)d.sc.done_lvl[di] <= d.cfg.concat_level) continue;
+    const u32 e = d.sc.done_e[di] & d.tab.mask;
+    const u64 k = a - abase[lo];
+    const u32 mn = LEVEL_M ? d.sc.r_meta_n[lo] : d.tab.vec_n[2 * (u64)e];
     if (k >= mn) continue;
     bool ok1, ok2 = true;
     u64 ma = vec_addr(d.tab, e, 0, 2 * k, &ok1);
@@ -1158,11 +1301,11 @@ __global__ void __launch_bounds__(kThreads) k_dense_arena(Dev d) {
     } else {
       end = d.tab.vec_n[2 * (u64)e + 1];
     }
-    if (c >= d.sc.r_dense_n[r] || end < pos) {
+    if (c > d.tab.last[e] || end < pos) {
       raise_err(ctl, ALTO_EDUP);
       continue;
     }
-    const u64 slot = d.sc.r_dense_base[r] + c;
+    const u64 slot = d.tab.dbase[e] + c;
     if (slot >= d.cfg.dense_cap) continue;
     u32 old = atomicExch(&d.sc.dense[slot].x, ep);
     if (old == ep) raise_err(ctl, ALTO_EDUP);
@@ -1179,7 +1322,7 @@ struct DenseScan {
   u64* dst;
   Ctl* ctlp;
   __device__ u64 size(const Ctl* ctl) const {
-    return (ctl->skip_dense || ctl->batch_err) ? 0 : ctl->dense_total;
+    return (ctl->skip_dense || ctl->batch_err) ? 0 : ctl->dense_total + ctl->chain_total;
   }
   __device__ u64 value(u64 j) const {
     uint4 v = dense[j];
@@ -1199,6 +1342,8 @@ struct DenseScan {
 __global__ void k_check2(Dev d) {
   Ctl* ctl = d.ctl;
   if (poisoned(ctl) || ctl->skip_dense) return;
+  // level M's spans come first; the slots after them are handed up, not emitted
+  if (ctl->chain_total && !ctl->batch_err) ctl->pay_total = d.sc.dst[ctl->dense_total];
   if (ctl->pay_count + ctl->pay_total > d.cfg.out_payload) {
     raise_err(ctl, ALTO_ENOSPC);
     ctl->skip_dense = 1;
@@ -1281,6 +1426,85 @@ __global__ void __launch_bounds__(kThreads) k_gather(Dev d, Batch b) {
   }
 }
 
+// Level l (M < l): the concatenations of its groups completing in this batch,
+// copied into the spans they reserved in their parents' payload vectors.  The
+// done list holds levels in non-increasing order (levels finalise bottom-up),
+// so the level's groups, and their dense slots, form one range.  A warp takes
+// 32 consecutive slots; each lane finds its slot's group by binary search,
+// then the warp copies the spans one after another.
+__global__ void __launch_bounds__(kThreads) k_chain_gather(Dev d, Batch b, int l) {
+  Ctl* ctl = d.ctl;
+  if (no_copy(ctl) || ctl->skip_dense) return;
+  const u32 ep = ctl->epoch;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  const u32* lvl = d.sc.done_lvl;
+  // [x0, x1): done indices of level l
+  u32 x0 = 0, x1 = nd;
+  {
+    u32 lo = 0, hi = nd;  // first index with level <= l
+    while (lo < hi) {
+      const u32 mid = (lo + hi) >> 1;
+      if ((int)lvl[mid] > l) lo = mid + 1;
+      else hi = mid;
+    }
+    x0 = lo;
+    hi = nd;  // first index with level < l
+    while (lo < hi) {
+      const u32 mid = (lo + hi) >> 1;
+      if ((int)lvl[mid] >= l) lo = mid + 1;
+      else hi = mid;
+    }
+    x1 = lo;
+  }
+  if (x0 >= x1) return;
+  const u64 j0 = d.sc.c_dense_base[x0], j1 = d.sc.c_dense_base[x1];
+  const int lane = threadIdx.x & 31;
+  const u64 gw = gtid() >> 5, nw = gstride() >> 5;
+  for (u64 jb = j0 + gw * 32; jb < j1; jb += nw * 32) {
+    const u64 j = jb + lane;
+    u32 len = 0, owner = kNone, pos = 0, P = 0;
+    u64 dp = 0;
+    if (j < j1 && j < d.cfg.dense_cap) {
+      u32 lo = x0, hi = x1;  // last index with slot base <= j
+      while (hi - lo > 1) {
+        const u32 mid = (lo + hi) >> 1;
+        if (d.sc.c_dense_base[mid] <= j) lo = mid;
+        else hi = mid;
+      }
+      const u32 e = d.sc.done_e[lo] & d.tab.mask;
+      const uint4 v = d.sc.dense[j];
+      const u32 par = d.tab.par[e] & d.tab.mask;
+      const u64 to = (d.tab.app[e] & kPos40) + (d.sc.dst[j] - d.sc.dst[d.sc.c_dense_base[lo]]);
+      bool good = v.x == ep && to + v.y <= d.tab.vec_n[2 * (u64)par + 1];
+      if (good && v.z == kNone) good = (u64)v.w + v.y <= b.n_payload;
+      if (good && v.z != kNone)
+        good = v.z <= d.tab.mask && (u64)v.w + v.y <= d.tab.vec_n[2 * (u64)v.z + 1];
+      if (good) {
+        len = v.y;
+        owner = v.z;
+        pos = v.w;
+        P = par;
+        dp = to;
+      }
+    }
+    const u32 cnt = (j1 - jb < 32) ? (u32)(j1 - jb) : 32u;
+    for (u32 k = 0; k < cnt; ++k) {
+      const u32 Lk = __shfl_sync(0xFFFFFFFFu, len, k);
+      if (Lk == 0) continue;
+      const u32 ow = __shfl_sync(0xFFFFFFFFu, owner, k);
+      const u32 ps = __shfl_sync(0xFFFFFFFFu, pos, k);
+      const u32 Pk = __shfl_sync(0xFFFFFFFFu, P, k);
+      const u64 dk = __shfl_sync(0xFFFFFFFFu, dp, k);
+      for (u32 q = lane; q < Lk; q += 32) {
+        const int32_t val = span_load(d, b, ow, ps, q);
+        bool ok;
+        const u64 a = vec_addr(d.tab, Pk, 1, dk + q, &ok);
+        if (ok) d.ar.pool[a] = val;
+      }
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
@@ -1344,7 +1568,7 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
           d.out_topk[to + q] = p;
         }
       }
-      if (l == M) {
+      if (M >= 0 && l >= M) {
         for (int vec = 0; vec < kVecs; ++vec) {
           el[vec] = (u64)d.tab.vec_n[2 * (u64)e + vec] * (vec == 0 ? 2 : 1);
           if (el[vec] == 0) continue;
@@ -1353,6 +1577,7 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
         }
       }
       d.tab.key[e] = kTomb;
+      d.tab.cur[e] = 0;  // a slot taken later may receive spans in the launch that inserts it
       atomicAdd(&s_del, 1u);
     }
     __syncthreads();
@@ -1363,7 +1588,7 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
       atomicAdd(&s_freed, (unsigned long long)s_cnt[j] * chunk_size(j));
     }
     __syncthreads();
-    if (mine && l == M) {
+    if (mine && M >= 0 && l >= M) {
       for (int vec = 0; vec < kVecs; ++vec) {
         if (el[vec] == 0) continue;
         const int jl = min(chunk_of(el[vec] - 1), kNumChunks - 1);
@@ -1531,13 +1756,183 @@ void launch_scan3(const LookbackState& lb, int num_sms, Ctl* ctl, const F& f0, c
 }
 
 template <class F>
-void launch_scan(alto_agg* h, const F& f, u64 cap, int site, cudaStream_t s) {
+void launch_scan(const LookbackState& lb, int num_sms, Ctl* ctl, const F& f, u64 cap, int site,
+                 u64 spin, cudaStream_t s) {
   u64 tiles = (cap + kScanTile - 1) / kScanTile;
   if (tiles == 0) tiles = 1;
-  int grid = (int)std::min<u64>(tiles, (u64)h->num_sms * 4);
-  h->launches += 1;
-  k_scan<F><<<grid, kScanThreads, 0, s>>>(f, h->lbs, h->d.ctl, site, &h->d.ctl->exit_ctr[site],
-                                          h->d.cfg.spin_limit);
+  int grid = (int)std::min<u64>(tiles, (u64)num_sms * 4);
+  k_scan<F><<<grid, kScanThreads, 0, s>>>(f, lb, ctl, site, &ctl->exit_ctr[site], spin);
+}
+
+// What one batch enqueues between k_begin and k_end, for the handle's push
+// and for the one-shot entry point alike.  `stage` (may be null) marks the
+// start of each profiling stage; `launches` counts the kernels.
+struct Pipeline {
+  Dev d;
+  SortBuffers* leaf_sort;
+  SortBuffers* up_sort;
+  LookbackState lbs;
+  int num_sms;
+  int tbits;
+  u32 nmax;
+  cudaStream_t s;
+  void (*stage)(void* ctx, int st, int64_t launches) = nullptr;
+  void* stage_ctx = nullptr;
+  int64_t launches = 0;
+  void enter(int st) {
+    if (stage) stage(stage_ctx, st, launches);
+  }
+};
+
+void enqueue_batch(Pipeline& p, const Batch& bt) {
+  Dev d = p.d;
+  cudaStream_t s = p.s;
+  const int D = d.cfg.depth;
+  const int M = d.cfg.concat_level;
+  const u32 nmax = p.nmax;
+  const int grid = p.num_sms * 8;   // kernels over fragments or leaves
+  const int sgrid = p.num_sms * 2;  // kernels over groups (fewer items)
+  const u64 spin = d.cfg.spin_limit;
+  int sl = 0;  // launches inside sort_pairs
+  int site = 0;
+  k_ingest<<<grid, kThreads, 0, s>>>(d, bt);
+  p.launches += 1;
+  const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK;
+  int set = 0;
+  if (leaf_sorted) {
+    // leaf level with TOPK: sort fragments by their leaf-parent group so that
+    // each group's candidates are contiguous for the segmented top-k
+    p.enter(1);
+    int cur = sort_pairs(&d.ctl->n, nmax, p.tbits, true, *p.leaf_sort, d.ctl, site, spin, p.num_sms,
+                         s, &sl);
+    p.launches += sl;
+    sl = 0;
+    d.sc.leaf_keys = p.leaf_sort->keys[cur];
+    d.sc.leaf_perm = p.leaf_sort->vals[cur];
+    p.enter(2);
+    SegFind f{d.sc.leaf_keys, d.sc.leaf_seg_start, d.sc.leaf_seg_of, &d.ctl->n, nmax,
+              &d.ctl->n_segs[D - 1]};
+    launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site + 4, spin, s);
+    k_reduce<true><<<grid, kThreads, 0, s>>>(d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
+                                             d.sc.leaf_seg_start, set);
+    p.launches += 2;
+  } else {
+    // leaf level without TOPK: accumulate into the table in arrival order
+    p.enter(2);
+    k_leaf_accumulate<<<grid, kThreads, 0, s>>>(d, bt);
+    k_up_finalize<true><<<sgrid, kThreads, 0, s>>>(d, bt, D - 1, set);
+    p.launches += 2;
+  }
+  site += 5;
+  p.enter(3);
+  // an atomic finalize also looks up the parent groups of the items it emits
+  bool looked_up = !leaf_sorted;
+  for (int l = D - 2; l >= 0; --l) {
+    set ^= 1;  // items written by the level below
+    if (!looked_up) {
+      k_items_lookup<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+      p.launches += 1;
+    }
+    if (d.cfg.score_op[l] != ALTO_SCORE_TOPK) {
+      k_up_accumulate<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+      k_up_finalize<false><<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+      p.launches += 2;
+      looked_up = true;
+      continue;
+    }
+    looked_up = false;
+    int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nmax, p.tbits, true, *p.up_sort, d.ctl, site, spin,
+                        p.num_sms, s, &sl);
+    p.launches += sl;
+    sl = 0;
+    site += 4;
+    d.sc.up_keys = p.up_sort->keys[c2];
+    d.sc.up_perm = p.up_sort->vals[c2];
+    SegFind f{d.sc.up_keys, d.sc.up_seg_start, nullptr, &d.ctl->n_segs[l + 1], nmax,
+              &d.ctl->n_segs[l]};
+    launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site++, spin, s);
+    k_reduce<false><<<grid, kThreads, 0, s>>>(d, bt, l, d.sc.up_keys, d.sc.up_perm,
+                                              d.sc.up_seg_start, set);
+    p.launches += 2;
+  }
+  // emission order
+  p.enter(4);
+  {
+    RankScan f{d.sc.mask, d.sc.prefix, &d.ctl->n};
+    launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site++, spin, s);
+  }
+  k_done_rank<<<sgrid, kThreads, 0, s>>>(d);
+  p.launches += 2;
+  const u32 dcap = d.sc.done_cap;
+  {
+    CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0,
+                 d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask,
+                 (M == D - 1) ? d.tab.bstate : nullptr, d.ctl};
+    CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
+    CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
+    launch_scan3(p.lbs, p.num_sms, d.ctl, f0, f1, f2, dcap, site, spin, s);
+    p.launches += 1;
+    site += 3;
+  }
+  const bool chain = M >= 0 && M < D - 1;
+  if (chain) {
+    ChainScan c[3];
+    for (int k = 0; k < 3; ++k) {
+      c[k].done_e = d.sc.done_e;
+      c[k].done_lvl = d.sc.done_lvl;
+      c[k].n_dev = &d.ctl->n_done;
+      c[k].cap = dcap;
+      c[k].which = k;
+      c[k].out_off = (k == 1) ? d.sc.c_arena_base : d.sc.c_dense_base;
+      c[k].tab = d.tab;
+      c[k].arena_pool = d.ar.pool;
+      c[k].ctlp = d.ctl;
+      c[k].M = M;
+      c[k].L = D - 1;
+    }
+    launch_scan3(p.lbs, p.num_sms, d.ctl, c[0], c[1], c[2], dcap, site, spin, s);
+    p.launches += 1;
+    site += 3;
+  }
+  k_check<<<1, 1, 0, s>>>(d);
+  p.launches += 1;
+  if (M >= 0) {
+    p.enter(5);
+    if (leaf_sorted) {
+      k_carry_alloc<false><<<sgrid, kThreads, 0, s>>>(d);
+      k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
+      k_carry_copy<<<grid, kThreads, 0, s>>>(d, bt);
+      p.enter(6);
+      k_dense_batch<<<grid, kThreads, 0, s>>>(d, bt);
+    } else {
+      k_carry_alloc<true><<<sgrid, kThreads, 0, s>>>(d);
+      k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
+      p.enter(6);
+      k_leaf_place<<<grid, kThreads, 0, s>>>(d, bt);
+    }
+    k_dense_arena<true><<<sgrid, kThreads, 0, s>>>(d);
+    p.launches += leaf_sorted ? 5 : 4;
+    if (chain) {
+      k_dense_arena<false><<<sgrid, kThreads, 0, s>>>(d);
+      p.launches += 1;
+    }
+    DenseScan fd{d.sc.dense, d.sc.dst, d.ctl};
+    launch_scan(p.lbs, p.num_sms, d.ctl, fd, d.cfg.dense_cap, site++, spin, s);
+    k_check2<<<1, 1, 0, s>>>(d);
+    p.launches += 2;
+    p.enter(7);
+    // levels below M hand their concatenations up, deepest first
+    for (int l = D - 1; chain && l > M; --l) {
+      k_chain_gather<<<grid, kThreads, 0, s>>>(d, bt, l);
+      p.launches += 1;
+    }
+    k_gather<<<grid, kThreads, 0, s>>>(d, bt);
+    p.launches += 1;
+  }
+  p.enter(8);
+  k_records<<<sgrid, kThreads, 0, s>>>(d);
+  k_sweep<<<sgrid, kThreads, 0, s>>>(d);
+  p.launches += 2;
 }
 
 void* dev_alloc(alto_agg* h, size_t bytes, cudaStream_t s) {
@@ -1581,10 +1976,7 @@ alto_status validate(const alto_agg_config* c) {
   for (int l = 0; l < c->depth; ++l) {
     if (c->payload_op[l] != ALTO_PAYLOAD_NONE && c->payload_op[l] != ALTO_PAYLOAD_CONCAT)
       return ALTO_EINVAL;
-    if (c->payload_op[l] == ALTO_PAYLOAD_CONCAT) {
-      ++nconcat;
-      if (l != c->depth - 1) return ALTO_EINVAL;  // the device path concatenates at the leaf-parent level
-    }
+    if (c->payload_op[l] == ALTO_PAYLOAD_CONCAT) ++nconcat;
     if (c->score_op[l] < ALTO_SCORE_NONE || c->score_op[l] > ALTO_SCORE_TOPK) return ALTO_EINVAL;
     if (c->score_op[l] == ALTO_SCORE_TOPK && (c->topk_k[l] < 1 || c->topk_k[l] > ALTO_MAX_TOPK))
       return ALTO_EINVAL;
@@ -1774,6 +2166,13 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     ALLOC(sc.dst, u64, dense_cap + 1);
     ALLOC(sc.lenscan, u64, nmax + 1);
   }
+  if (concat >= 0 && concat < D - 1) {
+    ALLOC(sc.c_dense_base, u64, done_cap + 1);
+    ALLOC(sc.c_arena_base, u64, done_cap + 1);
+    ALLOC(d.tab.par, u32, T);
+    ALLOC(d.tab.cidx, u32, T);
+    ALLOC(d.tab.app, u64, T);
+  }
   ALLOC(sc.pairset, u64, PS);
   sc.ps_mask = PS - 1;
   sc.done_cap = (u32)done_cap;
@@ -1798,6 +2197,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   cudaMemsetAsync(d.ctl, 0, sizeof(Ctl), s);
   cudaMemsetAsync(d.tab.key, 0xFF, sizeof(u64) * T, s);
   cudaMemsetAsync(d.tab.done_epoch, 0, sizeof(u32) * T, s);
+  cudaMemsetAsync(d.tab.cur, 0, sizeof(u64) * T, s);
   cudaMemsetAsync(sc.mask, 0, sizeof(u32) * nmax, s);
   cudaMemsetAsync(sc.pairset, 0, sizeof(u64) * PS, s);
   cudaMemsetAsync(h->leaf_sort.hist, 0, sizeof(u32) * 4 * 256, s);
@@ -1825,7 +2225,6 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
   if (b->n > 0 && h->d.cfg.has_score && b->score == nullptr) return ALTO_EINVAL;
   cudaStream_t s = (cudaStream_t)stream;
   Dev d = h->d;
-  const int D = cfg.depth;
   const u32 n = (u32)b->n;
   Batch bt;
   bt.tags = b->tags;
@@ -1834,148 +2233,45 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
   bt.score = h->d.cfg.has_score ? b->score : nullptr;
   bt.n = n;
   bt.n_payload = (u64)b->n_payload;
-  const u32 nmax = (u32)cfg.max_batch_fragments;
-  const int grid = h->num_sms * 8;          // kernels over fragments or leaves
-  const int sgrid = h->num_sms * 2;         // kernels over groups (fewer items)
-  const u64 spin = d.cfg.spin_limit;
-
   if (h->pushed % 127 == 0 && h->pushed > 0)
     cudaMemsetAsync(d.sc.pairset, 0, sizeof(u64) * (d.sc.ps_mask + 1), s);
   h->pushed += 1;
   h->last_stream = s;
   if (h->profiling) h->prof_pushes += 1;
-  StageClock clk(h, s);
-  int64_t l0 = h->launches;
-  int stage = 0;
-  auto stage_enter = [&](int st) {
-    if (h->profiling) h->stage_launches[stage] += h->launches - l0;
-    l0 = h->launches;
-    stage = st;
-    clk.enter(st);
+  struct Clock {
+    alto_agg* h;
+    StageClock clk;
+    int stage;
+    int64_t l0;
+  } ck{h, StageClock(h, s), 0, 0};
+  auto on_stage = [](void* ctx, int st, int64_t launches) {
+    Clock* c = (Clock*)ctx;
+    if (c->h->profiling) c->h->stage_launches[c->stage] += launches - c->l0;
+    c->l0 = launches;
+    c->stage = st;
+    c->clk.enter(st);
   };
-  int sl = 0;  // launches inside sort_pairs
-  clk.enter(0);
+  Pipeline p;
+  p.d = d;
+  p.leaf_sort = &h->leaf_sort;
+  p.up_sort = &h->up_sort;
+  p.lbs = h->lbs;
+  p.num_sms = h->num_sms;
+  p.tbits = h->tbits;
+  p.nmax = (u32)cfg.max_batch_fragments;
+  p.s = s;
+  p.stage = on_stage;
+  p.stage_ctx = &ck;
+  ck.clk.enter(0);
   k_begin<<<1, 1, 0, s>>>(d.ctl, n);
-  h->launches += 1;
-  if (n > 0) {
-    int site = 0;
-    k_ingest<<<grid, kThreads, 0, s>>>(d, bt);
-    h->launches += 1;
-    const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK;
-    int set = 0;
-    if (leaf_sorted) {
-      // leaf level with TOPK: sort fragments by their leaf-parent group so that
-      // each group's candidates are contiguous for the segmented top-k
-      stage_enter(1);
-      int cur = sort_pairs(&d.ctl->n, nmax, h->tbits, true, h->leaf_sort, d.ctl, site, spin,
-                           h->num_sms, s, &sl);
-      h->launches += sl;
-      sl = 0;
-      d.sc.leaf_keys = h->leaf_sort.keys[cur];
-      d.sc.leaf_perm = h->leaf_sort.vals[cur];
-      stage_enter(2);
-      {
-        SegFind f{d.sc.leaf_keys, d.sc.leaf_seg_start, d.sc.leaf_seg_of, &d.ctl->n, nmax,
-                  &d.ctl->n_segs[D - 1]};
-        launch_scan(h, f, nmax, site + 4, s);
-      }
-      k_reduce<true><<<grid, kThreads, 0, s>>>(d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
-                                               d.sc.leaf_seg_start, set);
-      h->launches += 1;
-    } else {
-      // leaf level without TOPK: accumulate into the table in arrival order
-      stage_enter(2);
-      k_leaf_accumulate<<<grid, kThreads, 0, s>>>(d, bt);
-      k_up_finalize<true><<<sgrid, kThreads, 0, s>>>(d, bt, D - 1, set);
-      h->launches += 2;
-    }
-    site += 5;
-    stage_enter(3);
-    // an atomic finalize also looks up the parent groups of the items it emits
-    bool looked_up = !leaf_sorted;
-    for (int l = D - 2; l >= 0; --l) {
-      set ^= 1;  // items written by the level below
-      if (!looked_up) {
-        k_items_lookup<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
-        h->launches += 1;
-      }
-      if (d.cfg.score_op[l] != ALTO_SCORE_TOPK) {
-        k_up_accumulate<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
-        k_up_finalize<false><<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
-        h->launches += 2;
-        looked_up = true;
-        continue;
-      }
-      looked_up = false;
-      int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nmax, h->tbits, true, h->up_sort, d.ctl, site,
-                          spin, h->num_sms, s, &sl);
-      h->launches += sl;
-      sl = 0;
-      site += 4;
-      d.sc.up_keys = h->up_sort.keys[c2];
-      d.sc.up_perm = h->up_sort.vals[c2];
-      SegFind f{d.sc.up_keys, d.sc.up_seg_start, nullptr, &d.ctl->n_segs[l + 1], nmax,
-                &d.ctl->n_segs[l]};
-      launch_scan(h, f, nmax, site++, s);
-      k_reduce<false><<<grid, kThreads, 0, s>>>(d, bt, l, d.sc.up_keys, d.sc.up_perm,
-                                                d.sc.up_seg_start, set);
-      h->launches += 1;
-    }
-    // emission order
-    stage_enter(4);
-    {
-      RankScan f{d.sc.mask, d.sc.prefix, &d.ctl->n};
-      launch_scan(h, f, nmax, site++, s);
-    }
-    k_done_rank<<<sgrid, kThreads, 0, s>>>(d);
-    h->launches += 1;
-    const u32 dcap = d.sc.done_cap;
-    {
-      CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0,
-                   d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask, d.tab.bstate, d.ctl};
-      CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
-      CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
-      launch_scan3(h->lbs, h->num_sms, d.ctl, f0, f1, f2, dcap, site, spin, s);
-      h->launches += 1;
-      site += 3;
-    }
-    k_check<<<1, 1, 0, s>>>(d);
-    h->launches += 1;
-    if (d.cfg.concat_level >= 0) {
-      stage_enter(5);
-      if (leaf_sorted) {
-        k_carry_alloc<false><<<sgrid, kThreads, 0, s>>>(d);
-        k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
-        k_carry_copy<<<grid, kThreads, 0, s>>>(d, bt);
-        stage_enter(6);
-        k_dense_batch<<<grid, kThreads, 0, s>>>(d, bt);
-      } else {
-        k_carry_alloc<true><<<sgrid, kThreads, 0, s>>>(d);
-        k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
-        stage_enter(6);
-        k_leaf_place<<<grid, kThreads, 0, s>>>(d, bt);
-      }
-      k_dense_arena<<<sgrid, kThreads, 0, s>>>(d);
-      h->launches += 4;
-      DenseScan fd{d.sc.dense, d.sc.dst, d.ctl};
-      launch_scan(h, fd, d.cfg.dense_cap, site++, s);
-      k_check2<<<1, 1, 0, s>>>(d);
-      h->launches += 1;
-      stage_enter(7);
-      k_gather<<<grid, kThreads, 0, s>>>(d, bt);
-      h->launches += 1;
-    }
-    stage_enter(8);
-    k_records<<<sgrid, kThreads, 0, s>>>(d);
-    k_sweep<<<sgrid, kThreads, 0, s>>>(d);
-    h->launches += 2;
-  } else {
-    stage_enter(8);
-  }
+  p.launches += 1;
+  if (n > 0) enqueue_batch(p, bt);
+  else p.enter(8);
   k_end<<<1, 1, 0, s>>>(d.ctl, n);
-  h->launches += 1;
-  stage_enter(ALTO_NUM_STAGES);
-  clk.finish();
+  p.launches += 1;
+  p.enter(ALTO_NUM_STAGES);
+  ck.clk.finish();
+  h->launches += p.launches;
   if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
   return ALTO_OK;
 }
@@ -2140,10 +2436,10 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   st.T = T;
   st.tbits = ilog2(T);
   st.done_cap = nmax * (u64)D;
-  st.dense_cap = nmax;
+  st.dense_cap = kNaMaxGroupsLevels;  // children of every level of one self-contained batch
   st.PS = next_pow2(std::max<u64>(2 * nmax * (u64)D, 1024));
   st.sort_tiles = nmax / 4096 + 2;
-  st.scan_tiles = std::max<u64>(st.done_cap, nmax) / kScanTile + 2;
+  st.scan_tiles = std::max<u64>(std::max<u64>(st.done_cap, st.dense_cap), nmax) / kScanTile + 2;
   Dev& d = st.d;
   memset(&d, 0, sizeof(d));
   d.ctl = cv.take<Ctl>(1);
@@ -2247,6 +2543,13 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
     sc.dense = cv.take<uint4>(st.dense_cap);
     sc.dst = cv.take<u64>(st.dense_cap + 1);
   }
+  if (concat >= 0 && concat < D - 1) {
+    sc.c_dense_base = cv.take<u64>(dc + 1);
+    sc.c_arena_base = cv.take<u64>(dc + 1);
+    d.tab.par = cv.take<u32>(T);
+    d.tab.cidx = cv.take<u32>(T);
+    d.tab.app = cv.take<u64>(T);
+  }
   sc.pairset = cv.take<u64>(st.PS);
   sc.ps_mask = st.PS - 1;
   sc.done_cap = (u32)dc;
@@ -2279,6 +2582,7 @@ __global__ void k_na_reset(Dev d, u32* hist, u64 T, u64 PS, u32 nmax) {
     d.tab.acc_smx[i] = 0;
     d.tab.acc_len[i] = 0;
     d.tab.acc_leaf[i] = make_uint4(0, 0, 0, 0);
+    d.tab.cur[i] = 0;
   }
   for (u64 i = tid; i < PS; i += stride) d.sc.pairset[i] = 0;
   for (u64 i = tid; i < nmax; i += stride) d.sc.mask[i] = 0;
@@ -2349,11 +2653,8 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
   d.cfg.out_topk = (u64)cap_topk;
 
   cudaStream_t s = (cudaStream_t)stream;
-  const int D = cfg.depth;
   const u32 n = (u32)b->n;
   const u32 nmax = (u32)kNaMaxFragments;
-  const int grid = num_sms * 8, sgrid = num_sms * 2;
-  const u64 spin = d.cfg.spin_limit;
   Batch bt;
   bt.tags = b->tags;
   bt.off = b->payload_off;
@@ -2362,94 +2663,19 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
   bt.n = n;
   bt.n_payload = (u64)b->n_payload;
 
-  k_na_reset<<<sgrid, kThreads, 0, s>>>(d, st.leaf_sort.hist, st.T, st.PS, nmax);
+  k_na_reset<<<num_sms * 2, kThreads, 0, s>>>(d, st.leaf_sort.hist, st.T, st.PS, nmax);
   k_begin<<<1, 1, 0, s>>>(d.ctl, n);
   if (n > 0) {
-    // the same stages, in the same order, as a push (see alto_agg_push_batch)
-    auto scan_grid = [&](u64 cap) {
-      u64 tiles = (cap + kScanTile - 1) / kScanTile;
-      return (int)std::min<u64>(std::max<u64>(tiles, 1), (u64)num_sms * 4);
-    };
-    int site = 0;
-    k_ingest<<<grid, kThreads, 0, s>>>(d, bt);
-    const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK;
-    int set = 0;
-    if (leaf_sorted) {
-      int cur = sort_pairs(&d.ctl->n, nmax, st.tbits, true, st.leaf_sort, d.ctl, site, spin, num_sms,
-                           s, nullptr);
-      d.sc.leaf_keys = st.leaf_sort.keys[cur];
-      d.sc.leaf_perm = st.leaf_sort.vals[cur];
-      SegFind f{d.sc.leaf_keys, d.sc.leaf_seg_start, d.sc.leaf_seg_of, &d.ctl->n, nmax,
-                &d.ctl->n_segs[D - 1]};
-      k_scan<SegFind><<<scan_grid(nmax), kScanThreads, 0, s>>>(f, st.lbs, d.ctl, site + 4,
-                                                             &d.ctl->exit_ctr[site + 4], spin);
-      k_reduce<true><<<grid, kThreads, 0, s>>>(d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
-                                               d.sc.leaf_seg_start, set);
-    } else {
-      k_leaf_accumulate<<<grid, kThreads, 0, s>>>(d, bt);
-      k_up_finalize<true><<<sgrid, kThreads, 0, s>>>(d, bt, D - 1, set);
-    }
-    site += 5;
-    bool looked_up = !leaf_sorted;
-    for (int l = D - 2; l >= 0; --l) {
-      set ^= 1;
-      if (!looked_up) k_items_lookup<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
-      if (d.cfg.score_op[l] != ALTO_SCORE_TOPK) {
-        k_up_accumulate<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
-        k_up_finalize<false><<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
-        looked_up = true;
-        continue;
-      }
-      looked_up = false;
-      int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nmax, st.tbits, true, st.up_sort, d.ctl, site, spin,
-                          num_sms, s, nullptr);
-      site += 4;
-      d.sc.up_keys = st.up_sort.keys[c2];
-      d.sc.up_perm = st.up_sort.vals[c2];
-      SegFind f{d.sc.up_keys, d.sc.up_seg_start, nullptr, &d.ctl->n_segs[l + 1], nmax,
-                &d.ctl->n_segs[l]};
-      k_scan<SegFind><<<scan_grid(nmax), kScanThreads, 0, s>>>(f, st.lbs, d.ctl, site,
-                                                             &d.ctl->exit_ctr[site], spin);
-      ++site;
-      k_reduce<false><<<grid, kThreads, 0, s>>>(d, bt, l, d.sc.up_keys, d.sc.up_perm,
-                                                d.sc.up_seg_start, set);
-    }
-    {
-      RankScan f{d.sc.mask, d.sc.prefix, &d.ctl->n};
-      k_scan<RankScan><<<scan_grid(nmax), kScanThreads, 0, s>>>(f, st.lbs, d.ctl, site,
-                                                              &d.ctl->exit_ctr[site], spin);
-      ++site;
-    }
-    k_done_rank<<<sgrid, kThreads, 0, s>>>(d);
-    const u32 dcap = d.sc.done_cap;
-    CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0,
-                 d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask, d.tab.bstate, d.ctl};
-    CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
-    CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
-    launch_scan3(st.lbs, num_sms, d.ctl, f0, f1, f2, dcap, site, spin, s);
-    site += 3;
-    k_check<<<1, 1, 0, s>>>(d);
-    if (d.cfg.concat_level >= 0) {
-      if (leaf_sorted) {
-        k_carry_alloc<false><<<sgrid, kThreads, 0, s>>>(d);
-        k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
-        k_carry_copy<<<grid, kThreads, 0, s>>>(d, bt);
-        k_dense_batch<<<grid, kThreads, 0, s>>>(d, bt);
-      } else {
-        k_carry_alloc<true><<<sgrid, kThreads, 0, s>>>(d);
-        k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
-        k_leaf_place<<<grid, kThreads, 0, s>>>(d, bt);
-      }
-      k_dense_arena<<<sgrid, kThreads, 0, s>>>(d);
-      DenseScan fd{d.sc.dense, d.sc.dst, d.ctl};
-      k_scan<DenseScan><<<scan_grid(d.cfg.dense_cap), kScanThreads, 0, s>>>(
-          fd, st.lbs, d.ctl, site, &d.ctl->exit_ctr[site], spin);
-      ++site;
-      k_check2<<<1, 1, 0, s>>>(d);
-      k_gather<<<grid, kThreads, 0, s>>>(d, bt);
-    }
-    k_records<<<sgrid, kThreads, 0, s>>>(d);
-    k_sweep<<<sgrid, kThreads, 0, s>>>(d);
+    Pipeline p;
+    p.d = d;
+    p.leaf_sort = &st.leaf_sort;
+    p.up_sort = &st.up_sort;
+    p.lbs = st.lbs;
+    p.num_sms = num_sms;
+    p.tbits = st.tbits;
+    p.nmax = nmax;
+    p.s = s;
+    enqueue_batch(p, bt);
   }
   k_end<<<1, 1, 0, s>>>(d.ctl, n);
   k_na_finish<<<1, 1, 0, s>>>(d.ctl, out_counts);

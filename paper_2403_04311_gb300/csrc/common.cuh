@@ -52,6 +52,8 @@ struct Ctl {
   u64 pay_total;           // payload elements emitted by this batch
   u64 topk_total;          // top-k pairs emitted by this batch
   u64 n_emit;              // records ranked by this batch
+  u64 chain_total;         // dense child slots of completing groups at levels M < l
+  u64 chain_arena;         // their buffered child spans
   u64 scan_total[kSites];  // totals written by scans
 };
 
@@ -158,6 +160,12 @@ struct Table {
   u64* dbase;      // [T] first dense child slot of a group completing this batch
   uint4* bstate;   // [T] where this batch's leaves go, one load per fragment:
                    //     {epoch, mode (1 arena, 2 dense), dense base lo, hi}
+  // CONCAT at a level M above the leaf parent: a group of a level l with
+  // M < l <= D-1 that completes is appended, as one child span, to its
+  // parent's arena vectors (the parent's cursor `cur` counts the spans)
+  u32* par;        // [T] parent entry the completed group was appended to
+  u32* cidx;       // [T] its child index in that parent
+  u64* app;        // [T] its reserved place there: span index << 40 | payload position
   int chain_len;   // D - 1
   u32 mask;        // T - 1
   int kk;          // stride of topk (largest k over levels)

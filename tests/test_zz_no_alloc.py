@@ -9,6 +9,7 @@ different batches, must give exactly the records, payload and top-k pairs of
 create + push_batch + drain on a fresh handle (exact equality: the results
 are integers and copied floats).  This file is collected last on purpose."""
 import ctypes
+import dataclasses
 
 import numpy as np
 import pytest
@@ -67,7 +68,9 @@ def _cases():
     # depth 4 with top-k and max levels, whole stream in one batch
     fact = make_factcheck(n_responses=8, batch=4096)
     assert fact.n_batches == 1
-    return [(tiny, tiny.batch(0)), (fact, fact.batch(0))]
+    # the same batch with the concatenation two levels above the fragments
+    fact_up = dataclasses.replace(fact, payload_op=(0, 1, 0, 0))
+    return [(tiny, tiny.batch(0)), (fact, fact.batch(0)), (fact_up, fact_up.batch(0))]
 
 
 def test_oneshot_noalloc_matches_regular_path_twice_in_a_row():
