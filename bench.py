@@ -240,7 +240,19 @@ def main():
             dist.barrier()
 
     stream = torch.cuda.current_stream()
-    caps = stream_caps(s)
+    if args.max_batches > 0:
+        # size the handle for the prefix only, so that a profiling run holds a
+        # few GB on the device rather than the whole stream's capacities
+        import dataclasses
+        nbp = min(args.max_batches, s.n_batches)
+        n_pref = int(s.batch_starts()[nbp])
+        s_caps = dataclasses.replace(
+            s, tags=s.tags[:, :n_pref], off=s.off[:n_pref + 1],
+            payload=s.payload[:int(s.off[n_pref])],
+            score=None if s.score is None else s.score[:n_pref], batch_sizes=s.batch_sizes[:nbp])
+        caps = stream_caps(s_caps)
+    else:
+        caps = stream_caps(s)
     agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, stream=stream, **caps)
     nb = s.n_batches if args.max_batches <= 0 else min(args.max_batches, s.n_batches)
     batches = [alto.to_device(s.batch(b)) for b in range(nb)]
