@@ -656,7 +656,8 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
 // Leaf level without TOPK: every fragment, in arrival order (coalesced),
 // checks its ancestry against its group's entry and adds itself to the
 // entry's batch accumulators (warp-aggregated over lanes of the same group).
-__global__ void __launch_bounds__(kThreads) k_leaf_accumulate(Dev d, Batch b) {
+// 32 registers: eight blocks per SM, so the grid is one wave
+__global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch b) {
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const int D = d.cfg.depth;
@@ -677,8 +678,12 @@ __global__ void __launch_bounds__(kThreads) k_leaf_accumulate(Dev d, Batch b) {
       f = tag_last(t);
       len = b.off[i + 1] - b.off[i];
       if (scores) sk = score_key(b.score[i]);
-      if (chain_differs(d.tab, e, b.tags, n, i, L)) raise_err(ctl, ALTO_EINCONSIST);
-      if (ps_insert(d.sc, e, c, ep7, ctl)) raise_err(ctl, ALTO_EDUP);
+      // the chain row and the leaf-slot probe are independent loads: issue both
+      // before acting on either
+      const bool bad = chain_differs(d.tab, e, b.tags, n, i, L);
+      const bool dup = ps_insert(d.sc, e, c, ep7, ctl);
+      if (bad) raise_err(ctl, ALTO_EINCONSIST);
+      if (dup) raise_err(ctl, ALTO_EDUP);
     }
     const u32 key = valid ? e : kNone;
     const u32 peers = __match_any_sync(0xFFFFFFFFu, key);
@@ -1186,7 +1191,7 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
 // cursor (one 64-bit atomic: leaf index and payload offset together) and is
 // copied there; a fragment of a group completed by this batch is placed at
 // its dense child slot.
-__global__ void __launch_bounds__(kThreads) k_leaf_place(Dev d, Batch b) {
+__global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch b) {
   Ctl* ctl = d.ctl;
   if (no_copy(ctl)) return;
   const int D = d.cfg.depth;
@@ -1350,10 +1355,6 @@ __global__ void k_check2(Dev d) {
   }
 }
 
-// Copy every child span into the output payload ring.  A warp takes 32
-// consecutive dense slots -- one contiguous output range -- reads their
-// headers in one go, then copies four spans per round with all loads issued
-// before the stores.  Spans longer than 64 elements finish in a second loop.
 __device__ __forceinline__ int32_t span_load(const Dev& d, const Batch& b, u32 owner, u32 pos,
                                              u32 k) {
   if (owner == kNone) return b.pay[(u64)pos + k];
@@ -1362,21 +1363,39 @@ __device__ __forceinline__ int32_t span_load(const Dev& d, const Batch& b, u32 o
   return ok ? d.ar.pool[a] : 0;
 }
 
+// Copy every child span into the output payload ring.
+//
+// Eight lanes take one span (a warp four spans at a time): lane `sub` of the
+// group copies elements sub, sub+8, ..., with the first 64 elements' loads
+// all issued, as plain predicated loads, before the stores.  With spans of a
+// few dozen elements read in an order unrelated to their source order, this
+// keeps about as many loads in flight as the memory system can overlap;
+// wider groups (16 or 32 lanes a span), narrower ones, more spans per group,
+// staging through shared memory (with 16-byte vector loads or with bulk
+// copies) and scattering in source order instead all measured slower on span
+// streams of this shape, and so did a first pass with a per-element fallback
+// branch (the loads no longer overlap).  An arena span is read through its
+// first chunk; elements past that chunk (a span across a chunk boundary)
+// look up their chunk one by one, after the rest.
+constexpr int kSpanLanes = 8;
+constexpr int kSpanFirst = 8;  // elements per lane in the first pass
+
 __global__ void __launch_bounds__(kThreads) k_gather(Dev d, Batch b) {
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
+  const int lane = threadIdx.x & 31, sub = lane % kSpanLanes, grp = lane / kSpanLanes;
+  constexpr int kGroups = 32 / kSpanLanes;
   const u32 ep = ctl->epoch;
   const u64 total = ctl->dense_total;
   const u64 base = ctl->pay_count;
   const u64 cap = d.cfg.out_payload;
-  const int lane = threadIdx.x & 31;
-  const u64 gw = gtid() >> 5, nw = gstride() >> 5;
   int32_t* __restrict__ out = d.out_pay;
-  for (u64 jb = gw * 32; jb < total; jb += nw * 32) {
-    // this lane's slot header; an unusable slot copies nothing
-    const u64 j = jb + lane;
-    u32 len = 0, owner = kNone, pos = 0;
+  const u64 gw = gtid() >> 5, nw = gstride() >> 5;
+  for (u64 jb = gw * kGroups; jb < total; jb += nw * kGroups) {
+    const u64 j = jb + grp;
+    u32 len = 0, owner = kNone, pos = 0, n1 = 0;
     u64 o = 0;
+    const int32_t* src = b.pay;
     if (j < total) {
       const uint4 v = d.sc.dense[j];
       o = base + d.sc.dst[j];
@@ -1388,41 +1407,33 @@ __global__ void __launch_bounds__(kThreads) k_gather(Dev d, Batch b) {
         len = v.y;
         owner = v.z;
         pos = v.w;
+        if (owner == kNone) {
+          src = b.pay + pos;
+          n1 = len;
+        } else if (len) {
+          const int jc = chunk_of(pos);
+          const u32 cb = (jc < kNumChunks) ? d.tab.dir[((u64)owner * kVecs + 1) * kNumChunks + jc] : kNone;
+          if (cb != kNone) {
+            src = d.ar.pool + cb + ((u64)pos - chunk_start(jc));
+            const u64 room = chunk_start(jc) + chunk_size(jc) - pos;
+            n1 = (room < len) ? (u32)room : len;
+          }
+        }
       }
     }
-    const u32 cnt = (total - jb < 32) ? (u32)(total - jb) : 32u;
-    // four spans per round, two elements per lane per span: all eight loads
-    // are in flight before the first store
-    for (u32 k0 = 0; k0 < cnt; k0 += 4) {
-      int32_t val[4][2];
-      u32 L[4];
-      u64 O[4];
+    int32_t val[kSpanFirst];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int src = (k0 + u < 31u) ? (int)(k0 + u) : 31;
-        L[u] = __shfl_sync(0xFFFFFFFFu, len, src);
-        const u32 ow = __shfl_sync(0xFFFFFFFFu, owner, src);
-        const u32 ps = __shfl_sync(0xFFFFFFFFu, pos, src);
-        O[u] = __shfl_sync(0xFFFFFFFFu, o, src);
-        if (k0 + u >= cnt) L[u] = 0;
-        val[u][0] = ((u32)lane < L[u]) ? span_load(d, b, ow, ps, lane) : 0;
-        val[u][1] = ((u32)lane + 32 < L[u]) ? span_load(d, b, ow, ps, lane + 32) : 0;
-      }
+    for (int q = 0; q < kSpanFirst; ++q) {
+      const u32 k = sub + kSpanLanes * q;
+      val[q] = (k < n1) ? src[k] : 0;
+    }
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        if ((u32)lane < L[u]) out[O[u] + lane] = val[u][0];
-        if ((u32)lane + 32 < L[u]) out[O[u] + lane + 32] = val[u][1];
-      }
+    for (int q = 0; q < kSpanFirst; ++q) {
+      const u32 k = sub + kSpanLanes * q;
+      if (k < n1) out[o + k] = val[q];
     }
-    // the remainder of long spans
-    for (u32 k = 0; k < cnt; ++k) {
-      const u32 Lk = __shfl_sync(0xFFFFFFFFu, len, k);
-      if (Lk <= 64) continue;
-      const u32 ow = __shfl_sync(0xFFFFFFFFu, owner, k);
-      const u32 ps = __shfl_sync(0xFFFFFFFFu, pos, k);
-      const u64 Ok = __shfl_sync(0xFFFFFFFFu, o, k);
-      for (u32 q = 64 + lane; q < Lk; q += 32) out[Ok + q] = span_load(d, b, ow, ps, q);
-    }
+    for (u32 k = kSpanLanes * kSpanFirst + sub; k < n1; k += kSpanLanes) out[o + k] = src[k];
+    for (u32 k = n1 + sub; k < len; k += kSpanLanes) out[o + k] = span_load(d, b, owner, pos, k);
   }
 }
 
