@@ -217,8 +217,14 @@ alto_status alto_agg_stats(alto_agg_t* h, void* stream, int64_t* open_groups,
  *   6 dense child placement + length scan                 7 payload gather
  *   8 records, frees, table sweep
  * `launches` counts every kernel the pushes launched (also when profiling is
- * off).  enable = 1 starts a fresh count, 0 stops recording events. */
+ * off).  enable = ALTO_PROFILE_STAGES (1) records an event at every stage
+ * boundary; ALTO_PROFILE_GATHER (2) records only the two around the payload
+ * gather (stage 7), so that the other kernel boundaries run as without
+ * profiling; either starts a fresh count.  0 stops recording events. */
 #define ALTO_NUM_STAGES 9
+#define ALTO_PROFILE_OFF 0
+#define ALTO_PROFILE_STAGES 1
+#define ALTO_PROFILE_GATHER 2
 typedef struct alto_profile {
   int64_t pushes;                          /* pushes since the last enable */
   int64_t launches;                        /* kernels those pushes launched */

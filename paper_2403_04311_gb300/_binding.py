@@ -210,8 +210,13 @@ def alto_agg_oneshot_noalloc(cfg, batch, out_records, cap_records, out_payload, 
         ctypes.c_void_p(out_counts), ctypes.c_void_p(stream))
 
 
-def alto_agg_profile(h, enable: bool) -> int:
-    return load_library().alto_agg_profile(h, 1 if enable else 0)
+PROFILE_OFF, PROFILE_STAGES, PROFILE_GATHER = 0, 1, 2
+
+
+def alto_agg_profile(h, enable) -> int:
+    """enable: False/0 off, True/1 every stage boundary, 2 the gather stage only."""
+    mode = PROFILE_STAGES if enable is True else int(enable)
+    return load_library().alto_agg_profile(h, mode)
 
 
 def alto_agg_profile_read(h):
@@ -301,7 +306,7 @@ class Aggregator:
     def stats(self):
         return alto_agg_stats(self._h, self.stream.cuda_stream)
 
-    def profile(self, enable: bool) -> int:
+    def profile(self, enable) -> int:
         return alto_agg_profile(self._h, enable)
 
     def profile_read(self):

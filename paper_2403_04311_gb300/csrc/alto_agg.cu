@@ -26,6 +26,7 @@
 #include <algorithm>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <vector>
 
@@ -293,6 +294,7 @@ __device__ __forceinline__ void chain_reserve(const Table& tab, u32 e, u32 P, u3
 // kernels
 // ---------------------------------------------------------------------------
 __global__ void k_begin(Ctl* ctl, u32 n) {
+  pdl_enter();
   ctl->epoch += 1;
   ctl->batch_err = 0;
   ctl->n_done = 0;
@@ -303,6 +305,7 @@ __global__ void k_begin(Ctl* ctl, u32 n) {
 }
 
 __global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   __shared__ u32 s_ins;
@@ -331,6 +334,7 @@ __global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
 
 // Items of level l are the level-(l+1) groups present in the batch.
 __global__ void __launch_bounds__(kThreads) k_items_lookup(Dev d, Batch b, int l, int in_set) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   __shared__ u32 s_ins;
@@ -384,6 +388,7 @@ template <bool LEAF>
 __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, const u32* skeys,
                                                      const u32* sperm, const u32* seg_start,
                                                      int in_set) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const int D = d.cfg.depth;
@@ -584,6 +589,7 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
 // ---------------------------------------------------------------------------
 // Items of level l: check ancestry against the entry and accumulate.
 __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int l, int in_set) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const u32 ni = min(ctl->n_segs[l + 1], d.cfg.n_max);
@@ -658,6 +664,7 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
 // entry's batch accumulators (warp-aggregated over lanes of the same group).
 // 32 registers: eight blocks per SM, so the grid is one wave
 __global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch b) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const int D = d.cfg.depth;
@@ -743,6 +750,7 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch b)
 // One thread per touched entry: merge, test completion, emit the next items.
 template <bool LEAF>
 __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l, int in_set) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const int D = d.cfg.depth;
@@ -862,6 +870,7 @@ struct RankScan {
 };
 
 __global__ void __launch_bounds__(kThreads) k_done_rank(Dev d) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const int D = d.cfg.depth, M = d.cfg.concat_level;
@@ -977,6 +986,7 @@ struct ChainScan {
 };
 
 __global__ void k_check(Dev d) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   bool bad = false;
@@ -1013,6 +1023,7 @@ constexpr int kMaxReq = 8;
 
 template <bool ATOMIC>
 __global__ void __launch_bounds__(kThreads) k_carry_alloc(Dev d) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (no_copy(ctl)) return;
   const u32 ep = ctl->epoch;
@@ -1111,6 +1122,7 @@ __global__ void __launch_bounds__(kThreads) k_carry_alloc(Dev d) {
 }
 
 __global__ void k_fix_tops(Ctl* ctl) {
+  pdl_enter();
   int j = threadIdx.x;
   if (j < kNumChunks && ctl->top[j] < 0) ctl->top[j] = 0;
 }
@@ -1119,6 +1131,7 @@ __global__ void k_fix_tops(Ctl* ctl) {
 // per leaf, over the sorted leaves.  A leaf's vector position is its group's
 // reserved base plus its offset inside the segment (written by the reduce).
 __global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch b) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (no_copy(ctl)) return;
   const int D = d.cfg.depth;
@@ -1158,6 +1171,7 @@ __global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch b) {
 
 // Dense child slots of completing CONCAT groups, from this batch's leaves.
 __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
   const int D = d.cfg.depth;
@@ -1192,6 +1206,7 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
 // copied there; a fragment of a group completed by this batch is placed at
 // its dense child slot.
 __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch b) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (no_copy(ctl)) return;
   const int D = d.cfg.depth;
@@ -1273,6 +1288,7 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch b) {
 // by done index.
 template <bool LEVEL_M>
 __global__ void __launch_bounds__(kThreads) k_dense_arena(Dev d) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
   const u32 ep = ctl->epoch;
@@ -1345,6 +1361,7 @@ struct DenseScan {
 };
 
 __global__ void k_check2(Dev d) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl) || ctl->skip_dense) return;
   // level M's spans come first; the slots after them are handed up, not emitted
@@ -1380,7 +1397,9 @@ __device__ __forceinline__ int32_t span_load(const Dev& d, const Batch& b, u32 o
 constexpr int kSpanLanes = 8;
 constexpr int kSpanFirst = 8;  // elements per lane in the first pass
 
-__global__ void __launch_bounds__(kThreads) k_gather(Dev d, Batch b) {
+// 32 registers: eight blocks per SM, the grid is one wave
+__global__ void __launch_bounds__(kThreads, 8) k_gather(Dev d, Batch b) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
   const int lane = threadIdx.x & 31, sub = lane % kSpanLanes, grp = lane / kSpanLanes;
@@ -1444,6 +1463,7 @@ __global__ void __launch_bounds__(kThreads) k_gather(Dev d, Batch b) {
 // 32 consecutive slots; each lane finds its slot's group by binary search,
 // then the warp copies the spans one after another.
 __global__ void __launch_bounds__(kThreads) k_chain_gather(Dev d, Batch b, int l) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
   const u32 ep = ctl->epoch;
@@ -1517,6 +1537,7 @@ __global__ void __launch_bounds__(kThreads) k_chain_gather(Dev d, Batch b, int l
 }
 
 __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   __shared__ u32 s_del;
@@ -1621,6 +1642,7 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
 // Turn deleted slots back into free ones where no probe chain runs through
 // them: a tombstone followed (after more tombstones) by a free slot.
 __global__ void __launch_bounds__(kThreads) k_sweep(Dev d) {
+  pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const u32 nd = min(ctl->n_done, d.sc.done_cap);
@@ -1648,6 +1670,7 @@ __global__ void __launch_bounds__(kThreads) k_sweep(Dev d) {
 }
 
 __global__ void k_end(Ctl* ctl, u32 n) {
+  pdl_enter();
   if (ctl->status != ALTO_OK) return;
   if (ctl->batch_err) {
     ctl->status = -(ctl->batch_err & 0xFF);
@@ -1660,6 +1683,7 @@ __global__ void k_end(Ctl* ctl, u32 n) {
 }
 
 __global__ void k_drain_reset(Ctl* ctl) {
+  pdl_enter();
   ctl->rec_count = 0;
   ctl->pay_count = 0;
   ctl->topk_count = 0;
@@ -1689,6 +1713,7 @@ struct alto_agg {
   int latched;
   // measurement hooks
   bool profiling;
+  int profile_mode;  // ALTO_PROFILE_STAGES or ALTO_PROFILE_GATHER
   cudaStream_t last_stream;
   int64_t prof_pushes;
   int64_t launches;
@@ -1718,12 +1743,17 @@ struct StageClock {
     }
     return e;
   }
-  // mark the start of stage `st` (stages must be entered in order)
+  // mark the start of stage `st` (stages must be entered in order); in gather
+  // mode only the boundaries around the gather stage get an event
   void enter(int st) {
     if (!h->profiling) return;
     while ((int)ev.size() <= st) {
-      cudaEvent_t e = take();
-      if (e) cudaEventRecord(e, s);
+      const int bnd = (int)ev.size();
+      cudaEvent_t e = nullptr;
+      if (h->profile_mode == ALTO_PROFILE_STAGES || bnd == 7 || bnd == 8) {
+        e = take();
+        if (e) cudaEventRecord(e, s);
+      }
       ev.push_back(e);
     }
   }
@@ -1762,7 +1792,7 @@ void launch_scan3(const LookbackState& lb, int num_sms, Ctl* ctl, const F& f0, c
   // a small persistent grid, so that hundreds of idle CTAs do not contend on
   // the tile and exit counters
   dim3 grid((unsigned)std::min<u64>(tiles, 32), 3);
-  k_scan3<F><<<grid, kScanThreads, 0, s>>>(f0, f1, f2, lb_region(lb, 0), lb_region(lb, 1),
+  launch_pdl(k_scan3<F>, grid, kScanThreads, 0, s, f0, f1, f2, lb_region(lb, 0), lb_region(lb, 1),
                                            lb_region(lb, 2), ctl, site, spin);
 }
 
@@ -1772,7 +1802,7 @@ void launch_scan(const LookbackState& lb, int num_sms, Ctl* ctl, const F& f, u64
   u64 tiles = (cap + kScanTile - 1) / kScanTile;
   if (tiles == 0) tiles = 1;
   int grid = (int)std::min<u64>(tiles, (u64)num_sms * 4);
-  k_scan<F><<<grid, kScanThreads, 0, s>>>(f, lb, ctl, site, &ctl->exit_ctr[site], spin);
+  launch_pdl(k_scan<F>, grid, kScanThreads, 0, s, f, lb, ctl, site, &ctl->exit_ctr[site], spin);
 }
 
 // What one batch enqueues between k_begin and k_end, for the handle's push
@@ -1795,6 +1825,21 @@ struct Pipeline {
   }
 };
 
+// Blocks of 256 threads of `kernel` resident per SM (cached per kernel): a
+// grid-stride kernel whose grid is exactly one wave has no ragged tail.
+int blocks_per_sm(const void* kernel) {
+  static std::mutex mu;
+  static std::vector<std::pair<const void*, int>> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  for (auto& kv : cache)
+    if (kv.first == kernel) return kv.second;
+  int nb = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kernel, kThreads, 0) != cudaSuccess || nb < 1)
+    nb = 1;
+  cache.emplace_back(kernel, nb);
+  return nb;
+}
+
 void enqueue_batch(Pipeline& p, const Batch& bt) {
   Dev d = p.d;
   cudaStream_t s = p.s;
@@ -1806,7 +1851,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   const u64 spin = d.cfg.spin_limit;
   int sl = 0;  // launches inside sort_pairs
   int site = 0;
-  k_ingest<<<grid, kThreads, 0, s>>>(d, bt);
+  launch_pdl(k_ingest, grid, kThreads, 0, s, d, bt);
   p.launches += 1;
   const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK;
   int set = 0;
@@ -1824,14 +1869,15 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     SegFind f{d.sc.leaf_keys, d.sc.leaf_seg_start, d.sc.leaf_seg_of, &d.ctl->n, nmax,
               &d.ctl->n_segs[D - 1]};
     launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site + 4, spin, s);
-    k_reduce<true><<<grid, kThreads, 0, s>>>(d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
+    launch_pdl(k_reduce<true>, p.num_sms * blocks_per_sm((const void*)k_reduce<true>), kThreads, 0, s, d, bt,
+               D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
                                              d.sc.leaf_seg_start, set);
     p.launches += 2;
   } else {
     // leaf level without TOPK: accumulate into the table in arrival order
     p.enter(2);
-    k_leaf_accumulate<<<grid, kThreads, 0, s>>>(d, bt);
-    k_up_finalize<true><<<sgrid, kThreads, 0, s>>>(d, bt, D - 1, set);
+    launch_pdl(k_leaf_accumulate, grid, kThreads, 0, s, d, bt);
+    launch_pdl(k_up_finalize<true>, sgrid, kThreads, 0, s, d, bt, D - 1, set);
     p.launches += 2;
   }
   site += 5;
@@ -1841,12 +1887,12 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   for (int l = D - 2; l >= 0; --l) {
     set ^= 1;  // items written by the level below
     if (!looked_up) {
-      k_items_lookup<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+      launch_pdl(k_items_lookup, sgrid, kThreads, 0, s, d, bt, l, set);
       p.launches += 1;
     }
     if (d.cfg.score_op[l] != ALTO_SCORE_TOPK) {
-      k_up_accumulate<<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
-      k_up_finalize<false><<<sgrid, kThreads, 0, s>>>(d, bt, l, set);
+      launch_pdl(k_up_accumulate, sgrid, kThreads, 0, s, d, bt, l, set);
+      launch_pdl(k_up_finalize<false>, sgrid, kThreads, 0, s, d, bt, l, set);
       p.launches += 2;
       looked_up = true;
       continue;
@@ -1862,7 +1908,8 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     SegFind f{d.sc.up_keys, d.sc.up_seg_start, nullptr, &d.ctl->n_segs[l + 1], nmax,
               &d.ctl->n_segs[l]};
     launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site++, spin, s);
-    k_reduce<false><<<grid, kThreads, 0, s>>>(d, bt, l, d.sc.up_keys, d.sc.up_perm,
+    launch_pdl(k_reduce<false>, p.num_sms * blocks_per_sm((const void*)k_reduce<false>), kThreads, 0, s, d,
+               bt, l, d.sc.up_keys, d.sc.up_perm,
                                               d.sc.up_seg_start, set);
     p.launches += 2;
   }
@@ -1872,7 +1919,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     RankScan f{d.sc.mask, d.sc.prefix, &d.ctl->n};
     launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site++, spin, s);
   }
-  k_done_rank<<<sgrid, kThreads, 0, s>>>(d);
+  launch_pdl(k_done_rank, sgrid, kThreads, 0, s, d);
   p.launches += 2;
   const u32 dcap = d.sc.done_cap;
   {
@@ -1905,44 +1952,47 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     p.launches += 1;
     site += 3;
   }
-  k_check<<<1, 1, 0, s>>>(d);
+  launch_pdl(k_check, 1, 1, 0, s, d);
   p.launches += 1;
   if (M >= 0) {
     p.enter(5);
     if (leaf_sorted) {
-      k_carry_alloc<false><<<sgrid, kThreads, 0, s>>>(d);
-      k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
-      k_carry_copy<<<grid, kThreads, 0, s>>>(d, bt);
+      launch_pdl(k_carry_alloc<false>, sgrid, kThreads, 0, s, d);
+      launch_pdl(k_fix_tops, 1, 32, 0, s, d.ctl);
+      launch_pdl(k_carry_copy, grid, kThreads, 0, s, d, bt);
       p.enter(6);
-      k_dense_batch<<<grid, kThreads, 0, s>>>(d, bt);
+      launch_pdl(k_dense_batch, grid, kThreads, 0, s, d, bt);
     } else {
-      k_carry_alloc<true><<<sgrid, kThreads, 0, s>>>(d);
-      k_fix_tops<<<1, 32, 0, s>>>(d.ctl);
+      launch_pdl(k_carry_alloc<true>, sgrid, kThreads, 0, s, d);
+      launch_pdl(k_fix_tops, 1, 32, 0, s, d.ctl);
       p.enter(6);
-      k_leaf_place<<<grid, kThreads, 0, s>>>(d, bt);
+      launch_pdl(k_leaf_place, grid, kThreads, 0, s, d, bt);
     }
-    k_dense_arena<true><<<sgrid, kThreads, 0, s>>>(d);
+    launch_pdl(k_dense_arena<true>, sgrid, kThreads, 0, s, d);
     p.launches += leaf_sorted ? 5 : 4;
     if (chain) {
-      k_dense_arena<false><<<sgrid, kThreads, 0, s>>>(d);
+      launch_pdl(k_dense_arena<false>, sgrid, kThreads, 0, s, d);
       p.launches += 1;
     }
     DenseScan fd{d.sc.dense, d.sc.dst, d.ctl};
     launch_scan(p.lbs, p.num_sms, d.ctl, fd, d.cfg.dense_cap, site++, spin, s);
-    k_check2<<<1, 1, 0, s>>>(d);
+    launch_pdl(k_check2, 1, 1, 0, s, d);
     p.launches += 2;
     p.enter(7);
     // levels below M hand their concatenations up, deepest first
     for (int l = D - 1; chain && l > M; --l) {
-      k_chain_gather<<<grid, kThreads, 0, s>>>(d, bt, l);
+      launch_pdl(k_chain_gather, p.num_sms * blocks_per_sm((const void*)k_chain_gather), kThreads, 0, s, d,
+                 bt, l);
       p.launches += 1;
     }
+    // plain stream order (no programmatic overlap with its neighbours): the
+    // gather is the stage the measurement hooks time on their own
     k_gather<<<grid, kThreads, 0, s>>>(d, bt);
     p.launches += 1;
   }
   p.enter(8);
-  k_records<<<sgrid, kThreads, 0, s>>>(d);
-  k_sweep<<<sgrid, kThreads, 0, s>>>(d);
+  launch_pdl(k_records, sgrid, kThreads, 0, s, d);
+  launch_pdl(k_sweep, sgrid, kThreads, 0, s, d);
   p.launches += 2;
 }
 
@@ -2033,6 +2083,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   h->drain_first = 0;
   h->latched = ALTO_OK;
   h->profiling = false;
+  h->profile_mode = ALTO_PROFILE_STAGES;
   h->last_stream = s;
   h->prof_pushes = 0;
   h->launches = 0;
@@ -2274,11 +2325,11 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
   p.stage = on_stage;
   p.stage_ctx = &ck;
   ck.clk.enter(0);
-  k_begin<<<1, 1, 0, s>>>(d.ctl, n);
+  launch_pdl(k_begin, 1, 1, 0, s, d.ctl, n);
   p.launches += 1;
   if (n > 0) enqueue_batch(p, bt);
   else p.enter(8);
-  k_end<<<1, 1, 0, s>>>(d.ctl, n);
+  launch_pdl(k_end, 1, 1, 0, s, d.ctl, n);
   p.launches += 1;
   p.enter(ALTO_NUM_STAGES);
   ck.clk.finish();
@@ -2308,7 +2359,7 @@ alto_status alto_agg_drain(alto_agg_t* h, void* stream, alto_drain* out) {
   out->payload = h->d.out_pay;
   out->n_topk = (int64_t)c.topk_count;
   out->topk = h->d.out_topk;
-  k_drain_reset<<<1, 1, 0, s>>>(h->d.ctl);
+  launch_pdl(k_drain_reset, 1, 1, 0, s, h->d.ctl);
   if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
   return ALTO_OK;
 }
@@ -2330,6 +2381,7 @@ alto_status alto_agg_profile(alto_agg_t* h, int enable) {
     if (h->last_stream || h->pushed) cudaStreamSynchronize(h->last_stream);
     collect_profile(h);
     h->profiling = true;
+    h->profile_mode = (enable == ALTO_PROFILE_GATHER) ? ALTO_PROFILE_GATHER : ALTO_PROFILE_STAGES;
     h->prof_pushes = 0;
     h->launches = 0;
     for (int i = 0; i < ALTO_NUM_STAGES; ++i) {
@@ -2573,6 +2625,7 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
 // the per-batch accumulators, the completion masks, the leaf-slot set, the
 // free-chunk stacks and the sort histogram.
 __global__ void k_na_reset(Dev d, u32* hist, u64 T, u64 PS, u32 nmax) {
+  pdl_enter();
   const u64 tid = (u64)blockIdx.x * blockDim.x + threadIdx.x;
   const u64 stride = (u64)gridDim.x * blockDim.x;
   if (tid == 0) {
@@ -2602,6 +2655,7 @@ __global__ void k_na_reset(Dev d, u32* hist, u64 T, u64 PS, u32 nmax) {
 
 // Counts of the call for the caller: {status, records, payload, top-k pairs}.
 __global__ void k_na_finish(const Ctl* ctl, int64_t* out) {
+  pdl_enter();
   out[0] = ctl->status;
   out[1] = (ctl->status == ALTO_OK) ? (int64_t)ctl->rec_count : 0;
   out[2] = (ctl->status == ALTO_OK) ? (int64_t)ctl->pay_count : 0;
@@ -2674,8 +2728,8 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
   bt.n = n;
   bt.n_payload = (u64)b->n_payload;
 
-  k_na_reset<<<num_sms * 2, kThreads, 0, s>>>(d, st.leaf_sort.hist, st.T, st.PS, nmax);
-  k_begin<<<1, 1, 0, s>>>(d.ctl, n);
+  launch_pdl(k_na_reset, num_sms * 2, kThreads, 0, s, d, st.leaf_sort.hist, st.T, st.PS, nmax);
+  launch_pdl(k_begin, 1, 1, 0, s, d.ctl, n);
   if (n > 0) {
     Pipeline p;
     p.d = d;
@@ -2688,8 +2742,8 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
     p.s = s;
     enqueue_batch(p, bt);
   }
-  k_end<<<1, 1, 0, s>>>(d.ctl, n);
-  k_na_finish<<<1, 1, 0, s>>>(d.ctl, out_counts);
+  launch_pdl(k_end, 1, 1, 0, s, d.ctl, n);
+  launch_pdl(k_na_finish, 1, 1, 0, s, d.ctl, out_counts);
   if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
   return ALTO_OK;
 }

@@ -57,6 +57,16 @@ struct Ctl {
   u64 scan_total[kSites];  // totals written by scans
 };
 
+// Programmatic dependent launch.  Every kernel of the library is launched
+// with programmatic stream serialization and first waits here until its
+// predecessor in the stream has completed and its memory is visible; nothing
+// of a batch reads state before the wait.  No kernel triggers its successor
+// early: the implicit trigger at exit already hides most of the boundary
+// (launch and memory flush), and an early trigger lets the kernel after next
+// take SM slots while two grids still run, which split one-wave grids into a
+// ragged second wave.
+__device__ __forceinline__ void pdl_enter() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // error priority: the class reported when a batch holds several defects
 __device__ __forceinline__ int err_priority(int code) {
   switch (code) {

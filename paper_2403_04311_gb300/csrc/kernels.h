@@ -1,9 +1,29 @@
 // Host-side launch interfaces shared between the library's translation units.
 #pragma once
 
+#include <utility>
+
 #include "common.cuh"
 
 namespace alto {
+
+// Launch with programmatic stream serialization: the kernel may be scheduled
+// while its predecessor finishes and waits for it in pdl_enter().
+template <typename... KArgs, typename... Args>
+inline void launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 struct SortBuffers {
   u32* keys[2];

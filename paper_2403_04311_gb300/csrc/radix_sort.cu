@@ -25,6 +25,7 @@ constexpr int kRadix = 256;
 
 __global__ void __launch_bounds__(256) k_sort_hist(const u32* n_dev, u32 n_cap, const u32* keys,
                                                    int passes, u32* hist, Ctl* ctl) {
+  pdl_enter();
   __shared__ u32 sh[4][kRadix];
   for (int i = threadIdx.x; i < 4 * kRadix; i += blockDim.x) (&sh[0][0])[i] = 0;
   __syncthreads();
@@ -50,6 +51,7 @@ __global__ void __launch_bounds__(256) k_sort_hist(const u32* n_dev, u32 n_cap, 
 
 // Exclusive scan of each pass's 256 digit counts; clears the histogram.
 __global__ void __launch_bounds__(256) k_sort_binbase(u32* hist, u32* bin_base, int passes) {
+  pdl_enter();
   __shared__ u32 s_w[kWarps];
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   for (int p = 0; p < passes; ++p) {
@@ -91,6 +93,7 @@ __global__ void __launch_bounds__(kSortThreads) k_onesweep(const u32* n_dev, u32
                                                            int shift, const u32* bin_base, u64* lb,
                                                            u64 lb_tiles, Ctl* ctl, int site,
                                                            u64 spin_limit) {
+  pdl_enter();
   __shared__ u32 whist[kWarps][kRadix];
   __shared__ u32 s_k[kSortTile];
   __shared__ u32 s_v[kSortTile];
@@ -208,14 +211,14 @@ int sort_pairs(const u32* n_dev, u32 n_cap, int bits, bool vals_identity, SortBu
   u32 tiles_cap = (n_cap + kSortTile - 1) / kSortTile;
   if (tiles_cap == 0) tiles_cap = 1;
   int hist_grid = num_sms * 2;
-  k_sort_hist<<<hist_grid, 256, 0, s>>>(n_dev, n_cap, b.keys[0], passes, b.hist, ctl);
-  k_sort_binbase<<<1, 256, 0, s>>>(b.hist, b.bin_base, passes);
+  launch_pdl(k_sort_hist, hist_grid, 256, 0, s, n_dev, n_cap, b.keys[0], passes, b.hist, ctl);
+  launch_pdl(k_sort_binbase, 1, 256, 0, s, b.hist, b.bin_base, passes);
   u32 g4 = (u32)num_sms * 4u;
   int grid = (int)(tiles_cap < g4 ? tiles_cap : g4);
   int cur = 0;
   for (int p = 0; p < passes; ++p) {
     const u32* vin = (p == 0 && vals_identity) ? nullptr : b.vals[cur];
-    k_onesweep<<<grid, kSortThreads, 0, s>>>(n_dev, n_cap, b.keys[cur], vin, b.keys[cur ^ 1],
+    launch_pdl(k_onesweep, grid, kSortThreads, 0, s, n_dev, n_cap, b.keys[cur], vin, b.keys[cur ^ 1],
                                              b.vals[cur ^ 1], 8 * p, b.bin_base + p * kRadix,
                                              b.lookback, b.lb_tiles, ctl, site_base + p,
                                              spin_limit);

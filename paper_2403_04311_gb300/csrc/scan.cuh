@@ -235,6 +235,7 @@ __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl
 template <class F>
 __global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ctl* ctl, int site,
                                                        u32* exit_ctr, u64 spin_limit) {
+  pdl_enter();
   scan_body(f, st, ctl, site, exit_ctr, spin_limit);
 }
 
@@ -244,6 +245,7 @@ template <class F>
 __global__ void __launch_bounds__(kScanThreads) k_scan3(F f0, F f1, F f2, LookbackState st0,
                                                         LookbackState st1, LookbackState st2,
                                                         Ctl* ctl, int site, u64 spin_limit) {
+  pdl_enter();
   const int y = blockIdx.y;
   const F& f = (y == 0) ? f0 : (y == 1) ? f1 : f2;
   const LookbackState st = (y == 0) ? st0 : (y == 1) ? st1 : st2;
