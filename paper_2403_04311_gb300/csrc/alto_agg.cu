@@ -109,6 +109,20 @@ __device__ __forceinline__ bool no_copy(const Ctl* c) {
 __device__ __forceinline__ u32 gtid() { return blockIdx.x * blockDim.x + threadIdx.x; }
 __device__ __forceinline__ u32 gstride() { return gridDim.x * blockDim.x; }
 
+// A place in a list whose length is the global `counter`, for every lane with
+// `want` (kNone for the others), with one atomic per warp: tens of thousands
+// of single appends to one address a batch serialise in one L2 slice.  All 32
+// lanes of the warp call it together.
+__device__ __forceinline__ u32 warp_take(bool want, u32* counter) {
+  const u32 m = __ballot_sync(0xFFFFFFFFu, want);
+  if (m == 0) return kNone;
+  const int leader = __ffs(m) - 1;
+  u32 base = 0;
+  if ((int)(threadIdx.x & 31) == leader) base = atomicAdd(counter, (u32)__popc(m));
+  base = __shfl_sync(0xFFFFFFFFu, base, leader);
+  return want ? base + __popc(m & lanemask_lt()) : kNone;
+}
+
 // ---------------------------------------------------------------------------
 // open-group hash table (linear probing; a slot index is the entry id)
 // ---------------------------------------------------------------------------
@@ -143,6 +157,11 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
         tab.acc_smx[h] = 0;
         tab.acc_len[h] = 0;
         tab.acc_leaf[h] = make_uint4(0, 0, 0, 0);
+        if (tags && l == tab.leaf_level) {
+          ulonglong2* cb = reinterpret_cast<ulonglong2*>(tab.cbits + 4 * (u64)h);
+          cb[0] = make_ulonglong2(0, 0);
+          cb[1] = make_ulonglong2(0, 0);
+        }
         tab.carry_epoch[h] = 0;
         *inserted = 1;
         return h;
@@ -178,6 +197,21 @@ __device__ bool ps_insert(const Scratch& sc, u32 e, u32 c, u32 ep7, Ctl* ctl) {
   }
   raise_err(ctl, ALTO_ENOSPC);
   return false;
+}
+
+// A leaf slot given twice.  Slots below 256 go through the leaf parent's
+// bitmap, which lives as long as the open group (so a slot repeated in a later
+// batch is caught too) and sits next to the group's other state in L2; the
+// others through the batch-local pair set.  Only for launches after the one
+// that inserted the entry (the insert clears the bitmap).
+__device__ __forceinline__ bool leaf_dup(const Table& tab, const Scratch& sc, u32 e, u32 c, u32 ep7,
+                                         Ctl* ctl) {
+  if (c < 256) {
+    const u64 bit = 1ull << (c & 63);
+    const u64 old = atomicOr((unsigned long long*)&tab.cbits[4 * (u64)e + (c >> 6)], (unsigned long long)bit);
+    return (old & bit) != 0;
+  }
+  return ps_insert(sc, e, c, ep7, ctl);
 }
 
 __device__ __forceinline__ bool chain_differs(const Table& tab, u32 e, const u64* tags, u64 n, u32 rep,
@@ -603,6 +637,7 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
   for (u32 x = gtid(); x < end; x += gstride()) {
     const bool valid = x < ni;
     u32 e = 0, rep = 0, c = 0, f = 0, done = 0, cs = 0, sk = 0;
+    bool first = false;
     if (valid) {
       e = d.sc.up_sort_keys0[x] & d.tab.mask;
       rep = it_rep[x];
@@ -614,8 +649,11 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
       cs = cf & 0x7FFFFFFFu;
       sk = it_skey[x];
       if (chain_differs(d.tab, e, b.tags, n, rep, l)) raise_err(ctl, ALTO_EINCONSIST);
-      if (atomicExch(&d.tab.touch[e], ep) != ep) {
-        const u32 pos = atomicAdd(&ctl->n_segs[l], 1u);
+      first = atomicExch(&d.tab.touch[e], ep) != ep;
+    }
+    {
+      const u32 pos = warp_take(first, &ctl->n_segs[l]);
+      if (first) {
         if (pos < d.cfg.n_max) list[pos] = e;
         d.tab.acc_rep[e] = rep;
       }
@@ -688,22 +726,19 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch b)
       // the chain row and the leaf-slot probe are independent loads: issue both
       // before acting on either
       const bool bad = chain_differs(d.tab, e, b.tags, n, i, L);
-      const bool dup = ps_insert(d.sc, e, c, ep7, ctl);
+      const bool dup = leaf_dup(d.tab, d.sc, e, c, ep7, ctl);
       if (bad) raise_err(ctl, ALTO_EINCONSIST);
       if (dup) raise_err(ctl, ALTO_EDUP);
     }
     const u32 key = valid ? e : kNone;
     const u32 peers = __match_any_sync(0xFFFFFFFFu, key);
+    bool first = false;  // this lane made the entry's first contribution of the batch
     if (__all_sync(0xFFFFFFFFu, peers == (1u << lane))) {
       // every lane its own group (the common case): plain atomics, no reductions
       if (valid) {
         uint4* rec = d.tab.acc_leaf + e;
         const u64 old = atomicAdd((unsigned long long*)&rec->x, (1ull << 40) | len);
-        if (old == 0) {
-          const u32 pos = atomicAdd(&ctl->n_segs[L], 1u);
-          if (pos < d.cfg.n_max) list[pos] = e;
-          d.tab.acc_rep[e] = i;
-        }
+        first = old == 0;
         atomicMax(&rec->z, c + 1);
         atomicMax(&rec->w, i + 1);
         if (f) {
@@ -712,37 +747,38 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch b)
         }
         if (scores) atomicMax(&d.tab.acc_smx[e], sk);
       }
-      continue;
-    }
-    const int leader = __ffs(peers) - 1;
-    const u32 cnt = __popc(peers);
-    const u32 m1 = __reduce_max_sync(peers, valid ? c + 1 : 0u);
-    const u32 cs1 = __reduce_max_sync(peers, valid ? i + 1 : 0u);
-    const u32 lsum = __reduce_add_sync(peers, len);
-    const u32 anyf = __reduce_or_sync(peers, f);
-    if (valid && lane == leader) {
-      // one returning atomic per group and warp: leaves and payload together
-      uint4* rec = d.tab.acc_leaf + e;
-      const u64 old = atomicAdd((unsigned long long*)&rec->x, ((unsigned long long)cnt << 40) | lsum);
-      if (old == 0) {
-        const u32 pos = atomicAdd(&ctl->n_segs[L], 1u);
-        if (pos < d.cfg.n_max) list[pos] = e;
-        d.tab.acc_rep[e] = i;
+    } else {
+      const int leader = __ffs(peers) - 1;
+      const u32 cnt = __popc(peers);
+      const u32 m1 = __reduce_max_sync(peers, valid ? c + 1 : 0u);
+      const u32 cs1 = __reduce_max_sync(peers, valid ? i + 1 : 0u);
+      const u32 lsum = __reduce_add_sync(peers, len);
+      const u32 anyf = __reduce_or_sync(peers, f);
+      if (valid && lane == leader) {
+        // one returning atomic per group and warp: leaves and payload together
+        uint4* rec = d.tab.acc_leaf + e;
+        const u64 old = atomicAdd((unsigned long long*)&rec->x, ((unsigned long long)cnt << 40) | lsum);
+        first = old == 0;
+        atomicMax(&rec->z, m1);
+        atomicMax(&rec->w, cs1);
       }
-      atomicMax(&rec->z, m1);
-      atomicMax(&rec->w, cs1);
-    }
-    if (anyf) {
-      const u32 fmin = __reduce_min_sync(peers, (valid && f) ? c : kNone);
-      const u32 fmax1 = __reduce_max_sync(peers, (valid && f) ? c + 1 : 0u);
-      if (valid && lane == leader && fmax1) {
-        atomicMin(&d.tab.acc_fmin[e], fmin);
-        atomicMax(&d.tab.acc_fmax1[e], fmax1);
+      if (anyf) {
+        const u32 fmin = __reduce_min_sync(peers, (valid && f) ? c : kNone);
+        const u32 fmax1 = __reduce_max_sync(peers, (valid && f) ? c + 1 : 0u);
+        if (valid && lane == leader && fmax1) {
+          atomicMin(&d.tab.acc_fmin[e], fmin);
+          atomicMax(&d.tab.acc_fmax1[e], fmax1);
+        }
+      }
+      if (scores) {
+        const u32 smx = __reduce_max_sync(peers, valid ? sk : 0u);
+        if (valid && lane == leader && smx) atomicMax(&d.tab.acc_smx[e], smx);
       }
     }
-    if (scores) {
-      const u32 smx = __reduce_max_sync(peers, valid ? sk : 0u);
-      if (valid && lane == leader && smx) atomicMax(&d.tab.acc_smx[e], smx);
+    const u32 pos = warp_take(first, &ctl->n_segs[L]);
+    if (first) {
+      if (pos < d.cfg.n_max) list[pos] = e;
+      d.tab.acc_rep[e] = i;
     }
   }
 }
@@ -768,63 +804,69 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
   u32* nx_cseq = d.sc.it_cseq[in_set ^ 1];
   u32* nx_skey = d.sc.it_skey[in_set ^ 1];
   const u64 n = b.n;
-  for (u32 s = gtid(); s < nt; s += gstride()) {
-    const u32 e = list[s] & d.tab.mask;
-    if (receives) chain_sync(d.tab, d.ar, ctl, e);
-    u32 cnt, m1, cs1;
-    u32 blen = 0;
-    if (LEAF) {
-      const uint4 a = d.tab.acc_leaf[e];
-      const u64 cl = ((u64)a.y << 32) | a.x;
-      cnt = (u32)(cl >> 40);
-      blen = (u32)(cl & ((1ull << 40) - 1));
-      m1 = a.z;
-      cs1 = a.w;
-      d.tab.acc_leaf[e] = make_uint4(0, 0, 0, 0);
-    } else {
-      cnt = d.tab.acc_cnt[e];
-      m1 = d.tab.acc_m1[e];
-      cs1 = d.tab.acc_cs1[e];
+  const u32 end = (nt + 31) & ~31u;  // whole warps iterate together
+  for (u32 s = gtid(); s < end; s += gstride()) {
+    const bool valid = s < nt;
+    u32 e = 0, rep = 0, cmax = 0, smn = 0, blen = 0;
+    bool complete = false;
+    if (valid) {
+      e = list[s] & d.tab.mask;
+      if (receives) chain_sync(d.tab, d.ar, ctl, e);
+      u32 cnt, m1, cs1;
+      if (LEAF) {
+        const uint4 a = d.tab.acc_leaf[e];
+        const u64 cl = ((u64)a.y << 32) | a.x;
+        cnt = (u32)(cl >> 40);
+        blen = (u32)(cl & ((1ull << 40) - 1));
+        m1 = a.z;
+        cs1 = a.w;
+        d.tab.acc_leaf[e] = make_uint4(0, 0, 0, 0);
+      } else {
+        cnt = d.tab.acc_cnt[e];
+        m1 = d.tab.acc_m1[e];
+        cs1 = d.tab.acc_cs1[e];
+      }
+      const u32 fmin = d.tab.acc_fmin[e];
+      const u32 fmax1 = d.tab.acc_fmax1[e], smx = d.tab.acc_smx[e];
+      rep = d.tab.acc_rep[e];
+      // reset the accumulators for the next batch
+      d.tab.acc_cnt[e] = 0;
+      d.tab.acc_m1[e] = 0;
+      d.tab.acc_fmin[e] = kNone;
+      d.tab.acc_fmax1[e] = 0;
+      d.tab.acc_cs1[e] = 0;
+      d.tab.acc_smx[e] = 0;
+      if (l > 0 && d.tab.up[e] != b.tags[(u64)(l - 1) * n + rep]) raise_err(ctl, ALTO_EINCONSIST);
+      const u32 last_old = d.tab.last[e];
+      u32 nl = last_old;
+      if (fmax1) {
+        if (fmin + 1 != fmax1) raise_err(ctl, ALTO_ELAST);
+        if (last_old != kNone && last_old != fmin) raise_err(ctl, ALTO_ELAST);
+        if (last_old == kNone) nl = fmin;
+      }
+      const u32 m1n = max(d.tab.maxc1[e], m1);
+      if (nl != kNone && m1n > nl + 1) raise_err(ctl, ALTO_ELAST);
+      const u32 comp = d.tab.completed[e] + cnt;
+      smn = max(d.tab.smax[e], smx);
+      complete = (nl != kNone) && (comp == nl + 1) && (m1n <= nl + 1);
+      d.tab.last[e] = nl;
+      d.tab.maxc1[e] = m1n;
+      d.tab.completed[e] = comp;
+      d.tab.smax[e] = smn;
+      cmax = cs1 ? cs1 - 1 : 0;
+      if (carry && !complete) {
+        // reserve this batch's leaves at the end of the group's arena vectors
+        const u32 v0 = d.tab.vec_n[2 * (u64)e], v1 = d.tab.vec_n[2 * (u64)e + 1];
+        d.tab.cur[e] = ((u64)v0 << 40) | v1;
+        d.tab.vec_n[2 * (u64)e] = v0 + cnt;
+        d.tab.vec_n[2 * (u64)e + 1] = v1 + blen;
+        d.tab.carry_epoch[e] = ep;
+        d.tab.bstate[e] = make_uint4(ep, 1u, 0u, 0u);
+      }
     }
-    const u32 fmin = d.tab.acc_fmin[e];
-    const u32 fmax1 = d.tab.acc_fmax1[e], smx = d.tab.acc_smx[e];
-    const u32 rep = d.tab.acc_rep[e];
-    // reset the accumulators for the next batch
-    d.tab.acc_cnt[e] = 0;
-    d.tab.acc_m1[e] = 0;
-    d.tab.acc_fmin[e] = kNone;
-    d.tab.acc_fmax1[e] = 0;
-    d.tab.acc_cs1[e] = 0;
-    d.tab.acc_smx[e] = 0;
-    if (l > 0 && d.tab.up[e] != b.tags[(u64)(l - 1) * n + rep]) raise_err(ctl, ALTO_EINCONSIST);
-    const u32 last_old = d.tab.last[e];
-    u32 nl = last_old;
-    if (fmax1) {
-      if (fmin + 1 != fmax1) raise_err(ctl, ALTO_ELAST);
-      if (last_old != kNone && last_old != fmin) raise_err(ctl, ALTO_ELAST);
-      if (last_old == kNone) nl = fmin;
-    }
-    const u32 m1n = max(d.tab.maxc1[e], m1);
-    if (nl != kNone && m1n > nl + 1) raise_err(ctl, ALTO_ELAST);
-    const u32 comp = d.tab.completed[e] + cnt;
-    const u32 smn = max(d.tab.smax[e], smx);
-    const bool complete = (nl != kNone) && (comp == nl + 1) && (m1n <= nl + 1);
-    d.tab.last[e] = nl;
-    d.tab.maxc1[e] = m1n;
-    d.tab.completed[e] = comp;
-    d.tab.smax[e] = smn;
-    const u32 cmax = cs1 ? cs1 - 1 : 0;
-    if (carry && !complete) {
-      // reserve this batch's leaves at the end of the group's arena vectors
-      const u32 v0 = d.tab.vec_n[2 * (u64)e], v1 = d.tab.vec_n[2 * (u64)e + 1];
-      d.tab.cur[e] = ((u64)v0 << 40) | v1;
-      d.tab.vec_n[2 * (u64)e] = v0 + cnt;
-      d.tab.vec_n[2 * (u64)e + 1] = v1 + blen;
-      d.tab.carry_epoch[e] = ep;
-      d.tab.bstate[e] = make_uint4(ep, 1u, 0u, 0u);
-    }
+    const u32 di = warp_take(complete, &ctl->n_done);
+    if (!valid) continue;
     if (complete) {
-      u32 di = atomicAdd(&ctl->n_done, 1u);
       if (di < d.sc.done_cap) {
         d.sc.done_e[di] = e;
         d.sc.done_lvl[di] = (u32)l;
@@ -2150,6 +2192,8 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(d.tab.acc_leaf, uint4, T);
   ALLOC(d.tab.dbase, u64, T);
   ALLOC(d.tab.bstate, uint4, T);
+  ALLOC(d.tab.cbits, u64, 4 * T);
+  d.tab.leaf_level = D - 1;
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
   d.tab.max_probe = (int)std::min<u64>(T, 1u << 16);
@@ -2535,6 +2579,8 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   d.tab.acc_leaf = cv.take<uint4>(T);
   d.tab.dbase = cv.take<u64>(T);
   d.tab.bstate = cv.take<uint4>(T);
+  d.tab.cbits = cv.take<u64>(4 * T);
+  d.tab.leaf_level = D - 1;
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
   d.tab.max_probe = (int)T;

@@ -176,6 +176,8 @@ struct Table {
   u32* par;        // [T] parent entry the completed group was appended to
   u32* cidx;       // [T] its child index in that parent
   u64* app;        // [T] its reserved place there: span index << 40 | payload position
+  u64* cbits;      // [T][4] leaf parents: leaf slots 0..255 seen while the group is open
+  int leaf_level;  // D - 1
   int chain_len;   // D - 1
   u32 mask;        // T - 1
   int kk;          // stride of topk (largest k over levels)

@@ -102,6 +102,20 @@ def test_bruteforce_streams_on_device():
         assert_same(o, g, f"{depth} {po} {so} {kk} {cuts}")
 
 
+def test_leaf_slot_repeated_in_a_later_batch():
+    """A leaf slot below 256 given again in a later batch while its group is
+    still open: the oracle and the device both report EDUP in that batch."""
+    for c in (0, 5, 255):
+        frags = [(((9, 0, 1), (90, c, 0)), [1], 0.0),
+                 (((9, 0, 1), (90, c, 0)), [2], 0.0),
+                 (((9, 0, 1), (90, c + 1, 1)), [3], 0.0)]
+        batches = [to_batch(p, 2, False) for p in split(frags, [1, 2])]
+        o = run_oracle_batches(2, [0, 1], [0, 0], [0, 0], batches)
+        _, g = run_gpu_batches(2, [0, 1], [0, 0], [0, 0], batches, small_caps(4, 16, 2))
+        assert [d.status for d in o] == [alto.OK, alto.EDUP]
+        assert [d[0] for d in g] == [alto.OK, alto.EDUP], c
+
+
 def test_nan_score_is_einval():
     frags = tree_fragments([2], score_fn=lambda k: float("nan") if k == 1 else 1.0)
     b = to_batch(frags, 2, True)
