@@ -162,7 +162,6 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
           cb[0] = make_ulonglong2(0, 0);
           cb[1] = make_ulonglong2(0, 0);
         }
-        tab.carry_epoch[h] = 0;
         *inserted = 1;
         return h;
       }
@@ -259,6 +258,77 @@ __device__ void free_chunk(const Arena& ar, Ctl* ctl, int j, u32 chunk) {
   if (chunk == kNone) return;
   int pos = atomicAdd(&ctl->top[j], 1);
   if ((u64)pos < ar.stack_cap[j]) ar.stack[ar.stack_off[j] + (u64)pos] = chunk;
+}
+
+// Chunks for the growth of each requesting lane's two vectors of entry e:
+// every class that starts in [old, new) of a vector (vector 0 holds two int32
+// per leaf).  One free-stack atomic per chunk class and warp; a stack may go
+// negative, and k_check clears that before anything is freed.  All 32 lanes
+// call it together.
+__device__ void warp_grow(const Table& tab, const Arena& ar, Ctl* ctl, bool want, u32 e, u64 old0,
+                          u64 new0, u64 old1, u64 new1) {
+  const int lane = threadIdx.x & 31;
+  int jf[kVecs], jl[kVecs];
+  const u64 olds[kVecs] = {old0, old1}, news[kVecs] = {new0, new1};
+#pragma unroll
+  for (int v = 0; v < kVecs; ++v) {
+    jf[v] = kNumChunks;
+    jl[v] = -1;
+    if (want && news[v] > olds[v]) {
+      jf[v] = (olds[v] == 0) ? 0 : chunk_of(olds[v] - 1) + 1;
+      jl[v] = chunk_of(news[v] - 1);
+      if (jl[v] >= kNumChunks) {
+        raise_err(ctl, ALTO_ENOSPC);
+        jl[v] = kNumChunks - 1;
+      }
+    }
+  }
+  const int lo = __reduce_min_sync(0xFFFFFFFFu, min(jf[0], jf[1]));
+  const int hi = __reduce_max_sync(0xFFFFFFFFu, max(jl[0], jl[1]));
+  u64 got = 0;
+  for (int j = lo; j <= hi; ++j) {
+    const bool w0 = j >= jf[0] && j <= jl[0];
+    const bool w1 = j >= jf[1] && j <= jl[1];
+    const u32 m0 = __ballot_sync(0xFFFFFFFFu, w0), m1 = __ballot_sync(0xFFFFFFFFu, w1);
+    const u32 cnt = __popc(m0) + __popc(m1);
+    if (cnt == 0) continue;
+    const int leader = __ffs(m0 | m1) - 1;
+    int old = 0;
+    u32 avail = 0;
+    unsigned long long bump = 0;
+    if (lane == leader) {
+      old = atomicSub(&ctl->top[j], (int)cnt);
+      avail = (old <= 0) ? 0u : min((u32)old, cnt);
+      if (cnt > avail)
+        bump = atomicAdd((unsigned long long*)&ctl->bump, (unsigned long long)(cnt - avail) * chunk_size(j));
+    }
+    old = __shfl_sync(0xFFFFFFFFu, old, leader);
+    avail = __shfl_sync(0xFFFFFFFFu, avail, leader);
+    bump = __shfl_sync(0xFFFFFFFFu, bump, leader);
+    const u32 lt = lanemask_lt();
+#pragma unroll
+    for (int v = 0; v < kVecs; ++v) {
+      if (!(v == 0 ? w0 : w1)) continue;
+      const u32 r = (v == 0) ? __popc(m0 & lt) : __popc(m0) + __popc(m1 & lt);
+      u32 c;
+      if (r < avail) {
+        c = ar.stack[ar.stack_off[j] + (u64)(old - 1 - (int)r)];
+      } else {
+        const u64 o = bump + (u64)(r - avail) * chunk_size(j);
+        if (o + chunk_size(j) > ar.elems) {
+          raise_err(ctl, ALTO_ENOSPC);
+          c = kNone;
+        } else {
+          c = (u32)o;
+        }
+      }
+      tab.dir[((u64)e * kVecs + v) * kNumChunks + j] = c;
+      if (c != kNone) got += chunk_size(j);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) got += __shfl_xor_sync(0xFFFFFFFFu, got, o);
+  if (lane == 0 && got) atomicAdd((unsigned long long*)&ctl->arena_used, (unsigned long long)got);
 }
 
 // ---------------------------------------------------------------------------
@@ -808,7 +878,8 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
   for (u32 s = gtid(); s < end; s += gstride()) {
     const bool valid = s < nt;
     u32 e = 0, rep = 0, cmax = 0, smn = 0, blen = 0;
-    bool complete = false;
+    bool complete = false, grows = false;
+    u64 gv[4] = {0, 0, 0, 0};  // old and new element counts of the two arena vectors
     if (valid) {
       e = list[s] & d.tab.mask;
       if (receives) chain_sync(d.tab, d.ar, ctl, e);
@@ -860,10 +931,16 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
         d.tab.cur[e] = ((u64)v0 << 40) | v1;
         d.tab.vec_n[2 * (u64)e] = v0 + cnt;
         d.tab.vec_n[2 * (u64)e + 1] = v1 + blen;
-        d.tab.carry_epoch[e] = ep;
         d.tab.bstate[e] = make_uint4(ep, 1u, 0u, 0u);
+        grows = true;
+        gv[0] = 2 * (u64)v0;
+        gv[1] = 2 * ((u64)v0 + cnt);
+        gv[2] = v1;
+        gv[3] = (u64)v1 + blen;
       }
     }
+    // the leaf level allocates the chunks of the reserved growth right here
+    if (LEAF && carry) warp_grow(d.tab, d.ar, ctl, grows, e, gv[0], gv[1], gv[2], gv[3]);
     const u32 di = warp_take(complete, &ctl->n_done);
     if (!valid) continue;
     if (complete) {
@@ -1040,6 +1117,9 @@ __global__ void k_check(Dev d) {
     raise_err(ctl, ALTO_ENOSPC);
     ctl->skip_dense = 1;
   }
+  // allocations of the level kernels may have taken a free stack below zero
+  for (int j = 0; j < kNumChunks; ++j)
+    if (ctl->top[j] < 0) ctl->top[j] = 0;
 }
 
 // Payload lengths of the leaves in sorted order, scanned: a leaf's position
@@ -1058,17 +1138,17 @@ struct LenScan {
   __device__ void total(Ctl*, u64 t) const { out_scan[size(nullptr)] = t; }
 };
 
-// Chunks for the arena ranges reserved by this batch's open CONCAT groups.
-// A block counts its requests per size class in shared memory and takes them
-// from the class's free stack (or the bump allocator) with one atomic each.
+// TOPK leaf level: chunks for the arena ranges reserved by this batch's open
+// CONCAT groups (the reduce recorded their old sizes per segment).  A block
+// counts its requests per size class in shared memory and takes them from the
+// class's free stack (or the bump allocator) with one atomic each.  (Without
+// TOPK the leaf finalize allocates these itself, per warp.)
 constexpr int kMaxReq = 8;
 
-template <bool ATOMIC>
 __global__ void __launch_bounds__(kThreads) k_carry_alloc(Dev d) {
   pdl_enter();
   Ctl* ctl = d.ctl;
   if (no_copy(ctl)) return;
-  const u32 ep = ctl->epoch;
   __shared__ u32 s_cnt[kNumChunks];
   __shared__ int s_old[kNumChunks];
   __shared__ u32 s_avail[kNumChunks];
@@ -1086,21 +1166,11 @@ __global__ void __launch_bounds__(kThreads) k_carry_alloc(Dev d) {
     u32 rr[kMaxReq];
     bool want = false;
     u64 old0 = 0, old1 = 0;
-    if (s < nseg) {
-      if (ATOMIC) {
-        e = d.sc.leaf_seg_start[s] & d.tab.mask;
-        want = d.tab.carry_epoch[e] == ep;
-        if (want) {
-          const u64 cu = d.tab.cur[e];
-          old0 = cu >> 40;
-          old1 = cu & ((1ull << 40) - 1);
-        }
-      } else if (d.sc.seg_carry[s] == 1u) {
-        e = d.sc.leaf_keys[d.sc.leaf_seg_start[s]] & d.tab.mask;
-        want = true;
-        old0 = d.sc.seg_vb0[s];
-        old1 = d.sc.seg_vb1[s];
-      }
+    if (s < nseg && d.sc.seg_carry[s] == 1u) {
+      e = d.sc.leaf_keys[d.sc.leaf_seg_start[s]] & d.tab.mask;
+      want = true;
+      old0 = d.sc.seg_vb0[s];
+      old1 = d.sc.seg_vb1[s];
     }
     if (want) {
       for (int vec = 0; vec < kVecs; ++vec) {
@@ -1296,29 +1366,46 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch b) {
         copy = true;
       }
     }
-    // the warp copies the tokens of its arena-bound fragments one after another
+    // arena-bound fragments: eight lanes copy one span, four spans at a time,
+    // the first 64 elements' loads all issued before the stores (as in the
+    // gather); the span's first chunk is looked up once, elements past it
+    // one by one
     u32 pending = __ballot_sync(0xFFFFFFFFu, copy);
+    const int sub = lane & 7, grp = lane >> 3;
     while (pending) {
-      const int src = __ffs(pending) - 1;
-      pending &= pending - 1;
+      u32 pm = pending;  // this group's span: the grp-th pending lane
+      for (int k = 0; k < grp; ++k) pm &= pm - 1;
+      for (int k = 0; k < 4; ++k) pending &= pending - 1;
+      const int src = pm ? __ffs(pm) - 1 : 0;
       const u32 se = __shfl_sync(0xFFFFFFFFu, e, src);
       const u32 so = __shfl_sync(0xFFFFFFFFu, o0, src);
-      const u32 sl = __shfl_sync(0xFFFFFFFFu, len, src);
+      const u32 sl0 = __shfl_sync(0xFFFFFFFFu, len, src);
       const u64 sp = __shfl_sync(0xFFFFFFFFu, ppos, src);
-      // positions before the end of the first chunk need no directory lookup
+      const u32 sl = pm ? sl0 : 0u;
+      if (sl == 0) continue;
       const int j1 = chunk_of(sp);
-      const u64 cend = chunk_start(j1) + chunk_size(j1);
+      const u64 room = chunk_start(j1) + chunk_size(j1) - sp;
       bool ok1;
       const u64 a1 = vec_addr(d.tab, se, 1, sp, &ok1);
-      for (u32 k = lane; k < sl; k += 32) {
-        const int32_t v = b.pay[(u64)so + k];
-        if (sp + k < cend) {
-          if (ok1) d.ar.pool[a1 + k] = v;
-        } else {
-          bool ok;
-          const u64 a = vec_addr(d.tab, se, 1, sp + k, &ok);
-          if (ok) d.ar.pool[a] = v;
-        }
+      const u32 n1 = ok1 ? ((room < sl) ? (u32)room : sl) : 0u;
+      const int32_t* src_p = b.pay + so;
+      int32_t* dst_p = d.ar.pool + a1;
+      int32_t v[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const u32 k = sub + 8 * q;
+        v[q] = (k < n1) ? src_p[k] : 0;
+      }
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const u32 k = sub + 8 * q;
+        if (k < n1) dst_p[k] = v[q];
+      }
+      for (u32 k = 64 + sub; k < n1; k += 8) dst_p[k] = src_p[k];
+      for (u32 k = n1 + sub; k < sl; k += 8) {
+        bool ok;
+        const u64 a = vec_addr(d.tab, se, 1, sp + k, &ok);
+        if (ok) d.ar.pool[a] = src_p[k];
       }
     }
   }
@@ -1999,19 +2086,18 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   if (M >= 0) {
     p.enter(5);
     if (leaf_sorted) {
-      launch_pdl(k_carry_alloc<false>, sgrid, kThreads, 0, s, d);
+      launch_pdl(k_carry_alloc, sgrid, kThreads, 0, s, d);
       launch_pdl(k_fix_tops, 1, 32, 0, s, d.ctl);
       launch_pdl(k_carry_copy, grid, kThreads, 0, s, d, bt);
       p.enter(6);
       launch_pdl(k_dense_batch, grid, kThreads, 0, s, d, bt);
     } else {
-      launch_pdl(k_carry_alloc<true>, sgrid, kThreads, 0, s, d);
-      launch_pdl(k_fix_tops, 1, 32, 0, s, d.ctl);
+      // the leaf finalize already allocated the carried leaves' chunks
       p.enter(6);
       launch_pdl(k_leaf_place, grid, kThreads, 0, s, d, bt);
     }
     launch_pdl(k_dense_arena<true>, sgrid, kThreads, 0, s, d);
-    p.launches += leaf_sorted ? 5 : 4;
+    p.launches += leaf_sorted ? 5 : 2;
     if (chain) {
       launch_pdl(k_dense_arena<false>, sgrid, kThreads, 0, s, d);
       p.launches += 1;
@@ -2187,7 +2273,6 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(d.tab.acc_smx, u32, T);
   ALLOC(d.tab.acc_rep, u32, T);
   ALLOC(d.tab.acc_len, u32, T);
-  ALLOC(d.tab.carry_epoch, u32, T);
   ALLOC(d.tab.cur, u64, T);
   ALLOC(d.tab.acc_leaf, uint4, T);
   ALLOC(d.tab.dbase, u64, T);
@@ -2574,7 +2659,6 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   d.tab.acc_smx = cv.take<u32>(T);
   d.tab.acc_rep = cv.take<u32>(T);
   d.tab.acc_len = cv.take<u32>(T);
-  d.tab.carry_epoch = cv.take<u32>(T);
   d.tab.cur = cv.take<u64>(T);
   d.tab.acc_leaf = cv.take<uint4>(T);
   d.tab.dbase = cv.take<u64>(T);

@@ -163,7 +163,6 @@ struct Table {
   u32* acc_smx;    // [T] largest score key of complete children
   u32* acc_rep;    // [T] a representative fragment
   u32* acc_len;    // [T] payload elements of this batch's leaves (leaf level)
-  u32* carry_epoch;// [T] epoch in which the entry's leaves go to its arena vectors
   u64* cur;        // [T] arena cursor: leaves << 40 | payload elements
   uint4* acc_leaf; // [T] leaf level, one sector per group: {leaves << 40 | payload
                    //     elements (as u64 in .x/.y), max child + 1, max seq + 1}
