@@ -281,10 +281,11 @@ def main():
     n_payload_step = int(d.payload.numel())
 
     # ---- timed region: device-resident inputs -------------------------------
-    # CUDA events on the push stream around the gather only (two per push), so
-    # that every other kernel boundary runs as it does without measurement
+    # CUDA events on the push stream around the two heaviest kernels only (the
+    # leaf accumulate and the gather, four events a push), so that every other
+    # kernel boundary runs as it does without measurement
     sampler = ClockSampler(local_rank)
-    agg.profile(alto.PROFILE_GATHER)
+    agg.profile(alto.PROFILE_HOT)
     barrier()
     torch.cuda.synchronize()
     sampler.start()
@@ -311,19 +312,33 @@ def main():
     alg_bytes = algorithmic_bytes(s)
     hbm_gbs, peak_kind = peaks()
 
-    # roofline of k_gather: the payload copy, whose bytes are all algorithmic
-    # (4 read + 4 written per emitted element), timed in the timed region
+    # rooflines of the two heaviest kernels, timed in the timed region, per
+    # launch (one launch each per push); the line's `roofline` is the one with
+    # the larger device time.  Algorithmic bytes per launch:
+    #   k_leaf_accumulate: per fragment its D tags, one payload offset, its
+    #     table slot (written by the ingest) and its score when scored;
+    #   k_gather: 4 bytes read + 4 written per emitted payload element.
     pushes = max(1, prof["pushes"])
-    gather_bytes = 8.0 * n_payload_step / s.n_batches
-    per_launch_ms = prof["stage_ms"]["gather"] / pushes
-    achieved = gather_bytes / (per_launch_ms / 1e3) / 1e9 if per_launch_ms > 0 else 0.0
-    traffic = None
+    frag_bytes = 8.0 * s.depth + 4.0 + 4.0 + (4.0 if s.score is not None else 0.0)
+    kernels = {
+        "k_leaf_accumulate": (frag_bytes * s.n / s.n_batches, prof["stage_ms"]["leaf_accumulate"] / pushes),
+        "k_gather": (8.0 * n_payload_step / s.n_batches, prof["stage_ms"]["gather"] / pushes),
+    }
+    traffic_all = {}
     tf = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tf):
         try:
-            traffic = json.load(open(tf)).get("k_gather")
+            traffic_all = json.load(open(tf))
         except Exception:
-            traffic = None
+            traffic_all = {}
+    rooflines = {}
+    for kname, (kbytes, kms) in kernels.items():
+        ach = kbytes / (kms / 1e3) / 1e9 if kms > 0 else 0.0
+        rooflines[kname] = {"bound": "hbm", "kernel": kname, "achieved": ach, "peak": hbm_gbs,
+                            "unit": "GB/s", "frac": ach / hbm_gbs, "peak_kind": peak_kind,
+                            "traffic": traffic_all.get(kname), "ms_per_launch": kms,
+                            "algorithmic_bytes_per_launch": kbytes}
+    dominant = max(kernels, key=lambda k: kernels[k][1])
 
     if args.max_batches > 0:
         # profiling runs stop here: the truncated stream cannot be replayed on
@@ -432,9 +447,8 @@ def main():
         "algorithmic_gbps": alg_bytes * world * args.steps / (ms / 1e3) / 1e9,
         "hbm_frac_path": alg_bytes * args.steps / (ms / 1e3) / 1e9 / hbm_gbs,
         "p50_batch_latency_us": p50, "p99_batch_latency_us": p99,
-        "roofline": {"bound": "hbm", "kernel": "k_gather", "achieved": achieved, "peak": hbm_gbs,
-                     "unit": "GB/s", "frac": achieved / hbm_gbs, "peak_kind": peak_kind,
-                     "traffic": traffic},
+        "roofline": rooflines[dominant],
+        "rooflines": rooflines,
         "stage_ms_per_step": stage_ms,
         "stage_note": f"separate pass of {args.profile_steps} step(s), an event at every stage boundary",
         "largest_stage": dom,

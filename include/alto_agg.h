@@ -208,23 +208,24 @@ alto_status alto_agg_stats(alto_agg_t* h, void* stream, int64_t* open_groups,
 
 /* Measurement hooks.  The paper has no counterpart: they exist so that the
  * benchmark can time the pipeline's stages on the device while it runs.
- * With profiling on, every push records a CUDA event at each stage boundary
- * on its stream; alto_agg_profile_read synchronises the handle's last push
+ * With profiling on, every push records CUDA events at stage boundaries on
+ * its stream; alto_agg_profile_read synchronises the handle's last push
  * stream and sums the elapsed times.  Stages, in push order:
- *   0 ingest (validate, table lookup, leaf-slot check)   1 leaf sort
- *   2 leaf segments + reduce                             3 upper levels
- *   4 emission order + offsets                            5 arena carry-over
- *   6 dense child placement + length scan                 7 payload gather
- *   8 records, frees, table sweep
+ *   0 ingest (validate, table lookup)      1 leaf sort (TOPK leaf level)
+ *   2 leaf accumulate (or segments+reduce) 3 leaf finalize
+ *   4 upper levels                         5 emission order + offsets
+ *   6 arena carry-over (TOPK leaf level)   7 dense child placement + length scan
+ *   8 payload gather                       9 records, frees, table sweep
  * `launches` counts every kernel the pushes launched (also when profiling is
  * off).  enable = ALTO_PROFILE_STAGES (1) records an event at every stage
- * boundary; ALTO_PROFILE_GATHER (2) records only the two around the payload
- * gather (stage 7), so that the other kernel boundaries run as without
- * profiling; either starts a fresh count.  0 stops recording events. */
-#define ALTO_NUM_STAGES 9
+ * boundary; ALTO_PROFILE_HOT (2) records only the events around the two
+ * heaviest kernels, the leaf accumulate (stage 2) and the payload gather
+ * (stage 8), so that the other kernel boundaries run as without profiling;
+ * either starts a fresh count.  0 stops recording events. */
+#define ALTO_NUM_STAGES 10
 #define ALTO_PROFILE_OFF 0
 #define ALTO_PROFILE_STAGES 1
-#define ALTO_PROFILE_GATHER 2
+#define ALTO_PROFILE_HOT 2
 typedef struct alto_profile {
   int64_t pushes;                          /* pushes since the last enable */
   int64_t launches;                        /* kernels those pushes launched */

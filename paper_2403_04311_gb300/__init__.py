@@ -11,7 +11,7 @@ from ._binding import (  # noqa: F401
     alto_drain, alto_agg_create, alto_agg_push_batch, alto_agg_drain, alto_agg_stats,
     alto_agg_destroy, alto_agg_profile, alto_agg_profile_read, alto_agg_oneshot_noalloc,
     load_library, make_config,
-    STAGE_NAMES, PROFILE_OFF, PROFILE_STAGES, PROFILE_GATHER,
+    STAGE_NAMES, PROFILE_OFF, PROFILE_STAGES, PROFILE_HOT,
 )
 from ._build import build  # noqa: F401
 from .device_batches import DeviceBatch, to_device  # noqa: F401

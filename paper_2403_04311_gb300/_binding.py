@@ -76,9 +76,9 @@ class alto_drain(ctypes.Structure):
     ]
 
 
-NUM_STAGES = 9
-STAGE_NAMES = ("ingest", "leaf_sort", "leaf_reduce", "upper_levels", "emit_order", "carry_over",
-               "dense_place", "gather", "records")
+NUM_STAGES = 10
+STAGE_NAMES = ("ingest", "leaf_sort", "leaf_accumulate", "leaf_finalize", "upper_levels",
+               "emit_order", "carry_over", "dense_place", "gather", "records")
 
 
 class alto_profile(ctypes.Structure):
@@ -210,11 +210,12 @@ def alto_agg_oneshot_noalloc(cfg, batch, out_records, cap_records, out_payload, 
         ctypes.c_void_p(out_counts), ctypes.c_void_p(stream))
 
 
-PROFILE_OFF, PROFILE_STAGES, PROFILE_GATHER = 0, 1, 2
+PROFILE_OFF, PROFILE_STAGES, PROFILE_HOT = 0, 1, 2
 
 
 def alto_agg_profile(h, enable) -> int:
-    """enable: False/0 off, True/1 every stage boundary, 2 the gather stage only."""
+    """enable: False/0 off, True/1 every stage boundary, 2 the leaf accumulate
+    and gather stages only."""
     mode = PROFILE_STAGES if enable is True else int(enable)
     return load_library().alto_agg_profile(h, mode)
 

@@ -1842,7 +1842,7 @@ struct alto_agg {
   int latched;
   // measurement hooks
   bool profiling;
-  int profile_mode;  // ALTO_PROFILE_STAGES or ALTO_PROFILE_GATHER
+  int profile_mode;  // ALTO_PROFILE_STAGES or ALTO_PROFILE_HOT
   cudaStream_t last_stream;
   int64_t prof_pushes;
   int64_t launches;
@@ -1872,14 +1872,15 @@ struct StageClock {
     }
     return e;
   }
-  // mark the start of stage `st` (stages must be entered in order); in gather
-  // mode only the boundaries around the gather stage get an event
+  // mark the start of stage `st` (stages must be entered in order); in the hot
+  // mode only the boundaries around the leaf accumulate and the gather get an
+  // event
   void enter(int st) {
     if (!h->profiling) return;
     while ((int)ev.size() <= st) {
       const int bnd = (int)ev.size();
       cudaEvent_t e = nullptr;
-      if (h->profile_mode == ALTO_PROFILE_STAGES || bnd == 7 || bnd == 8) {
+      if (h->profile_mode == ALTO_PROFILE_STAGES || bnd == 2 || bnd == 3 || bnd == 8 || bnd == 9) {
         e = take();
         if (e) cudaEventRecord(e, s);
       }
@@ -2004,13 +2005,15 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     p.launches += 2;
   } else {
     // leaf level without TOPK: accumulate into the table in arrival order
+    // (plain stream order: the measurement hooks time this kernel on its own)
     p.enter(2);
-    launch_pdl(k_leaf_accumulate, grid, kThreads, 0, s, d, bt);
+    k_leaf_accumulate<<<grid, kThreads, 0, s>>>(d, bt);
+    p.enter(3);
     launch_pdl(k_up_finalize<true>, sgrid, kThreads, 0, s, d, bt, D - 1, set);
     p.launches += 2;
   }
   site += 5;
-  p.enter(3);
+  p.enter(4);
   // an atomic finalize also looks up the parent groups of the items it emits
   bool looked_up = !leaf_sorted;
   for (int l = D - 2; l >= 0; --l) {
@@ -2043,7 +2046,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     p.launches += 2;
   }
   // emission order
-  p.enter(4);
+  p.enter(5);
   {
     RankScan f{d.sc.mask, d.sc.prefix, &d.ctl->n};
     launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site++, spin, s);
@@ -2084,16 +2087,16 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   launch_pdl(k_check, 1, 1, 0, s, d);
   p.launches += 1;
   if (M >= 0) {
-    p.enter(5);
+    p.enter(6);
     if (leaf_sorted) {
       launch_pdl(k_carry_alloc, sgrid, kThreads, 0, s, d);
       launch_pdl(k_fix_tops, 1, 32, 0, s, d.ctl);
       launch_pdl(k_carry_copy, grid, kThreads, 0, s, d, bt);
-      p.enter(6);
+      p.enter(7);
       launch_pdl(k_dense_batch, grid, kThreads, 0, s, d, bt);
     } else {
       // the leaf finalize already allocated the carried leaves' chunks
-      p.enter(6);
+      p.enter(7);
       launch_pdl(k_leaf_place, grid, kThreads, 0, s, d, bt);
     }
     launch_pdl(k_dense_arena<true>, sgrid, kThreads, 0, s, d);
@@ -2106,7 +2109,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     launch_scan(p.lbs, p.num_sms, d.ctl, fd, d.cfg.dense_cap, site++, spin, s);
     launch_pdl(k_check2, 1, 1, 0, s, d);
     p.launches += 2;
-    p.enter(7);
+    p.enter(8);
     // levels below M hand their concatenations up, deepest first
     for (int l = D - 1; chain && l > M; --l) {
       launch_pdl(k_chain_gather, p.num_sms * blocks_per_sm((const void*)k_chain_gather), kThreads, 0, s, d,
@@ -2118,7 +2121,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     k_gather<<<grid, kThreads, 0, s>>>(d, bt);
     p.launches += 1;
   }
-  p.enter(8);
+  p.enter(9);
   launch_pdl(k_records, sgrid, kThreads, 0, s, d);
   launch_pdl(k_sweep, sgrid, kThreads, 0, s, d);
   p.launches += 2;
@@ -2457,7 +2460,7 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
   launch_pdl(k_begin, 1, 1, 0, s, d.ctl, n);
   p.launches += 1;
   if (n > 0) enqueue_batch(p, bt);
-  else p.enter(8);
+  else p.enter(9);
   launch_pdl(k_end, 1, 1, 0, s, d.ctl, n);
   p.launches += 1;
   p.enter(ALTO_NUM_STAGES);
@@ -2510,7 +2513,7 @@ alto_status alto_agg_profile(alto_agg_t* h, int enable) {
     if (h->last_stream || h->pushed) cudaStreamSynchronize(h->last_stream);
     collect_profile(h);
     h->profiling = true;
-    h->profile_mode = (enable == ALTO_PROFILE_GATHER) ? ALTO_PROFILE_GATHER : ALTO_PROFILE_STAGES;
+    h->profile_mode = (enable == ALTO_PROFILE_HOT) ? ALTO_PROFILE_HOT : ALTO_PROFILE_STAGES;
     h->prof_pushes = 0;
     h->launches = 0;
     for (int i = 0; i < ALTO_NUM_STAGES; ++i) {
