@@ -46,7 +46,7 @@ TOKEN_VOCAB = 50257
 NONE, CONCAT = 0, 1
 S_NONE, S_MAX, S_TOPK = 0, 1, 2
 
-CONFIG_NAMES = ("tiny", "tiny64", "factcheck", "throughput", "tokens", "adversarial")
+CONFIG_NAMES = ("tiny", "tiny64", "factcheck", "throughput", "tokens", "adversarial", "tot")
 
 _U32 = np.uint64(0xFFFFFFFF)
 
@@ -426,6 +426,38 @@ def make_adversarial(n_leaves=64 * 2**20, hot_leaves=2**20, seed=5, batch=2 * 2*
         topk_k=(0,) * 5 + (8,), batch=batch, with_score=True)
 
 
+def make_tot(n_queries=2048, seed=7, batch=65536, iters=3, keep=5, thoughts=(30, 50), evals=3):
+    """Tree-of-Thoughts shaped (Sec. 6.1.2): each query runs `iters`
+    iterations; in iteration i every frontier node (the query itself, then
+    the `keep` best thoughts of each node of the previous iteration: 1, 5, 25
+    nodes) expands into U{30..50} thoughts, and every thought is evaluated
+    `evals` times (the leaves, each with an fp32 score and U{1..16} tokens).
+    Tags, D=3: level 0 = the query's iteration (children: its frontier
+    nodes), level 1 = a frontier node (children: its thoughts; TOPK(keep) by
+    score), level 2 = a thought (children: its evaluations; MAX of the
+    scores, CONCAT of their texts).  Queries start at staggered times; a
+    query's iteration i+1 arrives after its iteration i, and fragments are
+    shuffled within each iteration's window."""
+    rng = np.random.default_rng(seed)
+    fan = [keep ** i for i in range(iters)]                     # frontier nodes per iteration
+    it_counts = np.tile(np.asarray(fan, dtype=np.int64), n_queries)  # level-0 groups: (query, iter)
+    counts = _grow(rng, it_counts, [
+        lambda r, n: r.integers(thoughts[0], thoughts[1] + 1, size=n),
+        lambda r, n: np.full(n, evals, dtype=np.int64)])
+    gidx, cidx = _leaves_of(counts)
+    n = len(gidx[0])
+    g0 = gidx[0]                                   # level-0 group = query * iters + iteration
+    q, it = g0 // iters, g0 % iters
+    start = rng.random(n_queries) * iters          # query start, in iteration windows
+    key = start[q] + it + rng.random(n) * 0.999
+    order = np.argsort(key, kind="stable")
+    lens = rng.integers(1, 17, size=n)
+    return stream_from_leaves(
+        "tot", gidx, cidx, order, lens, rng,
+        payload_op=(NONE, NONE, CONCAT), score_op=(S_NONE, S_TOPK, S_MAX), topk_k=(0, keep, 0),
+        batch=batch, with_score=True, meta={"iters": iters, "keep": keep})
+
+
 def make_stream(name: str, small: bool = False) -> Stream:
     """Full-size stream by name, or a scaled-down stream of the same shape
     (``small=True``) that the CPU oracle finishes in seconds and that still
@@ -447,4 +479,6 @@ def make_stream(name: str, small: bool = False) -> Stream:
     if name == "adversarial":
         return (make_adversarial(n_leaves=3 * 2**16, hot_leaves=2**14, batch=2**14)
                 if small else make_adversarial())
+    if name == "tot":
+        return make_tot(n_queries=12, batch=4096) if small else make_tot()
     raise ValueError(f"unknown stream {name!r}; one of {CONFIG_NAMES}")

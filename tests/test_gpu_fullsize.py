@@ -63,7 +63,7 @@ def run_gpu(s, prefix_batches, drain_every):
     return drains
 
 
-@pytest.mark.parametrize("name", ["tiny", "factcheck", "throughput", "tokens", "adversarial"])
+@pytest.mark.parametrize("name", ["tiny", "factcheck", "throughput", "tokens", "adversarial", "tot"])
 def test_fullsize(name):
     s = make_stream(name)
     sizes = s.batch_sizes

@@ -25,7 +25,7 @@ def small_caps(n, payload, depth, k=8):
                 out_payload_elems=1 << 14, out_topk=4096, max_emit_children=4096)
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny64", "factcheck", "throughput", "tokens", "adversarial"])
+@pytest.mark.parametrize("name", ["tiny", "tiny64", "factcheck", "throughput", "tokens", "adversarial", "tot"])
 @pytest.mark.parametrize("drain_every", [1, 3])
 def test_workloads_small(name, drain_every):
     s = make_stream(name, small=True)

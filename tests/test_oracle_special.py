@@ -106,7 +106,7 @@ def group_table(s: Stream):
     return facts, pid, cid
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny64", "factcheck", "throughput", "tokens", "adversarial"])
+@pytest.mark.parametrize("name", ["tiny", "tiny64", "factcheck", "throughput", "tokens", "adversarial", "tot"])
 def test_invariants_on_workloads(name):
     s = make_stream(name, small=True)
     drains = oracle.run_stream(s, drain_every=2)
