@@ -16,6 +16,8 @@ from dataclasses import dataclass
 
 import numpy as np
 
+from .split_text import split_pieces, split_text  # noqa: F401
+
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "alto_oracle.cpp")
 _LIB = os.path.join(_HERE, "liboracle.so")
