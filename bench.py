@@ -174,6 +174,124 @@ def run_reference(args, s, rank, world):
     return line
 
 
+def run_split(args, rank, world):
+    """split_text (the fragmentation step in front of the aggregator) on 4,096
+    token streams x 24,414 tokens, sentences of U{1..64} tokens closed by a
+    delimiter: one step = one call over all streams (mark, two scans, write)."""
+    import numpy as np
+    from gen import make_split_input
+    si = make_split_input()
+    n_tok, n_src = len(si.tokens), len(si.src_id)
+    if args.impl == "reference":
+        import oracle
+        if rank != 0:
+            return None
+        k = max(1, int(n_src * min(1.0, args.ref_sample / n_tok)))  # streams per step
+        sl = slice(0, k)
+        sub_off = si.tok_off[:k + 1]
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            oracle.split_text(si.src_tags[:, sl], si.src_id[sl], sub_off, si.tokens[:int(sub_off[-1])], si.delims)
+        dt = time.perf_counter() - t0
+        value = int(sub_off[-1]) * args.steps / dt
+        return {"impl": "reference", "metric": "split_text tokens/s", "value": value, "unit": "tokens/s",
+                "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+                "config": {"workload": "split", "streams": n_src, "tokens": n_tok},
+                "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                                 "sample": f"first {k} streams per step, single thread"},
+                "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    import torch
+    import paper_2403_04311_gb300 as alto
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    stream = torch.cuda.current_stream()
+    dev = "cuda"
+    tags_d = torch.as_tensor(si.src_tags.view(np.int64), device=dev)
+    sid_d = torch.as_tensor(si.src_id.view(np.int32), device=dev)
+    off_d = torch.as_tensor(si.tok_off.astype(np.uint32).view(np.int32), device=dev)
+    tok_d = torch.as_tensor(si.tokens, device=dev)
+    cap = n_tok + n_src
+    out_tags = torch.empty(2 * cap, dtype=torch.int64, device=dev)
+    out_off = torch.empty(cap + 1, dtype=torch.int32, device=dev)
+    counts = torch.zeros(2, dtype=torch.int64, device=dev)
+    nbytes = alto.alto_split_scratch_bytes(n_src, n_tok)
+    scratch = torch.empty(nbytes + 256, dtype=torch.uint8, device=dev)
+    a = alto.alto_split_args()
+    a.n_src, a.n_tokens, a.depth_in, a.n_delims = n_src, n_tok, 1, len(si.delims)
+    for i, x in enumerate(si.delims):
+        a.delims[i] = x
+    a.src_tags, a.src_id, a.tok_off, a.tokens = tags_d.data_ptr(), sid_d.data_ptr(), off_d.data_ptr(), tok_d.data_ptr()
+    a.cap_frag, a.out_tags, a.out_off, a.out_counts = cap, out_tags.data_ptr(), out_off.data_ptr(), counts.data_ptr()
+    a.scratch, a.scratch_bytes = (scratch.data_ptr() + 255) & ~255, nbytes
+
+    def step():
+        if alto.alto_split_text(a, stream.cuda_stream) != alto.OK:
+            raise RuntimeError("split_text failed")
+
+    for _ in range(max(args.warmup, 1)):
+        step()
+    torch.cuda.synchronize()
+    st, n_frag = (int(x) for x in counts.cpu().tolist())
+    assert st == alto.OK
+    sampler = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
+    sampler.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    hbm_gbs, peak_kind = peaks()
+    # algorithmic bytes of one call: the tokens and the stream offsets and tags
+    # read, each piece's two tags and offset written
+    alg = 4.0 * n_tok + 4.0 * (n_src + 1) + 8.0 * n_src + 4.0 * n_src + n_frag * (16.0 + 4.0)
+    achieved = alg / (ms / 1e3) / 1e9
+    # end to end: tokens and offsets from pinned host memory, pieces back to the host
+    h_tok = torch.from_numpy(si.tokens).pin_memory()
+    h_off = torch.from_numpy(si.tok_off.astype(np.uint32).view(np.int32)).pin_memory()
+    h_tags = torch.empty(2 * n_frag, dtype=torch.int64).pin_memory()
+    h_poff = torch.empty(n_frag + 1, dtype=torch.int32).pin_memory()
+    torch.cuda.synchronize()
+    x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    x0.record(stream)
+    for _ in range(args.steps):
+        tok_d.copy_(h_tok, non_blocking=True)
+        off_d.copy_(h_off, non_blocking=True)
+        step()
+        h_tags.copy_(out_tags[:2 * n_frag], non_blocking=True)
+        h_poff.copy_(out_off[:n_frag + 1], non_blocking=True)
+    x1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = x0.elapsed_time(x1) / args.steps
+    cpu = None
+    if not args.no_cpu_baseline:
+        import oracle
+        k = 400
+        t0 = time.perf_counter()
+        oracle.split_text(si.src_tags[:, :k], si.src_id[:k], si.tok_off[:k + 1],
+                          si.tokens[:int(si.tok_off[k])], si.delims)
+        dt = time.perf_counter() - t0
+        cpu = {"value": int(si.tok_off[k]) / dt, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": f"first {k} of {n_src} streams ({int(si.tok_off[k])} tokens), single thread"}
+    return {"metric": "split_text tokens/s", "value": n_tok * world / (ms / 1e3), "unit": "tokens/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
+            "data": "synthetic",
+            "config": {"workload": "split", "streams": n_src, "tokens": n_tok, "pieces": n_frag,
+                       "l2": "inputs larger than L2 (no flush)"},
+            "roofline": {"bound": "hbm", "kernel": "split_text (mark, two scans, write)",
+                         "achieved": achieved, "peak": hbm_gbs, "unit": "GB/s",
+                         "frac": achieved / hbm_gbs, "peak_kind": peak_kind, "traffic": None},
+            "gpu_launches": 4 * args.steps, "clocks": clocks,
+            "e2e": {"value": n_tok * world / (e2e_ms / 1e3), "unit": "tokens/s",
+                    "h2d_bytes_per_step": int(4 * n_tok + 4 * (n_src + 1)),
+                    "d2h_bytes_per_step": int(16 * n_frag + 4 * (n_frag + 1))},
+            "cpu_baseline": cpu}
+
+
 def cpu_baseline(s, budget_s=20.0):
     """Oracle fragments/s on a bounded sample (batches in order until the
     budget is spent), one host thread."""
@@ -217,6 +335,12 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.workload == "split":
+        line = run_split(args, rank, world)
+        if rank == 0 and line is not None:
+            print(json.dumps(line), flush=True)
+        return
 
     from gen import make_stream
     s = make_stream(args.workload, small=args.small)

@@ -7,5 +7,5 @@ streams from here.
 """
 from .streams import (  # noqa: F401
     CONCAT, NONE, S_MAX, S_NONE, S_TOPK, TOKEN_VOCAB, Stream, CONFIG_NAMES,
-    make_stream, pack_tags, stream_from_leaves,
+    make_stream, pack_tags, stream_from_leaves, SplitInput, make_split_input,
 )

@@ -458,6 +458,43 @@ def make_tot(n_queries=2048, seed=7, batch=65536, iters=3, keep=5, thoughts=(30,
         batch=batch, with_score=True, meta={"iters": iters, "keep": keep})
 
 
+@dataclass
+class SplitInput:
+    """Token streams for split_text: streams x tokens, sentences of U{1..max_sentence}
+    tokens each closed by one of the delimiter ids, plus each stream's own tags
+    (one level: child s of a single source) and its id at the new level."""
+    tok_off: np.ndarray    # int64 [n_src + 1]
+    tokens: np.ndarray     # int32
+    delims: tuple
+    src_tags: np.ndarray   # uint64 [1, n_src]
+    src_id: np.ndarray     # uint32 [n_src]
+
+
+def make_split_input(n_streams=4096, tokens_per_stream=24414, seed=8, delims=(198, 13), max_sentence=64,
+                     empty_every=0):
+    rng = np.random.default_rng(seed)
+    lens = np.full(n_streams, tokens_per_stream, dtype=np.int64)
+    if empty_every:
+        lens[::empty_every] = 0
+    n = int(lens.sum())
+    tokens = _integers(rng, 0, TOKEN_VOCAB, n).astype(np.int32)
+    # ordinary tokens never collide with a delimiter id
+    dl = np.asarray(delims, dtype=np.int32)
+    hit = np.isin(tokens, dl)
+    tokens[hit] = (tokens[hit] + 1) % TOKEN_VOCAB
+    # a delimiter closes every sentence
+    gaps = rng.integers(1, max_sentence + 1, size=n // 1 + 1)
+    ends = np.cumsum(gaps) - 1
+    ends = ends[ends < n]
+    tokens[ends] = dl[rng.integers(0, len(dl), size=len(ends))]
+    tok_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    src_tags = pack_tags(np.full(n_streams, 9, dtype=np.uint64), np.arange(n_streams, dtype=np.uint64),
+                         (np.arange(n_streams) == n_streams - 1).astype(np.uint64))[None, :]
+    src_id = (rng.permutation(n_streams) + 1000).astype(np.uint32)
+    return SplitInput(tok_off=tok_off, tokens=tokens, delims=tuple(int(x) for x in delims),
+                      src_tags=np.ascontiguousarray(src_tags), src_id=src_id)
+
+
 def make_stream(name: str, small: bool = False) -> Stream:
     """Full-size stream by name, or a scaled-down stream of the same shape
     (``small=True``) that the CPU oracle finishes in seconds and that still

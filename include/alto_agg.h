@@ -267,6 +267,56 @@ alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg, const alto_batc
  * Always succeeds on a valid or poisoned handle. */
 alto_status alto_agg_destroy(alto_agg_t* h);
 
+/* ---- split_text: the fragmentation step before the aggregator ------------
+ *
+ * Sec. 3.1-3.2 (the split_text operator turns a text item of a Delimiter type
+ * into a stream of smaller Delimiter items, one level of hierarchy below it)
+ * and Sec. 4.2 (at a pmap entry every child keeps its parent's tags and gets
+ * one new tag).  Each of n_src token streams is cut after every delimiter
+ * token; piece k of stream s becomes a fragment whose tags are the stream's
+ * depth_in tags followed by (src_id[s], k, last = final piece).  A delimiter
+ * stays at the end of the piece it closes; a stream that ends with a
+ * delimiter has no trailing empty piece; an empty stream has one empty piece.
+ * The pieces tile the streams, so they need no copy: out_off indexes the
+ * input `tokens`, and {out_tags, out_off, tokens} is directly a batch for
+ * alto_agg_push_batch (depth depth_in + 1, n = n_frag) with the pieces in
+ * stream order.
+ *
+ * All pointers are device memory except `a` itself.  tok_off must start at 0,
+ * be non-decreasing and end at n_tokens.  out_tags is level-major with stride
+ * n_frag (the number of pieces, which the call computes): the caller gives
+ * capacity for cap_frag pieces, (depth_in + 1) * cap_frag tags and cap_frag + 1
+ * offsets.  Stream-ordered on `stream`, no synchronisation: the outcome is
+ * written to the device int64 out_counts[2] = {status, n_frag}, status
+ * ALTO_EINVAL for bad offsets, ALTO_ENOSPC when n_frag > cap_frag (nothing else
+ * is written then; n_frag is still the count needed).  `scratch` is device
+ * memory of at least alto_split_scratch_bytes(n_src, n_tokens) bytes, 256-byte
+ * aligned, owned by the caller; calls sharing a scratch must not overlap.  The
+ * return value is ALTO_EINVAL for bad host arguments (n_delims outside
+ * 1..ALTO_MAX_DELIMS, depth_in outside 0..ALTO_MAX_DEPTH-1, null pointers,
+ * too little scratch), ALTO_ECUDA if a launch fails, else ALTO_OK. */
+#define ALTO_MAX_DELIMS 32
+typedef struct alto_split_args {
+  int64_t n_src;              /* streams */
+  int64_t n_tokens;           /* tokens of all streams */
+  int32_t depth_in;           /* tags each stream carries, 0..ALTO_MAX_DEPTH-1 */
+  int32_t n_delims;           /* delimiter token ids, 1..ALTO_MAX_DELIMS */
+  int32_t delims[ALTO_MAX_DELIMS];
+  const uint64_t* src_tags;   /* [depth_in * n_src] level-major; may be NULL if depth_in == 0 */
+  const uint32_t* src_id;     /* [n_src] the streams' ids at the new level */
+  const uint32_t* tok_off;    /* [n_src + 1] */
+  const int32_t* tokens;      /* [n_tokens] */
+  int64_t cap_frag;
+  uint64_t* out_tags;         /* [(depth_in + 1) * n_frag] */
+  uint32_t* out_off;          /* [n_frag + 1] */
+  int64_t* out_counts;        /* [2]: status, n_frag */
+  void* scratch;
+  int64_t scratch_bytes;
+} alto_split_args;
+
+int64_t alto_split_scratch_bytes(int64_t n_src, int64_t n_tokens);
+alto_status alto_split_text(const alto_split_args* a, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -10,7 +10,7 @@ from ._binding import (  # noqa: F401
     RECORD_DTYPE, PAIR_DTYPE, Aggregator, Drain, alto_agg_config, alto_allocator, alto_batch,
     alto_drain, alto_agg_create, alto_agg_push_batch, alto_agg_drain, alto_agg_stats,
     alto_agg_destroy, alto_agg_profile, alto_agg_profile_read, alto_agg_oneshot_noalloc,
-    load_library, make_config,
+    load_library, make_config, alto_split_args, alto_split_scratch_bytes, alto_split_text, split_text,
     STAGE_NAMES, PROFILE_OFF, PROFILE_STAGES, PROFILE_HOT,
 )
 from ._build import build  # noqa: F401

@@ -87,9 +87,23 @@ class alto_profile(ctypes.Structure):
                 ("stage_launches", ctypes.c_int64 * NUM_STAGES)]
 
 
+MAX_DELIMS = 32
+
+
+class alto_split_args(ctypes.Structure):
+    _fields_ = [("n_src", ctypes.c_int64), ("n_tokens", ctypes.c_int64),
+                ("depth_in", ctypes.c_int32), ("n_delims", ctypes.c_int32),
+                ("delims", ctypes.c_int32 * MAX_DELIMS),
+                ("src_tags", ctypes.c_void_p), ("src_id", ctypes.c_void_p),
+                ("tok_off", ctypes.c_void_p), ("tokens", ctypes.c_void_p),
+                ("cap_frag", ctypes.c_int64), ("out_tags", ctypes.c_void_p),
+                ("out_off", ctypes.c_void_p), ("out_counts", ctypes.c_void_p),
+                ("scratch", ctypes.c_void_p), ("scratch_bytes", ctypes.c_int64)]
+
+
 EXPORTS = ("alto_agg_create", "alto_agg_push_batch", "alto_agg_drain", "alto_agg_stats",
            "alto_agg_profile", "alto_agg_profile_read", "alto_agg_oneshot_noalloc",
-           "alto_agg_destroy")
+           "alto_agg_destroy", "alto_split_scratch_bytes", "alto_split_text")
 
 _lib = None
 
@@ -123,6 +137,10 @@ def load_library(build: bool = True):
     lib.alto_agg_oneshot_noalloc.argtypes = [
         ctypes.POINTER(alto_agg_config), ctypes.POINTER(alto_batch), P, ctypes.c_int64, P,
         ctypes.c_int64, P, ctypes.c_int64, P, P]
+    lib.alto_split_scratch_bytes.restype = ctypes.c_int64
+    lib.alto_split_scratch_bytes.argtypes = [ctypes.c_int64, ctypes.c_int64]
+    lib.alto_split_text.restype = ctypes.c_int
+    lib.alto_split_text.argtypes = [ctypes.POINTER(alto_split_args), P]
     _lib = lib
     return lib
 
@@ -218,6 +236,54 @@ def alto_agg_profile(h, enable) -> int:
     and gather stages only."""
     mode = PROFILE_STAGES if enable is True else int(enable)
     return load_library().alto_agg_profile(h, mode)
+
+
+def alto_split_scratch_bytes(n_src: int, n_tokens: int) -> int:
+    return load_library().alto_split_scratch_bytes(n_src, n_tokens)
+
+
+def alto_split_text(args, stream=0) -> int:
+    return load_library().alto_split_text(ctypes.byref(args), ctypes.c_void_p(stream))
+
+
+def split_text(src_tags, src_id, tok_off, tokens, delims, cap_frag=None, stream=None):
+    """Device tensors in (src_tags uint64 [depth_in, n_src] or None, src_id
+    int32/uint32 [n_src], tok_off int32 [n_src + 1], tokens int32), device
+    tensors out: (status, n_frag, tags [depth_in + 1, n_frag] as int64 bits,
+    off [n_frag + 1] as int32).  Allocation only; every step runs in the
+    library's kernels."""
+    import torch
+    n_src = int(src_id.numel())
+    n_tokens = int(tokens.numel())
+    depth_in = 0 if src_tags is None else int(src_tags.shape[0])
+    cap = int(cap_frag) if cap_frag is not None else n_tokens + n_src
+    dev = tokens.device
+    stream = stream or torch.cuda.current_stream()
+    out_tags = torch.empty((depth_in + 1) * max(cap, 1), dtype=torch.int64, device=dev)
+    out_off = torch.empty(cap + 1, dtype=torch.int32, device=dev)
+    counts = torch.zeros(2, dtype=torch.int64, device=dev)
+    nbytes = alto_split_scratch_bytes(n_src, n_tokens)
+    scratch = torch.empty(max(nbytes, 256) + 256, dtype=torch.uint8, device=dev)
+    base = (scratch.data_ptr() + 255) & ~255
+    a = alto_split_args()
+    a.n_src, a.n_tokens, a.depth_in, a.n_delims = n_src, n_tokens, depth_in, len(delims)
+    for k, x in enumerate(delims):
+        a.delims[k] = int(x)
+    a.src_tags = src_tags.data_ptr() if src_tags is not None else None
+    a.src_id, a.tok_off = src_id.data_ptr(), tok_off.data_ptr()
+    a.tokens = tokens.data_ptr() if n_tokens else None
+    a.cap_frag = cap
+    a.out_tags, a.out_off, a.out_counts = out_tags.data_ptr(), out_off.data_ptr(), counts.data_ptr()
+    a.scratch, a.scratch_bytes = base, nbytes
+    st = alto_split_text(a, stream.cuda_stream)
+    if st != OK:
+        return st, 0, None, None
+    torch.cuda.current_stream().synchronize() if stream is None else stream.synchronize()
+    status, n_frag = (int(x) for x in counts.cpu().tolist())
+    if status != OK:
+        return status, n_frag, None, None
+    tags = out_tags[:(depth_in + 1) * n_frag].view(depth_in + 1, n_frag)
+    return status, n_frag, tags, out_off[:n_frag + 1]
 
 
 def alto_agg_profile_read(h):

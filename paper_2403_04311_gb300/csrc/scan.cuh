@@ -67,8 +67,10 @@ __device__ __forceinline__ ulonglong2 lb_read(LookbackState st, long long tile) 
 }
 
 // Sum of everything before `tile`, found by warp 0: each lane reads four
-// predecessors of a 128-tile window (lane l takes tiles top-l, top-l-32, ...);
-// the nearest inclusive prefix ends the walk.
+// predecessors of a 128-tile window (lane l takes tiles top-l, top-l-32, ...).
+// The nearest inclusive prefix ends the walk; only the tiles nearer than it
+// must have published (their aggregates), so a slow tile further back does
+// not hold this one up.
 __device__ __forceinline__ u64 lb_walk_warp(LookbackState st, u32 tile, u32 es, Ctl* ctl,
                                             u64 spin_limit) {
   const int lane = threadIdx.x & 31;
@@ -77,18 +79,23 @@ __device__ __forceinline__ u64 lb_walk_warp(LookbackState st, u32 tile, u32 es, 
   u64 spins = 0;
   while (top >= 0) {
     ulonglong2 dsc[4];
-    bool ready = true;
+    int stop = 128, wait = 128;  // nearest inclusive, nearest unpublished
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
       const long long p = top - lane - 32 * r;
       dsc[r] = make_ulonglong2(0, 0);
+      u32 kind = 2;  // before tile 0: an inclusive prefix of 0
       if (p >= 0) {
         dsc[r] = lb_read(st, p);
         const u32 f = (u32)dsc[r].y;
-        ready = ready && ((f >> 2) == es) && ((f & 3u) != 0);
+        kind = ((f >> 2) == es) ? (f & 3u) : 0u;
       }
+      const u32 inc = __ballot_sync(0xFFFFFFFFu, kind == 2u);
+      const u32 unp = __ballot_sync(0xFFFFFFFFu, kind == 0u);
+      if (inc && stop == 128) stop = 32 * r + __ffs(inc) - 1;
+      if (unp && wait == 128) wait = 32 * r + __ffs(unp) - 1;
     }
-    if (!__all_sync(0xFFFFFFFFu, ready)) {
+    if (wait < stop) {
       if (++spins > spin_limit || *(volatile int*)&ctl->abort) {
         if (lane == 0) raise_timeout(ctl);
         break;
@@ -96,15 +103,6 @@ __device__ __forceinline__ u64 lb_walk_warp(LookbackState st, u32 tile, u32 es, 
       // back off: every waiting warp polls the same few lines of descriptors
       __nanosleep(64);
       continue;
-    }
-    // nearest inclusive predecessor: smallest distance d = lane + 32 r
-    int stop = 128;
-#pragma unroll
-    for (int r = 0; r < 4; ++r) {
-      const long long p = top - lane - 32 * r;
-      const bool inc = (p < 0) || (((u32)dsc[r].y & 3u) == 2u);
-      const u32 m = __ballot_sync(0xFFFFFFFFu, inc);
-      if (m && stop == 128) stop = 32 * r + __ffs(m) - 1;
     }
     u64 v = 0;
 #pragma unroll
@@ -130,9 +128,25 @@ __device__ __forceinline__ u64 lb_walk_warp(LookbackState st, u32 tile, u32 es, 
 // Element values fit in 32 bits (counts, lengths, flags); prefixes are
 // 64-bit, tile-local prefixes 32-bit (a tile whose sum does not fit takes the
 // blocked order instead).  Shared memory is padded by one word per 32 so that
-// both access orders are free of bank conflicts.  The next tile's id is
-// taken while the current one is processed.
+// both access orders are free of bank conflicts.
+//
+// The look-back is one warp's job; the CTA's other warps would wait for it at
+// a barrier.  Instead, once the tile's aggregate is published, every thread
+// loads the NEXT tile's values into registers, so that those loads are in
+// flight while warp 0 walks back (value() only reads the scan's inputs).  The
+// next tile's id is taken one tile ahead for the same reason.
 __device__ __forceinline__ u32 scan_pad(u32 p) { return p + (p >> 5); }
+
+template <class F>
+__device__ __forceinline__ void scan_load(const F& f, u64 n, u32 tile, u32 ntiles, u32 (&r)[kScanItems]) {
+  const int t = threadIdx.x;
+  const u64 base = (u64)tile * kScanTile;
+#pragma unroll
+  for (int k = 0; k < kScanItems; ++k) {
+    const u64 i = base + (u64)(k * kScanThreads + t);
+    r[k] = (tile < ntiles && i < n) ? (u32)f.value(i) : 0u;
+  }
+}
 
 template <class F>
 __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl, int site,
@@ -143,25 +157,23 @@ __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl
   __shared__ u64 s_excl;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const u64 n = halted(ctl) ? 0 : f.size(ctl);
-  u64 ntiles = (n + kScanTile - 1) / kScanTile;
-  if (ntiles == 0) ntiles = 1;
-  if (ntiles > st.tiles) ntiles = st.tiles;
+  u64 ntiles64 = (n + kScanTile - 1) / kScanTile;
+  if (ntiles64 == 0) ntiles64 = 1;
+  if (ntiles64 > st.tiles) ntiles64 = st.tiles;
+  const u32 ntiles = (u32)ntiles64;
   const u32 es = epoch_site(ctl, site);
   if (t == 0) s_next = take_tile(ctl, site);
   __syncthreads();
-  for (;;) {
-    const u32 tile = s_next;
-    __syncthreads();
-    if (tile >= ntiles) break;
+  u32 tile = s_next;
+  __syncthreads();
+  u32 r[kScanItems];
+  scan_load(f, n, tile, ntiles, r);
+  while (tile < ntiles) {
     if (t == 0) s_next = take_tile(ctl, site);  // read after the barriers below
-    const u64 base = (u64)tile * kScanTile;
 #pragma unroll
-    for (int k = 0; k < kScanItems; ++k) {
-      const u32 p = (u32)(k * kScanThreads + t);
-      const u64 i = base + p;
-      s_v[scan_pad(p)] = (i < n) ? (u32)f.value(i) : 0u;
-    }
+    for (int k = 0; k < kScanItems; ++k) s_v[scan_pad((u32)(k * kScanThreads + t))] = r[k];
     __syncthreads();
+    const u64 base = (u64)tile * kScanTile;
     u32 w[kScanItems];
     u64 sum = 0;
 #pragma unroll
@@ -177,6 +189,7 @@ __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl
     }
     if (lane == 31) s_w[warp] = x;
     __syncthreads();
+    const u32 next = s_next;
     u64 wpre = 0, agg = 0;
 #pragma unroll
     for (int q = 0; q < kScanWarps; ++q) {
@@ -193,12 +206,12 @@ __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl
         rel += w[k];
       }
     }
+    if (warp == 0 && lane == 0) lb_publish(st, tile, es, tile == 0 ? 2u : 1u, agg);
+    // the next tile's loads go out while warp 0 walks back
+    scan_load(f, n, next, ntiles, r);
     if (warp == 0) {
       u64 excl = 0;
-      if (tile == 0) {
-        if (lane == 0) lb_publish(st, tile, es, 2u, agg);
-      } else {
-        if (lane == 0) lb_publish(st, tile, es, 1u, agg);
+      if (tile != 0) {
         excl = lb_walk_warp(st, tile, es, ctl, spin_limit);
         if (lane == 0) lb_publish(st, tile, es, 2u, excl + agg);
       }
@@ -228,8 +241,159 @@ __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl
       }
     }
     __syncthreads();
+    tile = next;
   }
   if (t == 0) finish_ctas(ctl, site, exit_ctr);
+}
+
+// ---------------------------------------------------------------------------
+// Large scans: reduce, then scan down, no look-back.  A persistent grid of G
+// CTAs splits the elements into G contiguous chunks of whole tiles.  The first
+// kernel writes each chunk's sum; the second has every CTA add up the sums of
+// the chunks before its own and scan its chunk tile by tile with a running
+// offset.  The input is read twice and the prefixes written once, all in
+// streaming order, which beats the look-back scan once the elements are many
+// times the CTAs' tiles (the look-back then walks back a whole wave of tiles).
+// ---------------------------------------------------------------------------
+template <class F>
+__device__ __forceinline__ void chunk_of_cta(const F& f, Ctl* ctl, u64* n_out, u64* lo, u64* hi) {
+  const u64 n = halted(ctl) ? 0 : f.size(ctl);
+  const u64 tiles = (n + kScanTile - 1) / kScanTile;
+  const u64 per = (tiles + gridDim.x - 1) / gridDim.x * kScanTile;
+  *n_out = n;
+  *lo = min(n, (u64)blockIdx.x * per);
+  *hi = min(n, *lo + per);
+}
+
+template <class F>
+__global__ void __launch_bounds__(kScanThreads) k_scan_reduce(F f, u64* part, Ctl* ctl) {
+  pdl_enter();
+  __shared__ u64 s_w[kScanWarps];
+  u64 n, lo, hi;
+  chunk_of_cta(f, ctl, &n, &lo, &hi);
+  u64 sum = 0;
+  for (u64 b = lo; b < hi; b += (u64)kScanThreads * kScanItems) {
+    u32 v[kScanItems];
+#pragma unroll
+    for (int k = 0; k < kScanItems; ++k) {
+      const u64 i = b + (u64)k * kScanThreads + threadIdx.x;
+      v[k] = (i < hi) ? (u32)f.value(i) : 0u;
+    }
+#pragma unroll
+    for (int k = 0; k < kScanItems; ++k) sum += v[k];
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+  if ((threadIdx.x & 31) == 0) s_w[threadIdx.x >> 5] = sum;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    u64 t = 0;
+    for (int q = 0; q < kScanWarps; ++q) t += s_w[q];
+    part[blockIdx.x] = t;
+  }
+}
+
+template <class F>
+__global__ void __launch_bounds__(kScanThreads) k_scan_down(F f, const u64* part, Ctl* ctl) {
+  pdl_enter();
+  __shared__ u32 s_v[kScanTile + kScanTile / 32];
+  __shared__ u64 s_w[kScanWarps];
+  __shared__ u64 s_off;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  u64 n, lo, hi;
+  chunk_of_cta(f, ctl, &n, &lo, &hi);
+  // offset of this chunk: the sums of the chunks before it (and the grand total)
+  {
+    u64 before = 0, all = 0;
+    for (u32 c = t; c < gridDim.x; c += kScanThreads) {
+      const u64 v = part[c];
+      if (c < blockIdx.x) before += v;
+      all += v;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      before += __shfl_xor_sync(0xFFFFFFFFu, before, o);
+      all += __shfl_xor_sync(0xFFFFFFFFu, all, o);
+    }
+    __shared__ u64 s_b[kScanWarps], s_a[kScanWarps];
+    if (lane == 0) {
+      s_b[warp] = before;
+      s_a[warp] = all;
+    }
+    __syncthreads();
+    if (t == 0) {
+      u64 b = 0, a = 0;
+      for (int q = 0; q < kScanWarps; ++q) {
+        b += s_b[q];
+        a += s_a[q];
+      }
+      s_off = b;
+      if (blockIdx.x == 0) f.total(ctl, a);
+    }
+    __syncthreads();
+  }
+  u64 off = s_off;
+  for (u64 base = lo; base < hi; base += kScanTile) {
+#pragma unroll
+    for (int k = 0; k < kScanItems; ++k) {
+      const u32 p = (u32)(k * kScanThreads + t);
+      const u64 i = base + p;
+      s_v[scan_pad(p)] = (i < hi) ? (u32)f.value(i) : 0u;
+    }
+    __syncthreads();
+    u32 w[kScanItems];
+    u64 sum = 0;
+#pragma unroll
+    for (int k = 0; k < kScanItems; ++k) {
+      w[k] = s_v[scan_pad((u32)(t * kScanItems + k))];
+      sum += w[k];
+    }
+    u64 x = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const u64 y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) s_w[warp] = x;
+    __syncthreads();
+    u64 wpre = 0, agg = 0;
+#pragma unroll
+    for (int q = 0; q < kScanWarps; ++q) {
+      const u64 c = s_w[q];
+      if (q < warp) wpre += c;
+      agg += c;
+    }
+    const bool narrow = agg < (1ull << 32);
+    u64 rel = wpre + (x - sum);
+    if (narrow) {
+#pragma unroll
+      for (int k = 0; k < kScanItems; ++k) {
+        s_v[scan_pad((u32)(t * kScanItems + k))] = (u32)rel;
+        rel += w[k];
+      }
+    }
+    __syncthreads();
+    if (narrow) {
+#pragma unroll
+      for (int k = 0; k < kScanItems; ++k) {
+        const u32 p = (u32)(k * kScanThreads + t);
+        const u64 i = base + p;
+        const u32 r0 = s_v[scan_pad(p)];
+        const u32 r1 = (p + 1 < (u32)kScanTile) ? s_v[scan_pad(p + 1)] : (u32)agg;
+        if (i < hi) f.out(i, off + r0, (u64)(r1 - r0));
+      }
+    } else {
+      u64 run = off + wpre + (x - sum);
+      const u64 first = base + (u64)t * kScanItems;
+#pragma unroll
+      for (int k = 0; k < kScanItems; ++k) {
+        if (first + k < hi) f.out(first + k, run, w[k]);
+        run += w[k];
+      }
+    }
+    off += agg;
+    __syncthreads();
+  }
 }
 
 template <class F>

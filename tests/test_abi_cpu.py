@@ -17,7 +17,7 @@ def declared_functions():
     for f in sorted(os.listdir(inc)):
         if f.endswith(".h"):
             txt = open(os.path.join(inc, f)).read()
-            names += re.findall(r"^alto_status\s+(alto_\w+)\s*\(", txt, flags=re.M)
+            names += re.findall(r"^(?:alto_status|int64_t)\s+(alto_\w+)\s*\(", txt, flags=re.M)
     return names
 
 
