@@ -16,6 +16,7 @@ from dataclasses import dataclass
 
 import numpy as np
 
+from .route import HASH, LEAST_LOADED, RouterOracle, splitmix64_mix  # noqa: F401
 from .split_text import split_pieces, split_text  # noqa: F401
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
