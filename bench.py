@@ -292,6 +292,82 @@ def run_split(args, rank, world):
             "cpu_baseline": cpu}
 
 
+def run_route(args, rank, world, R=8):
+    """Routing in front of R replicated aggregators: the throughput stream
+    (16M fragments, 1M batches) routed at level 1 with flows placed by load,
+    each batch partitioned into R sub-batches (tags, offsets, payload).  One
+    step = the whole stream."""
+    import numpy as np
+    from gen import make_stream
+    s = make_stream("throughput")
+    L = 1
+    if args.impl == "reference":
+        import oracle
+        if rank != 0:
+            return None
+        b0 = s.batch(0)
+        n = min(b0["n"], int(args.ref_sample))
+        sample = dict(n=n, tags=np.ascontiguousarray(b0["tags"][:, :n]), off=b0["off"][:n + 1],
+                      payload=b0["payload"][:int(b0["off"][n])], score=None)
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            oracle.RouterOracle(s.depth, L, R, oracle.LEAST_LOADED).route(sample)
+        dt = time.perf_counter() - t0
+        value = n * args.steps / dt
+        return {"impl": "reference", "metric": "routed fragments/s", "value": value, "unit": "fragments/s",
+                "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
+                "data": "synthetic", "config": {"workload": "route", "replicas": R, "level": L},
+                "cpu_baseline": {"value": value, "unit": "fragments/s", "cores": 1, "kind": "oracle",
+                                 "sample": f"first {n} fragments of batch 0 per step, single thread"},
+                "e2e": {"value": value, "unit": "fragments/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    import torch
+    import paper_2403_04311_gb300 as alto
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    stream = torch.cuda.current_stream()
+    st = s.batch_starts()
+    pay = int(max(s.off[b1] - s.off[b0] for b0, b1 in zip(st[:-1], st[1:])))
+    batches = [alto.to_device(s.batch(b)) for b in range(s.n_batches)]
+    rt = alto.Router(s.depth, L, R, alto.ROUTE_LEAST_LOADED, max_batch_fragments=int(max(s.batch_sizes)),
+                     max_batch_payload=pay, max_flows=1 << 22, stream=stream)
+
+    def step():
+        for db in batches:
+            if rt.route(db.tags, db.off, db.payload) != alto.OK:
+                raise RuntimeError("route failed")
+
+    for _ in range(max(args.warmup, 1)):
+        step()
+    torch.cuda.synchronize()
+    assert rt.counts()[0] == alto.OK
+    sampler = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
+    sampler.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    rt.close()
+    hbm_gbs, peak_kind = peaks()
+    # algorithmic bytes of a pass: every fragment's tags and offset read and
+    # written once, every payload element read and written once
+    alg = (8.0 * s.depth + 4.0) * 2 * s.n + 8.0 * s.payload.size
+    achieved = alg / (ms / 1e3) / 1e9
+    return {"metric": "routed fragments/s", "value": s.n * world / (ms / 1e3), "unit": "fragments/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+            "config": {"workload": "route", "stream": "throughput", "fragments": s.n, "replicas": R, "level": L,
+                       "policy": "least_loaded", "l2": "inputs larger than L2 (no flush)"},
+            "roofline": {"bound": "hbm", "kernel": "route (all kernels of a batch)", "achieved": achieved,
+                         "peak": hbm_gbs, "unit": "GB/s", "frac": achieved / hbm_gbs, "peak_kind": peak_kind,
+                         "traffic": None},
+            "gpu_launches": 15 * s.n_batches * args.steps, "clocks": clocks, "cpu_baseline": None,
+            "e2e": None}
+
+
 def cpu_baseline(s, budget_s=20.0):
     """Oracle fragments/s on a bounded sample (batches in order until the
     budget is spent), one host thread."""
@@ -336,8 +412,8 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
 
-    if args.workload == "split":
-        line = run_split(args, rank, world)
+    if args.workload in ("split", "route"):
+        line = (run_split if args.workload == "split" else run_route)(args, rank, world)
         if rank == 0 and line is not None:
             print(json.dumps(line), flush=True)
         return

@@ -317,6 +317,78 @@ typedef struct alto_split_args {
 int64_t alto_split_scratch_bytes(int64_t n_src, int64_t n_tokens);
 alto_status alto_split_text(const alto_split_args* a, void* stream);
 
+/* ---- routing by ancestry: the step in front of replicated aggregators ----
+ *
+ * Sec. 4.3: the aggregation at a pmap exit needs every element of a group at
+ * the same instance of the next stage, so all elements with the same
+ * ancestry tags go to the same instance (like ECMP, keyed on the tags), and a
+ * new flow may be placed by load instead of by a hash; Sec. 5: the
+ * controller picks replicas by these rules and by queue lengths.
+ *
+ * A flow is the group at the routing level L: fragments whose tags agree on
+ * levels 0..L (parent ids are unique per level, so (L, p_L) names it).
+ * ALTO_ROUTE_HASH places it at splitmix64(L << 32 | p_L) mod R.
+ * ALTO_ROUTE_LEAST_LOADED keeps a placed flow on its replica and deals the
+ * batch's new flows, in the order of their first fragment, round-robin over
+ * the replicas ordered by load at the start of the batch (fewest first, ties
+ * to the lower index), the load being the fragments routed to the replica so
+ * far.  alto_router_release forgets the flows whose groups the aggregator
+ * reported complete.  Each batch is partitioned stably: replica r's
+ * sub-batch holds its fragments in arrival order and is itself a batch for
+ * alto_agg_push_batch.
+ *
+ * Calls are stream-ordered and do not synchronise, except
+ * alto_router_counts.  Device-detected errors (bad payload offsets: EINVAL;
+ * flow table full: ENOSPC; a wait that ran out: ETIMEOUT) latch and poison
+ * the handle; the next call returns them. */
+#define ALTO_ROUTE_HASH 0
+#define ALTO_ROUTE_LEAST_LOADED 1
+#define ALTO_MAX_REPLICAS 1024
+
+typedef struct alto_router_config {
+  int32_t depth;               /* tags per fragment, 1..ALTO_MAX_DEPTH */
+  int32_t level;               /* routing level L, 0..depth-1 */
+  int32_t n_replicas;          /* R, 1..ALTO_MAX_REPLICAS */
+  int32_t policy;              /* ALTO_ROUTE_HASH or ALTO_ROUTE_LEAST_LOADED */
+  int64_t max_batch_fragments; /* n per batch, >= 1 */
+  int64_t max_batch_payload;   /* payload elements per batch */
+  int64_t max_flows;           /* LEAST_LOADED: flows placed at once (0: 2^20) */
+  int32_t with_score;          /* batches carry scores (routed along) */
+  int32_t reserved;
+} alto_router_config;
+
+typedef struct alto_router alto_router_t;
+
+/* The last batch's routing, all in device memory owned by the handle, valid
+ * until the next route or destroy.  Replica r's sub-batch: n_r =
+ * frag_off[r+1] - frag_off[r] fragments; tags at tags + depth * frag_off[r]
+ * (level-major with stride n_r); payload_off at payload_off + frag_off[r] + r
+ * (n_r + 1 offsets from 0); payload at payload + pay_off[r]; scores at
+ * score + frag_off[r]. */
+typedef struct alto_routed {
+  const uint32_t* replica;     /* [n] replica of each input fragment */
+  const uint32_t* perm;        /* [n] input fragments grouped by replica, in arrival order */
+  const int64_t* frag_off;     /* [R + 1] */
+  const int64_t* pay_off;      /* [R + 1] */
+  const uint64_t* tags;        /* [depth * n] */
+  const uint32_t* payload_off; /* [n + R] */
+  const int32_t* payload;      /* [n_payload] */
+  const float* score;          /* [n] or NULL */
+} alto_routed;
+
+alto_status alto_router_create(const alto_router_config* cfg, const alto_allocator* alloc, void* stream,
+                               alto_router_t** out);
+/* Route one batch (device buffers, borrowed until the stream reaches the work). */
+alto_status alto_router_route(alto_router_t* h, const alto_batch* b, void* stream, alto_routed* out);
+/* Synchronise and copy the last batch's frag_off and pay_off (R + 1 each) to
+ * host arrays; returns the latched status. */
+alto_status alto_router_counts(alto_router_t* h, void* stream, int64_t* frag_off, int64_t* pay_off);
+/* Forget the flows of the groups in `records` (device, as a drain returns
+ * them) that sit at the routing level. */
+alto_status alto_router_release(alto_router_t* h, const alto_record* records, int64_t n_records, void* stream);
+/* Free everything; NULL is OK. */
+alto_status alto_router_destroy(alto_router_t* h);
+
 #ifdef __cplusplus
 }
 #endif

@@ -11,6 +11,7 @@ from ._binding import (  # noqa: F401
     alto_drain, alto_agg_create, alto_agg_push_batch, alto_agg_drain, alto_agg_stats,
     alto_agg_destroy, alto_agg_profile, alto_agg_profile_read, alto_agg_oneshot_noalloc,
     load_library, make_config, alto_split_args, alto_split_scratch_bytes, alto_split_text, split_text,
+    Router, ROUTE_HASH, ROUTE_LEAST_LOADED,
     STAGE_NAMES, PROFILE_OFF, PROFILE_STAGES, PROFILE_HOT,
 )
 from ._build import build  # noqa: F401

@@ -101,9 +101,27 @@ class alto_split_args(ctypes.Structure):
                 ("scratch", ctypes.c_void_p), ("scratch_bytes", ctypes.c_int64)]
 
 
+ROUTE_HASH, ROUTE_LEAST_LOADED = 0, 1
+
+
+class alto_router_config(ctypes.Structure):
+    _fields_ = [("depth", ctypes.c_int32), ("level", ctypes.c_int32), ("n_replicas", ctypes.c_int32),
+                ("policy", ctypes.c_int32), ("max_batch_fragments", ctypes.c_int64),
+                ("max_batch_payload", ctypes.c_int64), ("max_flows", ctypes.c_int64),
+                ("with_score", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+class alto_routed(ctypes.Structure):
+    _fields_ = [("replica", ctypes.c_void_p), ("perm", ctypes.c_void_p), ("frag_off", ctypes.c_void_p),
+                ("pay_off", ctypes.c_void_p), ("tags", ctypes.c_void_p), ("payload_off", ctypes.c_void_p),
+                ("payload", ctypes.c_void_p), ("score", ctypes.c_void_p)]
+
+
 EXPORTS = ("alto_agg_create", "alto_agg_push_batch", "alto_agg_drain", "alto_agg_stats",
            "alto_agg_profile", "alto_agg_profile_read", "alto_agg_oneshot_noalloc",
-           "alto_agg_destroy", "alto_split_scratch_bytes", "alto_split_text")
+           "alto_agg_destroy", "alto_split_scratch_bytes", "alto_split_text",
+           "alto_router_create", "alto_router_route", "alto_router_counts", "alto_router_release",
+           "alto_router_destroy")
 
 _lib = None
 
@@ -141,6 +159,17 @@ def load_library(build: bool = True):
     lib.alto_split_scratch_bytes.argtypes = [ctypes.c_int64, ctypes.c_int64]
     lib.alto_split_text.restype = ctypes.c_int
     lib.alto_split_text.argtypes = [ctypes.POINTER(alto_split_args), P]
+    lib.alto_router_create.restype = ctypes.c_int
+    lib.alto_router_create.argtypes = [ctypes.POINTER(alto_router_config), ctypes.POINTER(alto_allocator), P,
+                                       ctypes.POINTER(P)]
+    lib.alto_router_route.restype = ctypes.c_int
+    lib.alto_router_route.argtypes = [P, ctypes.POINTER(alto_batch), P, ctypes.POINTER(alto_routed)]
+    lib.alto_router_counts.restype = ctypes.c_int
+    lib.alto_router_counts.argtypes = [P, P, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
+    lib.alto_router_release.restype = ctypes.c_int
+    lib.alto_router_release.argtypes = [P, P, ctypes.c_int64, P]
+    lib.alto_router_destroy.restype = ctypes.c_int
+    lib.alto_router_destroy.argtypes = [P]
     _lib = lib
     return lib
 
@@ -382,6 +411,95 @@ class Aggregator:
     def close(self):
         if getattr(self, "_h", None):
             alto_agg_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class Router:
+    """Owning wrapper around one alto_router handle: routes device batches to
+    R replicas and exposes each replica's sub-batch as device tensors."""
+
+    def __init__(self, depth, level, n_replicas, policy, *, max_batch_fragments, max_batch_payload,
+                 max_flows=0, with_score=False, stream=None, use_torch_allocator=True):
+        import torch
+        self._torch = torch
+        self.depth, self.level, self.R = depth, level, n_replicas
+        self.with_score = bool(with_score)
+        self.stream = stream if stream is not None else torch.cuda.current_stream()
+        self._alloc = _TorchAllocator(torch.cuda.current_device()) if use_torch_allocator else None
+        c = alto_router_config()
+        c.depth, c.level, c.n_replicas, c.policy = depth, level, n_replicas, policy
+        c.max_batch_fragments, c.max_batch_payload, c.max_flows = max_batch_fragments, max_batch_payload, max_flows
+        c.with_score = 1 if with_score else 0
+        h = ctypes.c_void_p()
+        a = self._alloc.struct if self._alloc is not None else None
+        st = load_library().alto_router_create(ctypes.byref(c), ctypes.byref(a) if a is not None else None,
+                                               ctypes.c_void_p(self.stream.cuda_stream), ctypes.byref(h))
+        if st != OK:
+            raise RuntimeError(f"alto_router_create failed: {STATUS_NAMES.get(st, st)}")
+        self._h = h
+        self.routed = alto_routed()
+
+    def route(self, tags, off, payload, score=None, n=None) -> int:
+        b = alto_batch()
+        b.n = int(tags.shape[-1]) if n is None else int(n)
+        b.depth = self.depth
+        b.tags = tags.data_ptr()
+        b.payload_off = off.data_ptr()
+        b.n_payload = int(payload.numel())
+        b.payload = payload.data_ptr() if payload.numel() else None
+        b.score = score.data_ptr() if score is not None else None
+        self._n = b.n
+        return load_library().alto_router_route(self._h, ctypes.byref(b), ctypes.c_void_p(self.stream.cuda_stream),
+                                                ctypes.byref(self.routed))
+
+    def counts(self):
+        """Synchronise; (status, frag_off [R+1], pay_off [R+1]) as numpy int64."""
+        import numpy as np
+        fo = (ctypes.c_int64 * (self.R + 1))()
+        po = (ctypes.c_int64 * (self.R + 1))()
+        st = load_library().alto_router_counts(self._h, ctypes.c_void_p(self.stream.cuda_stream), fo, po)
+        return st, np.frombuffer(fo, dtype=np.int64).copy(), np.frombuffer(po, dtype=np.int64).copy()
+
+    def outputs(self, frag_off, pay_off):
+        """Device views of the last routing: (replica, perm, [per replica (tags
+        (D, n_r), payload_off (n_r + 1), payload, score or None)])."""
+        torch = self._torch
+        r = self.routed
+        n = int(frag_off[-1])
+
+        def view(ptr, count, dtype, esize):
+            if count == 0 or not ptr:
+                return torch.zeros(0, dtype=dtype, device="cuda")
+            return torch.as_tensor(_DevView(ptr, count * esize), device="cuda").view(dtype)
+
+        replica = view(r.replica, n, torch.int32, 4)
+        perm = view(r.perm, n, torch.int32, 4)
+        tags = view(r.tags, self.depth * n, torch.int64, 8)
+        poff = view(r.payload_off, n + self.R, torch.int32, 4)
+        pay = view(r.payload, int(pay_off[-1]), torch.int32, 4)
+        score = view(r.score, n, torch.float32, 4) if self.with_score else None
+        parts = []
+        for k in range(self.R):
+            a, b = int(frag_off[k]), int(frag_off[k + 1])
+            nr = b - a
+            parts.append((tags[self.depth * a:self.depth * b].view(self.depth, nr),
+                          poff[a + k:b + k + 1], pay[int(pay_off[k]):int(pay_off[k + 1])],
+                          None if score is None else score[a:b]))
+        return replica, perm, parts
+
+    def release(self, records_ptr, n_records) -> int:
+        return load_library().alto_router_release(self._h, ctypes.c_void_p(records_ptr), int(n_records),
+                                                  ctypes.c_void_p(self.stream.cuda_stream))
+
+    def close(self):
+        if getattr(self, "_h", None):
+            load_library().alto_router_destroy(self._h)
             self._h = None
 
     def __del__(self):

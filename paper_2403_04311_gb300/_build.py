@@ -15,7 +15,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(HERE, "libalto_agg.so")
-SOURCES = ["alto_agg.cu", "radix_sort.cu", "split_text.cu"]
+SOURCES = ["alto_agg.cu", "radix_sort.cu", "split_text.cu", "route.cu"]
 HEADERS = ["common.cuh", "scan.cuh", "kernels.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]
