@@ -67,6 +67,8 @@ def _load():
                                  ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]
         lib.orc_drain.restype = ctypes.c_int
         lib.orc_drain.argtypes = [ctypes.c_void_p, ctypes.POINTER(_Drain)]
+        lib.orc_set_stream_release.restype = ctypes.c_int
+        lib.orc_set_stream_release.argtypes = [ctypes.c_void_p, ctypes.c_int]
         lib.orc_open_groups.restype = ctypes.c_int64
         lib.orc_open_groups.argtypes = [ctypes.c_void_p]
         lib.orc_destroy.restype = None
@@ -92,7 +94,7 @@ def _ptr(a):
 class Oracle:
     """Arrival-order reference aggregator over host arrays."""
 
-    def __init__(self, depth, payload_op, score_op, topk_k):
+    def __init__(self, depth, payload_op, score_op, topk_k, stream_release=False):
         lib = _load()
         self.depth = int(depth)
         po = np.asarray(list(payload_op) + [0] * (8 - len(payload_op)), dtype=np.int32)
@@ -101,10 +103,13 @@ class Oracle:
         self._h = lib.orc_create(self.depth, _ptr(po), _ptr(so), _ptr(kk))
         if not self._h:
             raise ValueError("invalid aggregation config")
+        if stream_release and lib.orc_set_stream_release(self._h, 1) != 0:
+            self.close()
+            raise ValueError("streaming release needs a CONCAT level")
 
     @classmethod
-    def for_stream(cls, stream):
-        return cls(stream.depth, stream.payload_op, stream.score_op, stream.topk_k)
+    def for_stream(cls, stream, stream_release=False):
+        return cls(stream.depth, stream.payload_op, stream.score_op, stream.topk_k, stream_release)
 
     def push(self, tags, off, payload, score=None, depth=None) -> int:
         tags = np.ascontiguousarray(tags, dtype=np.uint64)
@@ -148,10 +153,10 @@ class Oracle:
             pass
 
 
-def run_stream(stream, drain_every: int = 1):
+def run_stream(stream, drain_every: int = 1, stream_release: bool = False):
     """Push every batch of a generated stream and drain every
     ``drain_every`` batches (and at the end); returns the list of drains."""
-    o = Oracle.for_stream(stream)
+    o = Oracle.for_stream(stream, stream_release)
     out = []
     for b in range(stream.n_batches):
         o.push_batch(stream.batch(b))

@@ -28,6 +28,14 @@
 //    top-K thought selection of Sec. 6.1.2): MAX reports the largest leaf
 //    score of the subtree; TOPK lists the k children with the largest score
 //    (ties to the smaller child index), under IEEE-754 totalOrder.
+//  * Streaming release (optional; Sec. 3.2: the pmap's outputs are put back
+//    in order and passed on as a stream, not only once the whole group is
+//    in): at the end of each batch, a still-open CONCAT group whose run of
+//    complete children 0..r-1 grew past what it released before emits that
+//    run as a partial record (ops bit 0x80, n_children = r, completion seq =
+//    the latest completion among the run); the group's final record carries
+//    only the children not yet released.  Records of a batch are ordered by
+//    (completion seq, deeper level first).
 //
 // Error classes are collected per batch and the batch reports the one with
 // the highest priority (EINVAL > EDUP > EINCONSIST > ELAST > ECLOSED); the
@@ -98,6 +106,7 @@ struct OrcPair {  // 8 bytes
 struct Leaf {
   std::vector<int32_t> tokens;
   float score = 0.0f;
+  uint64_t seq = 0;           // arrival index (its completion seq)
 };
 
 struct Group {
@@ -111,6 +120,8 @@ struct Group {
   std::map<uint32_t, Leaf> leaves;           // level D-1: slot -> leaf
   uint32_t completed = 0;     // number of complete children
   bool emitted = false;
+  uint64_t done_seq = 0;      // completion seq, once emitted
+  uint32_t released = 0;      // streaming release: children 0..released-1 already emitted
 };
 
 // IEEE-754 totalOrder restricted to non-NaN values: the usual order, with
@@ -127,6 +138,14 @@ struct Oracle {
   int score_op[8] = {};
   int topk_k[8] = {};
   bool needs_score = false;
+  // Streaming release (Sec. 3.2: as each item of a pmap finishes, the stream
+  // is reconstituted in the original order and sent on in a streaming
+  // fashion): at the end of every batch, an open CONCAT group whose in-order
+  // prefix of complete children advanced emits that part of its payload as a
+  // partial record; its final record then holds only the rest.
+  bool stream_release = false;
+  int concat_level = -1;
+  std::set<uint32_t> touched;  // CONCAT-level groups that got fragments in this batch
 
   std::map<std::pair<int, uint32_t>, Group> groups;
   uint64_t seq_next = 0;       // global sequence number of the next fragment
@@ -145,10 +164,11 @@ struct Oracle {
   Group& group(int level, uint32_t id) { return groups[{level, id}]; }
 
   // Leaves of the subtree of (level, id), concatenated in child-index path
-  // order (Sec. 3.2: the stream is reconstituted in its original order).
-  void concat(int level, uint32_t id, std::vector<int32_t>& out) {
+  // order (Sec. 3.2: the stream is reconstituted in its original order);
+  // children from..to-1 of the group itself.
+  void concat_range(int level, uint32_t id, uint32_t from, uint32_t to, std::vector<int32_t>& out) {
     Group& g = group(level, id);
-    for (uint32_t c = 0; c <= g.last; ++c) {
+    for (uint32_t c = from; c < to; ++c) {
       if (level == depth - 1) {
         const Leaf& lf = g.leaves.at(c);
         out.insert(out.end(), lf.tokens.begin(), lf.tokens.end());
@@ -156,6 +176,26 @@ struct Oracle {
         concat(level + 1, g.child_group.at(c), out);
       }
     }
+  }
+  void concat(int level, uint32_t id, std::vector<int32_t>& out) {
+    concat_range(level, id, 0, group(level, id).last + 1, out);
+  }
+
+  // Child c of (level, id) is complete (a leaf that arrived, or an emitted
+  // group); its completion seq.
+  bool child_complete(int level, const Group& g, uint32_t c, uint64_t* seq) {
+    if (level == depth - 1) {
+      auto it = g.leaves.find(c);
+      if (it == g.leaves.end()) return false;
+      *seq = it->second.seq;
+      return true;
+    }
+    auto it = g.child_group.find(c);
+    if (it == g.child_group.end()) return false;
+    auto gi = groups.find({level + 1, it->second});
+    if (gi == groups.end() || !gi->second.emitted) return false;
+    *seq = gi->second.done_seq;
+    return true;
   }
 
   // Largest leaf score of the subtree of (level, id).
@@ -176,6 +216,7 @@ struct Oracle {
   void emit(int level, uint32_t id, uint64_t seq) {
     Group& g = group(level, id);
     g.emitted = true;
+    g.done_seq = seq;
     OrcRecord r{};
     r.completion_seq = seq;
     r.parent_id = id;
@@ -183,7 +224,11 @@ struct Oracle {
     r.level = static_cast<uint8_t>(level);
     r.ops = static_cast<uint8_t>(payload_op[level] | (score_op[level] << 2));
     r.payload_off = payload.size();
-    if (payload_op[level] == kPayloadConcat) concat(level, id, payload);
+    if (payload_op[level] == kPayloadConcat) {
+      // with streaming release, the children released earlier are not repeated
+      const uint32_t from = stream_release ? g.released : 0;
+      concat_range(level, id, from, g.last + 1, payload);
+    }
     r.payload_len = payload.size() - r.payload_off;
     r.topk_off = topk.size();
     r.topk_n = 0;
@@ -242,6 +287,7 @@ struct Oracle {
           Leaf& lf = g.leaves[c];
           lf.tokens.assign(tokens, tokens + len);
           lf.score = score;
+          lf.seq = seq;
         }
       }
       if (!g.any_child || c > g.max_child) g.max_child = c;
@@ -254,6 +300,7 @@ struct Oracle {
         }
       }
       if (g.has_last && g.max_child > g.last) errors.insert(kELast);
+      if (stream_release && l == concat_level) touched.insert(pid);
     }
     if (!errors.empty()) return;
     // the leaf is complete on arrival; pop levels while the group closes
@@ -263,6 +310,66 @@ struct Oracle {
       g.completed += 1;
       if (!complete(g)) break;
       emit(l, pid, seq);
+    }
+  }
+
+  // End of a batch with streaming release: every touched, still open CONCAT
+  // group whose in-order prefix of complete children advanced emits those
+  // children as a partial record (flag 0x80 in ops, no score or top-k;
+  // n_children = children released so far; completion seq = the largest
+  // completion seq among them);
+  // the batch's records are then put in (completion seq, deeper first) order.
+  void release_prefixes(size_t rec_base, size_t pay_base, size_t tk_base) {
+    struct Ev {
+      OrcRecord r;
+      std::vector<int32_t> pay;
+      std::vector<OrcPair> tk;
+    };
+    std::vector<Ev> ev;
+    for (size_t k = rec_base; k < records.size(); ++k) {
+      Ev e;
+      e.r = records[k];
+      e.pay.assign(payload.begin() + records[k].payload_off,
+                   payload.begin() + records[k].payload_off + records[k].payload_len);
+      e.tk.assign(topk.begin() + records[k].topk_off, topk.begin() + records[k].topk_off + records[k].topk_n);
+      ev.push_back(std::move(e));
+    }
+    const int M = concat_level;
+    for (uint32_t pid : touched) {
+      Group& g = group(M, pid);
+      if (g.emitted) continue;
+      uint32_t r1 = g.released;
+      uint64_t mx = 0, sq = 0;
+      while (child_complete(M, g, r1, &sq)) {
+        mx = std::max(mx, sq);
+        ++r1;
+      }
+      if (r1 == g.released) continue;
+      Ev e;
+      e.r = OrcRecord{};
+      e.r.completion_seq = mx;
+      e.r.parent_id = pid;
+      e.r.n_children = r1;
+      e.r.level = static_cast<uint8_t>(M);
+      e.r.ops = static_cast<uint8_t>(kPayloadConcat | 0x80);   // payload only, no score
+      concat_range(M, pid, g.released, r1, e.pay);
+      e.r.payload_len = e.pay.size();
+      g.released = r1;
+      ev.push_back(std::move(e));
+    }
+    std::stable_sort(ev.begin(), ev.end(), [](const Ev& a, const Ev& b) {
+      if (a.r.completion_seq != b.r.completion_seq) return a.r.completion_seq < b.r.completion_seq;
+      return a.r.level > b.r.level;
+    });
+    records.resize(rec_base);
+    payload.resize(pay_base);
+    topk.resize(tk_base);
+    for (Ev& e : ev) {
+      e.r.payload_off = payload.size();
+      payload.insert(payload.end(), e.pay.begin(), e.pay.end());
+      e.r.topk_off = topk.size();
+      topk.insert(topk.end(), e.tk.begin(), e.tk.end());
+      records.push_back(e.r);
     }
   }
 
@@ -285,6 +392,8 @@ struct Oracle {
         if (std::isnan(score[i])) errors.insert(kEInval);
     }
     uint64_t seq_base = seq_next;
+    const size_t rec_base = records.size(), pay_base = payload.size(), tk_base = topk.size();
+    touched.clear();
     if (errors.empty()) {
       std::vector<uint64_t> tag(depth);
       for (int64_t i = 0; i < n; ++i) {
@@ -293,6 +402,7 @@ struct Oracle {
                  needs_score ? score[i] : 0.0f, seq_base + i, errors);
       }
     }
+    if (errors.empty() && stream_release) release_prefixes(rec_base, pay_base, tk_base);
     seq_next += n;
     batches += 1;
     if (!errors.empty()) {
@@ -379,6 +489,18 @@ int orc_drain(void* h, orc_drain* out) {
   out->n_batches = o->batches - o->drain_first_batch;
   o->drain_first_batch = o->batches;
   return o->status;
+}
+
+// Streaming release at the CONCAT level (before the first push).
+int orc_set_stream_release(void* h, int on) {
+  Oracle* o = static_cast<Oracle*>(h);
+  if (o == nullptr || o->batches != 0) return kEInval;
+  o->concat_level = -1;
+  for (int l = 0; l < o->depth; ++l)
+    if (o->payload_op[l] == kPayloadConcat) o->concat_level = l;
+  if (on && o->concat_level < 0) return kEInval;
+  o->stream_release = on != 0;
+  return kOk;
 }
 
 // Number of groups that have fragments but have not been emitted.

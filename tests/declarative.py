@@ -10,6 +10,13 @@ the batch whose prefix first makes it complete; its completion sequence number
 is the smallest arrival index whose prefix makes it complete, found by trying
 every prefix.  Records are ordered by (completion seq, deeper level first).
 
+With streaming release (Sec. 3.2: the reordered outputs of a pmap flow on as
+a stream), after each batch every open group at the CONCAT level whose run of
+complete children 0..r-1 is longer than the run it already released gets a
+partial record for the new children (ops bit 0x80, n_children = r, seq = the
+latest completion seq among them, no score); a group's final record then
+carries only the children it had not released.
+
 Fragments are plain Python: ``(tags, tokens, score)`` with ``tags`` a tuple of
 ``(parent_id, child_index, last)`` per level, outermost first.
 """
@@ -112,7 +119,13 @@ def _closed(depth, frags, upto):
     return False
 
 
-def evaluate(depth, payload_op, score_op, topk_k, frags, batch_sizes, csr_ok=None):
+def _completion_seq(depth, frags, end, g):
+    """Smallest arrival index whose prefix makes group g complete."""
+    return next(x for x in range(end) if g in _Tree(depth, frags[:x + 1]).kids
+                and _Tree(depth, frags[:x + 1]).complete(g))
+
+
+def evaluate(depth, payload_op, score_op, topk_k, frags, batch_sizes, csr_ok=None, stream_release=False):
     """Per batch: (status, records, payload, topk).  After the first batch
     with an error every later batch reports the same status and nothing else.
     ``csr_ok[b] = False`` marks a batch whose offsets or scores are invalid.
@@ -122,6 +135,8 @@ def evaluate(depth, payload_op, score_op, topk_k, frags, batch_sizes, csr_ok=Non
     status = OK
     start = 0
     prev_complete = set()
+    released = {}                 # CONCAT-level group -> children released so far
+    cl = payload_op.index(1) if 1 in list(payload_op)[:depth] else None
     for b, nb in enumerate(batch_sizes):
         end = start + nb
         if status != OK:
@@ -146,21 +161,53 @@ def evaluate(depth, payload_op, score_op, topk_k, frags, batch_sizes, csr_ok=Non
         prev_complete = now
         recs = []
         for g in new:
-            # smallest arrival index whose prefix completes g
-            s = next(x for x in range(end) if g in _Tree(depth, frags[:x + 1]).kids
-                     and _Tree(depth, frags[:x + 1]).complete(g))
-            recs.append((s, -g[0], g))
+            recs.append((_completion_seq(depth, frags, end, g), -g[0], g, None))
+        if stream_release and cl is not None:
+            for g in tree.kids:
+                if g[0] != cl or g in now:
+                    continue
+                r, seqs = 0, []
+                while r in tree.kids[g]:
+                    if cl == depth - 1:
+                        seqs.append(tree.kids[g][r])
+                    else:
+                        child = (cl + 1, tree.kids[g][r])
+                        if not tree.complete(child):
+                            break
+                        seqs.append(_completion_seq(depth, frags, end, child))
+                    r += 1
+                r0 = released.get(g, 0)
+                if r > r0:
+                    recs.append((max(seqs[r0:r]), -cl, g, (r0, r)))
+                    released[g] = r
         recs.sort()
         payload, topk, records = [], [], []
-        for s, _, g in recs:
+        for s, _, g, part in recs:
             l, p = g
+            if part is not None:          # partial record: children part[0]..part[1]-1
+                rec = dict(completion_seq=s, parent_id=p, n_children=part[1], level=l, ops=1 | 0x80,
+                           payload_off=len(payload), topk_off=len(topk), topk_n=0, score=0.0)
+                for c in range(part[0], part[1]):
+                    sub = [tree.kids[g][c]] if l == depth - 1 else tree.leaves((l + 1, tree.kids[g][c]))
+                    for i in sub:
+                        payload.extend(frags[i][1])
+                rec["payload_len"] = len(payload) - rec["payload_off"]
+                records.append(rec)
+                continue
             last = tree.last(g)
             leaves = tree.leaves(g)
+            if stream_release and l == cl and released.get(g, 0):
+                skip = set()
+                for c in range(released[g]):
+                    skip.update([tree.kids[g][c]] if l == depth - 1 else tree.leaves((l + 1, tree.kids[g][c])))
+                payload_leaves = [i for i in leaves if i not in skip]
+            else:
+                payload_leaves = leaves
             rec = dict(completion_seq=s, parent_id=p, n_children=last + 1, level=l,
                        ops=payload_op[l] | (score_op[l] << 2), payload_off=len(payload),
                        topk_off=len(topk), topk_n=0, score=0.0)
             if payload_op[l] == 1:
-                for i in leaves:
+                for i in payload_leaves:
                     payload.extend(frags[i][1])
             rec["payload_len"] = len(payload) - rec["payload_off"]
             if score_op[l] != 0:

@@ -60,8 +60,8 @@ def cuts(n):
         yield sizes
 
 
-def run_oracle(depth, po, so, kk, frags, sizes, corrupt=None):
-    o = oracle.Oracle(depth, po, so, kk)
+def run_oracle(depth, po, so, kk, frags, sizes, corrupt=None, stream_release=False):
+    o = oracle.Oracle(depth, po, so, kk, stream_release=stream_release)
     with_score = any(s != 0 for s in so)
     res = []
     for b, part in enumerate(split(frags, sizes)):
@@ -74,9 +74,9 @@ def run_oracle(depth, po, so, kk, frags, sizes, corrupt=None):
     return res
 
 
-def compare(depth, po, so, kk, frags, sizes, status_only=False):
-    want = evaluate(depth, po, so, kk, frags, sizes)
-    got = run_oracle(depth, po, so, kk, frags, sizes)
+def compare(depth, po, so, kk, frags, sizes, status_only=False, stream_release=False):
+    want = evaluate(depth, po, so, kk, frags, sizes, stream_release=stream_release)
+    got = run_oracle(depth, po, so, kk, frags, sizes, stream_release=stream_release)
     for b, ((st, recs, pay, topk), d) in enumerate(zip(want, got)):
         assert d.status == st, (b, d.status, st, frags, sizes)
         if status_only or st != 0:
@@ -123,6 +123,21 @@ def test_bruteforce_valid(depth):
         compare(depth, po, so, kk, frags, sizes)
         count += 1
     assert count > 50
+
+
+@pytest.mark.parametrize("depth", [1, 2, 3])
+def test_bruteforce_stream_release(depth):
+    """Streaming release at every CONCAT level: partial records per batch
+    against the prefix of complete children recomputed from scratch."""
+    count = partial = 0
+    for frags, sizes, po, so, kk in _cases(depth, samples=8, seed=31):
+        if 1 not in po:
+            continue
+        compare(depth, po, so, kk, frags, sizes, stream_release=True)
+        want = evaluate(depth, po, so, kk, frags, sizes, stream_release=True)
+        partial += sum(1 for _st, recs, _p, _t in want for r in recs if r["ops"] & 0x80)
+        count += 1
+    assert count > 20 and partial > 10
 
 
 def test_bruteforce_forest():
