@@ -94,6 +94,20 @@ typedef int alto_status;
 #define ALTO_SCORE_MAX 1
 #define ALTO_SCORE_TOPK 2
 
+/* Streaming release (flags bit 0; Sec. 3.2: the outputs of a pmap are put
+ * back in order and passed on as a stream).  With the CONCAT level at the
+ * leaf parent (D-1), every push also emits, for each still-open CONCAT group
+ * whose run of present children 0..r-1 grew past the r it released before,
+ * a partial record: ops = CONCAT | ALTO_OPS_PARTIAL, n_children = r, payload
+ * = the newly released children's tokens in child order, score 0, no top-k,
+ * completion_seq = the latest arrival among those children.  The group's
+ * final record then carries only the children not released before (its other
+ * fields are unchanged).  Records stay in (completion_seq, deeper first)
+ * order.  EINVAL with no CONCAT level, with CONCAT above the leaf parent, and
+ * for alto_agg_oneshot_noalloc. */
+#define ALTO_FLAG_STREAM_RELEASE 1
+#define ALTO_OPS_PARTIAL 0x80
+
 /* Aggregator configuration (Sec. 5: the controller is told which queues are
  * pmap entry/exit points and which data is aggregated; here: the nesting
  * depth and what each level's exit computes).  Zero capacities take the
@@ -112,6 +126,7 @@ typedef struct alto_agg_config {
   int64_t out_topk;                       /* top-k pairs held between drains (default out_records) */
   int64_t max_emit_children;              /* children of CONCAT groups completing in one push (default 4*max_batch_fragments) */
   int64_t spin_limit;                     /* device wait cap in polls (default 2^20) */
+  int64_t flags;                          /* ALTO_FLAG_* (0: none) */
 } alto_agg_config;
 
 /* Device memory provider.  alloc returns device memory of at least `bytes`

@@ -21,6 +21,10 @@
 //               level between completes into one span of its parent's vectors
 //               (gathered level by level, bottom-up) before level M gathers.
 //   records     one record per completed group, top-k pairs; free entries
+//   streaming   (optional) an open leaf-parent CONCAT group whose first
+//               unreleased child came in the batch releases its run of
+//               present children as a partial record, placed and gathered
+//               like a completion; its buffer then drops those children [Sec. 3.2]
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -86,6 +90,10 @@ struct Scratch {
   u64* pairset;          // [ps_mask + 1]
   u64 ps_mask;
   u32 done_cap;
+  // streaming release
+  u32* done_part;        // [done_cap] 1: the done entry is a partial release (cleared by the records)
+  u32* bm;               // [bm_cap] per-batch presence bitmaps of the groups that release
+  u64 bm_cap;
 };
 
 struct Dev {
@@ -141,6 +149,7 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
         tab.completed[h] = 0;
         tab.maxc1[h] = 0;
         tab.smax[h] = 0;
+        if (tab.rel) tab.rel[h] = 0;
         if (tab.vec_n) {
           tab.vec_n[2 * (u64)h] = 0;
           tab.vec_n[2 * (u64)h + 1] = 0;
@@ -404,6 +413,7 @@ __global__ void k_begin(Ctl* ctl, u32 n) {
   ctl->n_done = 0;
   ctl->skip_dense = 0;
   ctl->dense_total = ctl->arena_total = ctl->pay_total = ctl->topk_total = ctl->n_emit = 0;
+  ctl->bm_used = 0;
   for (int l = 0; l < kMaxDepth; ++l) ctl->n_segs[l] = 0;
   ctl->n = (ctl->status == ALTO_OK) ? n : 0u;
 }
@@ -417,7 +427,7 @@ __global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
   __syncthreads();
   const int D = d.cfg.depth;
   const u32 ep7 = epoch7(ctl);
-  const bool sorted_leaf = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK;
+  const bool sorted_leaf = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK || d.cfg.stream;
   for (u32 i = gtid(); i < b.n; i += gstride()) {
     u32 o0 = b.off[i], o1 = b.off[i + 1];
     if (o1 < o0 || (u64)o1 > b.n_payload) raise_err(ctl, ALTO_EINVAL);
@@ -486,6 +496,70 @@ __device__ __forceinline__ u64 shfl_xor_u64(u64 v, int o) {
   return __shfl_xor_sync(0xFFFFFFFFu, v, o);
 }
 
+// Streaming release of leaf-parent entry e, whose child `rel` (its first
+// unreleased one) is in this batch's segment [j0, j1): the end r1 of the run
+// of present children rel, rel+1, ..., and in *pcs the latest arrival among
+// the segment's leaves in that run.  The candidates are the entry's buffered
+// leaves (the B entries of its meta vector, all with child >= rel) and the
+// segment's leaves; with K of them the first missing child is at most rel+K,
+// so a bitmap of K+1 bits, taken from the batch's bitmap scratch, holds the
+// whole run.  Returns rel when the scratch is full (ENOSPC).  All 32 lanes
+// call it together.
+__device__ u32 release_run(const Dev& d, const Batch& b, Ctl* ctl, u32 e, u32 rel, u32 j0, u32 j1,
+                           const u32* sperm, u32 n_items, u32* pcs) {
+  const int lane = threadIdx.x & 31;
+  const int L = d.cfg.depth - 1;
+  const u64 n = b.n;
+  const u32 B = d.tab.vec_n[2 * (u64)e];
+  const u64 K = (u64)B + (j1 - j0);
+  const u64 words = (K >> 5) + 1;
+  unsigned long long base = 0;
+  if (lane == 0) base = atomicAdd((unsigned long long*)&ctl->bm_used, (unsigned long long)words);
+  base = __shfl_sync(0xFFFFFFFFu, base, 0);
+  if (base + words > d.sc.bm_cap) {
+    if (lane == 0) raise_err(ctl, ALTO_ENOSPC);
+    *pcs = 0;
+    return rel;
+  }
+  u32* bm = d.sc.bm + base;
+  for (u64 w = lane; w < words; w += 32) bm[w] = 0;
+  __syncwarp();
+  const u64 span = words * 32;
+  for (u32 j = j0 + lane; j < j1; j += 32) {
+    const u32 x = min(sperm[j], n_items - 1);
+    const u32 c = tag_child(b.tags[(u64)L * n + x]);
+    if (c >= rel && (u64)(c - rel) < span) atomicOr(&bm[(c - rel) >> 5], 1u << ((c - rel) & 31));
+  }
+  for (u32 k = lane; k < B; k += 32) {
+    bool ok;
+    const u64 a = vec_addr(d.tab, e, 0, 2 * (u64)k, &ok);
+    if (!ok) continue;
+    const u32 c = (u32)d.ar.pool[a];
+    if (c >= rel && (u64)(c - rel) < span) atomicOr(&bm[(c - rel) >> 5], 1u << ((c - rel) & 31));
+  }
+  __syncwarp();
+  // first clear bit: K candidates cannot fill K+1 bits, so there is one
+  u32 z = kNone;
+  for (u64 wb = 0; wb < words && z == kNone; wb += 32) {
+    const u64 w = wb + lane;
+    u32 cand = kNone;
+    if (w < words) {
+      const u32 free_bits = ~__ldcg(&bm[w]);
+      if (free_bits) cand = (u32)(w * 32) + (u32)(__ffs(free_bits) - 1);
+    }
+    z = __reduce_min_sync(0xFFFFFFFFu, cand);
+  }
+  const u32 r1 = (z == kNone) ? rel : rel + z;
+  u32 mx = 0;
+  for (u32 j = j0 + lane; j < j1; j += 32) {
+    const u32 x = min(sperm[j], n_items - 1);
+    const u32 c = tag_child(b.tags[(u64)L * n + x]);
+    if (c >= rel && c < r1) mx = max(mx, x);
+  }
+  *pcs = __reduce_max_sync(0xFFFFFFFFu, mx);
+  return r1;
+}
+
 // One warp per group present at level l: reduce its items, merge with the
 // table entry, test completion, and emit the group as an item of level l-1.
 template <bool LEAF>
@@ -504,6 +578,7 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
   const bool carry = LEAF && d.cfg.concat_level >= 0;
   const bool receives = !LEAF && chain_parent(d.cfg, l);
   const bool hands_up = chain_level(d.cfg, l);
+  const bool strm = LEAF && d.cfg.stream;
   const u32 ep = ctl->epoch;
   const u32* it_rep = d.sc.it_rep[in_set];
   const u32* it_cseq = d.sc.it_cseq[in_set];
@@ -525,6 +600,8 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
     for (int q = 0; q < kMaxDepth; ++q) htag[q] = (q < l) ? b.tags[(u64)q * n + rep0] : 0ull;
     u32 cnt = 0, m1 = 0, fmin = kNone, fmax = 0, hasf = 0, cmax = 0, smx = 0, bad = 0;
     u64 lsum = 0;
+    const u32 rel = strm ? d.tab.rel[e] : 0u;
+    u32 hitrel = 0, below = 0;  // streaming: child `rel` came / a released child came again
     u32 running = 0;  // payload elements of the segment's earlier leaves (leaf level)
     for (u32 jb = j0; jb < j1; jb += 32) {
       const u32 j = jb + lane;
@@ -549,6 +626,10 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
         const u64 t = b.tags[(u64)l * n + rep];
         const u32 c = tag_child(t);
         m1 = max(m1, c + 1);
+        if (strm) {
+          hitrel |= (c == rel) ? 1u : 0u;
+          below |= (c < rel) ? 1u : 0u;
+        }
         if (tag_last(t)) {
           hasf = 1;
           fmin = min(fmin, c);
@@ -585,6 +666,21 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
     bad = __reduce_or_sync(0xFFFFFFFFu, bad);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) lsum += shfl_xor_u64(lsum, o);
+    u32 r1 = rel, pcs = 0;
+    if (strm) {
+      hitrel = __reduce_or_sync(0xFFFFFFFFu, hitrel);
+      below = __reduce_or_sync(0xFFFFFFFFu, below);
+      if (below && lane == 0) raise_err(ctl, ALTO_EDUP);
+      if (hitrel) {
+        // the same completion test as below: a group that completes emits its final record instead
+        const u32 lo = d.tab.last[e];
+        const u32 nl = (lo == kNone && hasf) ? fmin : lo;
+        const bool closes = nl != kNone && d.tab.completed[e] + cnt == nl + 1 &&
+                            max(d.tab.maxc1[e], m1) <= nl + 1;
+        if (!closes) r1 = release_run(d, b, ctl, e, rel, j0, j1, sperm, n_items, &pcs);
+      }
+      __syncwarp();
+    }
 
     if (topk) {
       // running top-k of complete children: lane q holds the q-th best
@@ -645,15 +741,22 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
       d.tab.maxc1[e] = m1n;
       d.tab.completed[e] = comp;
       d.tab.smax[e] = smn;
-      if (complete) {
+      // a completing group, or (streaming) a partial release, takes a done entry
+      if (complete || r1 > rel) {
+        const bool part = !complete;
+        const u32 cs = part ? pcs : cmax;
         u32 di = atomicAdd(&ctl->n_done, 1u);
         if (di < d.sc.done_cap) {
           d.sc.done_e[di] = e;
           d.sc.done_lvl[di] = (u32)l;
-          d.sc.done_cseq[di] = cmax;
+          d.sc.done_cseq[di] = cs;
           d.tab.done_epoch[e] = ep;
           d.tab.done_idx[e] = di;
-          if (cmax < n) atomicOr(&d.sc.mask[cmax], 1u << (D - 1 - l));
+          if (strm) {
+            d.sc.done_part[di] = part ? 1u : 0u;
+            d.tab.rnew[e] = part ? r1 : nl + 1;
+          }
+          if (cs < n) atomicOr(&d.sc.mask[cs], 1u << (D - 1 - l));
         } else {
           raise_err(ctl, ALTO_ENOSPC);
         }
@@ -1008,8 +1111,13 @@ __global__ void __launch_bounds__(kThreads) k_done_rank(Dev d) {
     d.sc.done_rank[di] = r;
     d.sc.r_done[r] = di;
     const u32 nch = d.tab.last[e] + 1;
-    d.sc.r_dense_n[r] = (l == M) ? nch : 0u;
-    d.sc.r_topk_n[r] = (d.cfg.score_op[l] == ALTO_SCORE_TOPK) ? min(nch, (u32)d.cfg.topk_k[l]) : 0u;
+    // streaming: children rel.. of the run that ends this batch (all of them
+    // up to the last for a final record); a partial record has no top-k
+    const bool part = d.cfg.stream && d.sc.done_part[di];
+    const u32 rel = (d.cfg.stream && l == M) ? d.tab.rel[e] : 0u;
+    const u32 rend = part ? d.tab.rnew[e] : nch;
+    d.sc.r_dense_n[r] = (l == M) ? rend - rel : 0u;
+    d.sc.r_topk_n[r] = (!part && d.cfg.score_op[l] == ALTO_SCORE_TOPK) ? min(nch, (u32)d.cfg.topk_k[l]) : 0u;
     d.sc.r_meta_n[r] = (l == M) ? d.tab.vec_n[2 * (u64)e] : 0u;
   }
 }
@@ -1301,7 +1409,9 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
     if (di >= nd) continue;
     const u32 c = tag_child(b.tags[(u64)(D - 1) * n + i]);
     if (c > d.tab.last[e]) continue;
-    const u64 slot = d.tab.dbase[e] + c;  // the group's first slot, from the count scan
+    const u32 rel = d.cfg.stream ? d.tab.rel[e] : 0u;  // children below were released earlier
+    if (c < rel) continue;
+    const u64 slot = d.tab.dbase[e] + (c - rel);  // the group's first slot, from the count scan
     if (slot >= d.cfg.dense_cap) continue;
     const u32 old = atomicExch(&d.sc.dense[slot].x, ep);
     if (old == ep) raise_err(ctl, ALTO_EDUP);
@@ -1451,11 +1561,15 @@ __global__ void __launch_bounds__(kThreads) k_dense_arena(Dev d) {
     } else {
       end = d.tab.vec_n[2 * (u64)e + 1];
     }
-    if (c > d.tab.last[e] || end < pos) {
+    // streaming: the buffer holds children rel.. only; a partial release
+    // places those below rnew and keeps the rest
+    const u32 rel = (LEVEL_M && d.cfg.stream) ? d.tab.rel[e] : 0u;
+    if (c > d.tab.last[e] || end < pos || c < rel) {
       raise_err(ctl, ALTO_EDUP);
       continue;
     }
-    const u64 slot = d.tab.dbase[e] + c;
+    if (LEVEL_M && d.cfg.stream && d.sc.done_part[di] && c >= d.tab.rnew[e]) continue;
+    const u64 slot = d.tab.dbase[e] + (c - rel);
     if (slot >= d.cfg.dense_cap) continue;
     u32 old = atomicExch(&d.sc.dense[slot].x, ep);
     if (old == ep) raise_err(ctl, ALTO_EDUP);
@@ -1665,6 +1779,122 @@ __global__ void __launch_bounds__(kThreads) k_chain_gather(Dev d, Batch b, int l
   }
 }
 
+// Streaming release, after the gather has copied the released spans out: one
+// warp per partial release drops the released children (below rnew) from its
+// group's buffer.  The kept meta entries and payload spans move down in
+// place, in their order (a destination never lies above its source, and a
+// warp reads each step's 32 entries, or 32 elements, before it writes them);
+// chunks of classes past the new sizes go back to the free stacks.
+__global__ void __launch_bounds__(kThreads) k_stream_compact(Dev d) {
+  pdl_enter();
+  Ctl* ctl = d.ctl;
+  if (no_copy(ctl) || ctl->skip_dense) return;
+  const int lane = threadIdx.x & 31;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  const u32 gw = gtid() >> 5, nw = gstride() >> 5;
+  u64 freed = 0;
+  for (u32 di = gw; di < nd; di += nw) {
+    if (!d.sc.done_part[di]) continue;
+    const u32 e = d.sc.done_e[di] & d.tab.mask;
+    const u32 r1 = d.tab.rnew[e];
+    const u32 m = d.tab.vec_n[2 * (u64)e], p = d.tab.vec_n[2 * (u64)e + 1];
+    u32 km = 0, kp = 0;  // kept entries and elements so far
+    for (u32 kb = 0; kb < m; kb += 32) {
+      const u32 k = kb + lane;
+      u32 c = 0, pos = 0, end = 0;
+      bool ok = false;
+      if (k < m) {
+        bool ok0, ok1 = true;
+        const u64 a = vec_addr(d.tab, e, 0, 2 * (u64)k, &ok0);
+        if (ok0) {
+          c = (u32)d.ar.pool[a];
+          pos = (u32)d.ar.pool[a + 1];
+        }
+        if (k + 1 < m) {
+          const u64 a2 = vec_addr(d.tab, e, 0, 2 * (u64)(k + 1) + 1, &ok1);
+          end = ok1 ? (u32)d.ar.pool[a2] : pos;
+        } else {
+          end = p;
+        }
+        ok = ok0 && ok1 && end >= pos && end <= p;
+      }
+      const bool keep = ok && c >= r1;
+      const u32 len = keep ? end - pos : 0u;
+      u32 incl = len;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      const u32 km_mask = __ballot_sync(0xFFFFFFFFu, keep);
+      const u32 nidx = km + __popc(km_mask & lanemask_lt());
+      const u32 npos = kp + incl - len;
+      __syncwarp();  // every lane has read this step's entries
+      if (keep) {
+        bool okw;
+        const u64 a = vec_addr(d.tab, e, 0, 2 * (u64)nidx, &okw);
+        if (okw) {
+          d.ar.pool[a] = (int32_t)c;
+          d.ar.pool[a + 1] = (int32_t)npos;
+        }
+      }
+      // the kept spans, one after another, 32 elements a step
+      u32 pend = km_mask;
+      while (pend) {
+        const int src = __ffs(pend) - 1;
+        pend &= pend - 1;
+        const u32 sp = __shfl_sync(0xFFFFFFFFu, pos, src);
+        const u32 dp = __shfl_sync(0xFFFFFFFFu, npos, src);
+        const u32 sl = __shfl_sync(0xFFFFFFFFu, len, src);
+        if (sp == dp) continue;
+        for (u32 q0 = 0; q0 < sl; q0 += 32) {
+          const u32 q = q0 + lane;
+          int32_t v = 0;
+          bool okr = false;
+          if (q < sl) {
+            const u64 a = vec_addr(d.tab, e, 1, (u64)sp + q, &okr);
+            if (okr) v = d.ar.pool[a];
+          }
+          __syncwarp();
+          if (okr) {
+            bool okw;
+            const u64 a = vec_addr(d.tab, e, 1, (u64)dp + q, &okw);
+            if (okw) d.ar.pool[a] = v;
+          }
+          __syncwarp();
+        }
+      }
+      km += __popc(km_mask);
+      kp += __shfl_sync(0xFFFFFFFFu, incl, 31);
+    }
+    // classes that start at or past the new sizes go back to the free stacks
+    if (lane < kVecs) {
+      const int vec = lane;
+      const u64 old_el = (vec == 0) ? 2 * (u64)m : (u64)p;
+      const u64 new_el = (vec == 0) ? 2 * (u64)km : (u64)kp;
+      if (old_el > new_el) {
+        const int jf = (new_el == 0) ? 0 : chunk_of(new_el - 1) + 1;
+        const int jl = min(chunk_of(old_el - 1), kNumChunks - 1);
+        for (int j = jf; j <= jl; ++j) {
+          u32* slot = &d.tab.dir[((u64)e * kVecs + vec) * kNumChunks + j];
+          if (*slot != kNone) {
+            free_chunk(d.ar, ctl, j, *slot);
+            freed += chunk_size(j);
+          }
+          *slot = kNone;
+        }
+      }
+    }
+    __syncwarp();
+    if (lane == 0) {
+      d.tab.vec_n[2 * (u64)e] = km;
+      d.tab.vec_n[2 * (u64)e + 1] = kp;
+      d.tab.rel[e] = r1;
+    }
+  }
+  if (freed) atomicAdd((unsigned long long*)&ctl->arena_used, (unsigned long long)(-(long long)freed));
+}
+
 __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
   pdl_enter();
   Ctl* ctl = d.ctl;
@@ -1692,12 +1922,17 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
     u32 e = 0;
     int l = 0;
     u64 el[kVecs] = {0, 0};
+    bool part = false;  // a partial release: the group stays open
     if (mine) {
       e = d.sc.done_e[di] & d.tab.mask;
       l = (int)d.sc.done_lvl[di];
       const u32 cs = d.sc.done_cseq[di];
       const u32 r = d.sc.done_rank[di];
       if (cs < d.cfg.n_max) d.sc.mask[cs] = 0;
+      if (d.cfg.stream) {
+        part = d.sc.done_part[di] != 0;
+        d.sc.done_part[di] = 0;
+      }
       if (!skip && r != kNone) {
         alto_record rec;
         rec.completion_seq = ctl->seq_base + cs;
@@ -1716,10 +1951,11 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
         rec.topk_off = to;
         rec.topk_n = (uint16_t)tn;
         rec.parent_id = (u32)d.tab.key[e];
-        rec.n_children = d.tab.last[e] + 1;
+        rec.n_children = part ? d.tab.rnew[e] : d.tab.last[e] + 1;
         rec.level = (uint8_t)l;
-        rec.ops = (uint8_t)(((l == M) ? 1 : 0) | (d.cfg.score_op[l] << 2));
-        rec.score = (d.cfg.score_op[l] != ALTO_SCORE_NONE) ? key_score(d.tab.smax[e]) : 0.0f;
+        rec.ops = part ? (uint8_t)(ALTO_PAYLOAD_CONCAT | ALTO_OPS_PARTIAL)
+                       : (uint8_t)(((l == M) ? 1 : 0) | (d.cfg.score_op[l] << 2));
+        rec.score = (!part && d.cfg.score_op[l] != ALTO_SCORE_NONE) ? key_score(d.tab.smax[e]) : 0.0f;
         d.out_rec[ctl->rec_count + r] = rec;
         for (u32 q = 0; q < tn; ++q) {
           const u64 v = d.tab.topk[(u64)e * d.tab.kk + q];
@@ -1729,7 +1965,7 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
           d.out_topk[to + q] = p;
         }
       }
-      if (M >= 0 && l >= M) {
+      if (M >= 0 && l >= M && !part) {
         for (int vec = 0; vec < kVecs; ++vec) {
           el[vec] = (u64)d.tab.vec_n[2 * (u64)e + vec] * (vec == 0 ? 2 : 1);
           if (el[vec] == 0) continue;
@@ -1737,9 +1973,11 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
           for (int j = 0; j <= jl; ++j) atomicAdd(&s_cnt[j], 1u);
         }
       }
-      d.tab.key[e] = kTomb;
-      d.tab.cur[e] = 0;  // a slot taken later may receive spans in the launch that inserts it
-      atomicAdd(&s_del, 1u);
+      if (!part) {
+        d.tab.key[e] = kTomb;
+        d.tab.cur[e] = 0;  // a slot taken later may receive spans in the launch that inserts it
+        atomicAdd(&s_del, 1u);
+      }
     }
     __syncthreads();
     // one push per chunk class for the whole block
@@ -1749,7 +1987,7 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
       atomicAdd(&s_freed, (unsigned long long)s_cnt[j] * chunk_size(j));
     }
     __syncthreads();
-    if (mine && M >= 0 && l >= M) {
+    if (mine && M >= 0 && l >= M && !part) {
       for (int vec = 0; vec < kVecs; ++vec) {
         if (el[vec] == 0) continue;
         const int jl = min(chunk_of(el[vec] - 1), kNumChunks - 1);
@@ -1983,7 +2221,8 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   int site = 0;
   launch_pdl(k_ingest, grid, kThreads, 0, s, d, bt);
   p.launches += 1;
-  const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK;
+  // streaming release needs each leaf parent's leaves together: the sorted path
+  const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK || d.cfg.stream;
   int set = 0;
   if (leaf_sorted) {
     // leaf level with TOPK: sort fragments by their leaf-parent group so that
@@ -2120,6 +2359,10 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     // gather is the stage the measurement hooks time on their own
     k_gather<<<grid, kThreads, 0, s>>>(d, bt);
     p.launches += 1;
+    if (d.cfg.stream) {
+      launch_pdl(k_stream_compact, sgrid, kThreads, 0, s, d);
+      p.launches += 1;
+    }
   }
   p.enter(9);
   launch_pdl(k_records, sgrid, kThreads, 0, s, d);
@@ -2174,6 +2417,10 @@ alto_status validate(const alto_agg_config* c) {
       return ALTO_EINVAL;
   }
   if (nconcat > 1) return ALTO_EINVAL;
+  if (c->flags & ~(int64_t)ALTO_FLAG_STREAM_RELEASE) return ALTO_EINVAL;
+  // streaming release needs the CONCAT level at the leaf parent
+  if ((c->flags & ALTO_FLAG_STREAM_RELEASE) && c->payload_op[c->depth - 1] != ALTO_PAYLOAD_CONCAT)
+    return ALTO_EINVAL;
   if (c->max_batch_fragments < 1 || c->max_batch_fragments >= (1ll << 30)) return ALTO_EINVAL;
   if (c->max_batch_payload < 0 || c->max_batch_payload >= (1ll << 32)) return ALTO_EINVAL;
   if (c->max_open_groups < 0 || c->max_open_groups > (1ll << 25)) return ALTO_EINVAL;
@@ -2281,6 +2528,11 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(d.tab.dbase, u64, T);
   ALLOC(d.tab.bstate, uint4, T);
   ALLOC(d.tab.cbits, u64, 4 * T);
+  const bool strm = (cfg.flags & ALTO_FLAG_STREAM_RELEASE) != 0;
+  if (strm) {
+    ALLOC(d.tab.rel, u32, T);
+    ALLOC(d.tab.rnew, u32, T);
+  }
   d.tab.leaf_level = D - 1;
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
@@ -2305,6 +2557,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     d.cfg.topk_k[l] = (l < D && cfg.score_op[l] == ALTO_SCORE_TOPK) ? cfg.topk_k[l] : 0;
   }
   d.cfg.has_score = has_score;
+  d.cfg.stream = strm;
   d.cfg.n_max = (u32)nmax;
   d.cfg.out_records = (u64)cfg.out_records;
   d.cfg.out_payload = (u64)cfg.out_payload_elems;
@@ -2370,6 +2623,14 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(sc.pairset, u64, PS);
   sc.ps_mask = PS - 1;
   sc.done_cap = (u32)done_cap;
+  if (strm) {
+    // presence bitmaps of one batch: a releasing group takes (candidates / 32 + 1)
+    // words, its candidates being the batch's leaves plus its buffered ones
+    // (two arena elements of metadata each)
+    sc.bm_cap = (nmax + (u64)cfg.arena_elems / 2) / 32 + nmax + 32;
+    ALLOC(sc.done_part, u32, done_cap);
+    ALLOC(sc.bm, u32, sc.bm_cap);
+  }
   const u64 scan_tiles = std::max<u64>(std::max<u64>(dense_cap, done_cap), nmax) / kScanTile + 2;
   ALLOC(h->lbs.desc, ulonglong2, 3 * scan_tiles);
   h->lbs.tiles = scan_tiles;
@@ -2398,6 +2659,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   cudaMemsetAsync(h->leaf_sort.lookback, 0, sizeof(u64) * sort_tiles * 256, s);
   cudaMemsetAsync(h->lbs.desc, 0, sizeof(ulonglong2) * 3 * scan_tiles, s);
   if (concat >= 0) cudaMemsetAsync(sc.dense, 0, sizeof(uint4) * std::max<u64>(dense_cap, 1), s);
+  if (strm) cudaMemsetAsync(sc.done_part, 0, sizeof(u32) * done_cap, s);
   if (cudaGetLastError() != cudaSuccess) {
     free_all(h, s);
     delete h;
@@ -2806,6 +3068,7 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
   alto_agg_config cfg = *cfg_in;
   if (cfg.max_batch_fragments == 0) cfg.max_batch_fragments = (int64_t)kNaMaxFragments;
   if (cfg.max_batch_payload == 0) cfg.max_batch_payload = (int64_t)kNaMaxPayload;
+  if (cfg.flags != 0) return ALTO_EINVAL;  // one batch: nothing to release in a stream
   alto_status v = validate(&cfg);
   if (v != ALTO_OK) return v;
   if (b->depth != cfg.depth || b->n < 0 || b->n_payload < 0) return ALTO_EINVAL;

@@ -54,6 +54,7 @@ struct Ctl {
   u64 n_emit;              // records ranked by this batch
   u64 chain_total;         // dense child slots of completing groups at levels M < l
   u64 chain_arena;         // their buffered child spans
+  u64 bm_used;             // streaming release: words of the presence bitmaps handed out
   u64 scan_total[kSites];  // totals written by scans
 };
 
@@ -176,6 +177,11 @@ struct Table {
   u32* cidx;       // [T] its child index in that parent
   u64* app;        // [T] its reserved place there: span index << 40 | payload position
   u64* cbits;      // [T][4] leaf parents: leaf slots 0..255 seen while the group is open
+  // streaming release (CONCAT at the leaf parent): children 0..rel-1 were
+  // released by partial records and are no longer buffered; rnew is where
+  // the release of the current batch ends (a partial or the final record)
+  u32* rel;        // [T]
+  u32* rnew;       // [T]
   int leaf_level;  // D - 1
   int chain_len;   // D - 1
   u32 mask;        // T - 1
@@ -197,6 +203,7 @@ struct Cfg {
   int score_op[kMaxDepth];
   int topk_k[kMaxDepth];
   bool has_score;
+  bool stream;          // streaming release at the CONCAT (leaf-parent) level
   u32 n_max;
   u64 out_records, out_payload, out_topk, dense_cap;
   u64 spin_limit;

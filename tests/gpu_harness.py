@@ -8,8 +8,9 @@ import oracle
 import paper_2403_04311_gb300 as alto
 
 
-def stream_caps(s, arena_factor=4):
-    """Capacities that hold a whole generated stream."""
+def stream_caps(s, arena_factor=4, stream_release=False):
+    """Capacities that hold a whole generated stream (with streaming release,
+    every fragment may also bring one partial record)."""
     D, n = s.depth, s.n
     groups = sum(len(np.unique(s.tags[l] >> np.uint64(32))) for l in range(D))
     st = s.batch_starts()
@@ -21,7 +22,7 @@ def stream_caps(s, arena_factor=4):
         max_open_groups=min(groups + 1024, 1 << 25),
         arena_elems=min(arena_factor * (int(s.payload.size) + 2 * n) + 64 * groups + (1 << 16),
                         (1 << 32) - 1),
-        out_records=groups + 16,
+        out_records=groups + 16 + (n if stream_release else 0),
         out_payload_elems=int(s.payload.size) + 16,
         out_topk=groups * kmax + 16,
         max_emit_children=n + 16,
@@ -50,8 +51,8 @@ def run_gpu_batches(depth, payload_op, score_op, topk_k, batches, caps, drain_af
     return pushes, drains
 
 
-def run_oracle_batches(depth, payload_op, score_op, topk_k, batches, drain_after=None):
-    o = oracle.Oracle(depth, payload_op, score_op, topk_k)
+def run_oracle_batches(depth, payload_op, score_op, topk_k, batches, drain_after=None, stream_release=False):
+    o = oracle.Oracle(depth, payload_op, score_op, topk_k, stream_release=stream_release)
     out = []
     for b, bt in enumerate(batches):
         o.push_batch(bt)
@@ -77,10 +78,12 @@ def assert_same(oracle_drains, gpu_drains, ctx=""):
         assert np.array_equal(tk.view(np.uint8), od.topk.view(np.uint8)), f"{ctx} drain {k}: top-k differs"
 
 
-def run_both_stream(s, drain_every=1, caps=None):
+def run_both_stream(s, drain_every=1, caps=None, stream_release=False):
     batches = [s.batch(b) for b in range(s.n_batches)]
     da = [((b + 1) % drain_every == 0) for b in range(s.n_batches)]
-    caps = caps or stream_caps(s)
+    caps = dict(caps or stream_caps(s, stream_release=stream_release))
+    if stream_release:
+        caps["stream_release"] = True
     _, g = run_gpu_batches(s.depth, s.payload_op, s.score_op, s.topk_k, batches, caps, da)
-    o = run_oracle_batches(s.depth, s.payload_op, s.score_op, s.topk_k, batches, da)
+    o = run_oracle_batches(s.depth, s.payload_op, s.score_op, s.topk_k, batches, da, stream_release)
     return o, g

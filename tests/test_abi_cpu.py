@@ -58,14 +58,31 @@ def _cfg(**kw):
     dict(max_batch_payload=-1),
     dict(max_open_groups=(1 << 25) + 1),
     dict(arena_elems=1 << 32),
+    dict(payload_op=[1, 0], stream_release=True),    # streaming release above the leaf parent
+    dict(payload_op=[0, 0], stream_release=True),    # streaming release without CONCAT
+    dict(flags=2),                                   # unknown flag
 ])
 def test_create_rejects_bad_configs_on_host(bad):
     lib = alto.load_library()
+    bad = dict(bad)
+    flags = bad.pop("flags", None)
     cfg = _cfg(**bad)
+    if flags is not None:
+        cfg.flags = flags
     h = ctypes.c_void_p(12345)
     st = lib.alto_agg_create(ctypes.byref(cfg), None, None, ctypes.byref(h))
     assert st == alto.EINVAL
     assert h.value == 12345  # untouched
+
+
+def test_noalloc_refuses_stream_release_on_host():
+    """One batch has nothing to release in a stream: refused before any device work."""
+    cfg = _cfg(stream_release=True)
+    b = alto.alto_batch()
+    b.depth = 2
+    counts = (ctypes.c_int64 * 4)()
+    st = alto.alto_agg_oneshot_noalloc(cfg, b, 0, 0, 0, 0, 0, 0, ctypes.addressof(counts), 0)
+    assert st == alto.EINVAL
 
 
 def test_null_arguments():
