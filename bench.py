@@ -12,6 +12,11 @@ timed region; they are far larger than L2 (tags 512 MB, payload 2.1 GB), so no
 flush is needed between steps.  Prints ONE JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload NAME] [--stream-release]
+
+--stream-release runs the same stream with streaming release (Sec. 3.2):
+open CONCAT groups also emit the in-order run of their present children
+after every push.
 
 --impl reference times the CPU oracle (the plain arrival-order definition) on
 this host's cores over a bounded sample of the same stream; it is the
@@ -46,7 +51,7 @@ def peaks():
         return 6800.0, "fallback"
 
 
-def stream_caps(s):
+def stream_caps(s, stream_release=False):
     import numpy as np
     D, n = s.depth, s.n
     st = s.batch_starts()
@@ -57,10 +62,12 @@ def stream_caps(s):
         max_batch_payload=max(1, max(pay_b)),
         max_open_groups=min(1 << 24, groups),
         arena_elems=min((1 << 32) - 1, 3 * (int(s.payload.size) + 2 * n) + 64 * groups),
-        out_records=groups + 16,
+        # with streaming release every fragment may also bring one partial record
+        out_records=groups + 16 + (n if stream_release else 0),
         out_payload_elems=int(s.payload.size) + 16,
         out_topk=groups * max(list(s.topk_k) + [1]) + 16,
         max_emit_children=n + 16,
+        stream_release=stream_release,
     )
 
 
@@ -147,7 +154,7 @@ def run_reference(args, s, rank, world):
                   score=None if b0["score"] is None else b0["score"][:n])
 
     def step():
-        o = oracle.Oracle.for_stream(s)
+        o = oracle.Oracle.for_stream(s, args.stream_release)
         o.push_batch(sample)
         d = o.drain()
         o.close()
@@ -165,7 +172,8 @@ def run_reference(args, s, rank, world):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
         "data": "synthetic", "config": {"workload": s.name, "fragments": s.n, "depth": s.depth,
-                                        "batch": int(s.batch_sizes[0])},
+                                        "batch": int(s.batch_sizes[0]),
+                                        "stream_release": bool(args.stream_release)},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": f"first {n} fragments of batch 0 of the {s.name} stream, "
                                    f"one batch per step, single thread"},
@@ -368,12 +376,12 @@ def run_route(args, rank, world, R=8):
             "e2e": None}
 
 
-def cpu_baseline(s, budget_s=20.0):
+def cpu_baseline(s, budget_s=20.0, stream_release=False):
     """Oracle fragments/s on a bounded sample (batches in order until the
     budget is spent), one host thread."""
     import oracle
     oracle.build()
-    o = oracle.Oracle.for_stream(s)
+    o = oracle.Oracle.for_stream(s, stream_release)
     done, t0 = 0, time.perf_counter()
     nb = 0
     for b in range(s.n_batches):
@@ -399,6 +407,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="throughput")
     ap.add_argument("--small", action="store_true", help="scaled-down stream (quick checks)")
+    ap.add_argument("--stream-release", action="store_true",
+                    help="streaming release of open CONCAT groups after every push")
     ap.add_argument("--ref-sample", type=float, default=250_000)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--latency-batches", type=int, default=16)
@@ -452,9 +462,9 @@ def main():
             s, tags=s.tags[:, :n_pref], off=s.off[:n_pref + 1],
             payload=s.payload[:int(s.off[n_pref])],
             score=None if s.score is None else s.score[:n_pref], batch_sizes=s.batch_sizes[:nbp])
-        caps = stream_caps(s_caps)
+        caps = stream_caps(s_caps, args.stream_release)
     else:
-        caps = stream_caps(s)
+        caps = stream_caps(s, args.stream_release)
     agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, stream=stream, **caps)
     nb = s.n_batches if args.max_batches <= 0 else min(args.max_batches, s.n_batches)
     batches = [alto.to_device(s.batch(b)) for b in range(nb)]
@@ -520,8 +530,16 @@ def main():
     #   k_gather: 4 bytes read + 4 written per emitted payload element.
     pushes = max(1, prof["pushes"])
     frag_bytes = 8.0 * s.depth + 4.0 + 4.0 + (4.0 if s.score is not None else 0.0)
+    # with streaming release (or TOPK at the leaf parent) the leaf level takes
+    # the sorted path: that stage is the segment scan + k_reduce<true>, which
+    # read per leaf its D tags, its offsets, its sorted position and write its
+    # segment offset
+    sorted_leaf = args.stream_release or s.score_op[s.depth - 1] == 2
+    leaf_name = "k_reduce_leaf" if sorted_leaf else "k_leaf_accumulate"
+    leaf_bytes = (8.0 * s.depth + 8.0 + 4.0 + 4.0 + (4.0 if s.score is not None else 0.0)) if sorted_leaf \
+        else frag_bytes
     kernels = {
-        "k_leaf_accumulate": (frag_bytes * s.n / s.n_batches, prof["stage_ms"]["leaf_accumulate"] / pushes),
+        leaf_name: (leaf_bytes * s.n / s.n_batches, prof["stage_ms"]["leaf_accumulate"] / pushes),
         "k_gather": (8.0 * n_payload_step / s.n_batches, prof["stage_ms"]["gather"] / pushes),
     }
     traffic_all = {}
@@ -634,7 +652,7 @@ def main():
         return
     cpu = None
     if not args.no_cpu_baseline and world == 1:
-        cpu = cpu_baseline(s)
+        cpu = cpu_baseline(s, stream_release=args.stream_release)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
@@ -642,7 +660,8 @@ def main():
         "config": {"workload": s.name, "fragments": s.n, "depth": s.depth,
                    "batch": int(s.batch_sizes[0]), "payload_tokens": int(s.payload.size),
                    "span_fraction": s.meta.get("span_fraction"),
-                   "l2": "inputs larger than L2 (no flush)", "parallelism": f"replicas x{world}"},
+                   "l2": "inputs larger than L2 (no flush)", "parallelism": f"replicas x{world}",
+                   "stream_release": bool(args.stream_release)},
         "payload_gbps": payload_bytes * world * args.steps / (ms / 1e3) / 1e9,
         "algorithmic_gbps": alg_bytes * world * args.steps / (ms / 1e3) / 1e9,
         "hbm_frac_path": alg_bytes * args.steps / (ms / 1e3) / 1e9 / hbm_gbs,

@@ -67,8 +67,9 @@ struct Scratch {
   u32* it_skey[2];       // items: largest score key of the child
   u32* seg_vb0;          // leaf segments: meta vector base (leaves)
   u32* seg_vb1;          // leaf segments: payload vector base (elements)
-  u32* seg_carry;        // leaf segments: 1 to the arena, 2 placed densely
-  u32* leaf_pos;         // [n_max] sorted leaf j: payload offset inside its segment
+  u32* seg_carry;        // leaf segments: 1 to the arena, 2 placed densely, 3 both (a partial release)
+  u32* leaf_pos;         // [n_max] sorted leaf j: payload offset inside its segment's buffered data
+  u32* leaf_mrank;       // [n_max] streaming, segments 3: meta index among the buffered leaves, kNone if placed
   u32* mask;             // [n_max] bit (D-1-l): a level-l group completes at this seq
   u32* prefix;           // [n_max] records completed before this seq
   u32* done_e;           // [done_cap]
@@ -91,7 +92,8 @@ struct Scratch {
   u64 ps_mask;
   u32 done_cap;
   // streaming release
-  u32* done_part;        // [done_cap] 1: the done entry is a partial release (cleared by the records)
+  u32* done_part;        // [done_cap] a partial release (cleared by the records): 1, or 2 when
+                         // children buffered by earlier batches were released (the buffer is compacted)
   u32* bm;               // [bm_cap] per-batch presence bitmaps of the groups that release
   u64 bm_cap;
 };
@@ -666,7 +668,7 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
     bad = __reduce_or_sync(0xFFFFFFFFu, bad);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) lsum += shfl_xor_u64(lsum, o);
-    u32 r1 = rel, pcs = 0;
+    u32 r1 = rel, pcs = 0, kept_n = 0, kept_len = 0;
     if (strm) {
       hitrel = __reduce_or_sync(0xFFFFFFFFu, hitrel);
       below = __reduce_or_sync(0xFFFFFFFFu, below);
@@ -678,6 +680,36 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
         const bool closes = nl != kNone && d.tab.completed[e] + cnt == nl + 1 &&
                             max(d.tab.maxc1[e], m1) <= nl + 1;
         if (!closes) r1 = release_run(d, b, ctl, e, rel, j0, j1, sperm, n_items, &pcs);
+        if (r1 > rel) {
+          // the segment's leaves below r1 are placed densely straight from the
+          // batch; the others are buffered, packed: their meta index and
+          // payload offset among the kept leaves
+          for (u32 jb = j0; jb < j1; jb += 32) {
+            const u32 j = jb + lane;
+            const bool valid = j < j1;
+            u32 c = 0, len = 0;
+            if (valid) {
+              const u32 x = min(sperm[j], n_items - 1);
+              c = tag_child(b.tags[(u64)l * n + x]);
+              len = b.off[x + 1] - b.off[x];
+            }
+            const bool keep = valid && c >= r1;
+            const u32 kl = keep ? len : 0u;
+            u32 incl = kl;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+              const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+              if (lane >= o) incl += y;
+            }
+            const u32 km = __ballot_sync(0xFFFFFFFFu, keep);
+            if (valid) {
+              d.sc.leaf_pos[j] = kept_len + incl - kl;
+              d.sc.leaf_mrank[j] = keep ? kept_n + __popc(km & lanemask_lt()) : kNone;
+            }
+            kept_n += __popc(km);
+            kept_len += __shfl_sync(0xFFFFFFFFu, incl, 31);
+          }
+        }
       }
       __syncwarp();
     }
@@ -753,7 +785,7 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
           d.tab.done_epoch[e] = ep;
           d.tab.done_idx[e] = di;
           if (strm) {
-            d.sc.done_part[di] = part ? 1u : 0u;
+            d.sc.done_part[di] = !part ? 0u : (d.tab.vec_n[2 * (u64)e] ? 2u : 1u);
             d.tab.rnew[e] = part ? r1 : nl + 1;
           }
           if (cs < n) atomicOr(&d.sc.mask[cs], 1u << (D - 1 - l));
@@ -762,13 +794,15 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
         }
       }
       if (carry) {
-        d.sc.seg_carry[s] = complete ? 2u : 1u;  // 1: to the arena, 2: placed densely
+        // 1: to the arena, 2: placed densely, 3: a partial release, both
+        const bool part = !complete && r1 > rel;
+        d.sc.seg_carry[s] = complete ? 2u : (part ? 3u : 1u);
         if (!complete) {
           const u32 v0 = d.tab.vec_n[2 * (u64)e], v1 = d.tab.vec_n[2 * (u64)e + 1];
           d.sc.seg_vb0[s] = v0;
           d.sc.seg_vb1[s] = v1;
-          d.tab.vec_n[2 * (u64)e] = v0 + (j1 - j0);
-          d.tab.vec_n[2 * (u64)e + 1] = v1 + (u32)lsum;
+          d.tab.vec_n[2 * (u64)e] = v0 + (part ? kept_n : (j1 - j0));
+          d.tab.vec_n[2 * (u64)e + 1] = v1 + (part ? kept_len : (u32)lsum);
         }
       }
       if (hands_up && complete) {
@@ -1274,7 +1308,7 @@ __global__ void __launch_bounds__(kThreads) k_carry_alloc(Dev d) {
     u32 rr[kMaxReq];
     bool want = false;
     u64 old0 = 0, old1 = 0;
-    if (s < nseg && d.sc.seg_carry[s] == 1u) {
+    if (s < nseg && (d.sc.seg_carry[s] == 1u || d.sc.seg_carry[s] == 3u)) {
       e = d.sc.leaf_keys[d.sc.leaf_seg_start[s]] & d.tab.mask;
       want = true;
       old0 = d.sc.seg_vb0[s];
@@ -1349,7 +1383,9 @@ __global__ void k_fix_tops(Ctl* ctl) {
 
 // Append the leaves of open CONCAT groups to their arena vectors: eight lanes
 // per leaf, over the sorted leaves.  A leaf's vector position is its group's
-// reserved base plus its offset inside the segment (written by the reduce).
+// reserved base plus its offset inside the segment (written by the reduce;
+// for a partial release, among the leaves it keeps).  (A lane per leaf with
+// the spans then copied four at a time, as in the gather, measured slower.)
 __global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch b) {
   pdl_enter();
   Ctl* ctl = d.ctl;
@@ -1361,15 +1397,20 @@ __global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch b) {
   const u32 g0 = gtid() >> 3, ng = gstride() >> 3;
   for (u32 j = g0; j < b.n; j += ng) {
     const u32 s = d.sc.leaf_seg_of[j];
-    if (s >= nseg || d.sc.seg_carry[s] != 1u) continue;
+    if (s >= nseg) continue;
+    const u32 sc_mode = d.sc.seg_carry[s];
+    if (sc_mode != 1u && sc_mode != 3u) continue;
     const u32 i = d.sc.leaf_perm[j];
     if (i >= b.n) continue;
     const u32 e = d.sc.leaf_keys[j] & d.tab.mask;
     const u32 s0 = d.sc.leaf_seg_start[s];
     if (s0 > j) continue;
+    // a partial release buffers only the leaves it keeps
+    const u32 mr = (sc_mode == 3u) ? d.sc.leaf_mrank[j] : j - s0;
+    if (mr == kNone) continue;
     const u32 o0 = b.off[i];
     const u32 len = b.off[i + 1] - o0;
-    const u64 mpos = (u64)d.sc.seg_vb0[s] + (j - s0);
+    const u64 mpos = (u64)d.sc.seg_vb0[s] + mr;
     const u64 ppos = (u64)d.sc.seg_vb1[s] + d.sc.leaf_pos[j];
     if (mpos >= d.tab.vec_n[2 * (u64)e] || ppos + len > d.tab.vec_n[2 * (u64)e + 1] ||
         (u64)o0 + len > b.n_payload)
@@ -1389,7 +1430,8 @@ __global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch b) {
   }
 }
 
-// Dense child slots of completing CONCAT groups, from this batch's leaves.
+// Dense child slots of completing CONCAT groups, from this batch's leaves
+// (and, streaming, of the leaves a partial release takes from the batch).
 __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
   pdl_enter();
   Ctl* ctl = d.ctl;
@@ -1401,7 +1443,9 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
   const u32 nseg = min(ctl->n_segs[D - 1], d.cfg.n_max);
   for (u32 j = gtid(); j < b.n; j += gstride()) {
     const u32 s = d.sc.leaf_seg_of[j];
-    if (s >= nseg || d.sc.seg_carry[s] != 2u) continue;
+    if (s >= nseg) continue;
+    const u32 sc_mode = d.sc.seg_carry[s];
+    if (sc_mode != 2u && sc_mode != 3u) continue;
     const u32 e = d.sc.leaf_keys[j] & d.tab.mask;
     const u32 i = d.sc.leaf_perm[j];
     if (i >= b.n || d.tab.done_epoch[e] != ep) continue;
@@ -1411,6 +1455,7 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
     if (c > d.tab.last[e]) continue;
     const u32 rel = d.cfg.stream ? d.tab.rel[e] : 0u;  // children below were released earlier
     if (c < rel) continue;
+    if (sc_mode == 3u && c >= d.tab.rnew[e]) continue;   // kept in the buffer
     const u64 slot = d.tab.dbase[e] + (c - rel);  // the group's first slot, from the count scan
     if (slot >= d.cfg.dense_cap) continue;
     const u32 old = atomicExch(&d.sc.dense[slot].x, ep);
@@ -1779,12 +1824,113 @@ __global__ void __launch_bounds__(kThreads) k_chain_gather(Dev d, Batch b, int l
   }
 }
 
-// Streaming release, after the gather has copied the released spans out: one
-// warp per partial release drops the released children (below rnew) from its
-// group's buffer.  The kept meta entries and payload spans move down in
-// place, in their order (a destination never lies above its source, and a
-// warp reads each step's 32 entries, or 32 elements, before it writes them);
-// chunks of classes past the new sizes go back to the free stacks.
+// Streaming release, after the gather has copied the released spans out:
+// drop the released children (those below rnew) of entry e from its buffer.
+// The kept meta entries and payload spans move down in place, in their order
+// (a destination never lies above its source, and the warp reads each step's
+// 32 entries, or 32 elements, before it writes them); chunks of classes past
+// the new sizes go back to the free stacks.  All 32 lanes call it together;
+// returns the elements freed (lanes 0 and 1).
+__device__ u64 compact_buffer(const Dev& d, Ctl* ctl, u32 e) {
+  const int lane = threadIdx.x & 31;
+  const u32 r1 = d.tab.rnew[e];
+  const u32 m = d.tab.vec_n[2 * (u64)e], p = d.tab.vec_n[2 * (u64)e + 1];
+  u32 km = 0, kp = 0;  // kept entries and elements so far
+  for (u32 kb = 0; kb < m; kb += 32) {
+    const u32 k = kb + lane;
+    u32 c = 0, pos = 0, end = 0;
+    bool ok = false;
+    if (k < m) {
+      bool ok0, ok1 = true;
+      const u64 a = vec_addr(d.tab, e, 0, 2 * (u64)k, &ok0);
+      if (ok0) {
+        c = (u32)d.ar.pool[a];
+        pos = (u32)d.ar.pool[a + 1];
+      }
+      if (k + 1 < m) {
+        const u64 a2 = vec_addr(d.tab, e, 0, 2 * (u64)(k + 1) + 1, &ok1);
+        end = ok1 ? (u32)d.ar.pool[a2] : pos;
+      } else {
+        end = p;
+      }
+      ok = ok0 && ok1 && end >= pos && end <= p;
+    }
+    const bool keep = ok && c >= r1;
+    const u32 len = keep ? end - pos : 0u;
+    u32 incl = len;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    const u32 kmask = __ballot_sync(0xFFFFFFFFu, keep);
+    const u32 nidx = km + __popc(kmask & lanemask_lt());
+    const u32 npos = kp + incl - len;
+    __syncwarp();  // every lane has read this step's entries
+    if (keep) {
+      bool okw;
+      const u64 a = vec_addr(d.tab, e, 0, 2 * (u64)nidx, &okw);
+      if (okw) {
+        d.ar.pool[a] = (int32_t)c;
+        d.ar.pool[a + 1] = (int32_t)npos;
+      }
+    }
+    // the kept spans, one after another, 32 elements a step
+    u32 pend = kmask;
+    while (pend) {
+      const int src = __ffs(pend) - 1;
+      pend &= pend - 1;
+      const u32 sp = __shfl_sync(0xFFFFFFFFu, pos, src);
+      const u32 dp = __shfl_sync(0xFFFFFFFFu, npos, src);
+      const u32 sl = __shfl_sync(0xFFFFFFFFu, len, src);
+      if (sp == dp) continue;
+      for (u32 q0 = 0; q0 < sl; q0 += 32) {
+        const u32 q = q0 + lane;
+        int32_t v = 0;
+        bool okr = false;
+        if (q < sl) {
+          const u64 a = vec_addr(d.tab, e, 1, (u64)sp + q, &okr);
+          if (okr) v = d.ar.pool[a];
+        }
+        __syncwarp();
+        if (okr) {
+          bool okw;
+          const u64 a = vec_addr(d.tab, e, 1, (u64)dp + q, &okw);
+          if (okw) d.ar.pool[a] = v;
+        }
+        __syncwarp();
+      }
+    }
+    km += __popc(kmask);
+    kp += __shfl_sync(0xFFFFFFFFu, incl, 31);
+  }
+  u64 freed = 0;
+  if (lane < kVecs) {
+    const int vec = lane;
+    const u64 old_el = (vec == 0) ? 2 * (u64)m : (u64)p;
+    const u64 new_el = (vec == 0) ? 2 * (u64)km : (u64)kp;
+    if (old_el > new_el) {
+      const int jf = (new_el == 0) ? 0 : chunk_of(new_el - 1) + 1;
+      const int jl = min(chunk_of(old_el - 1), kNumChunks - 1);
+      for (int j = jf; j <= jl; ++j) {
+        u32* slot = &d.tab.dir[((u64)e * kVecs + vec) * kNumChunks + j];
+        if (*slot != kNone) {
+          free_chunk(d.ar, ctl, j, *slot);
+          freed += chunk_size(j);
+        }
+        *slot = kNone;
+      }
+    }
+  }
+  __syncwarp();
+  if (lane == 0) {
+    d.tab.vec_n[2 * (u64)e] = km;
+    d.tab.vec_n[2 * (u64)e + 1] = kp;
+  }
+  return freed;
+}
+
+// One warp per partial release that took children buffered by earlier batches.
 __global__ void __launch_bounds__(kThreads) k_stream_compact(Dev d) {
   pdl_enter();
   Ctl* ctl = d.ctl;
@@ -1793,103 +1939,12 @@ __global__ void __launch_bounds__(kThreads) k_stream_compact(Dev d) {
   const u32 nd = min(ctl->n_done, d.sc.done_cap);
   const u32 gw = gtid() >> 5, nw = gstride() >> 5;
   u64 freed = 0;
-  for (u32 di = gw; di < nd; di += nw) {
-    if (!d.sc.done_part[di]) continue;
-    const u32 e = d.sc.done_e[di] & d.tab.mask;
-    const u32 r1 = d.tab.rnew[e];
-    const u32 m = d.tab.vec_n[2 * (u64)e], p = d.tab.vec_n[2 * (u64)e + 1];
-    u32 km = 0, kp = 0;  // kept entries and elements so far
-    for (u32 kb = 0; kb < m; kb += 32) {
-      const u32 k = kb + lane;
-      u32 c = 0, pos = 0, end = 0;
-      bool ok = false;
-      if (k < m) {
-        bool ok0, ok1 = true;
-        const u64 a = vec_addr(d.tab, e, 0, 2 * (u64)k, &ok0);
-        if (ok0) {
-          c = (u32)d.ar.pool[a];
-          pos = (u32)d.ar.pool[a + 1];
-        }
-        if (k + 1 < m) {
-          const u64 a2 = vec_addr(d.tab, e, 0, 2 * (u64)(k + 1) + 1, &ok1);
-          end = ok1 ? (u32)d.ar.pool[a2] : pos;
-        } else {
-          end = p;
-        }
-        ok = ok0 && ok1 && end >= pos && end <= p;
-      }
-      const bool keep = ok && c >= r1;
-      const u32 len = keep ? end - pos : 0u;
-      u32 incl = len;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-        if (lane >= o) incl += y;
-      }
-      const u32 km_mask = __ballot_sync(0xFFFFFFFFu, keep);
-      const u32 nidx = km + __popc(km_mask & lanemask_lt());
-      const u32 npos = kp + incl - len;
-      __syncwarp();  // every lane has read this step's entries
-      if (keep) {
-        bool okw;
-        const u64 a = vec_addr(d.tab, e, 0, 2 * (u64)nidx, &okw);
-        if (okw) {
-          d.ar.pool[a] = (int32_t)c;
-          d.ar.pool[a + 1] = (int32_t)npos;
-        }
-      }
-      // the kept spans, one after another, 32 elements a step
-      u32 pend = km_mask;
-      while (pend) {
-        const int src = __ffs(pend) - 1;
-        pend &= pend - 1;
-        const u32 sp = __shfl_sync(0xFFFFFFFFu, pos, src);
-        const u32 dp = __shfl_sync(0xFFFFFFFFu, npos, src);
-        const u32 sl = __shfl_sync(0xFFFFFFFFu, len, src);
-        if (sp == dp) continue;
-        for (u32 q0 = 0; q0 < sl; q0 += 32) {
-          const u32 q = q0 + lane;
-          int32_t v = 0;
-          bool okr = false;
-          if (q < sl) {
-            const u64 a = vec_addr(d.tab, e, 1, (u64)sp + q, &okr);
-            if (okr) v = d.ar.pool[a];
-          }
-          __syncwarp();
-          if (okr) {
-            bool okw;
-            const u64 a = vec_addr(d.tab, e, 1, (u64)dp + q, &okw);
-            if (okw) d.ar.pool[a] = v;
-          }
-          __syncwarp();
-        }
-      }
-      km += __popc(km_mask);
-      kp += __shfl_sync(0xFFFFFFFFu, incl, 31);
-    }
-    // classes that start at or past the new sizes go back to the free stacks
-    if (lane < kVecs) {
-      const int vec = lane;
-      const u64 old_el = (vec == 0) ? 2 * (u64)m : (u64)p;
-      const u64 new_el = (vec == 0) ? 2 * (u64)km : (u64)kp;
-      if (old_el > new_el) {
-        const int jf = (new_el == 0) ? 0 : chunk_of(new_el - 1) + 1;
-        const int jl = min(chunk_of(old_el - 1), kNumChunks - 1);
-        for (int j = jf; j <= jl; ++j) {
-          u32* slot = &d.tab.dir[((u64)e * kVecs + vec) * kNumChunks + j];
-          if (*slot != kNone) {
-            free_chunk(d.ar, ctl, j, *slot);
-            freed += chunk_size(j);
-          }
-          *slot = kNone;
-        }
-      }
-    }
-    __syncwarp();
-    if (lane == 0) {
-      d.tab.vec_n[2 * (u64)e] = km;
-      d.tab.vec_n[2 * (u64)e + 1] = kp;
-      d.tab.rel[e] = r1;
+  for (u32 db = gw * 32; db < nd; db += nw * 32) {
+    u32 todo = __ballot_sync(0xFFFFFFFFu, db + lane < nd && d.sc.done_part[db + lane] == 2u);
+    while (todo) {
+      const u32 di = db + (u32)(__ffs(todo) - 1);
+      todo &= todo - 1;
+      freed += compact_buffer(d, ctl, d.sc.done_e[di] & d.tab.mask);
     }
   }
   if (freed) atomicAdd((unsigned long long*)&ctl->arena_used, (unsigned long long)(-(long long)freed));
@@ -1932,6 +1987,7 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
       if (d.cfg.stream) {
         part = d.sc.done_part[di] != 0;
         d.sc.done_part[di] = 0;
+        if (part) d.tab.rel[e] = d.tab.rnew[e];  // the group goes on from the end of this release
       }
       if (!skip && r != kNone) {
         alto_record rec;
@@ -2359,12 +2415,13 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     // gather is the stage the measurement hooks time on their own
     k_gather<<<grid, kThreads, 0, s>>>(d, bt);
     p.launches += 1;
-    if (d.cfg.stream) {
-      launch_pdl(k_stream_compact, sgrid, kThreads, 0, s, d);
-      p.launches += 1;
-    }
   }
   p.enter(9);
+  if (d.cfg.stream) {
+    // the released spans are out: drop them from the buffers they came from
+    launch_pdl(k_stream_compact, sgrid, kThreads, 0, s, d);
+    p.launches += 1;
+  }
   launch_pdl(k_records, sgrid, kThreads, 0, s, d);
   launch_pdl(k_sweep, sgrid, kThreads, 0, s, d);
   p.launches += 2;
@@ -2629,6 +2686,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     // (two arena elements of metadata each)
     sc.bm_cap = (nmax + (u64)cfg.arena_elems / 2) / 32 + nmax + 32;
     ALLOC(sc.done_part, u32, done_cap);
+    ALLOC(sc.leaf_mrank, u32, nmax);
     ALLOC(sc.bm, u32, sc.bm_cap);
   }
   const u64 scan_tiles = std::max<u64>(std::max<u64>(dense_cap, done_cap), nmax) / kScanTile + 2;

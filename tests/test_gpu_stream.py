@@ -176,3 +176,64 @@ def test_released_child_again_is_edup():
     assert o[0].status == 0 and o[1].status == alto.EDUP
     assert g[0][0] == alto.OK and g[1][0] == alto.EDUP
 
+
+
+@pytest.mark.slow
+def test_stream_release_fullsize_throughput():
+    """The 16M-fragment throughput stream with streaming release, the bench's
+    capacities: the first two batches bit for bit against the oracle; over the
+    whole run, every leaf-parent group's partial records grow strictly and end
+    in one final record with n_children = last + 1, the records of every drain
+    are in strictly increasing (seq, deeper first) order, and for a seeded
+    sample of groups the released payloads, in record order, are the group's
+    leaves in child order."""
+    import bench
+    import oracle
+    s = make_stream("throughput")
+    D = s.depth
+    caps = bench.stream_caps(s, stream_release=True)
+    agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, **caps)
+    o = oracle.Oracle.for_stream(s, stream_release=True)
+    leaf_pid = (s.tags[D - 1] >> np.uint64(32)).astype(np.int64)
+    rng = np.random.default_rng(11)
+    sample = set(rng.choice(np.unique(leaf_pid), size=128, replace=False).tolist())
+    got_pay = {p: [] for p in sample}
+    pids, counts = np.unique(leaf_pid, return_counts=True)
+    n_leaves = dict(zip(pids.tolist(), counts.tolist()))
+    last_n, finals = {}, 0
+    for b in range(s.n_batches):
+        bt = s.batch(b)
+        db = alto.to_device(bt)
+        assert agg.push(db.tags, db.off, db.payload, db.score) == alto.OK
+        d = agg.drain()
+        assert d.status == alto.OK, b
+        rec, pay, _ = d.host()
+        if b < 2:
+            o.push_batch(bt)
+            od = o.drain()
+            assert np.array_equal(rec.view(np.uint8), od.records.view(np.uint8)), b
+            assert np.array_equal(pay, od.payload), b
+        keys = rec["completion_seq"].astype(np.int64) * 16 - rec["level"].astype(np.int64)
+        assert np.all(np.diff(keys) > 0), b
+        m = rec["level"] == D - 1
+        for r in rec[m]:
+            p, n_ch = int(r["parent_id"]), int(r["n_children"])
+            assert n_ch > last_n.get(p, 0), (b, p)
+            if int(r["ops"]) & 0x80:
+                last_n[p] = n_ch
+            else:
+                assert n_ch == n_leaves[p], (b, p)
+                last_n[p] = 1 << 40       # nothing may follow the final record
+                finals += 1
+            if p in sample:
+                got_pay[p].extend(pay[int(r["payload_off"]):int(r["payload_off"]) + int(r["payload_len"])].tolist())
+        del db
+    agg.close()
+    o.close()
+    assert finals == len(pids)
+    leaf_c = (s.tags[D - 1] & np.uint64(0x7FFFFFFF)).astype(np.int64)
+    for p in sample:
+        idx = np.flatnonzero(leaf_pid == p)
+        idx = idx[np.argsort(leaf_c[idx], kind="stable")]
+        want = np.concatenate([s.payload[s.off[i]:s.off[i + 1]] for i in idx]).tolist()
+        assert got_pay[p] == want, p
