@@ -489,6 +489,8 @@ def main():
         d = step()
     n_records_step = int(d.records.numel() // 48)
     n_payload_step = int(d.payload.numel())
+    # records of a step that are partial releases (ops byte at offset 41 of the 48)
+    n_partial_step = int(((d.records.view(-1, 48)[:, 41] & 0x80) != 0).sum().item()) if n_records_step else 0
 
     # ---- timed region: device-resident inputs -------------------------------
     # CUDA events on the push stream around the two heaviest kernels only (the
@@ -666,6 +668,7 @@ def main():
         "algorithmic_gbps": alg_bytes * world * args.steps / (ms / 1e3) / 1e9,
         "hbm_frac_path": alg_bytes * args.steps / (ms / 1e3) / 1e9 / hbm_gbs,
         "p50_batch_latency_us": p50, "p99_batch_latency_us": p99,
+        "records_per_step": n_records_step, "partial_records_per_step": n_partial_step,
         "roofline": rooflines[dominant],
         "rooflines": rooflines,
         "stage_ms_per_step": stage_ms,
