@@ -96,6 +96,8 @@ struct Scratch {
                          // children buffered by earlier batches were released (the buffer is compacted)
   u32* bm;               // [bm_cap] per-batch presence bitmaps of the groups that release
   u64 bm_cap;
+  u32* big_seg;          // [depth][big_cap] segments longer than kBigSeg, per level
+  u32 big_cap;
 };
 
 struct Dev {
@@ -416,6 +418,7 @@ __global__ void k_begin(Ctl* ctl, u32 n) {
   ctl->skip_dense = 0;
   ctl->dense_total = ctl->arena_total = ctl->pay_total = ctl->topk_total = ctl->n_emit = 0;
   ctl->bm_used = 0;
+  for (int l = 0; l < kMaxDepth; ++l) ctl->n_big[l] = 0;
   for (int l = 0; l < kMaxDepth; ++l) ctl->n_segs[l] = 0;
   ctl->n = (ctl->status == ALTO_OK) ? n : 0u;
 }
@@ -562,8 +565,298 @@ __device__ u32 release_run(const Dev& d, const Batch& b, Ctl* ctl, u32 e, u32 re
   return r1;
 }
 
+// Segments longer than this go to k_reduce_big (a block each) instead of a
+// warp: a hot group (a million children) would otherwise keep one warp busy
+// for the whole batch.
+constexpr u32 kBigSeg = 4096;
+constexpr int kBigThreads = 512;
+
+// What the reduce of level l reads and writes besides the table.
+template <bool LEAF>
+struct ReduceArgs {
+  int l;
+  const u32* skeys;
+  const u32* sperm;
+  const u32* seg_start;
+  const u32* it_rep;
+  const u32* it_cseq;
+  const u32* it_skey;
+  u32* nx_rep;
+  u32* nx_cseq;
+  u32* nx_skey;
+  u32 n_items;
+};
+
+template <bool LEAF>
+__device__ __forceinline__ ReduceArgs<LEAF> reduce_args(const Dev& d, const Batch& b, int l, const u32* skeys,
+                                                         const u32* sperm, const u32* seg_start, int in_set) {
+  ReduceArgs<LEAF> r;
+  r.l = l;
+  r.skeys = skeys;
+  r.sperm = sperm;
+  r.seg_start = seg_start;
+  r.it_rep = d.sc.it_rep[in_set];
+  r.it_cseq = d.sc.it_cseq[in_set];
+  r.it_skey = d.sc.it_skey[in_set];
+  r.nx_rep = d.sc.it_rep[in_set ^ 1];
+  r.nx_cseq = d.sc.it_cseq[in_set ^ 1];
+  r.nx_skey = d.sc.it_skey[in_set ^ 1];
+  r.n_items = LEAF ? b.n : min(d.ctl->n_segs[l + 1], d.cfg.n_max);
+  return r;
+}
+
+// One item of a segment: a leaf (LEAF) or a child group from the level below.
+struct Item {
+  u32 rep, done, cs, sk, len, c, last;
+};
+
+template <bool LEAF>
+__device__ __forceinline__ Item load_item(const Dev& d, const Batch& b, const ReduceArgs<LEAF>& r, u32 j) {
+  Item it;
+  const u32 x = min(r.sperm[j], r.n_items - 1);
+  if (LEAF) {
+    it.rep = x;
+    it.done = 1;
+    it.cs = x;
+    it.sk = d.cfg.has_score ? score_key(b.score[x]) : 0u;
+    it.len = b.off[x + 1] - b.off[x];
+  } else {
+    it.rep = r.it_rep[x];
+    const u32 cf = r.it_cseq[x];
+    it.done = cf >> 31;
+    it.cs = cf & 0x7FFFFFFFu;
+    it.sk = r.it_skey[x];
+    it.len = 0;
+  }
+  const u64 t = b.tags[(u64)r.l * b.n + it.rep];
+  it.c = tag_child(t);
+  it.last = tag_last(t);
+  return it;
+}
+
+// Per-segment reductions over its items.
+struct SegRed {
+  u32 cnt, m1, fmin, fmax, hasf, cmax, smx, bad, hitrel, below;
+  u64 lsum;
+  __device__ void init() {
+    cnt = m1 = fmax = hasf = cmax = smx = bad = hitrel = below = 0;
+    fmin = kNone;
+    lsum = 0;
+  }
+  __device__ void add(const Item& it, u32 rel, bool strm) {
+    m1 = max(m1, it.c + 1);
+    if (strm) {
+      hitrel |= (it.c == rel) ? 1u : 0u;
+      below |= (it.c < rel) ? 1u : 0u;
+    }
+    if (it.last) {
+      hasf = 1;
+      fmin = min(fmin, it.c);
+      fmax = max(fmax, it.c);
+    }
+    if (it.done) {
+      ++cnt;
+      cmax = max(cmax, it.cs);
+      smx = max(smx, it.sk);
+    }
+    lsum += it.len;
+  }
+  __device__ void warp_reduce() {
+    cnt = __reduce_add_sync(0xFFFFFFFFu, cnt);
+    m1 = __reduce_max_sync(0xFFFFFFFFu, m1);
+    fmin = __reduce_min_sync(0xFFFFFFFFu, fmin);
+    fmax = __reduce_max_sync(0xFFFFFFFFu, fmax);
+    hasf = __reduce_or_sync(0xFFFFFFFFu, hasf);
+    cmax = __reduce_max_sync(0xFFFFFFFFu, cmax);
+    smx = __reduce_max_sync(0xFFFFFFFFu, smx);
+    bad = __reduce_or_sync(0xFFFFFFFFu, bad);
+    hitrel = __reduce_or_sync(0xFFFFFFFFu, hitrel);
+    below = __reduce_or_sync(0xFFFFFFFFu, below);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) lsum += __shfl_xor_sync(0xFFFFFFFFu, lsum, o);
+  }
+  __device__ void merge(const SegRed& o) {
+    cnt += o.cnt;
+    m1 = max(m1, o.m1);
+    fmin = min(fmin, o.fmin);
+    fmax = max(fmax, o.fmax);
+    hasf |= o.hasf;
+    cmax = max(cmax, o.cmax);
+    smx = max(smx, o.smx);
+    bad |= o.bad;
+    hitrel |= o.hitrel;
+    below |= o.below;
+    lsum += o.lsum;
+  }
+};
+
+// The group's ancestry tags above level l, from its first item; an item
+// whose tags differ breaks the ancestry.
+struct Chain {
+  u64 t[kMaxDepth];
+};
+__device__ __forceinline__ Chain load_chain(const Batch& b, int l, u32 rep0) {
+  Chain h;
+#pragma unroll
+  for (int q = 0; q < kMaxDepth; ++q) h.t[q] = (q < l) ? b.tags[(u64)q * b.n + rep0] : 0ull;
+  return h;
+}
+__device__ __forceinline__ bool chain_bad(const Batch& b, int l, u32 rep, const Chain& h) {
+  bool bad = false;
+#pragma unroll
+  for (int q = 0; q < kMaxDepth; ++q)
+    if (q < l && b.tags[(u64)q * b.n + rep] != h.t[q]) bad = true;
+  return bad;
+}
+
+// Insert each lane's candidate (0 = none) into the warp's running top-K list
+// (lane q holds the q-th best, larger first).  All 32 lanes call it together.
+__device__ __forceinline__ void topk_insert(u64& best, u64 cand, int K) {
+  const int lane = threadIdx.x & 31;
+  const u64 thr = __shfl_sync(0xFFFFFFFFu, best, K - 1);
+  u32 pass = __ballot_sync(0xFFFFFFFFu, cand > thr);
+  while (pass) {
+    const int src = __ffs(pass) - 1;
+    pass &= pass - 1;
+    const u64 v = __shfl_sync(0xFFFFFFFFu, cand, src);
+    const u64 thr2 = __shfl_sync(0xFFFFFFFFu, best, K - 1);
+    if (v > thr2) {
+      const u32 pos = __popc(__ballot_sync(0xFFFFFFFFu, lane < K && best > v));
+      const u64 prev = __shfl_up_sync(0xFFFFFFFFu, best, 1);
+      if (lane >= (int)pos && lane < K) best = (lane == (int)pos) ? v : prev;
+    }
+  }
+}
+
+// Streaming release of a segment whose group stays open: the run's end r1,
+// and the kept leaves' meta indices and payload offsets (leaves below r1 are
+// placed densely straight from the batch; the others are buffered, packed).
+// All 32 lanes of one warp call it together.
+struct Release {
+  u32 r1, pcs, kept_n, kept_len;
+};
+
+template <bool LEAF>
+__device__ Release stream_release(const Dev& d, const Batch& b, Ctl* ctl, const ReduceArgs<LEAF>& r, u32 e,
+                                  u32 rel, u32 j0, u32 j1, const SegRed& red) {
+  const int lane = threadIdx.x & 31;
+  Release out{rel, 0, 0, 0};
+  // the same completion test as the finalize: a group that completes emits its final record instead
+  const u32 lo = d.tab.last[e];
+  const u32 nl = (lo == kNone && red.hasf) ? red.fmin : lo;
+  const bool closes = nl != kNone && d.tab.completed[e] + red.cnt == nl + 1 && max(d.tab.maxc1[e], red.m1) <= nl + 1;
+  if (closes) return out;
+  out.r1 = release_run(d, b, ctl, e, rel, j0, j1, r.sperm, r.n_items, &out.pcs);
+  if (out.r1 <= rel) return out;
+  for (u32 jb = j0; jb < j1; jb += 32) {
+    const u32 j = jb + lane;
+    const bool valid = j < j1;
+    u32 c = 0, len = 0;
+    if (valid) {
+      const u32 x = min(r.sperm[j], r.n_items - 1);
+      c = tag_child(b.tags[(u64)r.l * b.n + x]);
+      len = b.off[x + 1] - b.off[x];
+    }
+    const bool keep = valid && c >= out.r1;
+    const u32 kl = keep ? len : 0u;
+    u32 incl = kl;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    const u32 km = __ballot_sync(0xFFFFFFFFu, keep);
+    if (valid) {
+      d.sc.leaf_pos[j] = out.kept_len + incl - kl;
+      d.sc.leaf_mrank[j] = keep ? out.kept_n + __popc(km & lanemask_lt()) : kNone;
+    }
+    out.kept_n += __popc(km);
+    out.kept_len += __shfl_sync(0xFFFFFFFFu, incl, 31);
+  }
+  return out;
+}
+
+// Merge a reduced segment s of level l into its table entry e: checks,
+// completion test, done entry (or a partial release), carry mode, hand-up of
+// the concatenation, and the segment's item for level l-1.  One thread.
+template <bool LEAF>
+__device__ void finalize_segment(const Dev& d, const Batch& b, Ctl* ctl, const ReduceArgs<LEAF>& r, u32 s,
+                                 u32 e, u32 rep0, u32 nitems, const SegRed& red, u32 rel, const Release& rl) {
+  const int l = r.l;
+  const int D = d.cfg.depth;
+  const u64 n = b.n;
+  const bool carry = LEAF && d.cfg.concat_level >= 0;
+  const bool strm = LEAF && d.cfg.stream;
+  if (!LEAF && chain_parent(d.cfg, l)) chain_sync(d.tab, d.ar, ctl, e);
+  if (red.bad) raise_err(ctl, ALTO_EINCONSIST);
+  if (l > 0 && d.tab.up[e] != b.tags[(u64)(l - 1) * n + rep0]) raise_err(ctl, ALTO_EINCONSIST);
+  const u32 last_old = d.tab.last[e];
+  u32 nl = last_old;
+  if (red.hasf) {
+    if (red.fmin != red.fmax) raise_err(ctl, ALTO_ELAST);
+    if (last_old != kNone && last_old != red.fmin) raise_err(ctl, ALTO_ELAST);
+    if (last_old == kNone) nl = red.fmin;
+  }
+  const u32 m1n = max(d.tab.maxc1[e], red.m1);
+  if (nl != kNone && m1n > nl + 1) raise_err(ctl, ALTO_ELAST);
+  const u32 comp = d.tab.completed[e] + red.cnt;
+  const u32 smn = max(d.tab.smax[e], red.smx);
+  const bool complete = (nl != kNone) && (comp == nl + 1) && (m1n <= nl + 1);
+  d.tab.last[e] = nl;
+  d.tab.maxc1[e] = m1n;
+  d.tab.completed[e] = comp;
+  d.tab.smax[e] = smn;
+  const bool part = !complete && rl.r1 > rel;
+  // a completing group, or (streaming) a partial release, takes a done entry
+  if (complete || part) {
+    const u32 cs = part ? rl.pcs : red.cmax;
+    u32 di = atomicAdd(&ctl->n_done, 1u);
+    if (di < d.sc.done_cap) {
+      d.sc.done_e[di] = e;
+      d.sc.done_lvl[di] = (u32)l;
+      d.sc.done_cseq[di] = cs;
+      d.tab.done_epoch[e] = ctl->epoch;
+      d.tab.done_idx[e] = di;
+      if (strm) {
+        d.sc.done_part[di] = !part ? 0u : (d.tab.vec_n[2 * (u64)e] ? 2u : 1u);
+        d.tab.rnew[e] = part ? rl.r1 : nl + 1;
+      }
+      if (cs < n) atomicOr(&d.sc.mask[cs], 1u << (D - 1 - l));
+    } else {
+      raise_err(ctl, ALTO_ENOSPC);
+    }
+  }
+  if (carry) {
+    // 1: to the arena, 2: placed densely, 3: a partial release, both
+    d.sc.seg_carry[s] = complete ? 2u : (part ? 3u : 1u);
+    if (!complete) {
+      const u32 v0 = d.tab.vec_n[2 * (u64)e], v1 = d.tab.vec_n[2 * (u64)e + 1];
+      d.sc.seg_vb0[s] = v0;
+      d.sc.seg_vb1[s] = v1;
+      d.tab.vec_n[2 * (u64)e] = v0 + (part ? rl.kept_n : nitems);
+      d.tab.vec_n[2 * (u64)e + 1] = v1 + (part ? rl.kept_len : (u32)red.lsum);
+    }
+  }
+  if (chain_level(d.cfg, l) && complete) {
+    const u64 tp = b.tags[(u64)(l - 1) * n + rep0];
+    const u64 upp = (l > 1) ? b.tags[(u64)(l - 2) * n + rep0] : 0ull;
+    int ins = 0;
+    const u32 P = ht_find_or_insert(d.tab, ((u64)(l - 1) << 32) | tag_pid(tp), upp, ctl, &ins, b.tags, n,
+                                    rep0, l - 1);
+    if (ins) atomicAdd((unsigned long long*)&ctl->live_groups, 1ull);
+    const u64 total = (u64)d.tab.vec_n[2 * (u64)e + 1] + (LEAF ? red.lsum : 0ull);
+    chain_reserve(d.tab, e, P, tag_child(tp), total);
+  }
+  if (l > 0) {
+    r.nx_rep[s] = rep0;
+    r.nx_cseq[s] = (complete ? 0x80000000u : 0u) | red.cmax;
+    r.nx_skey[s] = smn;
+  }
+}
+
 // One warp per group present at level l: reduce its items, merge with the
 // table entry, test completion, and emit the group as an item of level l-1.
+// Segments longer than kBigSeg are listed for k_reduce_big.
 template <bool LEAF>
 __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, const u32* skeys,
                                                      const u32* sperm, const u32* seg_start,
@@ -571,81 +864,41 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
   pdl_enter();
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
-  const int D = d.cfg.depth;
   const u32 nseg = min(ctl->n_segs[l], d.cfg.n_max);
   const int lane = threadIdx.x & 31;
   const u32 gw = gtid() >> 5, nw = gstride() >> 5;
   const bool topk = d.cfg.score_op[l] == ALTO_SCORE_TOPK;
   const int K = d.cfg.topk_k[l];
-  const bool carry = LEAF && d.cfg.concat_level >= 0;
-  const bool receives = !LEAF && chain_parent(d.cfg, l);
-  const bool hands_up = chain_level(d.cfg, l);
   const bool strm = LEAF && d.cfg.stream;
-  const u32 ep = ctl->epoch;
-  const u32* it_rep = d.sc.it_rep[in_set];
-  const u32* it_cseq = d.sc.it_cseq[in_set];
-  const u32* it_skey = d.sc.it_skey[in_set];
-  u32* nx_rep = d.sc.it_rep[in_set ^ 1];
-  u32* nx_cseq = d.sc.it_cseq[in_set ^ 1];
-  u32* nx_skey = d.sc.it_skey[in_set ^ 1];
-  const u64 n = b.n;
-  const u32 n_items = LEAF ? b.n : min(ctl->n_segs[l + 1], d.cfg.n_max);
+  const ReduceArgs<LEAF> r = reduce_args<LEAF>(d, b, l, skeys, sperm, seg_start, in_set);
   for (u32 s = gw; s < nseg; s += nw) {
-    const u32 j1 = min(seg_start[s + 1], n_items);
+    const u32 j1 = min(seg_start[s + 1], r.n_items);
     const u32 j0 = min(seg_start[s], j1);
     if (j0 == j1) continue;
+    if (j1 - j0 > kBigSeg) {
+      if (lane == 0) {
+        const u32 q = atomicAdd(&ctl->n_big[l], 1u);
+        if (q < d.sc.big_cap) d.sc.big_seg[(u64)l * d.sc.big_cap + q] = s;
+        else raise_err(ctl, ALTO_ENOSPC);
+      }
+      continue;
+    }
     const u32 e = skeys[j0] & d.tab.mask;
-    const u32 x0 = min(sperm[j0], n_items - 1);
-    const u32 rep0 = LEAF ? x0 : it_rep[x0];
-    u64 htag[kMaxDepth];
-#pragma unroll
-    for (int q = 0; q < kMaxDepth; ++q) htag[q] = (q < l) ? b.tags[(u64)q * n + rep0] : 0ull;
-    u32 cnt = 0, m1 = 0, fmin = kNone, fmax = 0, hasf = 0, cmax = 0, smx = 0, bad = 0;
-    u64 lsum = 0;
+    const u32 rep0 = LEAF ? min(sperm[j0], r.n_items - 1) : r.it_rep[min(sperm[j0], r.n_items - 1)];
     const u32 rel = strm ? d.tab.rel[e] : 0u;
-    u32 hitrel = 0, below = 0;  // streaming: child `rel` came / a released child came again
+    const Chain htag = load_chain(b, l, rep0);
+    SegRed red;
+    red.init();
     u32 running = 0;  // payload elements of the segment's earlier leaves (leaf level)
     for (u32 jb = j0; jb < j1; jb += 32) {
       const u32 j = jb + lane;
       const bool valid = j < j1;
       u32 len = 0;
       if (valid) {
-        const u32 x = min(sperm[j], n_items - 1);
-        u32 rep, done, cs, sk;
-        if (LEAF) {
-          rep = x;
-          done = 1;
-          cs = x;
-          sk = d.cfg.has_score ? score_key(b.score[x]) : 0u;
-          len = b.off[x + 1] - b.off[x];
-        } else {
-          rep = it_rep[x];
-          u32 cf = it_cseq[x];
-          done = cf >> 31;
-          cs = cf & 0x7FFFFFFFu;
-          sk = it_skey[x];
-        }
-        const u64 t = b.tags[(u64)l * n + rep];
-        const u32 c = tag_child(t);
-        m1 = max(m1, c + 1);
-        if (strm) {
-          hitrel |= (c == rel) ? 1u : 0u;
-          below |= (c < rel) ? 1u : 0u;
-        }
-        if (tag_last(t)) {
-          hasf = 1;
-          fmin = min(fmin, c);
-          fmax = max(fmax, c);
-        }
-        if (done) {
-          ++cnt;
-          cmax = max(cmax, cs);
-          smx = max(smx, sk);
-        }
-        lsum += len;
-#pragma unroll
-        for (int q = 0; q < kMaxDepth; ++q)
-          if (q < l && b.tags[(u64)q * n + rep] != htag[q]) bad = 1;
+        const Item it = load_item<LEAF>(d, b, r, j);
+        red.add(it, rel, strm);
+        if (chain_bad(b, l, it.rep, htag)) red.bad = 1;
+        len = it.len;
       }
       if (LEAF) {
         u32 incl = len;
@@ -658,62 +911,13 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
         running += __shfl_sync(0xFFFFFFFFu, incl, 31);
       }
     }
-    cnt = __reduce_add_sync(0xFFFFFFFFu, cnt);
-    m1 = __reduce_max_sync(0xFFFFFFFFu, m1);
-    fmin = __reduce_min_sync(0xFFFFFFFFu, fmin);
-    fmax = __reduce_max_sync(0xFFFFFFFFu, fmax);
-    hasf = __reduce_or_sync(0xFFFFFFFFu, hasf);
-    cmax = __reduce_max_sync(0xFFFFFFFFu, cmax);
-    smx = __reduce_max_sync(0xFFFFFFFFu, smx);
-    bad = __reduce_or_sync(0xFFFFFFFFu, bad);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) lsum += shfl_xor_u64(lsum, o);
-    u32 r1 = rel, pcs = 0, kept_n = 0, kept_len = 0;
+    red.warp_reduce();
+    Release rl{rel, 0, 0, 0};
     if (strm) {
-      hitrel = __reduce_or_sync(0xFFFFFFFFu, hitrel);
-      below = __reduce_or_sync(0xFFFFFFFFu, below);
-      if (below && lane == 0) raise_err(ctl, ALTO_EDUP);
-      if (hitrel) {
-        // the same completion test as below: a group that completes emits its final record instead
-        const u32 lo = d.tab.last[e];
-        const u32 nl = (lo == kNone && hasf) ? fmin : lo;
-        const bool closes = nl != kNone && d.tab.completed[e] + cnt == nl + 1 &&
-                            max(d.tab.maxc1[e], m1) <= nl + 1;
-        if (!closes) r1 = release_run(d, b, ctl, e, rel, j0, j1, sperm, n_items, &pcs);
-        if (r1 > rel) {
-          // the segment's leaves below r1 are placed densely straight from the
-          // batch; the others are buffered, packed: their meta index and
-          // payload offset among the kept leaves
-          for (u32 jb = j0; jb < j1; jb += 32) {
-            const u32 j = jb + lane;
-            const bool valid = j < j1;
-            u32 c = 0, len = 0;
-            if (valid) {
-              const u32 x = min(sperm[j], n_items - 1);
-              c = tag_child(b.tags[(u64)l * n + x]);
-              len = b.off[x + 1] - b.off[x];
-            }
-            const bool keep = valid && c >= r1;
-            const u32 kl = keep ? len : 0u;
-            u32 incl = kl;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-              const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-              if (lane >= o) incl += y;
-            }
-            const u32 km = __ballot_sync(0xFFFFFFFFu, keep);
-            if (valid) {
-              d.sc.leaf_pos[j] = kept_len + incl - kl;
-              d.sc.leaf_mrank[j] = keep ? kept_n + __popc(km & lanemask_lt()) : kNone;
-            }
-            kept_n += __popc(km);
-            kept_len += __shfl_sync(0xFFFFFFFFu, incl, 31);
-          }
-        }
-      }
+      if (red.below && lane == 0) raise_err(ctl, ALTO_EDUP);
+      if (red.hitrel) rl = stream_release<LEAF>(d, b, ctl, r, e, rel, j0, j1, red);
       __syncwarp();
     }
-
     if (topk) {
       // running top-k of complete children: lane q holds the q-th best
       const u32 valid = min(d.tab.completed[e], (u32)K);
@@ -722,105 +926,107 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
         const u32 j = jb + lane;
         u64 cand = 0;
         if (j < j1) {
-          const u32 x = min(sperm[j], n_items - 1);
-          u32 rep, done, sk;
-          if (LEAF) {
-            rep = x;
-            done = 1;
-            sk = d.cfg.has_score ? score_key(b.score[x]) : 0u;
-          } else {
-            rep = it_rep[x];
-            done = it_cseq[x] >> 31;
-            sk = it_skey[x];
-          }
-          const u32 c = tag_child(b.tags[(u64)l * n + rep]);
-          if (done) cand = ((u64)sk << 32) | (u64)(~c);
+          const Item it = load_item<LEAF>(d, b, r, j);
+          if (it.done) cand = ((u64)it.sk << 32) | (u64)(~it.c);
         }
-        const u64 thr = __shfl_sync(0xFFFFFFFFu, best, K - 1);
-        u32 pass = __ballot_sync(0xFFFFFFFFu, cand > thr);
-        while (pass) {
-          const int src = __ffs(pass) - 1;
-          pass &= pass - 1;
-          const u64 v = __shfl_sync(0xFFFFFFFFu, cand, src);
-          const u64 thr2 = __shfl_sync(0xFFFFFFFFu, best, K - 1);
-          if (v > thr2) {
-            const u32 pos = __popc(__ballot_sync(0xFFFFFFFFu, lane < K && best > v));
-            const u64 prev = __shfl_up_sync(0xFFFFFFFFu, best, 1);
-            if (lane >= (int)pos && lane < K) best = (lane == (int)pos) ? v : prev;
-          }
-        }
+        topk_insert(best, cand, K);
       }
       if (lane < K) d.tab.topk[(u64)e * d.tab.kk + lane] = best;
     }
+    if (lane == 0) finalize_segment<LEAF>(d, b, ctl, r, s, e, rep0, j1 - j0, red, rel, rl);
+  }
+}
 
-    if (lane == 0) {
-      if (receives) chain_sync(d.tab, d.ar, ctl, e);
-      if (bad) raise_err(ctl, ALTO_EINCONSIST);
-      if (l > 0 && d.tab.up[e] != b.tags[(u64)(l - 1) * n + rep0]) raise_err(ctl, ALTO_EINCONSIST);
-      const u32 last_old = d.tab.last[e];
-      u32 nl = last_old;
-      if (hasf) {
-        if (fmin != fmax) raise_err(ctl, ALTO_ELAST);
-        if (last_old != kNone && last_old != fmin) raise_err(ctl, ALTO_ELAST);
-        if (last_old == kNone) nl = fmin;
+// The segments longer than kBigSeg, a block of kBigThreads each: the same
+// reductions with the block's warps over strided items, combined in shared
+// memory; each warp keeps a top-k of its items and warp 0 merges them with
+// the entry's list; a streaming release runs on warp 0.
+template <bool LEAF>
+__global__ void __launch_bounds__(kBigThreads) k_reduce_big(Dev d, Batch b, int l, const u32* skeys,
+                                                            const u32* sperm, const u32* seg_start,
+                                                            int in_set) {
+  pdl_enter();
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  constexpr int kW = kBigThreads / 32;
+  __shared__ SegRed s_red[kW];
+  __shared__ u64 s_topk[kW][kMaxTopk];
+  __shared__ u32 s_scan[kW];
+  const u32 nbig = min(ctl->n_big[l], d.sc.big_cap);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const bool topk = d.cfg.score_op[l] == ALTO_SCORE_TOPK;
+  const int K = d.cfg.topk_k[l];
+  const bool strm = LEAF && d.cfg.stream;
+  const ReduceArgs<LEAF> r = reduce_args<LEAF>(d, b, l, skeys, sperm, seg_start, in_set);
+  for (u32 q = blockIdx.x; q < nbig; q += gridDim.x) {
+    const u32 s = d.sc.big_seg[(u64)l * d.sc.big_cap + q];
+    const u32 j1 = min(seg_start[s + 1], r.n_items);
+    const u32 j0 = min(seg_start[s], j1);
+    const u32 e = skeys[j0] & d.tab.mask;
+    const u32 rep0 = LEAF ? min(sperm[j0], r.n_items - 1) : r.it_rep[min(sperm[j0], r.n_items - 1)];
+    const u32 rel = strm ? d.tab.rel[e] : 0u;
+    const Chain htag = load_chain(b, l, rep0);
+    SegRed red;
+    red.init();
+    u64 best = 0;
+    u32 running = 0;
+    // items in block-wide steps: reductions, the leaves' payload offsets
+    // (a block scan per step), and each warp's top-k
+    for (u32 jb = j0; jb < j1; jb += kBigThreads) {
+      const u32 j = jb + threadIdx.x;
+      const bool valid = j < j1;
+      u32 len = 0;
+      u64 cand = 0;
+      if (valid) {
+        const Item it = load_item<LEAF>(d, b, r, j);
+        red.add(it, rel, strm);
+        if (chain_bad(b, l, it.rep, htag)) red.bad = 1;
+        len = it.len;
+        if (it.done) cand = ((u64)it.sk << 32) | (u64)(~it.c);
       }
-      const u32 m1n = max(d.tab.maxc1[e], m1);
-      if (nl != kNone && m1n > nl + 1) raise_err(ctl, ALTO_ELAST);
-      const u32 comp = d.tab.completed[e] + cnt;
-      const u32 smn = max(d.tab.smax[e], smx);
-      const bool complete = (nl != kNone) && (comp == nl + 1) && (m1n <= nl + 1);
-      d.tab.last[e] = nl;
-      d.tab.maxc1[e] = m1n;
-      d.tab.completed[e] = comp;
-      d.tab.smax[e] = smn;
-      // a completing group, or (streaming) a partial release, takes a done entry
-      if (complete || r1 > rel) {
-        const bool part = !complete;
-        const u32 cs = part ? pcs : cmax;
-        u32 di = atomicAdd(&ctl->n_done, 1u);
-        if (di < d.sc.done_cap) {
-          d.sc.done_e[di] = e;
-          d.sc.done_lvl[di] = (u32)l;
-          d.sc.done_cseq[di] = cs;
-          d.tab.done_epoch[e] = ep;
-          d.tab.done_idx[e] = di;
-          if (strm) {
-            d.sc.done_part[di] = !part ? 0u : (d.tab.vec_n[2 * (u64)e] ? 2u : 1u);
-            d.tab.rnew[e] = part ? r1 : nl + 1;
-          }
-          if (cs < n) atomicOr(&d.sc.mask[cs], 1u << (D - 1 - l));
-        } else {
-          raise_err(ctl, ALTO_ENOSPC);
+      if (topk) topk_insert(best, cand, K);
+      if (LEAF) {
+        u32 incl = len;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+          if (lane >= o) incl += y;
         }
-      }
-      if (carry) {
-        // 1: to the arena, 2: placed densely, 3: a partial release, both
-        const bool part = !complete && r1 > rel;
-        d.sc.seg_carry[s] = complete ? 2u : (part ? 3u : 1u);
-        if (!complete) {
-          const u32 v0 = d.tab.vec_n[2 * (u64)e], v1 = d.tab.vec_n[2 * (u64)e + 1];
-          d.sc.seg_vb0[s] = v0;
-          d.sc.seg_vb1[s] = v1;
-          d.tab.vec_n[2 * (u64)e] = v0 + (part ? kept_n : (j1 - j0));
-          d.tab.vec_n[2 * (u64)e + 1] = v1 + (part ? kept_len : (u32)lsum);
+        if (lane == 31) s_scan[warp] = incl;
+        __syncthreads();
+        u32 wbase = 0, total = 0;
+        for (int w = 0; w < kW; ++w) {
+          const u32 v = s_scan[w];
+          if (w < warp) wbase += v;
+          total += v;
         }
-      }
-      if (hands_up && complete) {
-        const u64 tp = b.tags[(u64)(l - 1) * n + rep0];
-        const u64 upp = (l > 1) ? b.tags[(u64)(l - 2) * n + rep0] : 0ull;
-        int ins = 0;
-        const u32 P = ht_find_or_insert(d.tab, ((u64)(l - 1) << 32) | tag_pid(tp), upp, ctl, &ins,
-                                        b.tags, n, rep0, l - 1);
-        if (ins) atomicAdd((unsigned long long*)&ctl->live_groups, 1ull);
-        const u64 total = (u64)d.tab.vec_n[2 * (u64)e + 1] + (LEAF ? lsum : 0ull);
-        chain_reserve(d.tab, e, P, tag_child(tp), total);
-      }
-      if (l > 0) {
-        nx_rep[s] = rep0;
-        nx_cseq[s] = (complete ? 0x80000000u : 0u) | cmax;
-        nx_skey[s] = smn;
+        if (valid) d.sc.leaf_pos[j] = running + wbase + incl - len;
+        running += total;
+        __syncthreads();
       }
     }
+    red.warp_reduce();
+    if (lane == 0) s_red[warp] = red;
+    if (topk && lane < K) s_topk[warp][lane] = best;
+    __syncthreads();
+    if (warp == 0) {
+      SegRed all = s_red[0];
+      for (int w = 1; w < kW; ++w) all.merge(s_red[w]);
+      Release rl{rel, 0, 0, 0};
+      if (strm) {
+        if (all.below && lane == 0) raise_err(ctl, ALTO_EDUP);
+        if (all.hitrel) rl = stream_release<LEAF>(d, b, ctl, r, e, rel, j0, j1, all);
+        __syncwarp();
+      }
+      if (topk) {
+        const u32 valid = min(d.tab.completed[e], (u32)K);
+        u64 bt = (lane < (int)valid) ? d.tab.topk[(u64)e * d.tab.kk + lane] : 0ull;
+        for (int w = 0; w < kW; ++w) topk_insert(bt, (lane < K) ? s_topk[w][lane] : 0ull, K);
+        if (lane < K) d.tab.topk[(u64)e * d.tab.kk + lane] = bt;
+      }
+      if (lane == 0) finalize_segment<LEAF>(d, b, ctl, r, s, e, rep0, j1 - j0, all, rel, rl);
+    }
+    __syncthreads();
   }
 }
 
@@ -2295,9 +2501,10 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
               &d.ctl->n_segs[D - 1]};
     launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site + 4, spin, s);
     launch_pdl(k_reduce<true>, p.num_sms * blocks_per_sm((const void*)k_reduce<true>), kThreads, 0, s, d, bt,
-               D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
-                                             d.sc.leaf_seg_start, set);
-    p.launches += 2;
+               D - 1, d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
+    launch_pdl(k_reduce_big<true>, p.num_sms, kBigThreads, 0, s, d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
+               d.sc.leaf_seg_start, set);
+    p.launches += 3;
   } else {
     // leaf level without TOPK: accumulate into the table in arrival order
     // (plain stream order: the measurement hooks time this kernel on its own)
@@ -2336,9 +2543,10 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
               &d.ctl->n_segs[l]};
     launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site++, spin, s);
     launch_pdl(k_reduce<false>, p.num_sms * blocks_per_sm((const void*)k_reduce<false>), kThreads, 0, s, d,
-               bt, l, d.sc.up_keys, d.sc.up_perm,
-                                              d.sc.up_seg_start, set);
-    p.launches += 2;
+               bt, l, d.sc.up_keys, d.sc.up_perm, d.sc.up_seg_start, set);
+    launch_pdl(k_reduce_big<false>, p.num_sms, kBigThreads, 0, s, d, bt, l, d.sc.up_keys, d.sc.up_perm,
+               d.sc.up_seg_start, set);
+    p.launches += 3;
   }
   // emission order
   p.enter(5);
@@ -2678,6 +2886,8 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     ALLOC(d.tab.app, u64, T);
   }
   ALLOC(sc.pairset, u64, PS);
+  sc.big_cap = (u32)(nmax / kBigSeg + 1);
+  ALLOC(sc.big_seg, u32, (u64)D * sc.big_cap);
   sc.ps_mask = PS - 1;
   sc.done_cap = (u32)done_cap;
   if (strm) {
@@ -3069,6 +3279,9 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   sc.pairset = cv.take<u64>(st.PS);
   sc.ps_mask = st.PS - 1;
   sc.done_cap = (u32)dc;
+  // a one-shot batch is never longer than a warp's segment share
+  sc.big_cap = (u32)(nmax / kBigSeg + 1);
+  sc.big_seg = cv.take<u32>((u64)D * sc.big_cap);
   st.lbs.desc = cv.take<ulonglong2>(3 * st.scan_tiles);
   st.lbs.tiles = st.scan_tiles;
 }

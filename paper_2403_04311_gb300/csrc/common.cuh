@@ -55,6 +55,7 @@ struct Ctl {
   u64 chain_total;         // dense child slots of completing groups at levels M < l
   u64 chain_arena;         // their buffered child spans
   u64 bm_used;             // streaming release: words of the presence bitmaps handed out
+  u32 n_big[kMaxDepth];    // segments of level l longer than a warp's share, for the block reduce
   u64 scan_total[kSites];  // totals written by scans
 };
 
