@@ -552,11 +552,12 @@ def main():
         except Exception:
             traffic_all = {}
     rooflines = {}
+    traffic_key = s.name + ("+stream_release" if args.stream_release else "")
     for kname, (kbytes, kms) in kernels.items():
         ach = kbytes / (kms / 1e3) / 1e9 if kms > 0 else 0.0
         rooflines[kname] = {"bound": "hbm", "kernel": kname, "achieved": ach, "peak": hbm_gbs,
                             "unit": "GB/s", "frac": ach / hbm_gbs, "peak_kind": peak_kind,
-                            "traffic": traffic_all.get(s.name, {}).get(kname), "ms_per_launch": kms,
+                            "traffic": traffic_all.get(traffic_key, {}).get(kname), "ms_per_launch": kms,
                             "algorithmic_bytes_per_launch": kbytes}
     dominant = max(kernels, key=lambda k: kernels[k][1])
 
