@@ -148,11 +148,12 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
       u64 prev = atomicCAS((unsigned long long*)&tab.key[h], (unsigned long long)kEmpty,
                            (unsigned long long)key);
       if (prev == kEmpty) {
-        tab.up[h] = up;
-        tab.last[h] = kNone;
-        tab.completed[h] = 0;
-        tab.maxc1[h] = 0;
-        tab.smax[h] = 0;
+        // the whole record: up, last = none, nothing completed, accumulators zero
+        uint4* hw = reinterpret_cast<uint4*>(tab.hot + h);
+        hw[0] = make_uint4((u32)up, (u32)(up >> 32), kNone, 0);
+        hw[1] = make_uint4(0, 0, 0, 0);
+        hw[2] = make_uint4(kNone, 0, 0, 0);
+        hw[3] = make_uint4(0, 0, 0, 0);
         if (tab.rel) tab.rel[h] = 0;
         if (tab.vec_n) {
           tab.vec_n[2 * (u64)h] = 0;
@@ -161,15 +162,6 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
         if (tags) {
           for (int q = 0; q < l; ++q) tab.chain[(u64)h * tab.chain_len + q] = tags[(u64)q * n + rep];
         }
-        tab.touch[h] = 0;
-        tab.acc_cnt[h] = 0;
-        tab.acc_m1[h] = 0;
-        tab.acc_fmin[h] = kNone;
-        tab.acc_fmax1[h] = 0;
-        tab.acc_cs1[h] = 0;
-        tab.acc_smx[h] = 0;
-        tab.acc_len[h] = 0;
-        tab.acc_leaf[h] = make_uint4(0, 0, 0, 0);
         if (tags && l == tab.leaf_level) {
           ulonglong2* cb = reinterpret_cast<ulonglong2*>(tab.cbits + 4 * (u64)h);
           cb[0] = make_ulonglong2(0, 0);
@@ -742,9 +734,9 @@ __device__ Release stream_release(const Dev& d, const Batch& b, Ctl* ctl, const 
   const int lane = threadIdx.x & 31;
   Release out{rel, 0, 0, 0};
   // the same completion test as the finalize: a group that completes emits its final record instead
-  const u32 lo = d.tab.last[e];
+  const u32 lo = d.tab.hot[e].last;
   const u32 nl = (lo == kNone && red.hasf) ? red.fmin : lo;
-  const bool closes = nl != kNone && d.tab.completed[e] + red.cnt == nl + 1 && max(d.tab.maxc1[e], red.m1) <= nl + 1;
+  const bool closes = nl != kNone && d.tab.hot[e].completed + red.cnt == nl + 1 && max(d.tab.hot[e].maxc1, red.m1) <= nl + 1;
   if (closes) return out;
   out.r1 = release_run(d, b, ctl, e, rel, j0, j1, r.sperm, r.n_items, &out.pcs);
   if (out.r1 <= rel) return out;
@@ -789,23 +781,23 @@ __device__ void finalize_segment(const Dev& d, const Batch& b, Ctl* ctl, const R
   const bool strm = LEAF && d.cfg.stream;
   if (!LEAF && chain_parent(d.cfg, l)) chain_sync(d.tab, d.ar, ctl, e);
   if (red.bad) raise_err(ctl, ALTO_EINCONSIST);
-  if (l > 0 && d.tab.up[e] != b.tags[(u64)(l - 1) * n + rep0]) raise_err(ctl, ALTO_EINCONSIST);
-  const u32 last_old = d.tab.last[e];
+  if (l > 0 && d.tab.hot[e].up != b.tags[(u64)(l - 1) * n + rep0]) raise_err(ctl, ALTO_EINCONSIST);
+  const u32 last_old = d.tab.hot[e].last;
   u32 nl = last_old;
   if (red.hasf) {
     if (red.fmin != red.fmax) raise_err(ctl, ALTO_ELAST);
     if (last_old != kNone && last_old != red.fmin) raise_err(ctl, ALTO_ELAST);
     if (last_old == kNone) nl = red.fmin;
   }
-  const u32 m1n = max(d.tab.maxc1[e], red.m1);
+  const u32 m1n = max(d.tab.hot[e].maxc1, red.m1);
   if (nl != kNone && m1n > nl + 1) raise_err(ctl, ALTO_ELAST);
-  const u32 comp = d.tab.completed[e] + red.cnt;
-  const u32 smn = max(d.tab.smax[e], red.smx);
+  const u32 comp = d.tab.hot[e].completed + red.cnt;
+  const u32 smn = max(d.tab.hot[e].smax, red.smx);
   const bool complete = (nl != kNone) && (comp == nl + 1) && (m1n <= nl + 1);
-  d.tab.last[e] = nl;
-  d.tab.maxc1[e] = m1n;
-  d.tab.completed[e] = comp;
-  d.tab.smax[e] = smn;
+  d.tab.hot[e].last = nl;
+  d.tab.hot[e].maxc1 = m1n;
+  d.tab.hot[e].completed = comp;
+  d.tab.hot[e].smax = smn;
   const bool part = !complete && rl.r1 > rel;
   // a completing group, or (streaming) a partial release, takes a done entry
   if (complete || part) {
@@ -815,7 +807,7 @@ __device__ void finalize_segment(const Dev& d, const Batch& b, Ctl* ctl, const R
       d.sc.done_e[di] = e;
       d.sc.done_lvl[di] = (u32)l;
       d.sc.done_cseq[di] = cs;
-      d.tab.done_epoch[e] = ctl->epoch;
+      d.tab.hot[e].done_epoch = ctl->epoch;
       d.tab.done_idx[e] = di;
       if (strm) {
         d.sc.done_part[di] = !part ? 0u : (d.tab.vec_n[2 * (u64)e] ? 2u : 1u);
@@ -854,9 +846,156 @@ __device__ void finalize_segment(const Dev& d, const Batch& b, Ctl* ctl, const R
   }
 }
 
-// One warp per group present at level l: reduce its items, merge with the
-// table entry, test completion, and emit the group as an item of level l-1.
-// Segments longer than kBigSeg are listed for k_reduce_big.
+// Segments of at most kSmallSeg items are reduced by eight lanes (a warp takes
+// four at a time): most groups have a few dozen children or fewer, and a
+// whole warp per group left most lanes idle.
+constexpr u32 kSmallSeg = 32;
+
+// A small segment [j0, j1) by the eight lanes of `gmask` (sub = lane index in
+// the group): up to four items a lane, all loaded before they are combined;
+// the top-k of a TOPK level merged by the group's first lane.
+template <bool LEAF>
+__device__ __forceinline__ void reduce_small(const Dev& d, const Batch& b, Ctl* ctl, const ReduceArgs<LEAF>& r,
+                                             u32 s, u32 j0, u32 j1, u32 gmask, int sub, bool topk, int K) {
+  const u32 e = r.skeys[j0] & d.tab.mask;
+  const u32 rep0 = LEAF ? min(r.sperm[j0], r.n_items - 1) : r.it_rep[min(r.sperm[j0], r.n_items - 1)];
+  const Chain htag = load_chain(b, r.l, rep0);
+  SegRed red;
+  red.init();
+  u64 cand[kSmallSeg / 8];
+  u32 len[kSmallSeg / 8];
+#pragma unroll
+  for (int q = 0; q < (int)(kSmallSeg / 8); ++q) {
+    const u32 j = j0 + 8 * q + sub;
+    cand[q] = 0;
+    len[q] = 0;
+    if (j < j1) {
+      const Item it = load_item<LEAF>(d, b, r, j);
+      red.add(it, 0, false);
+      if (chain_bad(b, r.l, it.rep, htag)) red.bad = 1;
+      len[q] = it.len;
+      if (it.done) cand[q] = ((u64)it.sk << 32) | (u64)(~it.c);
+    }
+  }
+  if (LEAF) {
+    // payload offset of each leaf inside the segment
+    u32 running = 0;
+#pragma unroll
+    for (int q = 0; q < (int)(kSmallSeg / 8); ++q) {
+      u32 incl = len[q];
+#pragma unroll
+      for (int o = 1; o < 8; o <<= 1) {
+        const u32 y = __shfl_up_sync(gmask, incl, o, 8);
+        if (sub >= o) incl += y;
+      }
+      const u32 j = j0 + 8 * q + sub;
+      if (j < j1) d.sc.leaf_pos[j] = running + incl - len[q];
+      running += __shfl_sync(gmask, incl, 7, 8);
+    }
+  }
+  red.cnt = __reduce_add_sync(gmask, red.cnt);
+  red.m1 = __reduce_max_sync(gmask, red.m1);
+  red.fmin = __reduce_min_sync(gmask, red.fmin);
+  red.fmax = __reduce_max_sync(gmask, red.fmax);
+  red.hasf = __reduce_or_sync(gmask, red.hasf);
+  red.cmax = __reduce_max_sync(gmask, red.cmax);
+  red.smx = __reduce_max_sync(gmask, red.smx);
+  red.bad = __reduce_or_sync(gmask, red.bad);
+#pragma unroll
+  for (int o = 4; o > 0; o >>= 1) red.lsum += __shfl_xor_sync(gmask, red.lsum, o, 8);
+  if (topk) {
+    // the group's first lane keeps the list, best first, in local memory
+    u64 list[kMaxTopk];
+    int have = 0;
+    if (sub == 0) {
+      have = (int)min(d.tab.hot[e].completed, (u32)K);
+      for (int i = 0; i < have; ++i) list[i] = d.tab.topk[(u64)e * d.tab.kk + i];
+    }
+#pragma unroll
+    for (int q = 0; q < (int)(kSmallSeg / 8); ++q) {
+      for (int t = 0; t < 8; ++t) {
+        const u64 v = __shfl_sync(gmask, cand[q], t, 8);
+        if (sub != 0 || v == 0) continue;
+        if (have == K && v <= list[K - 1]) continue;
+        int pos = have < K ? have : K - 1;
+        while (pos > 0 && list[pos - 1] < v) {
+          list[pos] = list[pos - 1];
+          --pos;
+        }
+        list[pos] = v;
+        if (have < K) ++have;
+      }
+    }
+    if (sub == 0)
+      for (int i = 0; i < K; ++i) d.tab.topk[(u64)e * d.tab.kk + i] = (i < have) ? list[i] : 0ull;
+  }
+  if (sub == 0) finalize_segment<LEAF>(d, b, ctl, r, s, e, rep0, j1 - j0, red, 0u, Release{0, 0, 0, 0});
+}
+
+// A segment by the whole warp (32 lanes).
+template <bool LEAF>
+__device__ __forceinline__ void reduce_warp(const Dev& d, const Batch& b, Ctl* ctl, const ReduceArgs<LEAF>& r,
+                                            u32 s, u32 j0, u32 j1, bool topk, int K, bool strm) {
+  const int lane = threadIdx.x & 31;
+  const u32 e = r.skeys[j0] & d.tab.mask;
+  const u32 rep0 = LEAF ? min(r.sperm[j0], r.n_items - 1) : r.it_rep[min(r.sperm[j0], r.n_items - 1)];
+  const u32 rel = strm ? d.tab.rel[e] : 0u;
+  const Chain htag = load_chain(b, r.l, rep0);
+  SegRed red;
+  red.init();
+  u32 running = 0;  // payload elements of the segment's earlier leaves (leaf level)
+  for (u32 jb = j0; jb < j1; jb += 32) {
+    const u32 j = jb + lane;
+    const bool valid = j < j1;
+    u32 len = 0;
+    if (valid) {
+      const Item it = load_item<LEAF>(d, b, r, j);
+      red.add(it, rel, strm);
+      if (chain_bad(b, r.l, it.rep, htag)) red.bad = 1;
+      len = it.len;
+    }
+    if (LEAF) {
+      u32 incl = len;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (valid) d.sc.leaf_pos[j] = running + incl - len;
+      running += __shfl_sync(0xFFFFFFFFu, incl, 31);
+    }
+  }
+  red.warp_reduce();
+  Release rl{rel, 0, 0, 0};
+  if (strm) {
+    if (red.below && lane == 0) raise_err(ctl, ALTO_EDUP);
+    if (red.hitrel) rl = stream_release<LEAF>(d, b, ctl, r, e, rel, j0, j1, red);
+    __syncwarp();
+  }
+  if (topk) {
+    // running top-k of complete children: lane q holds the q-th best
+    const u32 valid = min(d.tab.hot[e].completed, (u32)K);
+    u64 best = (lane < (int)valid) ? d.tab.topk[(u64)e * d.tab.kk + lane] : 0ull;
+    for (u32 jb = j0; jb < j1; jb += 32) {
+      const u32 j = jb + lane;
+      u64 cand = 0;
+      if (j < j1) {
+        const Item it = load_item<LEAF>(d, b, r, j);
+        if (it.done) cand = ((u64)it.sk << 32) | (u64)(~it.c);
+      }
+      topk_insert(best, cand, K);
+    }
+    if (lane < K) d.tab.topk[(u64)e * d.tab.kk + lane] = best;
+  }
+  if (lane == 0) finalize_segment<LEAF>(d, b, ctl, r, s, e, rep0, j1 - j0, red, rel, rl);
+}
+
+// The groups present at level l: reduce their items, merge with the table
+// entries, test completion, and emit each group as an item of level l-1.  A
+// warp takes four segments at a time: the small ones by eight lanes each,
+// the others one after another by the whole warp; segments longer than
+// kBigSeg are listed for k_reduce_big.  (A streaming release needs the whole
+// warp, so with it every segment takes the warp path.)
 template <bool LEAF>
 __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, const u32* skeys,
                                                      const u32* sperm, const u32* seg_start,
@@ -865,75 +1004,38 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const u32 nseg = min(ctl->n_segs[l], d.cfg.n_max);
-  const int lane = threadIdx.x & 31;
+  const int lane = threadIdx.x & 31, grp = lane >> 3, sub = lane & 7;
+  const u32 gmask = 0xFFu << (8 * grp);
   const u32 gw = gtid() >> 5, nw = gstride() >> 5;
   const bool topk = d.cfg.score_op[l] == ALTO_SCORE_TOPK;
   const int K = d.cfg.topk_k[l];
   const bool strm = LEAF && d.cfg.stream;
   const ReduceArgs<LEAF> r = reduce_args<LEAF>(d, b, l, skeys, sperm, seg_start, in_set);
-  for (u32 s = gw; s < nseg; s += nw) {
-    const u32 j1 = min(seg_start[s + 1], r.n_items);
-    const u32 j0 = min(seg_start[s], j1);
-    if (j0 == j1) continue;
-    if (j1 - j0 > kBigSeg) {
-      if (lane == 0) {
-        const u32 q = atomicAdd(&ctl->n_big[l], 1u);
-        if (q < d.sc.big_cap) d.sc.big_seg[(u64)l * d.sc.big_cap + q] = s;
-        else raise_err(ctl, ALTO_ENOSPC);
-      }
-      continue;
+  for (u32 sb = gw * 4; sb < nseg; sb += nw * 4) {
+    const u32 s = sb + grp;
+    u32 j0 = 0, j1 = 0;
+    if (s < nseg) {
+      j1 = min(seg_start[s + 1], r.n_items);
+      j0 = min(seg_start[s], j1);
     }
-    const u32 e = skeys[j0] & d.tab.mask;
-    const u32 rep0 = LEAF ? min(sperm[j0], r.n_items - 1) : r.it_rep[min(sperm[j0], r.n_items - 1)];
-    const u32 rel = strm ? d.tab.rel[e] : 0u;
-    const Chain htag = load_chain(b, l, rep0);
-    SegRed red;
-    red.init();
-    u32 running = 0;  // payload elements of the segment's earlier leaves (leaf level)
-    for (u32 jb = j0; jb < j1; jb += 32) {
-      const u32 j = jb + lane;
-      const bool valid = j < j1;
-      u32 len = 0;
-      if (valid) {
-        const Item it = load_item<LEAF>(d, b, r, j);
-        red.add(it, rel, strm);
-        if (chain_bad(b, l, it.rep, htag)) red.bad = 1;
-        len = it.len;
-      }
-      if (LEAF) {
-        u32 incl = len;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-          if (lane >= o) incl += y;
+    const bool small = !strm && j1 > j0 && j1 - j0 <= kSmallSeg;
+    if (small) reduce_small<LEAF>(d, b, ctl, r, s, j0, j1, gmask, sub, topk, K);
+    u32 rest = __ballot_sync(0xFFFFFFFFu, sub == 0 && j1 > j0 && !small);
+    while (rest) {
+      const int g = (__ffs(rest) - 1) >> 3;
+      rest &= rest - 1;
+      const u32 s2 = sb + g;
+      const u32 a0 = __shfl_sync(0xFFFFFFFFu, j0, 8 * g), a1 = __shfl_sync(0xFFFFFFFFu, j1, 8 * g);
+      if (a1 - a0 > kBigSeg) {
+        if (lane == 0) {
+          const u32 q = atomicAdd(&ctl->n_big[l], 1u);
+          if (q < d.sc.big_cap) d.sc.big_seg[(u64)l * d.sc.big_cap + q] = s2;
+          else raise_err(ctl, ALTO_ENOSPC);
         }
-        if (valid) d.sc.leaf_pos[j] = running + incl - len;
-        running += __shfl_sync(0xFFFFFFFFu, incl, 31);
+        continue;
       }
+      reduce_warp<LEAF>(d, b, ctl, r, s2, a0, a1, topk, K, strm);
     }
-    red.warp_reduce();
-    Release rl{rel, 0, 0, 0};
-    if (strm) {
-      if (red.below && lane == 0) raise_err(ctl, ALTO_EDUP);
-      if (red.hitrel) rl = stream_release<LEAF>(d, b, ctl, r, e, rel, j0, j1, red);
-      __syncwarp();
-    }
-    if (topk) {
-      // running top-k of complete children: lane q holds the q-th best
-      const u32 valid = min(d.tab.completed[e], (u32)K);
-      u64 best = (lane < (int)valid) ? d.tab.topk[(u64)e * d.tab.kk + lane] : 0ull;
-      for (u32 jb = j0; jb < j1; jb += 32) {
-        const u32 j = jb + lane;
-        u64 cand = 0;
-        if (j < j1) {
-          const Item it = load_item<LEAF>(d, b, r, j);
-          if (it.done) cand = ((u64)it.sk << 32) | (u64)(~it.c);
-        }
-        topk_insert(best, cand, K);
-      }
-      if (lane < K) d.tab.topk[(u64)e * d.tab.kk + lane] = best;
-    }
-    if (lane == 0) finalize_segment<LEAF>(d, b, ctl, r, s, e, rep0, j1 - j0, red, rel, rl);
   }
 }
 
@@ -1019,7 +1121,7 @@ __global__ void __launch_bounds__(kBigThreads) k_reduce_big(Dev d, Batch b, int 
         __syncwarp();
       }
       if (topk) {
-        const u32 valid = min(d.tab.completed[e], (u32)K);
+        const u32 valid = min(d.tab.hot[e].completed, (u32)K);
         u64 bt = (lane < (int)valid) ? d.tab.topk[(u64)e * d.tab.kk + lane] : 0ull;
         for (int w = 0; w < kW; ++w) topk_insert(bt, (lane < K) ? s_topk[w][lane] : 0ull, K);
         if (lane < K) d.tab.topk[(u64)e * d.tab.kk + lane] = bt;
@@ -1062,13 +1164,13 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
       cs = cf & 0x7FFFFFFFu;
       sk = it_skey[x];
       if (chain_differs(d.tab, e, b.tags, n, rep, l)) raise_err(ctl, ALTO_EINCONSIST);
-      first = atomicExch(&d.tab.touch[e], ep) != ep;
+      first = atomicExch(&d.tab.hot[e].touch, ep) != ep;
     }
     {
       const u32 pos = warp_take(first, &ctl->n_segs[l]);
       if (first) {
         if (pos < d.cfg.n_max) list[pos] = e;
-        d.tab.acc_rep[e] = rep;
+        d.tab.hot[e].acc_rep = rep;
       }
     }
     // lanes past the end form their own group; the whole warp takes part
@@ -1077,14 +1179,14 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
     if (__all_sync(0xFFFFFFFFu, peers0 == (1u << (threadIdx.x & 31)))) {
       if (valid) {
         if (done) {
-          atomicAdd(&d.tab.acc_cnt[e], 1u);
-          atomicMax(&d.tab.acc_cs1[e], cs + 1);
-          if (sk) atomicMax(&d.tab.acc_smx[e], sk);
+          atomicAdd((unsigned long long*)&d.tab.hot[e].acc_cl, 1ull << 40);
+          atomicMax(&d.tab.hot[e].acc_cs1, cs + 1);
+          if (sk) atomicMax(&d.tab.hot[e].acc_smx, sk);
         }
-        atomicMax(&d.tab.acc_m1[e], c + 1);
+        atomicMax(&d.tab.hot[e].acc_m1, c + 1);
         if (f) {
-          atomicMin(&d.tab.acc_fmin[e], c);
-          atomicMax(&d.tab.acc_fmax1[e], c + 1);
+          atomicMin(&d.tab.hot[e].acc_fmin, c);
+          atomicMax(&d.tab.hot[e].acc_fmax1, c + 1);
         }
       }
       continue;
@@ -1099,12 +1201,12 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
       const u32 cs1 = __reduce_max_sync(peers, (valid && done) ? cs + 1 : 0u);
       const u32 smx = __reduce_max_sync(peers, (valid && done) ? sk : 0u);
       if (valid && (int)(threadIdx.x & 31) == leader) {
-        if (cnt) atomicAdd(&d.tab.acc_cnt[e], cnt);
-        if (m1) atomicMax(&d.tab.acc_m1[e], m1);
-        if (fmin != kNone) atomicMin(&d.tab.acc_fmin[e], fmin);
-        if (fmax1) atomicMax(&d.tab.acc_fmax1[e], fmax1);
-        if (cs1) atomicMax(&d.tab.acc_cs1[e], cs1);
-        if (smx) atomicMax(&d.tab.acc_smx[e], smx);
+        if (cnt) atomicAdd((unsigned long long*)&d.tab.hot[e].acc_cl, (unsigned long long)cnt << 40);
+        if (m1) atomicMax(&d.tab.hot[e].acc_m1, m1);
+        if (fmin != kNone) atomicMin(&d.tab.hot[e].acc_fmin, fmin);
+        if (fmax1) atomicMax(&d.tab.hot[e].acc_fmax1, fmax1);
+        if (cs1) atomicMax(&d.tab.hot[e].acc_cs1, cs1);
+        if (smx) atomicMax(&d.tab.hot[e].acc_smx, smx);
       }
     }
   }
@@ -1149,16 +1251,16 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch b)
     if (__all_sync(0xFFFFFFFFu, peers == (1u << lane))) {
       // every lane its own group (the common case): plain atomics, no reductions
       if (valid) {
-        uint4* rec = d.tab.acc_leaf + e;
-        const u64 old = atomicAdd((unsigned long long*)&rec->x, (1ull << 40) | len);
+        Hot* rec = d.tab.hot + e;
+        const u64 old = atomicAdd((unsigned long long*)&rec->acc_cl, (1ull << 40) | len);
         first = old == 0;
-        atomicMax(&rec->z, c + 1);
-        atomicMax(&rec->w, i + 1);
+        atomicMax(&rec->acc_m1, c + 1);
+        atomicMax(&rec->acc_cs1, i + 1);
         if (f) {
-          atomicMin(&d.tab.acc_fmin[e], c);
-          atomicMax(&d.tab.acc_fmax1[e], c + 1);
+          atomicMin(&d.tab.hot[e].acc_fmin, c);
+          atomicMax(&d.tab.hot[e].acc_fmax1, c + 1);
         }
-        if (scores) atomicMax(&d.tab.acc_smx[e], sk);
+        if (scores) atomicMax(&d.tab.hot[e].acc_smx, sk);
       }
     } else {
       const int leader = __ffs(peers) - 1;
@@ -1169,29 +1271,29 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch b)
       const u32 anyf = __reduce_or_sync(peers, f);
       if (valid && lane == leader) {
         // one returning atomic per group and warp: leaves and payload together
-        uint4* rec = d.tab.acc_leaf + e;
-        const u64 old = atomicAdd((unsigned long long*)&rec->x, ((unsigned long long)cnt << 40) | lsum);
+        Hot* rec = d.tab.hot + e;
+        const u64 old = atomicAdd((unsigned long long*)&rec->acc_cl, ((unsigned long long)cnt << 40) | lsum);
         first = old == 0;
-        atomicMax(&rec->z, m1);
-        atomicMax(&rec->w, cs1);
+        atomicMax(&rec->acc_m1, m1);
+        atomicMax(&rec->acc_cs1, cs1);
       }
       if (anyf) {
         const u32 fmin = __reduce_min_sync(peers, (valid && f) ? c : kNone);
         const u32 fmax1 = __reduce_max_sync(peers, (valid && f) ? c + 1 : 0u);
         if (valid && lane == leader && fmax1) {
-          atomicMin(&d.tab.acc_fmin[e], fmin);
-          atomicMax(&d.tab.acc_fmax1[e], fmax1);
+          atomicMin(&d.tab.hot[e].acc_fmin, fmin);
+          atomicMax(&d.tab.hot[e].acc_fmax1, fmax1);
         }
       }
       if (scores) {
         const u32 smx = __reduce_max_sync(peers, valid ? sk : 0u);
-        if (valid && lane == leader && smx) atomicMax(&d.tab.acc_smx[e], smx);
+        if (valid && lane == leader && smx) atomicMax(&d.tab.hot[e].acc_smx, smx);
       }
     }
     const u32 pos = warp_take(first, &ctl->n_segs[L]);
     if (first) {
       if (pos < d.cfg.n_max) list[pos] = e;
-      d.tab.acc_rep[e] = i;
+      d.tab.hot[e].acc_rep = i;
     }
   }
 }
@@ -1226,47 +1328,35 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
     if (valid) {
       e = list[s] & d.tab.mask;
       if (receives) chain_sync(d.tab, d.ar, ctl, e);
-      u32 cnt, m1, cs1;
-      if (LEAF) {
-        const uint4 a = d.tab.acc_leaf[e];
-        const u64 cl = ((u64)a.y << 32) | a.x;
-        cnt = (u32)(cl >> 40);
-        blen = (u32)(cl & ((1ull << 40) - 1));
-        m1 = a.z;
-        cs1 = a.w;
-        d.tab.acc_leaf[e] = make_uint4(0, 0, 0, 0);
-      } else {
-        cnt = d.tab.acc_cnt[e];
-        m1 = d.tab.acc_m1[e];
-        cs1 = d.tab.acc_cs1[e];
-      }
-      const u32 fmin = d.tab.acc_fmin[e];
-      const u32 fmax1 = d.tab.acc_fmax1[e], smx = d.tab.acc_smx[e];
-      rep = d.tab.acc_rep[e];
-      // reset the accumulators for the next batch
-      d.tab.acc_cnt[e] = 0;
-      d.tab.acc_m1[e] = 0;
-      d.tab.acc_fmin[e] = kNone;
-      d.tab.acc_fmax1[e] = 0;
-      d.tab.acc_cs1[e] = 0;
-      d.tab.acc_smx[e] = 0;
-      if (l > 0 && d.tab.up[e] != b.tags[(u64)(l - 1) * n + rep]) raise_err(ctl, ALTO_EINCONSIST);
-      const u32 last_old = d.tab.last[e];
+      // the entry's record in four 16-byte loads; the accumulators are reset
+      // for the next batch with two stores
+      uint4* hw = reinterpret_cast<uint4*>(d.tab.hot + e);
+      const uint4 h0 = hw[0], a = hw[1], f = hw[2], h3 = hw[3];
+      const u64 cl = ((u64)a.y << 32) | a.x;
+      const u32 cnt = (u32)(cl >> 40), m1 = a.z, cs1 = a.w;
+      if (LEAF) blen = (u32)(cl & kPos40);
+      const u32 fmin = f.x, fmax1 = f.y, smx = f.z;
+      rep = f.w;
+      hw[1] = make_uint4(0, 0, 0, 0);
+      hw[2] = make_uint4(kNone, 0, 0, 0);
+      const u64 up_e = ((u64)h0.y << 32) | h0.x;
+      if (l > 0 && up_e != b.tags[(u64)(l - 1) * n + rep]) raise_err(ctl, ALTO_EINCONSIST);
+      const u32 last_old = h0.z;
       u32 nl = last_old;
       if (fmax1) {
         if (fmin + 1 != fmax1) raise_err(ctl, ALTO_ELAST);
         if (last_old != kNone && last_old != fmin) raise_err(ctl, ALTO_ELAST);
         if (last_old == kNone) nl = fmin;
       }
-      const u32 m1n = max(d.tab.maxc1[e], m1);
+      const u32 m1n = max(h3.x, m1);
       if (nl != kNone && m1n > nl + 1) raise_err(ctl, ALTO_ELAST);
-      const u32 comp = d.tab.completed[e] + cnt;
-      smn = max(d.tab.smax[e], smx);
+      const u32 comp = h0.w + cnt;
+      smn = max(h3.y, smx);
       complete = (nl != kNone) && (comp == nl + 1) && (m1n <= nl + 1);
-      d.tab.last[e] = nl;
-      d.tab.maxc1[e] = m1n;
-      d.tab.completed[e] = comp;
-      d.tab.smax[e] = smn;
+      d.tab.hot[e].last = nl;
+      d.tab.hot[e].maxc1 = m1n;
+      d.tab.hot[e].completed = comp;
+      d.tab.hot[e].smax = smn;
       cmax = cs1 ? cs1 - 1 : 0;
       if (carry && !complete) {
         // reserve this batch's leaves at the end of the group's arena vectors
@@ -1291,7 +1381,7 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
         d.sc.done_e[di] = e;
         d.sc.done_lvl[di] = (u32)l;
         d.sc.done_cseq[di] = cmax;
-        d.tab.done_epoch[e] = ep;
+        d.tab.hot[e].done_epoch = ep;
         d.tab.done_idx[e] = di;
         if (cmax < n) atomicOr(&d.sc.mask[cmax], 1u << (D - 1 - l));
       } else {
@@ -1350,7 +1440,7 @@ __global__ void __launch_bounds__(kThreads) k_done_rank(Dev d) {
     }
     d.sc.done_rank[di] = r;
     d.sc.r_done[r] = di;
-    const u32 nch = d.tab.last[e] + 1;
+    const u32 nch = d.tab.hot[e].last + 1;
     // streaming: children rel.. of the run that ends this batch (all of them
     // up to the last for a final record); a partial record has no top-k
     const bool part = d.cfg.stream && d.sc.done_part[di];
@@ -1420,7 +1510,7 @@ struct ChainScan {
   __device__ u64 value(u64 i) const {
     if ((int)done_lvl[i] <= M) return 0;
     const u32 e = done_e[i] & tab.mask;
-    return (which == 0) ? (u64)tab.last[e] + 1 : (u64)tab.vec_n[2 * (u64)e];
+    return (which == 0) ? (u64)tab.hot[e].last + 1 : (u64)tab.vec_n[2 * (u64)e];
   }
   __device__ void out(u64 i, u64 excl, u64 v) const {
     if (which == 2) return;
@@ -1654,11 +1744,11 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
     if (sc_mode != 2u && sc_mode != 3u) continue;
     const u32 e = d.sc.leaf_keys[j] & d.tab.mask;
     const u32 i = d.sc.leaf_perm[j];
-    if (i >= b.n || d.tab.done_epoch[e] != ep) continue;
+    if (i >= b.n || d.tab.hot[e].done_epoch != ep) continue;
     const u32 di = d.tab.done_idx[e];
     if (di >= nd) continue;
     const u32 c = tag_child(b.tags[(u64)(D - 1) * n + i]);
-    if (c > d.tab.last[e]) continue;
+    if (c > d.tab.hot[e].last) continue;
     const u32 rel = d.cfg.stream ? d.tab.rel[e] : 0u;  // children below were released earlier
     if (c < rel) continue;
     if (sc_mode == 3u && c >= d.tab.rnew[e]) continue;   // kept in the buffer
@@ -1815,7 +1905,7 @@ __global__ void __launch_bounds__(kThreads) k_dense_arena(Dev d) {
     // streaming: the buffer holds children rel.. only; a partial release
     // places those below rnew and keeps the rest
     const u32 rel = (LEVEL_M && d.cfg.stream) ? d.tab.rel[e] : 0u;
-    if (c > d.tab.last[e] || end < pos || c < rel) {
+    if (c > d.tab.hot[e].last || end < pos || c < rel) {
       raise_err(ctl, ALTO_EDUP);
       continue;
     }
@@ -2213,11 +2303,11 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
         rec.topk_off = to;
         rec.topk_n = (uint16_t)tn;
         rec.parent_id = (u32)d.tab.key[e];
-        rec.n_children = part ? d.tab.rnew[e] : d.tab.last[e] + 1;
+        rec.n_children = part ? d.tab.rnew[e] : d.tab.hot[e].last + 1;
         rec.level = (uint8_t)l;
         rec.ops = part ? (uint8_t)(ALTO_PAYLOAD_CONCAT | ALTO_OPS_PARTIAL)
                        : (uint8_t)(((l == M) ? 1 : 0) | (d.cfg.score_op[l] << 2));
-        rec.score = (!part && d.cfg.score_op[l] != ALTO_SCORE_NONE) ? key_score(d.tab.smax[e]) : 0.0f;
+        rec.score = (!part && d.cfg.score_op[l] != ALTO_SCORE_NONE) ? key_score(d.tab.hot[e].smax) : 0.0f;
         d.out_rec[ctl->rec_count + r] = rec;
         for (u32 q = 0; q < tn; ++q) {
           const u64 v = d.tab.topk[(u64)e * d.tab.kk + q];
@@ -2765,12 +2855,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(d.ctl, Ctl, 1);
   // table
   ALLOC(d.tab.key, u64, T);
-  ALLOC(d.tab.up, u64, T);
-  ALLOC(d.tab.last, u32, T);
-  ALLOC(d.tab.completed, u32, T);
-  ALLOC(d.tab.maxc1, u32, T);
-  ALLOC(d.tab.smax, u32, T);
-  ALLOC(d.tab.done_epoch, u32, T);
+  ALLOC(d.tab.hot, Hot, T);
   ALLOC(d.tab.done_idx, u32, T);
   if (concat >= 0) {
     ALLOC(d.tab.vec_n, u32, 2 * T);
@@ -2779,17 +2864,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   if (kk > 0) ALLOC(d.tab.topk, u64, T * (u64)kk);
   d.tab.chain_len = std::max((D - 1 + 1) & ~1, 2);  // even: read as 16-byte pairs
   ALLOC(d.tab.chain, u64, T * (u64)d.tab.chain_len);
-  ALLOC(d.tab.touch, u32, T);
-  ALLOC(d.tab.acc_cnt, u32, T);
-  ALLOC(d.tab.acc_m1, u32, T);
-  ALLOC(d.tab.acc_fmin, u32, T);
-  ALLOC(d.tab.acc_fmax1, u32, T);
-  ALLOC(d.tab.acc_cs1, u32, T);
-  ALLOC(d.tab.acc_smx, u32, T);
-  ALLOC(d.tab.acc_rep, u32, T);
-  ALLOC(d.tab.acc_len, u32, T);
   ALLOC(d.tab.cur, u64, T);
-  ALLOC(d.tab.acc_leaf, uint4, T);
   ALLOC(d.tab.dbase, u64, T);
   ALLOC(d.tab.bstate, uint4, T);
   ALLOC(d.tab.cbits, u64, 4 * T);
@@ -2919,7 +2994,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   // initial state
   cudaMemsetAsync(d.ctl, 0, sizeof(Ctl), s);
   cudaMemsetAsync(d.tab.key, 0xFF, sizeof(u64) * T, s);
-  cudaMemsetAsync(d.tab.done_epoch, 0, sizeof(u32) * T, s);
+  cudaMemsetAsync(d.tab.hot, 0, sizeof(Hot) * T, s);
   cudaMemsetAsync(d.tab.cur, 0, sizeof(u64) * T, s);
   cudaMemsetAsync(sc.mask, 0, sizeof(u32) * nmax, s);
   cudaMemsetAsync(sc.pairset, 0, sizeof(u64) * PS, s);
@@ -3169,12 +3244,7 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   memset(&d, 0, sizeof(d));
   d.ctl = cv.take<Ctl>(1);
   d.tab.key = cv.take<u64>(T);
-  d.tab.up = cv.take<u64>(T);
-  d.tab.last = cv.take<u32>(T);
-  d.tab.completed = cv.take<u32>(T);
-  d.tab.maxc1 = cv.take<u32>(T);
-  d.tab.smax = cv.take<u32>(T);
-  d.tab.done_epoch = cv.take<u32>(T);
+  d.tab.hot = cv.take<Hot>(T);
   d.tab.done_idx = cv.take<u32>(T);
   if (concat >= 0) {
     d.tab.vec_n = cv.take<u32>(2 * T);
@@ -3183,17 +3253,7 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   if (kk > 0) d.tab.topk = cv.take<u64>(T * (u64)kk);
   d.tab.chain_len = std::max((D - 1 + 1) & ~1, 2);  // even: read as 16-byte pairs
   d.tab.chain = cv.take<u64>(T * (u64)d.tab.chain_len);
-  d.tab.touch = cv.take<u32>(T);
-  d.tab.acc_cnt = cv.take<u32>(T);
-  d.tab.acc_m1 = cv.take<u32>(T);
-  d.tab.acc_fmin = cv.take<u32>(T);
-  d.tab.acc_fmax1 = cv.take<u32>(T);
-  d.tab.acc_cs1 = cv.take<u32>(T);
-  d.tab.acc_smx = cv.take<u32>(T);
-  d.tab.acc_rep = cv.take<u32>(T);
-  d.tab.acc_len = cv.take<u32>(T);
   d.tab.cur = cv.take<u64>(T);
-  d.tab.acc_leaf = cv.take<uint4>(T);
   d.tab.dbase = cv.take<u64>(T);
   d.tab.bstate = cv.take<uint4>(T);
   d.tab.cbits = cv.take<u64>(4 * T);
@@ -3303,15 +3363,11 @@ __global__ void k_na_reset(Dev d, u32* hist, u64 T, u64 PS, u32 nmax) {
   }
   for (u64 i = tid; i < T; i += stride) {
     d.tab.key[i] = kEmpty;
-    d.tab.touch[i] = 0;
-    d.tab.acc_cnt[i] = 0;
-    d.tab.acc_m1[i] = 0;
-    d.tab.acc_fmin[i] = kNone;
-    d.tab.acc_fmax1[i] = 0;
-    d.tab.acc_cs1[i] = 0;
-    d.tab.acc_smx[i] = 0;
-    d.tab.acc_len[i] = 0;
-    d.tab.acc_leaf[i] = make_uint4(0, 0, 0, 0);
+    uint4* hw = reinterpret_cast<uint4*>(d.tab.hot + i);
+    hw[0] = make_uint4(0, 0, kNone, 0);
+    hw[1] = make_uint4(0, 0, 0, 0);
+    hw[2] = make_uint4(kNone, 0, 0, 0);
+    hw[3] = make_uint4(0, 0, 0, 0);
     d.tab.cur[i] = 0;
   }
   for (u64 i = tid; i < PS; i += stride) d.sc.pairset[i] = 0;

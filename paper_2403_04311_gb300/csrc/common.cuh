@@ -142,32 +142,37 @@ __device__ __forceinline__ u64 chunk_size(int j) { return 1ull << (kChunk0Log + 
 // ---------------------------------------------------------------------------
 // device-resident state, handed to kernels by value
 // ---------------------------------------------------------------------------
+// The fields of an open-group entry that the level kernels read and write
+// together, in one 64-byte record (one access brings them all; a
+// structure-of-arrays table spread them over a dozen cache lines).  The
+// batch accumulators are zero between batches (acc_fmin: kNone).
+struct __align__(64) Hot {
+  u64 up;          // tag one level up
+  u32 last;        // last child index or kNone
+  u32 completed;   // complete children so far
+  u64 acc_cl;      // this batch: complete children << 40 | payload elements (leaf level)
+  u32 acc_m1;      // this batch: largest child index + 1
+  u32 acc_cs1;     // this batch: largest completion seq + 1 of complete children
+  u32 acc_fmin;    // this batch: smallest flagged child index (kNone = none)
+  u32 acc_fmax1;   // this batch: largest flagged child index + 1 (0 = none)
+  u32 acc_smx;     // this batch: largest score key of complete children
+  u32 acc_rep;     // this batch: a representative fragment
+  u32 maxc1;       // largest child index seen + 1
+  u32 smax;        // largest score key over complete children (0 = none)
+  u32 touch;       // epoch of the batch that last touched the entry (upper levels)
+  u32 done_epoch;  // epoch of the batch that completed the group
+};
+static_assert(sizeof(Hot) == 64, "one 64-byte record per entry");
+
 struct Table {
   u64* key;        // [T] (level << 32 | parent_id), kEmpty, kTomb
-  u64* up;         // [T] tag one level up
-  u32* last;       // [T] last child index or kNone
-  u32* completed;  // [T] complete children so far
-  u32* maxc1;      // [T] largest child index seen + 1
-  u32* smax;       // [T] largest score key over complete children (0 = none)
-  u32* done_epoch; // [T] epoch of the batch that completed the group
+  Hot* hot;        // [T]
   u32* done_idx;   // [T] index in the batch's done list
   u32* vec_n;      // [T][2] CONCAT level: leaves in meta vector, elements in payload vector
   u32* dir;        // [T][2][kNumChunks] CONCAT level: chunk offsets in the arena
   u64* topk;       // [T][kk] TOPK levels: best (score_key << 32 | ~child) first
   u64* chain;      // [T][D-1] tags 0..l-1 of the group's first fragment (ancestry)
-  // per-batch accumulators of the atomic upper-level path (zero between batches)
-  u32* touch;      // [T] epoch of the batch that last touched the entry
-  u32* acc_cnt;    // [T] complete children in this batch
-  u32* acc_m1;     // [T] largest child index + 1 in this batch
-  u32* acc_fmin;   // [T] smallest flagged child index (kNone = none)
-  u32* acc_fmax1;  // [T] largest flagged child index + 1 (0 = none)
-  u32* acc_cs1;    // [T] largest completion seq + 1 of complete children
-  u32* acc_smx;    // [T] largest score key of complete children
-  u32* acc_rep;    // [T] a representative fragment
-  u32* acc_len;    // [T] payload elements of this batch's leaves (leaf level)
   u64* cur;        // [T] arena cursor: leaves << 40 | payload elements
-  uint4* acc_leaf; // [T] leaf level, one sector per group: {leaves << 40 | payload
-                   //     elements (as u64 in .x/.y), max child + 1, max seq + 1}
   u64* dbase;      // [T] first dense child slot of a group completing this batch
   uint4* bstate;   // [T] where this batch's leaves go, one load per fragment:
                    //     {epoch, mode (1 arena, 2 dense), dense base lo, hi}
