@@ -71,7 +71,8 @@ struct Scratch {
   u32* leaf_pos;         // [n_max] sorted leaf j: payload offset inside its segment's buffered data
   u32* leaf_mrank;       // [n_max] streaming, segments 3: meta index among the buffered leaves, kNone if placed
   u32* mask;             // [n_max] bit (D-1-l): a level-l group completes at this seq
-  u32* prefix;           // [n_max] records completed before this seq
+  u32* mblk;             // [n_max/32 + 1] completions at the seqs of each run of 32
+  u32* prefix;           // [n_max/32 + 1] completions before each run of 32 seqs
   u32* done_e;           // [done_cap]
   u32* done_lvl;
   u32* done_cseq;
@@ -813,7 +814,10 @@ __device__ void finalize_segment(const Dev& d, const Batch& b, Ctl* ctl, const R
         d.sc.done_part[di] = !part ? 0u : (d.tab.vec_n[2 * (u64)e] ? 2u : 1u);
         d.tab.rnew[e] = part ? rl.r1 : nl + 1;
       }
-      if (cs < n) atomicOr(&d.sc.mask[cs], 1u << (D - 1 - l));
+      if (cs < n) {
+        atomicOr(&d.sc.mask[cs], 1u << (D - 1 - l));
+        atomicAdd(&d.sc.mblk[cs >> 5], 1u);
+      }
     } else {
       raise_err(ctl, ALTO_ENOSPC);
     }
@@ -1383,7 +1387,10 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
         d.sc.done_cseq[di] = cmax;
         d.tab.hot[e].done_epoch = ep;
         d.tab.done_idx[e] = di;
-        if (cmax < n) atomicOr(&d.sc.mask[cmax], 1u << (D - 1 - l));
+        if (cmax < n) {
+          atomicOr(&d.sc.mask[cmax], 1u << (D - 1 - l));
+          atomicAdd(&d.sc.mblk[cmax >> 5], 1u);
+        }
       } else {
         raise_err(ctl, ALTO_ENOSPC);
       }
@@ -1410,14 +1417,19 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
 }
 
 // Emission rank of each completed group: records completed at earlier
-// arrival indices, plus the deeper groups completed at the same index.
+// arrival indices, plus the deeper groups completed at the same index.  The
+// scan runs over runs of 32 seqs (their completion counts); a group adds the
+// completions of its run's earlier seqs from the per-seq level masks.
 struct RankScan {
-  const u32* mask;
+  const u32* mblk;
   u32* prefix;
   const u32* n_dev;
-  __device__ u64 size(const Ctl*) const { return *n_dev; }
-  __device__ u64 value(u64 i) const { return __popc(mask[i]); }
-  __device__ void out(u64 i, u64 excl, u64) const { prefix[i] = (u32)excl; }
+  __device__ u64 size(const Ctl*) const { return (*n_dev + 31) >> 5; }
+  __device__ u64 value(u64 i) const { return mblk[i]; }
+  // only runs that completed a group are ever looked up
+  __device__ void out(u64 i, u64 excl, u64 v) const {
+    if (v) prefix[i] = (u32)excl;
+  }
   __device__ void total(Ctl* ctl, u64 t) const { ctl->n_emit = t; }
 };
 
@@ -1432,7 +1444,21 @@ __global__ void __launch_bounds__(kThreads) k_done_rank(Dev d) {
     const int l = (int)d.sc.done_lvl[di];
     const u32 cs = d.sc.done_cseq[di];
     const int bit = D - 1 - l;
-    const u32 r = (cs < ctl->n) ? d.sc.prefix[cs] + __popc(d.sc.mask[cs] & ((1u << bit) - 1u)) : kNone;
+    u32 r = kNone;
+    if (cs < ctl->n) {
+      // the run's earlier seqs: its 32 masks are one 128-byte line
+      const u32 b0 = cs & ~31u;
+      const uint4* m4 = reinterpret_cast<const uint4*>(d.sc.mask + b0);
+      u32 before = 0;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const uint4 v = m4[q];
+        const u32 s0 = b0 + 4 * q;
+        before += (s0 < cs ? __popc(v.x) : 0) + (s0 + 1 < cs ? __popc(v.y) : 0) +
+                  (s0 + 2 < cs ? __popc(v.z) : 0) + (s0 + 3 < cs ? __popc(v.w) : 0);
+      }
+      r = d.sc.prefix[cs >> 5] + before + __popc(d.sc.mask[cs] & ((1u << bit) - 1u));
+    }
     if (r >= nd) {
       raise_err(ctl, ALTO_EINCONSIST);
       d.sc.done_rank[di] = kNone;
@@ -1865,7 +1891,8 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch b) {
 // Dense child slots from the arena: spans buffered by earlier batches (and,
 // above the leaf parent, handed up earlier in this batch).  LEVEL_M: the
 // groups of level M, by emission rank; otherwise the groups of levels M < l,
-// by done index.
+// by done index.  (A warp per group with buffered spans, in place of the
+// binary search, measured slower: a few groups hold most of the spans.)
 template <bool LEVEL_M>
 __global__ void __launch_bounds__(kThreads) k_dense_arena(Dev d) {
   pdl_enter();
@@ -2279,7 +2306,10 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
       l = (int)d.sc.done_lvl[di];
       const u32 cs = d.sc.done_cseq[di];
       const u32 r = d.sc.done_rank[di];
-      if (cs < d.cfg.n_max) d.sc.mask[cs] = 0;
+      if (cs < d.cfg.n_max) {
+        d.sc.mask[cs] = 0;
+        d.sc.mblk[cs >> 5] = 0;
+      }
       if (d.cfg.stream) {
         part = d.sc.done_part[di] != 0;
         d.sc.done_part[di] = 0;
@@ -2521,7 +2551,9 @@ void launch_scan(const LookbackState& lb, int num_sms, Ctl* ctl, const F& f, u64
                  u64 spin, cudaStream_t s) {
   u64 tiles = (cap + kScanTile - 1) / kScanTile;
   if (tiles == 0) tiles = 1;
-  int grid = (int)std::min<u64>(tiles, (u64)num_sms * 4);
+  // one CTA per SM: at a million elements more CTAs only add idle ones that
+  // contend on the tile counter (measured: 13.8 us at 152 CTAs, 16 us at 608)
+  int grid = (int)std::min<u64>(tiles, (u64)num_sms);
   launch_pdl(k_scan<F>, grid, kScanThreads, 0, s, f, lb, ctl, site, &ctl->exit_ctr[site], spin);
 }
 
@@ -2641,8 +2673,8 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   // emission order
   p.enter(5);
   {
-    RankScan f{d.sc.mask, d.sc.prefix, &d.ctl->n};
-    launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site++, spin, s);
+    RankScan f{d.sc.mblk, d.sc.prefix, &d.ctl->n};
+    launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax / 32 + 1, site++, spin, s);
   }
   launch_pdl(k_done_rank, sgrid, kThreads, 0, s, d);
   p.launches += 2;
@@ -2864,10 +2896,10 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   if (kk > 0) ALLOC(d.tab.topk, u64, T * (u64)kk);
   d.tab.chain_len = std::max((D - 1 + 1) & ~1, 2);  // even: read as 16-byte pairs
   ALLOC(d.tab.chain, u64, T * (u64)d.tab.chain_len);
+  ALLOC(d.tab.cbits, u64, 4 * T);
   ALLOC(d.tab.cur, u64, T);
   ALLOC(d.tab.dbase, u64, T);
   ALLOC(d.tab.bstate, uint4, T);
-  ALLOC(d.tab.cbits, u64, 4 * T);
   const bool strm = (cfg.flags & ALTO_FLAG_STREAM_RELEASE) != 0;
   if (strm) {
     ALLOC(d.tab.rel, u32, T);
@@ -2935,7 +2967,8 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(sc.seg_vb1, u32, nmax);
   ALLOC(sc.seg_carry, u32, nmax);
   ALLOC(sc.leaf_pos, u32, nmax);
-  ALLOC(sc.mask, u32, nmax);
+  ALLOC(sc.mask, u32, (nmax + 31) / 32 * 32);   // whole runs of 32
+  ALLOC(sc.mblk, u32, nmax / 32 + 1);
   ALLOC(sc.prefix, u32, nmax);
   ALLOC(sc.done_e, u32, done_cap);
   ALLOC(sc.done_lvl, u32, done_cap);
@@ -2996,7 +3029,8 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   cudaMemsetAsync(d.tab.key, 0xFF, sizeof(u64) * T, s);
   cudaMemsetAsync(d.tab.hot, 0, sizeof(Hot) * T, s);
   cudaMemsetAsync(d.tab.cur, 0, sizeof(u64) * T, s);
-  cudaMemsetAsync(sc.mask, 0, sizeof(u32) * nmax, s);
+  cudaMemsetAsync(sc.mask, 0, sizeof(u32) * ((nmax + 31) / 32 * 32), s);
+  cudaMemsetAsync(sc.mblk, 0, sizeof(u32) * (nmax / 32 + 1), s);
   cudaMemsetAsync(sc.pairset, 0, sizeof(u64) * PS, s);
   cudaMemsetAsync(h->leaf_sort.hist, 0, sizeof(u32) * 4 * 256, s);
   cudaMemsetAsync(h->leaf_sort.lookback, 0, sizeof(u64) * sort_tiles * 256, s);
@@ -3253,10 +3287,10 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   if (kk > 0) d.tab.topk = cv.take<u64>(T * (u64)kk);
   d.tab.chain_len = std::max((D - 1 + 1) & ~1, 2);  // even: read as 16-byte pairs
   d.tab.chain = cv.take<u64>(T * (u64)d.tab.chain_len);
+  d.tab.cbits = cv.take<u64>(4 * T);
   d.tab.cur = cv.take<u64>(T);
   d.tab.dbase = cv.take<u64>(T);
   d.tab.bstate = cv.take<uint4>(T);
-  d.tab.cbits = cv.take<u64>(4 * T);
   d.tab.leaf_level = D - 1;
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
@@ -3311,7 +3345,8 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   sc.seg_vb1 = cv.take<u32>(nmax);
   sc.seg_carry = cv.take<u32>(nmax);
   sc.leaf_pos = cv.take<u32>(nmax);
-  sc.mask = cv.take<u32>(nmax);
+  sc.mask = cv.take<u32>((nmax + 31) / 32 * 32);
+  sc.mblk = cv.take<u32>(nmax / 32 + 1);
   sc.prefix = cv.take<u32>(nmax);
   const u64 dc = st.done_cap;
   sc.done_e = cv.take<u32>(dc);
@@ -3371,7 +3406,8 @@ __global__ void k_na_reset(Dev d, u32* hist, u64 T, u64 PS, u32 nmax) {
     d.tab.cur[i] = 0;
   }
   for (u64 i = tid; i < PS; i += stride) d.sc.pairset[i] = 0;
-  for (u64 i = tid; i < nmax; i += stride) d.sc.mask[i] = 0;
+  for (u64 i = tid; i < (nmax + 31) / 32 * 32; i += stride) d.sc.mask[i] = 0;
+  for (u64 i = tid; i < nmax / 32 + 1; i += stride) d.sc.mblk[i] = 0;
   for (u64 i = tid; i < 4 * 256; i += stride) hist[i] = 0;
 }
 

@@ -182,14 +182,17 @@ struct Table {
   u32* par;        // [T] parent entry the completed group was appended to
   u32* cidx;       // [T] its child index in that parent
   u64* app;        // [T] its reserved place there: span index << 40 | payload position
-  u64* cbits;      // [T][4] leaf parents: leaf slots 0..255 seen while the group is open
+  // [T][4] leaf parents: leaf slots 0..255 seen while the group is open (kept
+  // apart from the chain rows: sharing their lines with these atomics made the
+  // leaf accumulate slower)
+  u64* cbits;
   // streaming release (CONCAT at the leaf parent): children 0..rel-1 were
   // released by partial records and are no longer buffered; rnew is where
   // the release of the current batch ends (a partial or the final record)
   u32* rel;        // [T]
   u32* rnew;       // [T]
   int leaf_level;  // D - 1
-  int chain_len;   // D - 1
+  int chain_len;   // D - 1, rounded up to even
   u32 mask;        // T - 1
   int kk;          // stride of topk (largest k over levels)
   int max_probe;
