@@ -599,25 +599,50 @@ def main():
     h2d = sum(h["tags"].numel() * 8 + h["off"].numel() * 4 + h["payload"].numel() * 4 +
               (h["score"].numel() * 4 if h["score"] is not None else 0) for h in host)
 
+    # Copies overlap the pushes as a user of the API would run them: every
+    # batch's inputs go up on a copy stream and its push waits for them only;
+    # the step's records and payload come back on a second copy stream, while
+    # the next step's inputs go up.  The next step's pushes reuse the output
+    # ring (reset by the drain), so they wait for that read-back.
+    cs_in = torch.cuda.Stream()
+    cs_out = torch.cuda.Stream()
+    flags = {"out": None}
+
     def e2e_step():
-        for hb, db in zip(host, dev):
-            db.tags.copy_(hb["tags"], non_blocking=True)
-            db.off.copy_(hb["off"], non_blocking=True)
-            db.payload.copy_(hb["payload"], non_blocking=True)
-            if hb["score"] is not None:
-                db.score.copy_(hb["score"], non_blocking=True)
+        cs_in.wait_stream(stream)  # the device batch buffers are free once the previous pushes ran
+        ready = []
+        with torch.cuda.stream(cs_in):
+            for hb, db in zip(host, dev):
+                db.tags.copy_(hb["tags"], non_blocking=True)
+                db.off.copy_(hb["off"], non_blocking=True)
+                db.payload.copy_(hb["payload"], non_blocking=True)
+                if hb["score"] is not None:
+                    db.score.copy_(hb["score"], non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(cs_in)
+                ready.append(ev)
+        if flags["out"] is not None:
+            stream.wait_event(flags["out"])
+        for db, ev in zip(dev, ready):
+            stream.wait_event(ev)
             st = agg.push(db.tags, db.off, db.payload, db.score)
             if st != alto.OK:
                 raise RuntimeError(f"push failed: {st}")
         d = agg.drain()
         nr = d.records.numel()
         npay = d.payload.numel()
-        rec_host[:nr].copy_(d.records, non_blocking=True)
-        pay_host[:npay].copy_(d.payload, non_blocking=True)
-        torch.cuda.synchronize()
+        cs_out.wait_stream(stream)
+        with torch.cuda.stream(cs_out):
+            rec_host[:nr].copy_(d.records, non_blocking=True)
+            pay_host[:npay].copy_(d.payload, non_blocking=True)
+            ev = torch.cuda.Event()
+            ev.record(cs_out)
+        flags["out"] = ev
         return nr + npay * 4
 
     e2e_step()
+    torch.cuda.synchronize()
+    flags["out"] = None
     barrier()
     torch.cuda.synchronize()
     e_start = torch.cuda.Event(enable_timing=True)
@@ -627,6 +652,8 @@ def main():
     d2h = 0
     for _ in range(e_steps):
         d2h = e2e_step()
+    stream.wait_stream(cs_out)
+    stream.wait_stream(cs_in)
     e_end.record(stream)
     torch.cuda.synchronize()
     e_ms = e_start.elapsed_time(e_end)
