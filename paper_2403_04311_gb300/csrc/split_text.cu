@@ -98,8 +98,10 @@ struct SplitScan {
   }
 };
 
-__device__ __forceinline__ void put_piece(const SplitDev& d, u64 stride, u64 s, u64 f, u32 end, bool last) {
-  const u64 first = (u64)d.ends[d.tok_off[s]] + d.empt[s];
+// Piece f (of `stride`) of stream s, ending at token `end`; `first` is the
+// stream's first piece index.
+__device__ __forceinline__ void put_piece(const SplitDev& d, u64 stride, u64 s, u64 f, u32 end, bool last,
+                                          u64 first) {
   d.out_off[f + 1] = end;
   for (int l = 0; l < d.depth_in; ++l) d.out_tags[(u64)l * stride + f] = d.src_tags[(u64)l * d.n_src + s];
   d.out_tags[(u64)d.depth_in * stride + f] =
@@ -108,7 +110,11 @@ __device__ __forceinline__ void put_piece(const SplitDev& d, u64 stride, u64 s, 
 
 // Each warp takes one contiguous range of tokens: lane 0 finds the stream of
 // its first token by binary search once, and the warp steps forward from
-// there, 32 tokens at a time (four rounds' loads in flight).
+// there, 32 tokens at a time (four rounds' loads in flight).  A piece's index
+// is the range's first index (one load) plus the pieces the warp has ended
+// since (ballots), and the current stream's first piece index is kept in
+// registers, so a piece costs no dependent load of its own; the next step's
+// tokens are loaded before this step's pieces are written.
 constexpr int kSplitRounds = 4;
 
 __global__ void __launch_bounds__(kSplitThreads) k_split_write(SplitDev d) {
@@ -143,31 +149,53 @@ __global__ void __launch_bounds__(kSplitThreads) k_split_write(SplitDev d) {
     }
     s = __shfl_sync(0xFFFFFFFFu, s, 0);
   }
+  // pieces ended before this warp's range, and the current stream's first piece
+  u64 done = (lo < hi) ? (u64)d.ends[lo] : 0;
+  u64 first_s = (lo < hi) ? (u64)d.ends[d.tok_off[s]] + d.empt[s] : 0;
+  u32 empt_s = (lo < hi) ? d.empt[s] : 0;
+  bool end[kSplitRounds];
+#pragma unroll
+  for (int r = 0; r < kSplitRounds; ++r) {
+    const u64 p = lo + 32ull * r + lane;
+    end[r] = p < hi && (is_delim(d, d.tokens[p]) || d.endmark[p]);
+  }
   for (u64 base = lo; base < hi; base += step) {
-    bool end[kSplitRounds];
+    u32 m[kSplitRounds];
+#pragma unroll
+    for (int r = 0; r < kSplitRounds; ++r) m[r] = __ballot_sync(0xFFFFFFFFu, end[r]);
+    // the next step's tokens go out before this step's pieces are written
+    const u64 nb = base + step;
 #pragma unroll
     for (int r = 0; r < kSplitRounds; ++r) {
-      const u64 p = base + 32ull * r + lane;
+      const u64 p = nb + 32ull * r + lane;
       end[r] = p < hi && (is_delim(d, d.tokens[p]) || d.endmark[p]);
     }
 #pragma unroll
     for (int r = 0; r < kSplitRounds; ++r) {
       const u64 p = base + 32ull * r + lane;
-      if (!end[r]) continue;
-      u64 sp = s;
-      while (sp + 1 < d.n_src && d.tok_off[sp + 1] <= p) ++sp;
-      const u64 f = (u64)d.ends[p] + d.empt[sp];
-      put_piece(d, n_frag, sp, f, (u32)(p + 1), p + 1 == d.tok_off[sp + 1]);
+      if ((m[r] >> lane) & 1u) {
+        u64 sp = s;
+        while (sp + 1 < d.n_src && d.tok_off[sp + 1] <= p) ++sp;
+        const u64 k = done + __popc(m[r] & lanemask_lt());  // = ends[p]
+        const u32 em = (sp == s) ? empt_s : d.empt[sp];
+        const u64 fs = (sp == s) ? first_s : (u64)d.ends[d.tok_off[sp]] + d.empt[sp];
+        put_piece(d, n_frag, sp, k + em, (u32)(p + 1), p + 1 == d.tok_off[sp + 1], fs);
+      }
+      done += __popc(m[r]);
     }
-    // the stream of the next round's first token
-    const u64 nb = base + step;
+    // the stream of the next step's first token
+    const u64 s0 = s;
     while (s + 1 < d.n_src && d.tok_off[s + 1] <= nb) ++s;
+    if (s != s0 && nb < hi) {
+      empt_s = d.empt[s];
+      first_s = (u64)d.ends[d.tok_off[s]] + empt_s;
+    }
   }
   for (u64 st = (u64)blockIdx.x * blockDim.x + threadIdx.x; st < d.n_src; st += (u64)gridDim.x * blockDim.x) {
     const u32 a = d.tok_off[st];
     if (d.tok_off[st + 1] != a) continue;
     const u64 f = (u64)d.ends[a] + d.empt[st];
-    put_piece(d, n_frag, st, f, a, true);
+    put_piece(d, n_frag, st, f, a, true, f);
   }
 }
 
@@ -265,7 +293,13 @@ extern "C" alto_status alto_split_text(const alto_split_args* a, void* stream) {
     launch_pdl(k_scan_reduce<SplitScan>, rgrid, kScanThreads, 0, s, ft, part, d.ctl);
     launch_pdl(k_scan_down<SplitScan>, rgrid, kScanThreads, 0, s, ft, (const u64*)part, d.ctl);
   }
-  launch_pdl(k_split_write, sms * 8, kSplitThreads, 0, s, d);
+  // every warp owns a fixed token range: the grid is exactly the warps that
+  // fit on the GPU at once (a second wave would run its ranges after the first)
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_split_write, kSplitThreads, 0) != cudaSuccess ||
+      per_sm < 1)
+    per_sm = 1;
+  launch_pdl(k_split_write, sms * per_sm, kSplitThreads, 0, s, d);
   if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
   return ALTO_OK;
 }
