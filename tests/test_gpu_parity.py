@@ -166,3 +166,37 @@ def test_determinism_repeated_runs():
         assert a[0] == b[0]
         assert np.array_equal(a[1].view(np.uint8), b[1].view(np.uint8))
         assert np.array_equal(a[2], b[2])
+
+
+def _wide_topk_stream(n_children, leaves_per_child, batches, seed):
+    """Depth 2: one source whose level-0 group has n_children child groups
+    (TOPK(5) over them, CONCAT inside each), all in a shuffled order."""
+    rng = np.random.default_rng(seed)
+    frags = []
+    for c in range(n_children):
+        for k in range(leaves_per_child):
+            tags = ((1, c, c == n_children - 1), (100 + c, k, k == leaves_per_child - 1))
+            frags.append((tags, rng.integers(0, 1000, size=int(rng.integers(1, 6))).tolist(),
+                          float(rng.standard_normal())))
+    order = rng.permutation(len(frags))
+    frags = [frags[i] for i in order]
+    cuts = np.linspace(0, len(frags), batches + 1).astype(int)
+    return [frags[a:b] for a, b in zip(cuts[:-1], cuts[1:])]
+
+
+@pytest.mark.parametrize("n_children,batches", [(10_000, 1), (12_000, 3)])
+def test_topk_level_with_a_segment_longer_than_a_warp_share(n_children, batches):
+    """An upper TOPK level whose group has more than 4,096 items in one batch
+    takes the block-wide reduce; bit for bit against the oracle."""
+    parts = _wide_topk_stream(n_children, 2, batches, seed=n_children)
+    bts = [to_batch(p, 2, True) for p in parts]
+    n = max(b["n"] for b in bts)
+    pay = max(len(b["payload"]) for b in bts)
+    caps = dict(max_batch_fragments=n, max_batch_payload=pay, max_open_groups=1 << 16, arena_elems=1 << 22,
+                out_records=n_children + 64, out_payload_elems=sum(len(b["payload"]) for b in bts) + 64,
+                out_topk=64, max_emit_children=2 * n_children * 2 + 64)
+    po, so, kk = [0, 1], [2, 1], [5, 0]
+    _, g = run_gpu_batches(2, po, so, kk, bts, caps)
+    o = run_oracle_batches(2, po, so, kk, bts)
+    assert all(d.status == 0 for d in o)
+    assert_same(o, g, f"wide topk {n_children}/{batches}")

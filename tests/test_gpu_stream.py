@@ -237,3 +237,13 @@ def test_stream_release_fullsize_throughput():
         idx = idx[np.argsort(leaf_c[idx], kind="stable")]
         want = np.concatenate([s.payload[s.off[i]:s.off[i + 1]] for i in idx]).tolist()
         assert got_pay[p] == want, p
+
+
+def test_stream_release_on_a_segment_longer_than_a_warp_share():
+    """One group of 20,000 children in blocks of 1,000 in shuffled block order,
+    8,192-fragment batches: its segment in a batch is longer than 4,096 leaves
+    (the block-wide reduce), and releases both take leaves straight from the
+    batch and drop buffered ones."""
+    s = _groups_stream(1, 20_000, 6, lambda rng, n: [c for b in rng.permutation(n // 1000)
+                                                       for c in range(1000 * b, 1000 * (b + 1))], 8192, seed=3)
+    assert _check(s, 1) > 0
