@@ -290,7 +290,7 @@ def run_split(args, rank, world):
             "data": "synthetic",
             "config": {"workload": "split", "streams": n_src, "tokens": n_tok, "pieces": n_frag,
                        "l2": "inputs larger than L2 (no flush)"},
-            "roofline": {"bound": "hbm", "kernel": "split_text (mark, two scans, write)",
+            "roofline": {"bound": "hbm", "kernel": "split_text (mark, count, range scan, write)",
                          "achieved": achieved, "peak": hbm_gbs, "unit": "GB/s",
                          "frac": achieved / hbm_gbs, "peak_kind": peak_kind, "traffic": None},
             "gpu_launches": 4 * args.steps, "clocks": clocks,

@@ -246,156 +246,6 @@ __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl
   if (t == 0) finish_ctas(ctl, site, exit_ctr);
 }
 
-// ---------------------------------------------------------------------------
-// Large scans: reduce, then scan down, no look-back.  A persistent grid of G
-// CTAs splits the elements into G contiguous chunks of whole tiles.  The first
-// kernel writes each chunk's sum; the second has every CTA add up the sums of
-// the chunks before its own and scan its chunk tile by tile with a running
-// offset.  The input is read twice and the prefixes written once, all in
-// streaming order, which beats the look-back scan once the elements are many
-// times the CTAs' tiles (the look-back then walks back a whole wave of tiles).
-// ---------------------------------------------------------------------------
-template <class F>
-__device__ __forceinline__ void chunk_of_cta(const F& f, Ctl* ctl, u64* n_out, u64* lo, u64* hi) {
-  const u64 n = halted(ctl) ? 0 : f.size(ctl);
-  const u64 tiles = (n + kScanTile - 1) / kScanTile;
-  const u64 per = (tiles + gridDim.x - 1) / gridDim.x * kScanTile;
-  *n_out = n;
-  *lo = min(n, (u64)blockIdx.x * per);
-  *hi = min(n, *lo + per);
-}
-
-template <class F>
-__global__ void __launch_bounds__(kScanThreads) k_scan_reduce(F f, u64* part, Ctl* ctl) {
-  pdl_enter();
-  __shared__ u64 s_w[kScanWarps];
-  u64 n, lo, hi;
-  chunk_of_cta(f, ctl, &n, &lo, &hi);
-  u64 sum = 0;
-  for (u64 b = lo; b < hi; b += (u64)kScanThreads * kScanItems) {
-    u32 v[kScanItems];
-#pragma unroll
-    for (int k = 0; k < kScanItems; ++k) {
-      const u64 i = b + (u64)k * kScanThreads + threadIdx.x;
-      v[k] = (i < hi) ? (u32)f.value(i) : 0u;
-    }
-#pragma unroll
-    for (int k = 0; k < kScanItems; ++k) sum += v[k];
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
-  if ((threadIdx.x & 31) == 0) s_w[threadIdx.x >> 5] = sum;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    u64 t = 0;
-    for (int q = 0; q < kScanWarps; ++q) t += s_w[q];
-    part[blockIdx.x] = t;
-  }
-}
-
-template <class F>
-__global__ void __launch_bounds__(kScanThreads) k_scan_down(F f, const u64* part, Ctl* ctl) {
-  pdl_enter();
-  __shared__ u32 s_v[kScanTile + kScanTile / 32];
-  __shared__ u64 s_w[kScanWarps];
-  __shared__ u64 s_off;
-  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-  u64 n, lo, hi;
-  chunk_of_cta(f, ctl, &n, &lo, &hi);
-  // offset of this chunk: the sums of the chunks before it (and the grand total)
-  {
-    u64 before = 0, all = 0;
-    for (u32 c = t; c < gridDim.x; c += kScanThreads) {
-      const u64 v = part[c];
-      if (c < blockIdx.x) before += v;
-      all += v;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      before += __shfl_xor_sync(0xFFFFFFFFu, before, o);
-      all += __shfl_xor_sync(0xFFFFFFFFu, all, o);
-    }
-    __shared__ u64 s_b[kScanWarps], s_a[kScanWarps];
-    if (lane == 0) {
-      s_b[warp] = before;
-      s_a[warp] = all;
-    }
-    __syncthreads();
-    if (t == 0) {
-      u64 b = 0, a = 0;
-      for (int q = 0; q < kScanWarps; ++q) {
-        b += s_b[q];
-        a += s_a[q];
-      }
-      s_off = b;
-      if (blockIdx.x == 0) f.total(ctl, a);
-    }
-    __syncthreads();
-  }
-  u64 off = s_off;
-  for (u64 base = lo; base < hi; base += kScanTile) {
-#pragma unroll
-    for (int k = 0; k < kScanItems; ++k) {
-      const u32 p = (u32)(k * kScanThreads + t);
-      const u64 i = base + p;
-      s_v[scan_pad(p)] = (i < hi) ? (u32)f.value(i) : 0u;
-    }
-    __syncthreads();
-    u32 w[kScanItems];
-    u64 sum = 0;
-#pragma unroll
-    for (int k = 0; k < kScanItems; ++k) {
-      w[k] = s_v[scan_pad((u32)(t * kScanItems + k))];
-      sum += w[k];
-    }
-    u64 x = sum;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const u64 y = __shfl_up_sync(0xFFFFFFFFu, x, o);
-      if (lane >= o) x += y;
-    }
-    if (lane == 31) s_w[warp] = x;
-    __syncthreads();
-    u64 wpre = 0, agg = 0;
-#pragma unroll
-    for (int q = 0; q < kScanWarps; ++q) {
-      const u64 c = s_w[q];
-      if (q < warp) wpre += c;
-      agg += c;
-    }
-    const bool narrow = agg < (1ull << 32);
-    u64 rel = wpre + (x - sum);
-    if (narrow) {
-#pragma unroll
-      for (int k = 0; k < kScanItems; ++k) {
-        s_v[scan_pad((u32)(t * kScanItems + k))] = (u32)rel;
-        rel += w[k];
-      }
-    }
-    __syncthreads();
-    if (narrow) {
-#pragma unroll
-      for (int k = 0; k < kScanItems; ++k) {
-        const u32 p = (u32)(k * kScanThreads + t);
-        const u64 i = base + p;
-        const u32 r0 = s_v[scan_pad(p)];
-        const u32 r1 = (p + 1 < (u32)kScanTile) ? s_v[scan_pad(p + 1)] : (u32)agg;
-        if (i < hi) f.out(i, off + r0, (u64)(r1 - r0));
-      }
-    } else {
-      u64 run = off + wpre + (x - sum);
-      const u64 first = base + (u64)t * kScanItems;
-#pragma unroll
-      for (int k = 0; k < kScanItems; ++k) {
-        if (first + k < hi) f.out(first + k, run, w[k]);
-        run += w[k];
-      }
-    }
-    off += agg;
-    __syncthreads();
-  }
-}
-
 template <class F>
 __global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ctl* ctl, int site,
                                                        u32* exit_ctr, u64 spin_limit) {

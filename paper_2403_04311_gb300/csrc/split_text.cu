@@ -3,16 +3,18 @@
 // into a stream of smaller Delimiter items; Sec. 4.2: at a pmap entry every
 // child keeps its parent's tags and gets one new tag), on one GB300.
 //
-// After the scratch is cleared, three launches:
+// After the scratch is cleared:
 //   mark    per stream: check its offsets, flag its last token
-//   count   piece ends over the tokens (a delimiter, or a stream's last
-//           token): a reduce-then-scan, two streaming passes (a look-back scan
-//           would walk back a whole wave of tiles at 100M tokens); empty
-//           streams over the streams: a look-back scan
+//   empty   empty streams before each stream (a look-back scan over streams)
+//   count   every warp owns one contiguous range of tokens and counts the
+//           piece ends in it (a delimiter, or a stream's last token), and for
+//           every stream starting in it the ends before that start
+//   ranges  the ends before each range (a look-back scan over the ranges)
 //   write   per piece end, and per empty stream: the piece's fragment index
 //           (piece ends before it + empty streams before its stream), its
 //           tags, and its end offset.  Pieces tile the token buffer, so a
 //           piece starts where the previous one ends and nothing is copied.
+// The tokens are read twice (count, write); no per-token array is written.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -27,6 +29,10 @@ namespace {
 
 constexpr int kSplitThreads = 256;
 
+// count and write split the tokens into the same ranges, one a warp
+constexpr u64 kSplitStep = 128;         // tokens a warp looks at per step (4 rounds of 32)
+constexpr u64 kSplitMaxWarps = 1u << 15;
+
 struct SplitDev {
   Ctl* ctl;
   int32_t delims[ALTO_MAX_DELIMS];
@@ -38,8 +44,12 @@ struct SplitDev {
   const u32* tok_off;
   const int32_t* tokens;
   unsigned char* endmark;  // [n_tokens] last token of a non-empty stream
-  u32* ends;    // [n_tokens + 1] piece ends before each token
   u32* empt;    // [n_src + 1] empty streams before each stream
+  u32* sloc;    // [n_src] piece ends between its range's first token and the stream's first token
+  u32* wcnt;    // [nwarps] piece ends in each range
+  u32* wpre;    // [nwarps + 1] piece ends before each range
+  u64 range;    // tokens per range (a multiple of kSplitStep)
+  u32 nwarps;
   u64* out_tags;
   u32* out_off;
   int64_t* out_counts;
@@ -78,25 +88,100 @@ __global__ void __launch_bounds__(kSplitThreads) k_split_mark(SplitDev d) {
   }
 }
 
-// which 0: piece ends over the tokens; 1: empty streams over the streams; 2: none
+// which 0: piece ends before each range; 1: empty streams over the streams
 struct SplitScan {
   SplitDev d;
   int which;
-  __device__ u64 size(const Ctl*) const { return (which == 0) ? d.n_tokens : (which == 1) ? d.n_src : 0; }
+  __device__ u64 size(const Ctl*) const { return (which == 0) ? d.nwarps : d.n_src; }
   __device__ u64 value(u64 i) const {
-    if (which == 0) return (is_delim(d, d.tokens[i]) || d.endmark[i]) ? 1u : 0u;
+    if (which == 0) return d.wcnt[i];
     return (d.tok_off[i + 1] == d.tok_off[i]) ? 1u : 0u;
   }
   __device__ void out(u64 i, u64 excl, u64) const {
-    if (which == 0) d.ends[i] = (u32)excl;
-    else if (which == 1) d.empt[i] = (u32)excl;
+    if (which == 0) d.wpre[i] = (u32)excl;
+    else d.empt[i] = (u32)excl;
   }
   __device__ void total(Ctl* ctl, u64 t) const {
-    if (which == 0) d.ends[d.n_tokens] = (u32)t;
-    else if (which == 1) d.empt[d.n_src] = (u32)t;
-    if (which < 2) ctl->scan_total[which] = t;
+    if (which == 0) d.wpre[d.nwarps] = (u32)t;
+    else d.empt[d.n_src] = (u32)t;
+    ctl->scan_total[which] = t;
   }
 };
+
+// The range [lo, hi) of warp w.
+__device__ __forceinline__ void split_range(const SplitDev& d, u64 w, u64* lo, u64* hi) {
+  *lo = min(d.n_tokens, w * d.range);
+  *hi = min(d.n_tokens, *lo + d.range);
+}
+
+// Piece ends before token a, the first token of a stream s (a < n_tokens:
+// its range's count before the range plus the stream's own count in it).
+__device__ __forceinline__ u64 ends_before_start(const SplitDev& d, u64 s, u64 a) {
+  return (a < d.n_tokens) ? (u64)d.wpre[a / d.range] + d.sloc[s] : (u64)d.wpre[d.nwarps];
+}
+
+// The four rounds' end flags of the step at `base` (false past hi).
+__device__ __forceinline__ void load_ends(const SplitDev& d, u64 base, u64 hi, bool (&end)[4]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const u64 p = base + 32ull * r + lane;
+    end[r] = p < hi && (is_delim(d, d.tokens[p]) || d.endmark[p]);
+  }
+}
+
+// First stream whose first token is at or after `lo`.
+__device__ __forceinline__ u64 first_stream_from(const SplitDev& d, u64 lo) {
+  u64 a = 0, b = d.n_src;
+  while (a < b) {
+    const u64 mid = (a + b) >> 1;
+    if (d.tok_off[mid] < lo) a = mid + 1;
+    else b = mid;
+  }
+  return a;
+}
+
+// Per range: its piece ends, and for every stream starting in it the ends
+// between the range's first token and the stream's first token.
+__global__ void __launch_bounds__(kSplitThreads) k_split_count(SplitDev d) {
+  pdl_enter();
+  Ctl* ctl = d.ctl;
+  if (ctl->batch_err != 0 || *(volatile int*)&ctl->abort != 0) return;
+  const int lane = threadIdx.x & 31;
+  const u64 w = ((u64)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  if (w >= d.nwarps) return;
+  u64 lo, hi;
+  split_range(d, w, &lo, &hi);
+  u64 ns = 0;  // next stream to start in this range
+  if (lo < hi) {
+    if (lane == 0) ns = first_stream_from(d, lo);
+    ns = __shfl_sync(0xFFFFFFFFu, ns, 0);
+  }
+  u32 done = 0;
+  bool end[4];
+  load_ends(d, lo, hi, end);
+  for (u64 base = lo; base < hi; base += kSplitStep) {
+    u32 m[4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) m[r] = __ballot_sync(0xFFFFFFFFu, end[r]);
+    load_ends(d, base + kSplitStep, hi, end);  // the next step's loads go out now
+    const u64 top = min(base + kSplitStep, hi);
+    while (ns < d.n_src && d.tok_off[ns] < top) {
+      const u32 t = (u32)(d.tok_off[ns] - base);
+      u32 c = done;
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        if ((u32)r < (t >> 5)) c += __popc(m[r]);
+        else if ((u32)r == (t >> 5)) c += __popc(m[r] & ((1u << (t & 31)) - 1u));
+      }
+      if (lane == 0) d.sloc[ns] = c;
+      ++ns;
+    }
+#pragma unroll
+    for (int r = 0; r < 4; ++r) done += __popc(m[r]);
+  }
+  if (lane == 0) d.wcnt[w] = done;
+}
 
 // Piece f (of `stride`) of stream s, ending at token `end`; `first` is the
 // stream's first piece index.
@@ -108,15 +193,11 @@ __device__ __forceinline__ void put_piece(const SplitDev& d, u64 stride, u64 s, 
       ((u64)d.src_id[s] << 32) | ((u64)(last ? 1u : 0u) << 31) | ((f - first) & 0x7FFFFFFFull);
 }
 
-// Each warp takes one contiguous range of tokens: lane 0 finds the stream of
-// its first token by binary search once, and the warp steps forward from
-// there, 32 tokens at a time (four rounds' loads in flight).  A piece's index
-// is the range's first index (one load) plus the pieces the warp has ended
-// since (ballots), and the current stream's first piece index is kept in
-// registers, so a piece costs no dependent load of its own; the next step's
-// tokens are loaded before this step's pieces are written.
-constexpr int kSplitRounds = 4;
-
+// Per range: each piece end's fragment index is the ends before the range
+// (one load) plus the ends the warp has passed (ballots) plus the empty
+// streams before its stream; the current stream's first piece index stays in
+// registers, and the next step's tokens are loaded before this step's pieces
+// are written.
 __global__ void __launch_bounds__(kSplitThreads) k_split_write(SplitDev d) {
   pdl_enter();
   Ctl* ctl = d.ctl;
@@ -130,12 +211,9 @@ __global__ void __launch_bounds__(kSplitThreads) k_split_write(SplitDev d) {
   }
   if (!ok || n_frag > d.cap) return;
   const int lane = threadIdx.x & 31;
-  const u64 gw = ((u64)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const u64 nw = ((u64)gridDim.x * blockDim.x) >> 5;
-  const u64 step = 32ull * kSplitRounds;
-  const u64 per = (d.n_tokens + nw - 1) / nw;
-  const u64 lo = min(d.n_tokens, (per + step - 1) / step * step * gw);
-  const u64 hi = min(d.n_tokens, lo + (per + step - 1) / step * step);
+  const u64 w = ((u64)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  u64 lo = 0, hi = 0;
+  if (w < d.nwarps) split_range(d, w, &lo, &hi);
   u64 s = 0;
   if (lo < hi) {
     if (lane == 0) {
@@ -149,36 +227,26 @@ __global__ void __launch_bounds__(kSplitThreads) k_split_write(SplitDev d) {
     }
     s = __shfl_sync(0xFFFFFFFFu, s, 0);
   }
-  // pieces ended before this warp's range, and the current stream's first piece
-  u64 done = (lo < hi) ? (u64)d.ends[lo] : 0;
-  u64 first_s = (lo < hi) ? (u64)d.ends[d.tok_off[s]] + d.empt[s] : 0;
+  u64 done = (lo < hi) ? (u64)d.wpre[w] : 0;
   u32 empt_s = (lo < hi) ? d.empt[s] : 0;
-  bool end[kSplitRounds];
+  u64 first_s = (lo < hi) ? ends_before_start(d, s, d.tok_off[s]) + empt_s : 0;
+  bool end[4];
+  load_ends(d, lo, hi, end);
+  for (u64 base = lo; base < hi; base += kSplitStep) {
+    u32 m[4];
 #pragma unroll
-  for (int r = 0; r < kSplitRounds; ++r) {
-    const u64 p = lo + 32ull * r + lane;
-    end[r] = p < hi && (is_delim(d, d.tokens[p]) || d.endmark[p]);
-  }
-  for (u64 base = lo; base < hi; base += step) {
-    u32 m[kSplitRounds];
+    for (int r = 0; r < 4; ++r) m[r] = __ballot_sync(0xFFFFFFFFu, end[r]);
+    const u64 nb = base + kSplitStep;
+    load_ends(d, nb, hi, end);  // the next step's loads go out now
 #pragma unroll
-    for (int r = 0; r < kSplitRounds; ++r) m[r] = __ballot_sync(0xFFFFFFFFu, end[r]);
-    // the next step's tokens go out before this step's pieces are written
-    const u64 nb = base + step;
-#pragma unroll
-    for (int r = 0; r < kSplitRounds; ++r) {
-      const u64 p = nb + 32ull * r + lane;
-      end[r] = p < hi && (is_delim(d, d.tokens[p]) || d.endmark[p]);
-    }
-#pragma unroll
-    for (int r = 0; r < kSplitRounds; ++r) {
+    for (int r = 0; r < 4; ++r) {
       const u64 p = base + 32ull * r + lane;
       if ((m[r] >> lane) & 1u) {
         u64 sp = s;
         while (sp + 1 < d.n_src && d.tok_off[sp + 1] <= p) ++sp;
-        const u64 k = done + __popc(m[r] & lanemask_lt());  // = ends[p]
+        const u64 k = done + __popc(m[r] & lanemask_lt());  // piece ends before p
         const u32 em = (sp == s) ? empt_s : d.empt[sp];
-        const u64 fs = (sp == s) ? first_s : (u64)d.ends[d.tok_off[sp]] + d.empt[sp];
+        const u64 fs = (sp == s) ? first_s : ends_before_start(d, sp, d.tok_off[sp]) + em;
         put_piece(d, n_frag, sp, k + em, (u32)(p + 1), p + 1 == d.tok_off[sp + 1], fs);
       }
       done += __popc(m[r]);
@@ -188,13 +256,13 @@ __global__ void __launch_bounds__(kSplitThreads) k_split_write(SplitDev d) {
     while (s + 1 < d.n_src && d.tok_off[s + 1] <= nb) ++s;
     if (s != s0 && nb < hi) {
       empt_s = d.empt[s];
-      first_s = (u64)d.ends[d.tok_off[s]] + empt_s;
+      first_s = ends_before_start(d, s, d.tok_off[s]) + empt_s;
     }
   }
   for (u64 st = (u64)blockIdx.x * blockDim.x + threadIdx.x; st < d.n_src; st += (u64)gridDim.x * blockDim.x) {
     const u32 a = d.tok_off[st];
     if (d.tok_off[st + 1] != a) continue;
-    const u64 f = (u64)d.ends[a] + d.empt[st];
+    const u64 f = ends_before_start(d, st, a) + d.empt[st];
     put_piece(d, n_frag, st, f, a, true, f);
   }
 }
@@ -202,22 +270,26 @@ __global__ void __launch_bounds__(kSplitThreads) k_split_write(SplitDev d) {
 u64 align256(u64 x) { return (x + 255) & ~255ull; }
 
 struct SplitLayout {
-  u64 ctl, desc, ends, empt, mark, total;
+  u64 ctl, desc, empt, sloc, wcnt, wpre, mark, total;
   u64 tiles;
 };
 
 SplitLayout split_layout(u64 n_src, u64 n_tokens) {
   SplitLayout L;
-  L.tiles = std::max(n_src, n_tokens) / kScanTile + 2;
+  L.tiles = std::max<u64>(n_src, kSplitMaxWarps) / kScanTile + 2;
   u64 o = 0;
   L.ctl = o;
   o += align256(sizeof(Ctl));
   L.desc = o;
-  o += align256(3 * L.tiles * sizeof(ulonglong2));
-  L.ends = o;
-  o += align256((n_tokens + 1) * sizeof(u32));
+  o += align256(2 * L.tiles * sizeof(ulonglong2));
   L.empt = o;
   o += align256((n_src + 1) * sizeof(u32));
+  L.sloc = o;
+  o += align256(n_src * sizeof(u32));
+  L.wcnt = o;
+  o += align256(kSplitMaxWarps * sizeof(u32));
+  L.wpre = o;
+  o += align256((kSplitMaxWarps + 1) * sizeof(u32));
   L.mark = o;
   o += align256(std::max<u64>(n_tokens, 1));
   L.total = o;
@@ -262,44 +334,52 @@ extern "C" alto_status alto_split_text(const alto_split_args* a, void* stream) {
   d.tok_off = a->tok_off;
   d.tokens = a->tokens;
   d.endmark = base + L.mark;
-  d.ends = (u32*)(base + L.ends);
   d.empt = (u32*)(base + L.empt);
+  d.sloc = (u32*)(base + L.sloc);
+  d.wcnt = (u32*)(base + L.wcnt);
+  d.wpre = (u32*)(base + L.wpre);
   d.out_tags = a->out_tags;
   d.out_off = a->out_off;
   d.out_counts = a->out_counts;
   LookbackState lb;
   lb.desc = (ulonglong2*)(base + L.desc);
   lb.tiles = L.tiles;
-  // the control block, the look-back descriptors and the last-token marks start empty
-  cudaMemsetAsync(base + L.ctl, 0, L.ends - L.ctl, s);
+  // the control block and the look-back descriptors start empty, and so do
+  // the last-token marks
+  cudaMemsetAsync(base + L.ctl, 0, L.empt - L.ctl, s);
   cudaMemsetAsync(base + L.mark, 0, std::max<u64>(d.n_tokens, 1), s);
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return ALTO_ECUDA;
+  // count and write give every warp one fixed token range: the grid is
+  // exactly the warps that fit on the GPU at once (a second wave would run
+  // its ranges after the first)
+  int pc = 0, pw = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&pc, k_split_count, kSplitThreads, 0) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&pw, k_split_write, kSplitThreads, 0) != cudaSuccess)
+    return ALTO_ECUDA;
+  const u64 wpb = kSplitThreads / 32;
+  const u64 blocks = std::max<u64>(1, std::min<u64>((u64)sms * (u64)std::max(1, std::min(pc, pw)),
+                                                      kSplitMaxWarps / wpb));
+  d.nwarps = (u32)(blocks * wpb);
+  const u64 per = (d.n_tokens + d.nwarps - 1) / d.nwarps;
+  d.range = std::max<u64>(kSplitStep, (per + kSplitStep - 1) / kSplitStep * kSplitStep);
   const u64 spin = 1ull << 20;
   launch_pdl(k_split_begin, 1, 1, 0, s, d.ctl);
   const int sgrid = (int)std::min<u64>((d.n_src + kSplitThreads - 1) / kSplitThreads + 1, (u64)sms * 8);
   launch_pdl(k_split_mark, sgrid, kSplitThreads, 0, s, d);
-  {
-    // streams: a look-back scan over the first descriptor region; tokens: a
-    // reduce-then-scan whose chunk sums live in the second region
-    SplitScan fs{d, 1}, ft{d, 0};
-    const u64 stiles = std::max<u64>((d.n_src + kScanTile - 1) / kScanTile, 1);
-    launch_pdl(k_scan<SplitScan>, (int)std::min<u64>(stiles, (u64)sms * 4), kScanThreads, 0, s, fs, lb,
-               d.ctl, 1, &d.ctl->exit_ctr[1], spin);
-    u64* part = reinterpret_cast<u64*>(lb.desc + lb.tiles);
-    const int rgrid = (int)std::min<u64>((u64)sms * 4, 2 * lb.tiles);
-    launch_pdl(k_scan_reduce<SplitScan>, rgrid, kScanThreads, 0, s, ft, part, d.ctl);
-    launch_pdl(k_scan_down<SplitScan>, rgrid, kScanThreads, 0, s, ft, (const u64*)part, d.ctl);
-  }
-  // every warp owns a fixed token range: the grid is exactly the warps that
-  // fit on the GPU at once (a second wave would run its ranges after the first)
-  int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_split_write, kSplitThreads, 0) != cudaSuccess ||
-      per_sm < 1)
-    per_sm = 1;
-  launch_pdl(k_split_write, sms * per_sm, kSplitThreads, 0, s, d);
+  SplitScan fs{d, 1}, fw{d, 0};
+  LookbackState lb1 = lb;
+  lb1.desc += lb.tiles;
+  const u64 stiles = std::max<u64>((d.n_src + kScanTile - 1) / kScanTile, 1);
+  launch_pdl(k_scan<SplitScan>, (int)std::min<u64>(stiles, (u64)sms), kScanThreads, 0, s, fs, lb1, d.ctl, 1,
+             &d.ctl->exit_ctr[1], spin);
+  launch_pdl(k_split_count, (int)blocks, kSplitThreads, 0, s, d);
+  const u64 wtiles = std::max<u64>((d.nwarps + kScanTile - 1) / kScanTile, 1);
+  launch_pdl(k_scan<SplitScan>, (int)std::min<u64>(wtiles, (u64)sms), kScanThreads, 0, s, fw, lb, d.ctl, 0,
+             &d.ctl->exit_ctr[0], spin);
+  launch_pdl(k_split_write, (int)blocks, kSplitThreads, 0, s, d);
   if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
   return ALTO_OK;
 }
