@@ -437,7 +437,9 @@ __global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
                               b.n, i, D - 1);
     if (ins) atomicAdd(&s_ins, 1u);
     d.sc.leaf_sort_keys0[i] = e;
-    // the sorted (TOPK) leaf path checks leaf slots here; the accumulate does otherwise
+    // the sorted (TOPK) leaf path checks leaf slots here, spread over the
+    // whole grid (in the reduce, a hot group's checks would all fall to the
+    // block that reduces its segment); the accumulate does otherwise
     if (sorted_leaf && ps_insert(d.sc, e, tag_child(t), ep7, ctl)) raise_err(ctl, ALTO_EDUP);
   }
   __syncthreads();
@@ -1707,7 +1709,9 @@ __global__ void k_fix_tops(Ctl* ctl) {
 // per leaf, over the sorted leaves.  A leaf's vector position is its group's
 // reserved base plus its offset inside the segment (written by the reduce;
 // for a partial release, among the leaves it keeps).  (A lane per leaf with
-// the spans then copied four at a time, as in the gather, measured slower.)
+// the spans then copied four at a time, as in the gather, measured slower;
+// so did a warp per carried segment, which leaves a hot group's tens of
+// thousands of leaves to one warp.)
 __global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch b) {
   pdl_enter();
   Ctl* ctl = d.ctl;

@@ -213,6 +213,8 @@ int sort_pairs(const u32* n_dev, u32 n_cap, int bits, bool vals_identity, SortBu
   int hist_grid = num_sms * 2;
   launch_pdl(k_sort_hist, hist_grid, 256, 0, s, n_dev, n_cap, b.keys[0], passes, b.hist, ctl);
   launch_pdl(k_sort_binbase, 1, 256, 0, s, b.hist, b.bin_base, passes);
+  // four CTAs per SM (one per SM measured slower: each CTA then takes about
+  // two tiles in turn, and a tile's look-back waits on the one before)
   u32 g4 = (u32)num_sms * 4u;
   int grid = (int)(tiles_cap < g4 ? tiles_cap : g4);
   int cur = 0;
