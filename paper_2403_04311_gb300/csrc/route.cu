@@ -548,7 +548,7 @@ extern "C" alto_status alto_router_route(alto_router_t* h, const alto_batch* b, 
   if (cfg.policy == ALTO_ROUTE_LEAST_LOADED) {
     RankScan2 f{d};
     const u64 tiles = std::max<u64>(((u64)cfg.max_batch_fragments + kScanTile - 1) / kScanTile, 1);
-    launch_pdl(k_scan<RankScan2>, (int)std::min<u64>(tiles, (u64)h->num_sms), kScanThreads, 0, s, f,
+    launch_pdl(k_scan<RankScan2>, (int)std::min<u64>(tiles, (u64)h->num_sms * 4), kScanThreads, 0, s, f,
                h->lbs, d.ctl, 8, &d.ctl->exit_ctr[8], spin);
     launch_pdl(k_rt_order, 1, 1024, 0, s, d);
     launch_pdl(k_rt_place, grid, kRT, 0, s, d);
@@ -570,7 +570,7 @@ extern "C" alto_status alto_router_route(alto_router_t* h, const alto_batch* b, 
   {
     PermLenScan f{d};
     const u64 tiles = std::max<u64>(((u64)cfg.max_batch_fragments + kScanTile - 1) / kScanTile, 1);
-    launch_pdl(k_scan<PermLenScan>, (int)std::min<u64>(tiles, (u64)h->num_sms), kScanThreads, 0, s, f,
+    launch_pdl(k_scan<PermLenScan>, (int)std::min<u64>(tiles, (u64)h->num_sms * 4), kScanThreads, 0, s, f,
                h->lbs, d.ctl, 9, &d.ctl->exit_ctr[9], spin);
   }
   launch_pdl(k_rt_scatter, grid, kRT, 0, s, d);
