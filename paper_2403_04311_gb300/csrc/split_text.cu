@@ -30,7 +30,9 @@ namespace {
 constexpr int kSplitThreads = 256;
 
 // count and write split the tokens into the same ranges, one a warp
-constexpr u64 kSplitStep = 128;         // tokens a warp looks at per step (4 rounds of 32)
+constexpr int kSplitRounds = 4;         // rounds of loads a warp keeps in flight
+constexpr u64 kSplitRound = 128;        // tokens a round: four consecutive ones a lane
+constexpr u64 kSplitStep = kSplitRounds * kSplitRound;
 constexpr u64 kSplitMaxWarps = 1u << 15;
 
 struct SplitDev {
@@ -120,13 +122,47 @@ __device__ __forceinline__ u64 ends_before_start(const SplitDev& d, u64 s, u64 a
   return (a < d.n_tokens) ? (u64)d.wpre[a / d.range] + d.sloc[s] : (u64)d.wpre[d.nwarps];
 }
 
-// The four rounds' end flags of the step at `base` (false past hi).
-__device__ __forceinline__ void load_ends(const SplitDev& d, u64 base, u64 hi, bool (&end)[4]) {
+// The end flags of the step at `base`: in round r, lane l owns tokens
+// base + 128r + 4l .. +3 (bit k of f[r]: token 4l + k; none past hi).  With a
+// 16-byte aligned token buffer a lane reads its four tokens and their four
+// last-token marks with one load each.
+__device__ __forceinline__ u32 end_bit(const SplitDev& d, int32_t tok, u32 mark) {
+  return (is_delim(d, tok) || mark) ? 1u : 0u;
+}
+__device__ __forceinline__ void load_flags(const SplitDev& d, u64 base, u64 hi, bool vec, u32 (&f)[kSplitRounds]) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
-  for (int r = 0; r < 4; ++r) {
-    const u64 p = base + 32ull * r + lane;
-    end[r] = p < hi && (is_delim(d, d.tokens[p]) || d.endmark[p]);
+  for (int r = 0; r < kSplitRounds; ++r) {
+    const u64 p = base + kSplitRound * r + 4ull * lane;
+    u32 m = 0;
+    if (vec && p + 4 <= hi) {
+      const int4 t = *reinterpret_cast<const int4*>(d.tokens + p);
+      const u32 mk = *reinterpret_cast<const u32*>(d.endmark + p);
+      m = end_bit(d, t.x, mk & 0xFFu) | (end_bit(d, t.y, (mk >> 8) & 0xFFu) << 1) |
+          (end_bit(d, t.z, (mk >> 16) & 0xFFu) << 2) | (end_bit(d, t.w, mk >> 24) << 3);
+    } else {
+      for (int k = 0; k < 4; ++k)
+        if (p + k < hi) m |= end_bit(d, d.tokens[p + k], d.endmark[p + k]) << k;
+    }
+    f[r] = m;
+  }
+}
+
+// Per round: the ends of the lanes before this one, and the round's total.
+__device__ __forceinline__ void round_counts(const u32 (&f)[kSplitRounds], u32 (&excl)[kSplitRounds],
+                                             u32 (&tot)[kSplitRounds]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int r = 0; r < kSplitRounds; ++r) {
+    const u32 c = __popc(f[r]);
+    u32 incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const u32 y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    excl[r] = incl - c;
+    tot[r] = __shfl_sync(0xFFFFFFFFu, incl, 31);
   }
 }
 
@@ -157,28 +193,33 @@ __global__ void __launch_bounds__(kSplitThreads) k_split_count(SplitDev d) {
     if (lane == 0) ns = first_stream_from(d, lo);
     ns = __shfl_sync(0xFFFFFFFFu, ns, 0);
   }
+  const bool vec = (reinterpret_cast<uintptr_t>(d.tokens) & 15) == 0;
   u32 done = 0;
-  bool end[4];
-  load_ends(d, lo, hi, end);
+  u32 f[kSplitRounds];
+  load_flags(d, lo, hi, vec, f);
   for (u64 base = lo; base < hi; base += kSplitStep) {
-    u32 m[4];
+    u32 excl[kSplitRounds], tot[kSplitRounds], fc[kSplitRounds];
+    round_counts(f, excl, tot);
 #pragma unroll
-    for (int r = 0; r < 4; ++r) m[r] = __ballot_sync(0xFFFFFFFFu, end[r]);
-    load_ends(d, base + kSplitStep, hi, end);  // the next step's loads go out now
+    for (int r = 0; r < kSplitRounds; ++r) fc[r] = f[r];
+    load_flags(d, base + kSplitStep, hi, vec, f);  // the next step's loads go out now
     const u64 top = min(base + kSplitStep, hi);
     while (ns < d.n_src && d.tok_off[ns] < top) {
       const u32 t = (u32)(d.tok_off[ns] - base);
+      const u32 rr = t / (u32)kSplitRound, ll = (t % (u32)kSplitRound) >> 2, kk = t & 3u;
       u32 c = done;
 #pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        if ((u32)r < (t >> 5)) c += __popc(m[r]);
-        else if ((u32)r == (t >> 5)) c += __popc(m[r] & ((1u << (t & 31)) - 1u));
+      for (int r = 0; r < kSplitRounds; ++r) {
+        const u32 ex = __shfl_sync(0xFFFFFFFFu, excl[r], ll);
+        const u32 fl = __shfl_sync(0xFFFFFFFFu, fc[r], ll);
+        if ((u32)r < rr) c += tot[r];
+        else if ((u32)r == rr) c += ex + __popc(fl & ((1u << kk) - 1u));
       }
       if (lane == 0) d.sloc[ns] = c;
       ++ns;
     }
 #pragma unroll
-    for (int r = 0; r < 4; ++r) done += __popc(m[r]);
+    for (int r = 0; r < kSplitRounds; ++r) done += tot[r];
   }
   if (lane == 0) d.wcnt[w] = done;
 }
@@ -230,26 +271,32 @@ __global__ void __launch_bounds__(kSplitThreads) k_split_write(SplitDev d) {
   u64 done = (lo < hi) ? (u64)d.wpre[w] : 0;
   u32 empt_s = (lo < hi) ? d.empt[s] : 0;
   u64 first_s = (lo < hi) ? ends_before_start(d, s, d.tok_off[s]) + empt_s : 0;
-  bool end[4];
-  load_ends(d, lo, hi, end);
+  const bool vec = (reinterpret_cast<uintptr_t>(d.tokens) & 15) == 0;
+  u32 f[kSplitRounds];
+  load_flags(d, lo, hi, vec, f);
   for (u64 base = lo; base < hi; base += kSplitStep) {
-    u32 m[4];
+    u32 excl[kSplitRounds], tot[kSplitRounds], fc[kSplitRounds];
+    round_counts(f, excl, tot);
 #pragma unroll
-    for (int r = 0; r < 4; ++r) m[r] = __ballot_sync(0xFFFFFFFFu, end[r]);
+    for (int r = 0; r < kSplitRounds; ++r) fc[r] = f[r];
     const u64 nb = base + kSplitStep;
-    load_ends(d, nb, hi, end);  // the next step's loads go out now
+    load_flags(d, nb, hi, vec, f);  // the next step's loads go out now
 #pragma unroll
-    for (int r = 0; r < 4; ++r) {
-      const u64 p = base + 32ull * r + lane;
-      if ((m[r] >> lane) & 1u) {
+    for (int r = 0; r < kSplitRounds; ++r) {
+      u32 bits = fc[r];
+      u64 k = done + excl[r];  // piece ends before this lane's first token of the round
+      while (bits) {
+        const int b = __ffs(bits) - 1;
+        bits &= bits - 1;
+        const u64 p = base + kSplitRound * r + 4ull * lane + b;
         u64 sp = s;
         while (sp + 1 < d.n_src && d.tok_off[sp + 1] <= p) ++sp;
-        const u64 k = done + __popc(m[r] & lanemask_lt());  // piece ends before p
         const u32 em = (sp == s) ? empt_s : d.empt[sp];
         const u64 fs = (sp == s) ? first_s : ends_before_start(d, sp, d.tok_off[sp]) + em;
         put_piece(d, n_frag, sp, k + em, (u32)(p + 1), p + 1 == d.tok_off[sp + 1], fs);
+        ++k;
       }
-      done += __popc(m[r]);
+      done += tot[r];
     }
     // the stream of the next step's first token
     const u64 s0 = s;

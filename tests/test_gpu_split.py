@@ -20,11 +20,17 @@ from gpu_harness import assert_same, run_gpu_batches, run_oracle_batches
 pytestmark = pytest.mark.gpu
 
 
-def gpu_split(src_tags, src_id, tok_off, tokens, delims, cap=None):
+def gpu_split(src_tags, src_id, tok_off, tokens, delims, cap=None, misalign=False):
     st_t = None if src_tags.shape[0] == 0 else torch.as_tensor(src_tags.view(np.int64), device="cuda")
     sid = torch.as_tensor(np.asarray(src_id, dtype=np.uint32).view(np.int32), device="cuda")
     off = torch.as_tensor(np.asarray(tok_off, dtype=np.uint32).view(np.int32), device="cuda")
     tok = torch.as_tensor(np.asarray(tokens, dtype=np.int32), device="cuda")
+    if misalign:
+        # the same tokens one element into a larger buffer: 4-byte but not
+        # 16-byte aligned, so every token is read on its own
+        buf = torch.zeros(tok.numel() + 1, dtype=torch.int32, device="cuda")
+        buf[1:] = tok
+        tok = buf[1:]
     st, n, tags, poff = alto.split_text(st_t, sid, off, tok, list(delims), cap_frag=cap)
     if st != alto.OK:
         return st, n, None, None
@@ -60,6 +66,18 @@ def test_split_matches_oracle(n_src, max_len, depth_in, long_one):
     st, n, tags, poff = gpu_split(src_tags, src_id, off, toks, delims)
     assert st == alto.OK
     assert n == want_tags.shape[1]
+    assert np.array_equal(tags, want_tags)
+    assert np.array_equal(poff, want_off)
+
+
+@pytest.mark.parametrize("n_src,max_len", [(7, 30), (2000, 40)])
+def test_split_unaligned_tokens(n_src, max_len):
+    rng = np.random.default_rng(n_src + 1)
+    delims = [3, 7, 11]
+    src_tags, src_id, off, toks = _random_case(rng, n_src, max_len, delims, 1, n_src > 100)
+    want_tags, want_off = oracle.split_text(src_tags, src_id, off, toks, delims)
+    st, n, tags, poff = gpu_split(src_tags, src_id, off, toks, delims, misalign=True)
+    assert st == alto.OK and n == want_tags.shape[1]
     assert np.array_equal(tags, want_tags)
     assert np.array_equal(poff, want_off)
 
