@@ -306,7 +306,8 @@ alto_status alto_agg_destroy(alto_agg_t* h);
  * ALTO_EINVAL for bad offsets, ALTO_ENOSPC when n_frag > cap_frag (nothing else
  * is written then; n_frag is still the count needed).  `scratch` is device
  * memory of at least alto_split_scratch_bytes(n_src, n_tokens) bytes, 256-byte
- * aligned, owned by the caller; calls sharing a scratch must not overlap.  The
+ * aligned, owned by the caller; calls sharing a scratch must not overlap.
+ * `tokens` is read fastest 16-byte aligned (four tokens a load).  The
  * return value is ALTO_EINVAL for bad host arguments (n_delims outside
  * 1..ALTO_MAX_DELIMS, depth_in outside 0..ALTO_MAX_DEPTH-1, null pointers,
  * too little scratch), ALTO_ECUDA if a launch fails, else ALTO_OK. */
