@@ -3,15 +3,21 @@
 //
 // One push runs this stream-ordered pipeline (no host synchronisation):
 //   ingest      validate offsets/scores; find-or-insert each fragment's
-//               leaf-parent group (level D-1) in the open-group hash table;
-//               flag a leaf slot given twice in the batch              [Sec. 4.2]
-//   sort        stable onesweep radix sort of fragments by table slot      [Sec. 4.3]
-//   segments    decoupled look-back scan finds each group's run
-//   reduce      one warp per group: count complete children, last-flag and
-//               child-index checks, ancestry consistency, max score, top-k;
-//               merge with the table entry and test completion          [Sec. 3.1]
-//   levels      the groups present at level l become the items of level l-1:
-//               table lookup, sort, segments, reduce again, up to level 0 [Sec. 4.2]
+//               leaf-parent group (level D-1) in the open-group hash table
+//                                                                       [Sec. 4.2]
+//   leaf level  count complete children, last-flag and child-index checks,
+//               ancestry consistency, max score, top-k; merge with the table
+//               entry and test completion                               [Sec. 3.1]
+//               - without TOPK: every fragment, in arrival order, adds itself
+//                 to its group's 64-byte table record (warp-aggregated
+//                 atomics) and flags a repeated leaf slot; one pass over the
+//                 touched groups then merges and tests them
+//               - with TOPK (or streaming release): a stable onesweep radix
+//                 sort by table slot, a look-back scan for each group's run,
+//                 and a reduce by eight lanes, a warp or a block per run
+//                 (segmented top-k)                                     [Sec. 4.3]
+//   levels      the groups present at level l become the items of level l-1,
+//               in the same two forms, up to level 0                    [Sec. 4.2]
 //   emit order  completed groups ranked by (completion seq, deeper first)
 //   CONCAT      open groups: append their leaves to per-group arena vectors;
 //               completing groups: place every child span at slot
