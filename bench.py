@@ -71,6 +71,33 @@ def stream_caps(s, stream_release=False):
     )
 
 
+def init_dist(world, backend=None):
+    """One process per GPU under torchrun (RANK, WORLD_SIZE, MASTER_ADDR from the
+    environment): NCCL with GPUs, gloo without; None for one process."""
+    if world <= 1:
+        return None
+    import torch
+    import torch.distributed as dist
+    dist.init_process_group(backend or ("nccl" if torch.cuda.is_available() else "gloo"))
+    return dist
+
+
+def max_over_ranks(x, dist):
+    """The largest x over all ranks (every rank gets it)."""
+    if dist is None:
+        return float(x)
+    import torch
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
 class ClockSampler:
     """nvidia-smi clocks and throttle reasons during the timed region."""
 
@@ -213,6 +240,7 @@ def run_split(args, rank, world):
     import torch
     import paper_2403_04311_gb300 as alto
     torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    dist = init_dist(world)
     stream = torch.cuda.current_stream()
     dev = "cuda"
     tags_d = torch.as_tensor(si.src_tags.view(np.int64), device=dev)
@@ -243,6 +271,8 @@ def run_split(args, rank, world):
     st, n_frag = (int(x) for x in counts.cpu().tolist())
     assert st == alto.OK
     sampler = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
+    barrier(dist)
+    torch.cuda.synchronize()
     sampler.start()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
@@ -250,8 +280,9 @@ def run_split(args, rank, world):
         step()
     e1.record(stream)
     torch.cuda.synchronize()
+    barrier(dist)
     clocks = sampler.stop()
-    ms = e0.elapsed_time(e1) / args.steps
+    ms = max_over_ranks(e0.elapsed_time(e1), dist) / args.steps
     hbm_gbs, peak_kind = peaks()
     # algorithmic bytes of one call: the tokens and the stream offsets and tags
     # read, each piece's two tags and offset written
@@ -273,9 +304,11 @@ def run_split(args, rank, world):
         h_poff.copy_(out_off[:n_frag + 1], non_blocking=True)
     x1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = x0.elapsed_time(x1) / args.steps
+    e2e_ms = max_over_ranks(x0.elapsed_time(x1), dist) / args.steps
+    if dist is not None:
+        dist.destroy_process_group()
     cpu = None
-    if not args.no_cpu_baseline:
+    if not args.no_cpu_baseline and world == 1:
         import oracle
         k = 400
         t0 = time.perf_counter()
@@ -293,7 +326,7 @@ def run_split(args, rank, world):
             "roofline": {"bound": "hbm", "kernel": "split_text (mark, count, range scan, write)",
                          "achieved": achieved, "peak": hbm_gbs, "unit": "GB/s",
                          "frac": achieved / hbm_gbs, "peak_kind": peak_kind, "traffic": None},
-            "gpu_launches": 4 * args.steps, "clocks": clocks,
+            "gpu_launches": 6 * args.steps, "clocks": clocks,
             "e2e": {"value": n_tok * world / (e2e_ms / 1e3), "unit": "tokens/s",
                     "h2d_bytes_per_step": int(4 * n_tok + 4 * (n_src + 1)),
                     "d2h_bytes_per_step": int(16 * n_frag + 4 * (n_frag + 1))},
@@ -332,6 +365,7 @@ def run_route(args, rank, world, R=8):
     import torch
     import paper_2403_04311_gb300 as alto
     torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    dist = init_dist(world)
     stream = torch.cuda.current_stream()
     st = s.batch_starts()
     pay = int(max(s.off[b1] - s.off[b0] for b0, b1 in zip(st[:-1], st[1:])))
@@ -349,6 +383,8 @@ def run_route(args, rank, world, R=8):
     torch.cuda.synchronize()
     assert rt.counts()[0] == alto.OK
     sampler = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
+    barrier(dist)
+    torch.cuda.synchronize()
     sampler.start()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
@@ -356,9 +392,83 @@ def run_route(args, rank, world, R=8):
         step()
     e1.record(stream)
     torch.cuda.synchronize()
+    barrier(dist)
     clocks = sampler.stop()
-    ms = e0.elapsed_time(e1) / args.steps
+    ms = max_over_ranks(e0.elapsed_time(e1), dist) / args.steps
+
+    # end to end: every batch's tags, offsets and payload from pinned host
+    # memory on a copy stream (a batch's routing waits for its own upload),
+    # and the replicas' batches (tags, offsets, payload) back on a second one;
+    # the next routing reuses the output buffers, so it waits for that read-back
+    hosts = []
+    for b in range(s.n_batches):
+        hb = s.batch(b)
+        hosts.append((torch.from_numpy(hb["tags"].view(np.int64)).pin_memory(),
+                      torch.from_numpy(hb["off"].view(np.int32)).pin_memory(),
+                      torch.from_numpy(hb["payload"]).pin_memory(), hb["n"], len(hb["payload"])))
+    n_max = int(max(s.batch_sizes))
+    h_tags = torch.empty(s.depth * n_max, dtype=torch.int64).pin_memory()
+    h_poff = torch.empty(n_max + R, dtype=torch.int32).pin_memory()
+    h_pay = torch.empty(max(pay, 1), dtype=torch.int32).pin_memory()
+    cs_in, cs_out = torch.cuda.Stream(), torch.cuda.Stream()
+
+    def e2e_step():
+        cs_in.wait_stream(stream)
+        ready = []
+        with torch.cuda.stream(cs_in):
+            for (ht, ho, hp, _n, _p), db in zip(hosts, batches):
+                db.tags.copy_(ht, non_blocking=True)
+                db.off.copy_(ho, non_blocking=True)
+                db.payload.copy_(hp, non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(cs_in)
+                ready.append(ev)
+        out_done = None
+        moved = 0
+        for (_ht, _ho, _hp, n_b, p_b), db, ev in zip(hosts, batches, ready):
+            stream.wait_event(ev)
+            if out_done is not None:
+                stream.wait_event(out_done)
+            if rt.route(db.tags, db.off, db.payload) != alto.OK:
+                raise RuntimeError("route failed")
+            t_all, o_all, p_all = rt.all_outputs(n_b, p_b)
+            cs_out.wait_stream(stream)
+            with torch.cuda.stream(cs_out):
+                h_tags[:s.depth * n_b].copy_(t_all, non_blocking=True)
+                h_poff[:n_b + R].copy_(o_all, non_blocking=True)
+                h_pay[:p_b].copy_(p_all, non_blocking=True)
+                out_done = torch.cuda.Event()
+                out_done.record(cs_out)
+            moved += 8 * s.depth * n_b + 4 * (n_b + R) + 4 * p_b
+        return moved
+
+    e2e_step()
+    torch.cuda.synchronize()
+    barrier(dist)
+    x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    x0.record(stream)
+    for _ in range(args.steps):
+        d2h = e2e_step()
+    stream.wait_stream(cs_out)
+    x1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(x0.elapsed_time(x1), dist) / args.steps
+    h2d = sum(ht.numel() * 8 + ho.numel() * 4 + hp.numel() * 4 for ht, ho, hp, _n, _p in hosts)
     rt.close()
+    if dist is not None:
+        dist.destroy_process_group()
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        import oracle
+        b0 = s.batch(0)
+        n = min(b0["n"], 250_000)
+        sample = dict(n=n, tags=np.ascontiguousarray(b0["tags"][:, :n]), off=b0["off"][:n + 1],
+                      payload=b0["payload"][:int(b0["off"][n])], score=None)
+        t0 = time.perf_counter()
+        oracle.RouterOracle(s.depth, L, R, oracle.LEAST_LOADED).route(sample)
+        dt = time.perf_counter() - t0
+        cpu = {"value": n / dt, "unit": "fragments/s", "cores": 1, "kind": "oracle",
+               "sample": f"first {n} fragments of batch 0, single thread"}
     hbm_gbs, peak_kind = peaks()
     # algorithmic bytes of a pass: every fragment's tags and offset read and
     # written once, every payload element read and written once
@@ -372,8 +482,9 @@ def run_route(args, rank, world, R=8):
             "roofline": {"bound": "hbm", "kernel": "route (all kernels of a batch)", "achieved": achieved,
                          "peak": hbm_gbs, "unit": "GB/s", "frac": achieved / hbm_gbs, "peak_kind": peak_kind,
                          "traffic": None},
-            "gpu_launches": 15 * s.n_batches * args.steps, "clocks": clocks, "cpu_baseline": None,
-            "e2e": None}
+            "gpu_launches": 15 * s.n_batches * args.steps, "clocks": clocks, "cpu_baseline": cpu,
+            "e2e": {"value": s.n * world / (e2e_ms / 1e3), "unit": "fragments/s",
+                    "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}}
 
 
 def cpu_baseline(s, budget_s=20.0, stream_release=False):
@@ -442,14 +553,7 @@ def main():
     import paper_2403_04311_gb300 as alto
 
     torch.cuda.set_device(local_rank)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
-
-    def barrier():
-        if dist is not None:
-            dist.barrier()
+    dist = init_dist(world)
 
     stream = torch.cuda.current_stream()
     if args.max_batches > 0:
@@ -498,7 +602,7 @@ def main():
     # kernel boundary runs as it does without measurement
     sampler = ClockSampler(local_rank)
     agg.profile(alto.PROFILE_HOT)
-    barrier()
+    barrier(dist)
     torch.cuda.synchronize()
     sampler.start()
     t_start = torch.cuda.Event(enable_timing=True)
@@ -508,15 +612,11 @@ def main():
         step()
     t_end.record(stream)
     torch.cuda.synchronize()
-    barrier()
+    barrier(dist)
     clocks = sampler.stop()
     _st, prof = agg.profile_read()
     agg.profile(False)
-    ms = t_start.elapsed_time(t_end)
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(t_start.elapsed_time(t_end), dist)
     ms_per_step = ms / args.steps
     frags_per_step = s.n
     value = frags_per_step * world * args.steps / (ms / 1e3)
@@ -643,7 +743,7 @@ def main():
     e2e_step()
     torch.cuda.synchronize()
     flags["out"] = None
-    barrier()
+    barrier(dist)
     torch.cuda.synchronize()
     e_start = torch.cuda.Event(enable_timing=True)
     e_end = torch.cuda.Event(enable_timing=True)
@@ -656,11 +756,7 @@ def main():
     stream.wait_stream(cs_in)
     e_end.record(stream)
     torch.cuda.synchronize()
-    e_ms = e_start.elapsed_time(e_end)
-    if dist is not None:
-        t = torch.tensor([e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e_ms = float(t.item())
+    e_ms = max_over_ranks(e_start.elapsed_time(e_end), dist)
     e2e_value = frags_per_step * world * e_steps / (e_ms / 1e3)
 
     # ---- per-batch latency: push + drain, host clock -------------------------

@@ -498,6 +498,22 @@ class Router:
                           None if score is None else score[a:b]))
         return replica, perm, parts
 
+    def all_outputs(self, n, n_payload):
+        """Device views of the last routing's whole partition, every replica's
+        batch in turn: tags (D * n, each replica's block level-major), payload
+        offsets (n + R: each replica's n_r + 1), payload (n_payload)."""
+        torch = self._torch
+        r = self.routed
+
+        def view(ptr, count, dtype, esize):
+            if count == 0 or not ptr:
+                return torch.zeros(0, dtype=dtype, device="cuda")
+            return torch.as_tensor(_DevView(ptr, count * esize), device="cuda").view(dtype)
+
+        return (view(r.tags, self.depth * int(n), torch.int64, 8),
+                view(r.payload_off, int(n) + self.R, torch.int32, 4),
+                view(r.payload, int(n_payload), torch.int32, 4))
+
     def release(self, records_ptr, n_records) -> int:
         return load_library().alto_router_release(self._h, ctypes.c_void_p(records_ptr), int(n_records),
                                                   ctypes.c_void_p(self.stream.cuda_stream))
