@@ -105,6 +105,7 @@ struct Scratch {
   u64 bm_cap;
   u32* big_seg;          // [depth][big_cap] segments longer than kBigSeg, per level
   u32 big_cap;
+  u32* rel_seg;          // [n_max] streaming: small leaf segments whose groups release a run
 };
 
 struct Dev {
@@ -417,6 +418,7 @@ __global__ void k_begin(Ctl* ctl, u32 n) {
   ctl->skip_dense = 0;
   ctl->dense_total = ctl->arena_total = ctl->pay_total = ctl->topk_total = ctl->n_emit = 0;
   ctl->bm_used = 0;
+  ctl->n_rel = 0;
   for (int l = 0; l < kMaxDepth; ++l) ctl->n_big[l] = 0;
   for (int l = 0; l < kMaxDepth; ++l) ctl->n_segs[l] = 0;
   ctl->n = (ctl->status == ALTO_OK) ? n : 0u;
@@ -871,6 +873,8 @@ __device__ __forceinline__ void reduce_small(const Dev& d, const Batch& b, Ctl* 
                                              u32 s, u32 j0, u32 j1, u32 gmask, int sub, bool topk, int K) {
   const u32 e = r.skeys[j0] & d.tab.mask;
   const u32 rep0 = LEAF ? min(r.sperm[j0], r.n_items - 1) : r.it_rep[min(r.sperm[j0], r.n_items - 1)];
+  const bool strm = LEAF && d.cfg.stream;
+  const u32 rel = strm ? d.tab.rel[e] : 0u;
   const Chain htag = load_chain(b, r.l, rep0);
   SegRed red;
   red.init();
@@ -883,7 +887,7 @@ __device__ __forceinline__ void reduce_small(const Dev& d, const Batch& b, Ctl* 
     len[q] = 0;
     if (j < j1) {
       const Item it = load_item<LEAF>(d, b, r, j);
-      red.add(it, 0, false);
+      red.add(it, rel, strm);
       if (chain_bad(b, r.l, it.rep, htag)) red.bad = 1;
       len[q] = it.len;
       if (it.done) cand[q] = ((u64)it.sk << 32) | (u64)(~it.c);
@@ -915,6 +919,27 @@ __device__ __forceinline__ void reduce_small(const Dev& d, const Batch& b, Ctl* 
   red.bad = __reduce_or_sync(gmask, red.bad);
 #pragma unroll
   for (int o = 4; o > 0; o >>= 1) red.lsum += __shfl_xor_sync(gmask, red.lsum, o, 8);
+  if (strm) {
+    // a group that stays open and whose first unreleased child came releases
+    // a run: that needs a whole warp, so the segment is left to k_reduce_rel
+    red.hitrel = __reduce_or_sync(gmask, red.hitrel);
+    red.below = __reduce_or_sync(gmask, red.below);
+    if (red.below && sub == 0) raise_err(ctl, ALTO_EDUP);
+    if (red.hitrel) {
+      const u32 lo = d.tab.hot[e].last;
+      const u32 nl = (lo == kNone && red.hasf) ? red.fmin : lo;
+      const bool closes = nl != kNone && d.tab.hot[e].completed + red.cnt == nl + 1 &&
+                          max(d.tab.hot[e].maxc1, red.m1) <= nl + 1;
+      if (!closes) {
+        if (sub == 0) {
+          const u32 q = atomicAdd(&ctl->n_rel, 1u);
+          if (q < d.cfg.n_max) d.sc.rel_seg[q] = s;
+          else raise_err(ctl, ALTO_ENOSPC);
+        }
+        return;
+      }
+    }
+  }
   if (topk) {
     // the group's first lane keeps the list, best first, in local memory
     u64 list[kMaxTopk];
@@ -1006,8 +1031,8 @@ __device__ __forceinline__ void reduce_warp(const Dev& d, const Batch& b, Ctl* c
 // entries, test completion, and emit each group as an item of level l-1.  A
 // warp takes four segments at a time: the small ones by eight lanes each,
 // the others one after another by the whole warp; segments longer than
-// kBigSeg are listed for k_reduce_big.  (A streaming release needs the whole
-// warp, so with it every segment takes the warp path.)
+// kBigSeg are listed for k_reduce_big.  (A small segment whose group makes a
+// streaming release is listed for k_reduce_rel: the release needs a warp.)
 template <bool LEAF>
 __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, const u32* skeys,
                                                      const u32* sperm, const u32* seg_start,
@@ -1030,7 +1055,7 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
       j1 = min(seg_start[s + 1], r.n_items);
       j0 = min(seg_start[s], j1);
     }
-    const bool small = !strm && j1 > j0 && j1 - j0 <= kSmallSeg;
+    const bool small = j1 > j0 && j1 - j0 <= kSmallSeg;
     if (small) reduce_small<LEAF>(d, b, ctl, r, s, j0, j1, gmask, sub, topk, K);
     u32 rest = __ballot_sync(0xFFFFFFFFu, sub == 0 && j1 > j0 && !small);
     while (rest) {
@@ -1048,6 +1073,26 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
       }
       reduce_warp<LEAF>(d, b, ctl, r, s2, a0, a1, topk, K, strm);
     }
+  }
+}
+
+// Streaming release: the small segments whose groups release a run, a warp each.
+__global__ void __launch_bounds__(kThreads) k_reduce_rel(Dev d, Batch b, const u32* skeys, const u32* sperm,
+                                                         const u32* seg_start, int in_set) {
+  pdl_enter();
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  const int l = d.cfg.depth - 1;
+  const u32 nrel = min(ctl->n_rel, d.cfg.n_max);
+  const u32 gw = gtid() >> 5, nw = gstride() >> 5;
+  const bool topk = d.cfg.score_op[l] == ALTO_SCORE_TOPK;
+  const int K = d.cfg.topk_k[l];
+  const ReduceArgs<true> r = reduce_args<true>(d, b, l, skeys, sperm, seg_start, in_set);
+  for (u32 q = gw; q < nrel; q += nw) {
+    const u32 s = d.sc.rel_seg[q];
+    const u32 j1 = min(seg_start[s + 1], r.n_items);
+    const u32 j0 = min(seg_start[s], j1);
+    if (j0 < j1) reduce_warp<true>(d, b, ctl, r, s, j0, j1, topk, K, true);
   }
 }
 
@@ -2638,6 +2683,11 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     launch_pdl(k_reduce_big<true>, p.num_sms, kBigThreads, 0, s, d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
                d.sc.leaf_seg_start, set);
     p.launches += 3;
+    if (d.cfg.stream) {
+      launch_pdl(k_reduce_rel, p.num_sms * blocks_per_sm((const void*)k_reduce_rel), kThreads, 0, s, d, bt,
+                 d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
+      p.launches += 1;
+    }
   } else {
     // leaf level without TOPK: accumulate into the table in arrival order
     // (plain stream order: the measurement hooks time this kernel on its own)
@@ -3017,6 +3067,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     ALLOC(sc.done_part, u32, done_cap);
     ALLOC(sc.leaf_mrank, u32, nmax);
     ALLOC(sc.bm, u32, sc.bm_cap);
+    ALLOC(sc.rel_seg, u32, nmax);
   }
   const u64 scan_tiles = std::max<u64>(std::max<u64>(dense_cap, done_cap), nmax) / kScanTile + 2;
   ALLOC(h->lbs.desc, ulonglong2, 3 * scan_tiles);

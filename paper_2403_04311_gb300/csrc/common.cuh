@@ -56,6 +56,7 @@ struct Ctl {
   u64 chain_arena;         // their buffered child spans
   u64 bm_used;             // streaming release: words of the presence bitmaps handed out
   u32 n_big[kMaxDepth];    // segments of level l longer than a warp's share, for the block reduce
+  u32 n_rel;               // streaming: small leaf segments left to the warp reduce
   u64 scan_total[kSites];  // totals written by scans
 };
 
