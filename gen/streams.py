@@ -395,7 +395,7 @@ def make_adversarial(n_leaves=64 * 2**20, hot_leaves=2**20, seed=5, batch=2 * 2*
             break
         n_roots *= 2
     tg, tc = _trim(counts, n_tail)
-    # the hot chain: its own source/root/... with one leaf-parent of hot_leaves
+    # the hot chain: its own group at every level above, with one leaf parent of hot_leaves
     hot_counts = [np.ones(1, dtype=np.int64)] * 5 + [np.array([hot_leaves], dtype=np.int64)]
     hg, hc = _leaves_of(hot_counts)
     D = 6
