@@ -1,4 +1,4 @@
-"""Full-size parity: every workload at its BASELINE size, through the C ABI,
+"""Full-size parity: every workload at its full published size, through the C ABI,
 with the capacities bench.py uses.
 
 * the oracle runs on a prefix of the stream (about two million fragments) and
