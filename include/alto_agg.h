@@ -58,9 +58,11 @@
  * parent tags, or two different child groups in one slot within one batch
  * (EINCONSIST); two different last children, or a child index above the last
  * (ELAST); table, arena or output capacity exceeded (ENOSPC); a device-side
- * wait that ran past its iteration cap (ETIMEOUT).  Inputs outside that scope
- * (for example a fragment for a group that was already emitted) give
- * undefined records but never a fault or a hang.
+ * wait that ran past its iteration cap (ETIMEOUT).  A full open-group table
+ * and a wait that ran out stop the batch where they happen, so a defect that
+ * would be found later in the same batch is not reported.  Inputs outside
+ * that scope (for example a fragment for a group that was already emitted)
+ * give undefined records but never a fault or a hang.
  */
 #ifndef ALTO_AGG_H
 #define ALTO_AGG_H

@@ -183,8 +183,13 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
     }
     h = (h + 1) & tab.mask;
   }
+  // The table is full: the batch stops here.  The caller gets kNone and
+  // stores entry 0 where an index is needed, so that nothing indexes out of
+  // bounds; the abort keeps every later kernel of the batch from treating
+  // entry 0 as this group (which would report false duplicates).
   raise_err(ctl, ALTO_ENOSPC);
-  return 0;
+  *(volatile int*)&ctl->abort = 1;
+  return kNone;
 }
 
 // Batch-local set of (entry, child) slots; returns true if already present.
@@ -444,7 +449,8 @@ __global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
     u32 e = ht_find_or_insert(d.tab, ((u64)(D - 1) << 32) | tag_pid(t), up, ctl, &ins, b.tags,
                               b.n, i, D - 1);
     if (ins) atomicAdd(&s_ins, 1u);
-    d.sc.leaf_sort_keys0[i] = e;
+    d.sc.leaf_sort_keys0[i] = (e == kNone) ? 0u : e;
+    if (e == kNone) continue;
     // the sorted (TOPK) leaf path checks leaf slots here, spread over the
     // whole grid (in the reduce, a hot group's checks would all fall to the
     // block that reduces its segment); the accumulate does otherwise
@@ -472,7 +478,8 @@ __global__ void __launch_bounds__(kThreads) k_items_lookup(Dev d, Batch b, int l
     int ins = 0;
     u32 e = ht_find_or_insert(d.tab, ((u64)l << 32) | tag_pid(t), up, ctl, &ins, b.tags, b.n, rep, l);
     if (ins) atomicAdd(&s_ins, 1u);
-    d.sc.up_sort_keys0[x] = e;
+    d.sc.up_sort_keys0[x] = (e == kNone) ? 0u : e;
+    if (e == kNone) continue;
     if (ps_insert(d.sc, e, tag_child(t), ep7, ctl)) raise_err(ctl, ALTO_EINCONSIST);
   }
   __syncthreads();
@@ -851,7 +858,7 @@ __device__ void finalize_segment(const Dev& d, const Batch& b, Ctl* ctl, const R
                                     rep0, l - 1);
     if (ins) atomicAdd((unsigned long long*)&ctl->live_groups, 1ull);
     const u64 total = (u64)d.tab.vec_n[2 * (u64)e + 1] + (LEAF ? red.lsum : 0ull);
-    chain_reserve(d.tab, e, P, tag_child(tp), total);
+    if (P != kNone) chain_reserve(d.tab, e, P, tag_child(tp), total);
   }
   if (l > 0) {
     r.nx_rep[s] = rep0;
@@ -1459,7 +1466,8 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
       const u32 e2 = ht_find_or_insert(d.tab, ((u64)(l - 1) << 32) | tag_pid(tp), upp, ctl, &ins,
                                        b.tags, n, rep, l - 1);
       if (ins) atomicAdd(&s_ins, 1u);
-      d.sc.up_sort_keys0[s] = e2;
+      d.sc.up_sort_keys0[s] = (e2 == kNone) ? 0u : e2;
+      if (e2 == kNone) continue;
       if (ps_insert(d.sc, e2, tag_child(tp), ep7, ctl)) raise_err(ctl, ALTO_EINCONSIST);
       if (hands_up && complete)
         chain_reserve(d.tab, e, e2, tag_child(tp), (u64)d.tab.vec_n[2 * (u64)e + 1] + blen);

@@ -144,6 +144,26 @@ def test_output_capacity_is_enospc():
     assert g[0][0] == alto.ENOSPC
 
 
+@pytest.mark.parametrize("leaf", ["accumulate", "topk", "stream_release"])
+def test_full_open_group_table_is_enospc(leaf):
+    """2,001 open groups in one batch and a table of 1,024 slots: the inserts
+    that find no slot end the batch with ENOSPC, and no other class (the
+    unplaced groups must not be taken for one another, which would read as
+    repeated leaf slots), on each leaf form."""
+    frags = tree_fragments([2] * 2000)
+    n_pay = sum(len(f[1]) for f in frags)
+    topk = leaf == "topk"
+    caps = small_caps(len(frags), n_pay, 2)
+    caps.update(max_open_groups=16, stream_release=(leaf == "stream_release"))
+    agg = alto.Aggregator(2, [0, 1], [0, 2 if topk else 0], [0, 2 if topk else 0], **caps)
+    db = alto.to_device(to_batch(frags, 2, topk))
+    assert agg.push(db.tags, db.off, db.payload, db.score if topk else None) == alto.OK
+    d = agg.drain()
+    assert d.status == alto.ENOSPC
+    assert agg.drain().status == alto.ENOSPC      # latched
+    agg.close()
+
+
 def test_host_argument_errors_do_not_poison():
     frags = tree_fragments([2, 1])
     agg = alto.Aggregator(2, [0, 1], [0, 0], None, **small_caps(4, 16, 2))
