@@ -146,42 +146,73 @@ __device__ __forceinline__ u32 warp_take(bool want, u32* counter) {
 // ---------------------------------------------------------------------------
 // open-group hash table (linear probing; a slot index is the entry id)
 // ---------------------------------------------------------------------------
+// Find the entry of `key`, or insert it.  A slot is empty, deleted (a
+// tombstone: its group was emitted) or holds a key.  The walk from the home
+// slot ends at the key or at the first empty slot; a key is new when it has
+// not been met by then, and it takes the first deleted slot of the walk if
+// there was one, else that empty slot.  Taking deleted slots keeps a table
+// sized near the groups open at once from filling with tombstones.
+//
+// Within one launch slots only go from empty or deleted to a key, so every
+// thread inserting the same key aims at the same first free slot unless that
+// slot was taken meanwhile, and then its compare-and-swap fails: the thread
+// walks again from that slot (the slots before it hold other keys for good).
+// No key is ever placed twice, and a walk only grows while other threads take
+// free slots, so it ends.  A key lies within max_probe slots of home; a walk
+// that reaches that distance with no free slot met finds the table full.
 __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, int* inserted,
                                   const u64* tags = nullptr, u64 n = 0, u32 rep = 0, int l = 0) {
-  u32 h = (u32)mix64(key) & tab.mask;
-  for (int p = 0; p < tab.max_probe; ++p) {
-    u64 cur = ((volatile u64*)tab.key)[h];
-    if (cur == key) return h;
-    if (cur == kEmpty) {
-      u64 prev = atomicCAS((unsigned long long*)&tab.key[h], (unsigned long long)kEmpty,
-                           (unsigned long long)key);
-      if (prev == kEmpty) {
-        // the whole record: up, last = none, nothing completed, accumulators zero
-        uint4* hw = reinterpret_cast<uint4*>(tab.hot + h);
-        hw[0] = make_uint4((u32)up, (u32)(up >> 32), kNone, 0);
-        hw[1] = make_uint4(0, 0, 0, 0);
-        hw[2] = make_uint4(kNone, 0, 0, 0);
-        hw[3] = make_uint4(0, 0, 0, 0);
-        if (tab.rel) tab.rel[h] = 0;
-        if (tab.vec_n) {
-          tab.vec_n[2 * (u64)h] = 0;
-          tab.vec_n[2 * (u64)h + 1] = 0;
-        }
-        if (tags) {
-          for (int q = 0; q < l; ++q) tab.chain[(u64)h * tab.chain_len + q] = tags[(u64)q * n + rep];
-        }
-        if (tags && l == tab.leaf_level) {
-          ulonglong2* cb = reinterpret_cast<ulonglong2*>(tab.cbits + 4 * (u64)h);
-          cb[0] = make_ulonglong2(0, 0);
-          cb[1] = make_ulonglong2(0, 0);
-        }
-        *inserted = 1;
-        return h;
+  const u32 home = (u32)mix64(key) & tab.mask;
+  const u32 reach = (u32)tab.max_probe;  // at most the table size
+  u32 h = home, dist = 0;
+  u32 free_at = kNone;  // first deleted slot of the walk
+  for (;;) {
+    if (dist < reach) {
+      const u64 cur = ((volatile u64*)tab.key)[h];
+      if (cur == key) return h;
+      if (cur == kTomb && free_at == kNone) free_at = h;
+      if (cur != kEmpty) {
+        h = (h + 1) & tab.mask;
+        ++dist;
+        continue;
       }
-      if (prev == key) return h;
-      continue;  // another key took the slot: read it again, then move on
+    } else if (free_at == kNone) {
+      break;
     }
-    h = (h + 1) & tab.mask;
+    // the key is not in the table: take the first free slot of the walk
+    const u32 t = (free_at != kNone) ? free_at : h;
+    const u64 want = (free_at != kNone) ? kTomb : kEmpty;
+    const u64 prev = atomicCAS((unsigned long long*)&tab.key[t], (unsigned long long)want,
+                               (unsigned long long)key);
+    if (prev == want) {
+      // the whole record: up, last = none, nothing completed, accumulators zero
+      uint4* hw = reinterpret_cast<uint4*>(tab.hot + t);
+      hw[0] = make_uint4((u32)up, (u32)(up >> 32), kNone, 0);
+      hw[1] = make_uint4(0, 0, 0, 0);
+      hw[2] = make_uint4(kNone, 0, 0, 0);
+      hw[3] = make_uint4(0, 0, 0, 0);
+      if (tab.rel) tab.rel[t] = 0;
+      if (tab.vec_n) {
+        tab.vec_n[2 * (u64)t] = 0;
+        tab.vec_n[2 * (u64)t + 1] = 0;
+      }
+      if (tags) {
+        for (int q = 0; q < l; ++q) tab.chain[(u64)t * tab.chain_len + q] = tags[(u64)q * n + rep];
+      }
+      if (tags && l == tab.leaf_level) {
+        ulonglong2* cb = reinterpret_cast<ulonglong2*>(tab.cbits + 4 * (u64)t);
+        cb[0] = make_ulonglong2(0, 0);
+        cb[1] = make_ulonglong2(0, 0);
+      }
+      *inserted = 1;
+      return t;
+    }
+    if (prev == key) return t;
+    // another key took the slot: walk again from it (its distance from home
+    // is below reach, so the subtraction does not wrap)
+    h = t;
+    dist = (t - home) & tab.mask;
+    free_at = kNone;
   }
   // The table is full: the batch stops here.  The caller gets kNone and
   // stores entry 0 where an index is needed, so that nothing indexes out of
