@@ -93,18 +93,38 @@ __global__ void k_rt_begin(RDev d, u32 n) {
   for (int r = threadIdx.x; r < d.R; r += blockDim.x) d.counts[r] = 0;
 }
 
+// The flow's slot, inserted if new.  A walk from the home slot ends at the
+// key or at the first free slot; a new key takes the first released slot
+// (tombstone) it passed, else that free slot, so that released flows do not
+// fill the table.  Slots only go from free or released to a key within a
+// launch: a lost compare-and-swap means another key took the slot, and the
+// walk goes on from there; a key lies within fprobe slots of home.
 __device__ u32 flow_find_or_insert(const RDev& d, u64 key) {
-  u32 h = (u32)mix64(key) & d.fmask;
-  for (int p = 0; p < d.fprobe; ++p) {
-    const u64 cur = ((volatile u64*)d.fkey)[h];
-    if (cur == key) return h;
-    if (cur == kEmpty) {
-      const u64 prev = atomicCAS((unsigned long long*)&d.fkey[h], (unsigned long long)kEmpty,
-                                 (unsigned long long)key);
-      if (prev == kEmpty || prev == key) return h;
-      continue;  // another key took the slot: read it again
+  const u32 home = (u32)mix64(key) & d.fmask;
+  const u32 reach = (u32)d.fprobe;  // at most the table size
+  u32 h = home, dist = 0;
+  u32 tomb_at = kNone;
+  for (;;) {
+    if (dist < reach) {
+      const u64 cur = ((volatile u64*)d.fkey)[h];
+      if (cur == key) return h;
+      if (cur == kTomb && tomb_at == kNone) tomb_at = h;
+      if (cur != kEmpty) {
+        h = (h + 1) & d.fmask;
+        ++dist;
+        continue;
+      }
+    } else if (tomb_at == kNone) {
+      break;
     }
-    h = (h + 1) & d.fmask;  // occupied by another key, or a released slot
+    const u32 t = (tomb_at != kNone) ? tomb_at : h;
+    const u64 want = (tomb_at != kNone) ? kTomb : kEmpty;
+    const u64 prev = atomicCAS((unsigned long long*)&d.fkey[t], (unsigned long long)want,
+                               (unsigned long long)key);
+    if (prev == want || prev == key) return t;
+    h = t;  // its distance from home is below reach: no wrap
+    dist = (t - home) & d.fmask;
+    tomb_at = kNone;
   }
   raise_err(d.ctl, ALTO_ENOSPC);
   return kNone;

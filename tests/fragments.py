@@ -63,3 +63,37 @@ def tree_fragments(shape, rng=None, depth=None, id_base=100, score_fn=None, tok_
         sc = score_fn(k) if score_fn else float(k % 5) - 2.0
         frags.append((tuple(tags), tok, sc))
     return frags
+
+
+def window_stream(n_groups, n_children, window, batch, seed, topk=False):
+    """Depth 2: one source (level 0) with n_groups leaf-parent groups (level
+    1) of n_children leaves each, children in a random order; at most
+    `window` groups are open at once (a group starts when one ends), the
+    leaves of the open ones interleaved at random."""
+    from gen.streams import Stream
+
+    rng = np.random.default_rng(seed)
+    live, nxt, g_of, c_of = [], 0, [], []
+    while nxt < n_groups or live:
+        while len(live) < window and nxt < n_groups:
+            live.append([nxt, list(rng.permutation(n_children))])
+            nxt += 1
+        k = int(rng.integers(0, len(live)))
+        g_of.append(live[k][0])
+        c_of.append(live[k][1].pop(0))
+        if not live[k][1]:
+            live.pop(k)
+    g = np.asarray(g_of, np.uint64)
+    c = np.asarray(c_of, np.uint64)
+    n = len(g)
+    tags = np.zeros((2, n), np.uint64)
+    tags[0] = (np.uint64(1) << np.uint64(32)) | ((g == n_groups - 1).astype(np.uint64) << np.uint64(31)) | g
+    tags[1] = ((np.uint64(1000) + g) << np.uint64(32)) | ((c == n_children - 1).astype(np.uint64) << np.uint64(31)) | c
+    lens = rng.integers(0, 5, size=n)
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    payload = rng.integers(0, 1 << 30, size=int(off[-1])).astype(np.int32)
+    score = rng.standard_normal(n).astype(np.float32) if topk else None
+    sizes = [batch] * (n // batch) + ([n % batch] if n % batch else [])
+    return Stream(name="window", depth=2, payload_op=(0, 1), score_op=(0, 2 if topk else 0),
+                  topk_k=(0, 3 if topk else 0), tags=tags, off=off, payload=payload, score=score,
+                  batch_sizes=np.asarray(sizes), meta={})

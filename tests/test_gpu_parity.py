@@ -10,7 +10,7 @@ torch = pytest.importorskip("torch")
 
 import oracle
 import paper_2403_04311_gb300 as alto
-from fragments import split, to_batch, tree_fragments
+from fragments import split, to_batch, tree_fragments, window_stream
 from gen import make_stream
 from gpu_harness import (assert_same, run_both_stream, run_gpu_batches, run_oracle_batches,
                          stream_caps)
@@ -164,39 +164,6 @@ def test_full_open_group_table_is_enospc(leaf):
     agg.close()
 
 
-def _window_stream(n_groups, n_children, window, batch, seed, topk=False):
-    """Depth 2: one source (level 0) with n_groups leaf-parent groups (level
-    1) of n_children leaves each, children in a random order; at most
-    `window` groups are open at once (a group starts when one ends), the
-    leaves of the open ones interleaved at random."""
-    from gen.streams import Stream
-    rng = np.random.default_rng(seed)
-    live, nxt, g_of, c_of = [], 0, [], []
-    while nxt < n_groups or live:
-        while len(live) < window and nxt < n_groups:
-            live.append([nxt, list(rng.permutation(n_children))])
-            nxt += 1
-        k = int(rng.integers(0, len(live)))
-        g_of.append(live[k][0])
-        c_of.append(live[k][1].pop(0))
-        if not live[k][1]:
-            live.pop(k)
-    g = np.asarray(g_of, np.uint64)
-    c = np.asarray(c_of, np.uint64)
-    n = len(g)
-    tags = np.zeros((2, n), np.uint64)
-    tags[0] = (np.uint64(1) << np.uint64(32)) | ((g == n_groups - 1).astype(np.uint64) << np.uint64(31)) | g
-    tags[1] = ((np.uint64(1000) + g) << np.uint64(32)) | ((c == n_children - 1).astype(np.uint64) << np.uint64(31)) | c
-    lens = rng.integers(0, 5, size=n)
-    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
-    payload = rng.integers(0, 1 << 30, size=int(off[-1])).astype(np.int32)
-    score = rng.standard_normal(n).astype(np.float32) if topk else None
-    sizes = [batch] * (n // batch) + ([n % batch] if n % batch else [])
-    return Stream(name="window", depth=2, payload_op=(0, 1), score_op=(0, 2 if topk else 0),
-                  topk_k=(0, 3 if topk else 0), tags=tags, off=off, payload=payload, score=score,
-                  batch_sizes=np.asarray(sizes), meta={})
-
-
 @pytest.mark.parametrize("leaf", ["accumulate", "topk", "stream_release"])
 def test_small_table_reuses_deleted_slots(leaf):
     """20,000 groups through a 1,024-slot table, never more than 200 of them
@@ -204,7 +171,7 @@ def test_small_table_reuses_deleted_slots(leaf):
     the slots of emitted groups.  Without that, slots left deleted behind
     live keys fill the table within about fifty batches (ENOSPC); with it,
     every drain matches the oracle bit for bit."""
-    s = _window_stream(20_000, 4, 200, 256, seed=7, topk=(leaf == "topk"))
+    s = window_stream(20_000, 4, 200, 256, seed=7, topk=(leaf == "topk"))
     caps = stream_caps(s)
     caps["max_open_groups"] = 256                 # 1,024 slots
     o, g = run_both_stream(s, drain_every=1, caps=caps, stream_release=(leaf == "stream_release"))

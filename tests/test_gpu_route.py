@@ -14,6 +14,7 @@ torch = pytest.importorskip("torch")
 
 import oracle
 import paper_2403_04311_gb300 as alto
+from fragments import window_stream
 from gen import make_stream
 
 pytestmark = pytest.mark.gpu
@@ -84,17 +85,23 @@ def test_route_errors():
     rt.close()
 
 
-def test_route_release_and_aggregate():
+@pytest.mark.parametrize("stream", ["factcheck", "window"])
+def test_route_release_and_aggregate(stream):
     """Route at level 1 into R GPU aggregators, release completed flows from
     their device records, and compare with the oracle router + one oracle
     aggregator: replicas match batch by batch, and every group at level >= 1
-    gets the record the whole stream gives."""
-    s = make_stream("factcheck", small=True)
+    gets the record the whole stream gives.  "window" sends 20,000 flows, at
+    most 200 of them live at once, through a flow table of 1,024 slots: new
+    flows must take the slots of released ones."""
+    if stream == "window":
+        s, max_flows = window_stream(20_000, 4, 200, 256, seed=7), 256
+    else:
+        s, max_flows = make_stream("factcheck", small=True), 0
     L, R = 1, 4
     bsz = int(max(s.batch_sizes))
     pay = int(max(s.off[b1] - s.off[b0] for b0, b1 in zip(s.batch_starts()[:-1], s.batch_starts()[1:])))
     rt = alto.Router(s.depth, L, R, alto.ROUTE_LEAST_LOADED, max_batch_fragments=bsz, max_batch_payload=pay,
-                     with_score=True)
+                     max_flows=max_flows, with_score=s.score is not None)
     ro = oracle.RouterOracle(s.depth, L, R, oracle.LEAST_LOADED)
     from gpu_harness import stream_caps
     caps = stream_caps(s)
