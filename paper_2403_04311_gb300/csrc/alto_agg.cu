@@ -2551,7 +2551,8 @@ struct alto_agg {
   LookbackState lbs;
   Ctl* h_ctl;  // pinned host copy for drain
   std::vector<void*> blocks;
-  u64 pushed;
+  u64 pushed;    // batches pushed, empty ones included
+  u64 launched;  // batches that launched work (the device's batch epochs)
   u64 drain_first;
   int latched;
   // measurement hooks
@@ -2945,6 +2946,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   h->use_async = (alloc == nullptr);
   if (alloc) h->alloc = *alloc;
   h->pushed = 0;
+  h->launched = 0;
   h->drain_first = 0;
   h->latched = ALTO_OK;
   h->profiling = false;
@@ -3167,8 +3169,16 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
   bt.score = h->d.cfg.has_score ? b->score : nullptr;
   bt.n = n;
   bt.n_payload = (u64)b->n_payload;
-  if (h->pushed % 127 == 0 && h->pushed > 0)
+  if (n == 0) {
+    // nothing arrives: no group changes, nothing completes or is released
+    h->pushed += 1;
+    return ALTO_OK;
+  }
+  // the pair set's keys carry a 7-bit batch epoch (the device counts batches
+  // that launch work): clear it before an epoch value comes round again
+  if (h->launched % 127 == 0 && h->launched > 0)
     cudaMemsetAsync(d.sc.pairset, 0, sizeof(u64) * (d.sc.ps_mask + 1), s);
+  h->launched += 1;
   h->pushed += 1;
   h->last_stream = s;
   if (h->profiling) h->prof_pushes += 1;

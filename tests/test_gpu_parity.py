@@ -179,6 +179,32 @@ def test_small_table_reuses_deleted_slots(leaf):
     assert_same(o, g, f"window/{leaf}")
 
 
+def _empty_batch(s):
+    return dict(n=0, seq_base=0, tags=np.zeros((s.depth, 0), np.uint64), off=np.zeros(1, np.uint32),
+                payload=np.zeros(0, np.int32), score=None if s.score is None else np.zeros(0, np.float32))
+
+
+@pytest.mark.parametrize("name,stream_release", [("factcheck", False), ("throughput", False),
+                                                 ("throughput", True)])
+def test_empty_batches_are_no_ops(name, stream_release):
+    """An empty batch before, between and after the stream's batches, and a
+    drain after nothing but empty pushes: every drain equals the oracle's,
+    which is given the same empty batches (no group changes, nothing is
+    emitted or released)."""
+    s = make_stream(name, small=True)
+    batches = [_empty_batch(s), _empty_batch(s)]
+    for b in range(s.n_batches):
+        batches += [s.batch(b), _empty_batch(s)]
+    caps = stream_caps(s, stream_release=stream_release)
+    if stream_release:
+        caps["stream_release"] = True
+    _, g = run_gpu_batches(s.depth, s.payload_op, s.score_op, s.topk_k, batches, caps)
+    o = run_oracle_batches(s.depth, s.payload_op, s.score_op, s.topk_k, batches, stream_release=stream_release)
+    assert all(d.status == 0 for d in o)
+    assert_same(o, g, f"{name} with empty batches")
+    assert len(g[0][1]) == 0 and len(g[1][1]) == 0
+
+
 def test_host_argument_errors_do_not_poison():
     frags = tree_fragments([2, 1])
     agg = alto.Aggregator(2, [0, 1], [0, 0], None, **small_caps(4, 16, 2))
