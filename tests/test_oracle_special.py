@@ -149,3 +149,36 @@ def test_invariants_on_workloads(name):
                 assert np.array_equal(got, want)
                 total += int(r["payload_len"])
         assert total == s.payload.size
+
+
+def _empty(s):
+    return dict(n=0, seq_base=0, tags=np.zeros((s.depth, 0), np.uint64), off=np.zeros(1, np.uint32),
+                payload=np.zeros(0, np.int32), score=None if s.score is None else np.zeros(0, np.float32))
+
+
+@pytest.mark.parametrize("name", ["tiny", "factcheck", "throughput", "adversarial", "tot"])
+@pytest.mark.parametrize("stream_release", [False, True])
+def test_empty_batches_change_nothing(name, stream_release):
+    """An empty batch brings no fragment, so no group changes (Sec. 3.1: only
+    a delimiter closes a stream): with empty batches before, between and
+    after the stream's batches, the drains after the empty ones hold
+    nothing and the others equal the run without them."""
+    s = make_stream(name, small=True)
+    plain = oracle.Oracle.for_stream(s, stream_release=stream_release)
+    mixed = oracle.Oracle.for_stream(s, stream_release=stream_release)
+    mixed.push_batch(_empty(s))
+    assert len(mixed.drain().records) == 0
+    for b in range(s.n_batches):
+        bt = s.batch(b)
+        plain.push_batch(bt)
+        mixed.push_batch(bt)
+        mixed.push_batch(_empty(s))
+        want, got = plain.drain(), mixed.drain()
+        assert got.status == want.status == 0
+        assert np.array_equal(got.records.view(np.uint8), want.records.view(np.uint8)), b
+        assert np.array_equal(got.payload, want.payload), b
+        assert np.array_equal(got.topk.view(np.uint8), want.topk.view(np.uint8)), b
+        mixed.push_batch(_empty(s))
+        assert len(mixed.drain().records) == 0
+    plain.close()
+    mixed.close()
