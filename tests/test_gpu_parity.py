@@ -205,6 +205,65 @@ def test_empty_batches_are_no_ops(name, stream_release):
     assert len(g[0][1]) == 0 and len(g[1][1]) == 0
 
 
+def _deep_forest(seed, n_roots=4, depth=8):
+    """Random trees of the largest depth, fanout 1-2 per level and 1-40
+    leaves per leaf parent, with each level's parent ids remapped to the
+    top of the u32 range (the first group met at a level gets 0xFFFFFFFF)."""
+    rng = np.random.default_rng(seed)
+
+    def shape(d):
+        if d == 1:
+            return int(rng.integers(1, 41))
+        return [shape(d - 1) for _ in range(int(rng.integers(1, 3)))]
+
+    frags = []
+    for r in range(n_roots):
+        frags += tree_fragments(shape(depth), id_base=100_000 * (r + 1),
+                                score_fn=lambda k: float(rng.standard_normal()),
+                                tok_fn=lambda k: [int(x) for x in rng.integers(0, 50257, int(rng.integers(0, 5)))])
+    remap = [{} for _ in range(depth)]
+    out = []
+    for tags, tok, sc in frags:
+        nt = []
+        for l, (p_, c, last) in enumerate(tags):
+            m = remap[l].setdefault(p_, 0xFFFFFFFF - len(remap[l]))
+            nt.append((m, c, last))
+        out.append((tuple(nt), tok, sc))
+    order = rng.permutation(len(out))
+    out = [out[i] for i in order]
+    cuts = sorted(rng.choice(np.arange(1, len(out)), size=4, replace=False).tolist())
+    sizes = [b - a for a, b in zip([0] + cuts, cuts + [len(out)])]
+    return out, sizes
+
+
+@pytest.mark.parametrize("ops", [
+    # CONCAT at the leaf parent, TOPK(32) over its level's groups, MAX above
+    dict(payload_op=[0, 0, 0, 0, 0, 0, 0, 1], score_op=[0, 0, 1, 0, 0, 0, 2, 0],
+         topk_k=[0, 0, 0, 0, 0, 0, 32, 0]),
+    # CONCAT four levels above the leaf parent, TOPK(32) over leaves, MAX at the root
+    dict(payload_op=[0, 0, 0, 1, 0, 0, 0, 0], score_op=[1, 0, 0, 0, 0, 0, 0, 2],
+         topk_k=[0, 0, 0, 0, 0, 0, 0, 32]),
+])
+@pytest.mark.parametrize("seed", [1, 2])
+def test_depth8_top_ids_and_k32(ops, seed):
+    """The largest depth (8 tags), parent ids at the top of the u32 range
+    (0xFFFFFFFF included) and the largest k (32, above and below the child
+    counts), in five batches of a random arrival order, bit for bit against
+    the oracle."""
+    D = 8
+    frags, sizes = _deep_forest(seed, depth=D)
+    batches = [to_batch(part, D, True) for part in split(frags, sizes)]
+    n_pay = max(int(b["off"][-1]) for b in batches)
+    caps = small_caps(max(sizes), n_pay, D)
+    caps.update(arena_elems=1 << 22, out_records=1 << 14, out_payload_elems=1 << 16, out_topk=1 << 16,
+                max_emit_children=1 << 14)
+    _, g = run_gpu_batches(D, ops["payload_op"], ops["score_op"], ops["topk_k"], batches, caps)
+    o = run_oracle_batches(D, ops["payload_op"], ops["score_op"], ops["topk_k"], batches)
+    assert all(d.status == 0 for d in o)
+    assert sum(len(d.records) for d in o) > 100
+    assert_same(o, g, f"depth 8 seed {seed}")
+
+
 def test_host_argument_errors_do_not_poison():
     frags = tree_fragments([2, 1])
     agg = alto.Aggregator(2, [0, 1], [0, 0], None, **small_caps(4, 16, 2))
