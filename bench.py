@@ -525,6 +525,8 @@ def main():
     ap.add_argument("--latency-batches", type=int, default=16)
     ap.add_argument("--profile-steps", type=int, default=2,
                     help="steps of the separate stage-breakdown pass")
+    ap.add_argument("--max-open-groups", type=int, default=0,
+                    help="open-group table capacity (default: every group of the stream)")
     ap.add_argument("--max-batches", type=int, default=0,
                     help="profiling only: push just the first B batches per step")
     args = ap.parse_args()
@@ -569,6 +571,8 @@ def main():
         caps = stream_caps(s_caps, args.stream_release)
     else:
         caps = stream_caps(s, args.stream_release)
+    if args.max_open_groups > 0:
+        caps["max_open_groups"] = args.max_open_groups
     agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, stream=stream, **caps)
     nb = s.n_batches if args.max_batches <= 0 else min(args.max_batches, s.n_batches)
     batches = [alto.to_device(s.batch(b)) for b in range(nb)]
@@ -787,7 +791,8 @@ def main():
                    "batch": int(s.batch_sizes[0]), "payload_tokens": int(s.payload.size),
                    "span_fraction": s.meta.get("span_fraction"),
                    "l2": "inputs larger than L2 (no flush)", "parallelism": f"replicas x{world}",
-                   "stream_release": bool(args.stream_release)},
+                   "stream_release": bool(args.stream_release),
+                   "max_open_groups": int(caps["max_open_groups"])},
         "payload_gbps": payload_bytes * world * args.steps / (ms / 1e3) / 1e9,
         "algorithmic_gbps": alg_bytes * world * args.steps / (ms / 1e3) / 1e9,
         "hbm_frac_path": alg_bytes * args.steps / (ms / 1e3) / 1e9 / hbm_gbs,
