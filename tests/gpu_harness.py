@@ -8,6 +8,13 @@ import oracle
 import paper_2403_04311_gb300 as alto
 
 
+def small_caps(n, payload, depth, k=8):
+    """Capacities for hand-built streams of a few thousand fragments."""
+    return dict(max_batch_fragments=max(n, 1), max_batch_payload=max(payload, 1),
+                max_open_groups=4096, arena_elems=1 << 16, out_records=4096,
+                out_payload_elems=1 << 14, out_topk=4096, max_emit_children=4096)
+
+
 def stream_caps(s, arena_factor=4, stream_release=False):
     """Capacities that hold a whole generated stream (with streaming release,
     every fragment may also bring one partial record)."""
@@ -87,3 +94,53 @@ def run_both_stream(s, drain_every=1, caps=None, stream_release=False):
     _, g = run_gpu_batches(s.depth, s.payload_op, s.score_op, s.topk_k, batches, caps, da)
     o = run_oracle_batches(s.depth, s.payload_op, s.score_op, s.topk_k, batches, da, stream_release)
     return o, g
+
+
+def route_release_and_aggregate(s, L=1, R=4, max_flows=0):
+    """Route stream s at level L into R GPU aggregators, release completed
+    flows from the aggregators' device records, and check it against the
+    oracle router and one oracle aggregator over the whole stream: replicas
+    match batch by batch, and every group at level >= L gets the record the
+    whole stream gives it (Sec. 4.3)."""
+    bsz = int(max(s.batch_sizes))
+    pay = int(max(s.off[b1] - s.off[b0] for b0, b1 in zip(s.batch_starts()[:-1], s.batch_starts()[1:])))
+    rt = alto.Router(s.depth, L, R, alto.ROUTE_LEAST_LOADED, max_batch_fragments=bsz, max_batch_payload=pay,
+                     max_flows=max_flows, with_score=s.score is not None)
+    ro = oracle.RouterOracle(s.depth, L, R, oracle.LEAST_LOADED)
+    caps = stream_caps(s)
+    aggs = [alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, **caps) for _ in range(R)]
+    whole = oracle.run_stream(s, drain_every=1)
+    want = {}
+    for d in whole:
+        for r in d.records:
+            if int(r["level"]) >= L:
+                want[(int(r["level"]), int(r["parent_id"]))] = (
+                    int(r["n_children"]), d.payload[int(r["payload_off"]):int(r["payload_off"]) + int(r["payload_len"])].tolist())
+    got = {}
+    for b in range(s.n_batches):
+        bt = s.batch(b)
+        db = alto.to_device(bt)
+        assert rt.route(db.tags, db.off, db.payload, db.score) == alto.OK
+        st, fo, po = rt.counts()
+        assert st == alto.OK
+        replica, _, _, _ = ro.route(bt)
+        rep_d, _, parts = rt.outputs(fo, po)
+        assert np.array_equal(rep_d.cpu().numpy(), replica)
+        for r in range(R):
+            t, o, p, sc = parts[r]
+            if t.shape[1]:
+                assert aggs[r].push(t.contiguous(), o, p, sc) == alto.OK
+            d = aggs[r].drain()
+            assert d.status == alto.OK
+            rec, payl, _ = d.host()
+            if len(rec):
+                assert rt.release(d.records.data_ptr(), len(rec)) == alto.OK
+            ro.release(rec)
+            for x in rec:
+                if int(x["level"]) >= L:
+                    got[(int(x["level"]), int(x["parent_id"]))] = (
+                        int(x["n_children"]), payl[int(x["payload_off"]):int(x["payload_off"]) + int(x["payload_len"])].tolist())
+    for a in aggs:
+        a.close()
+    rt.close()
+    assert got == want

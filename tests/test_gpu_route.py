@@ -14,8 +14,8 @@ torch = pytest.importorskip("torch")
 
 import oracle
 import paper_2403_04311_gb300 as alto
-from fragments import window_stream
 from gen import make_stream
+from gpu_harness import route_release_and_aggregate
 
 pytestmark = pytest.mark.gpu
 
@@ -85,62 +85,12 @@ def test_route_errors():
     rt.close()
 
 
-@pytest.mark.parametrize("stream", ["factcheck", "window"])
-def test_route_release_and_aggregate(stream):
+def test_route_release_and_aggregate():
     """Route at level 1 into R GPU aggregators, release completed flows from
     their device records, and compare with the oracle router + one oracle
     aggregator: replicas match batch by batch, and every group at level >= 1
-    gets the record the whole stream gives.  "window" sends 20,000 flows, at
-    most 200 of them live at once, through a flow table of 1,024 slots: new
-    flows must take the slots of released ones."""
-    if stream == "window":
-        s, max_flows = window_stream(20_000, 4, 200, 256, seed=7), 256
-    else:
-        s, max_flows = make_stream("factcheck", small=True), 0
-    L, R = 1, 4
-    bsz = int(max(s.batch_sizes))
-    pay = int(max(s.off[b1] - s.off[b0] for b0, b1 in zip(s.batch_starts()[:-1], s.batch_starts()[1:])))
-    rt = alto.Router(s.depth, L, R, alto.ROUTE_LEAST_LOADED, max_batch_fragments=bsz, max_batch_payload=pay,
-                     max_flows=max_flows, with_score=s.score is not None)
-    ro = oracle.RouterOracle(s.depth, L, R, oracle.LEAST_LOADED)
-    from gpu_harness import stream_caps
-    caps = stream_caps(s)
-    aggs = [alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, **caps) for _ in range(R)]
-    whole = oracle.run_stream(s, drain_every=1)
-    want = {}
-    for d in whole:
-        for r in d.records:
-            if int(r["level"]) >= L:
-                want[(int(r["level"]), int(r["parent_id"]))] = (
-                    int(r["n_children"]), d.payload[int(r["payload_off"]):int(r["payload_off"]) + int(r["payload_len"])].tolist())
-    got = {}
-    for b in range(s.n_batches):
-        bt = s.batch(b)
-        db = alto.to_device(bt)
-        assert rt.route(db.tags, db.off, db.payload, db.score) == alto.OK
-        st, fo, po = rt.counts()
-        assert st == alto.OK
-        replica, _, _, oparts = ro.route(bt)
-        rep_d, _, parts = rt.outputs(fo, po)
-        assert np.array_equal(rep_d.cpu().numpy(), replica)
-        for r in range(R):
-            t, o, p, sc = parts[r]
-            if t.shape[1]:
-                assert aggs[r].push(t.contiguous(), o, p, sc) == alto.OK
-            d = aggs[r].drain()
-            assert d.status == alto.OK
-            rec, payl, _ = d.host()
-            if len(rec):
-                assert rt.release(d.records.data_ptr(), len(rec)) == alto.OK
-            ro.release(rec)
-            for x in rec:
-                if int(x["level"]) >= L:
-                    got[(int(x["level"]), int(x["parent_id"]))] = (
-                        int(x["n_children"]), payl[int(x["payload_off"]):int(x["payload_off"]) + int(x["payload_len"])].tolist())
-    for a in aggs:
-        a.close()
-    rt.close()
-    assert got == want
+    gets the record the whole stream gives."""
+    route_release_and_aggregate(make_stream("factcheck", small=True))
 
 
 @pytest.mark.slow
