@@ -110,6 +110,14 @@ typedef int alto_status;
 #define ALTO_FLAG_STREAM_RELEASE 1
 #define ALTO_OPS_PARTIAL 0x80
 
+/* Two output rings (flags bit 1): pushes fill one ring while the records,
+ * payload and top-k pairs of the previous drain stay in the other, and every
+ * drain swaps them.  What a drain returns then stays valid through the next
+ * drain, until the first push after it (or destroy), instead of until the
+ * next push, so the caller can copy it out while later pushes run.  Takes
+ * twice the output capacities' memory.  EINVAL for alto_agg_oneshot_noalloc. */
+#define ALTO_FLAG_DOUBLE_RING 2
+
 /* Aggregator configuration (Sec. 5: the controller is told which queues are
  * pmap entry/exit points and which data is aggregated; here: the nesting
  * depth and what each level's exit computes).  Zero capacities take the
@@ -181,7 +189,9 @@ typedef struct alto_topk_pair {
 } alto_topk_pair;
 
 /* Everything completed since the previous drain.  All pointers are device
- * memory owned by the handle, valid until the next push, drain or destroy. */
+ * memory owned by the handle, valid until the next push, drain or destroy
+ * (with ALTO_FLAG_DOUBLE_RING: through the next drain, until the first push
+ * after it, or destroy). */
 typedef struct alto_drain {
   int64_t n_records;
   const alto_record* records;

@@ -6,7 +6,7 @@ it in-tree and binds it with ctypes.  There is no CPU implementation here.
 """
 from ._binding import (  # noqa: F401
     EXPORTS, OK, EINVAL, ENOMEM, ENOSPC, EDUP, ELAST, EINCONSIST, ECLOSED, ETIMEOUT, ECUDA,
-    STATUS_NAMES, PAYLOAD_NONE, PAYLOAD_CONCAT, SCORE_NONE, SCORE_MAX, SCORE_TOPK, FLAG_STREAM_RELEASE, OPS_PARTIAL,
+    STATUS_NAMES, PAYLOAD_NONE, PAYLOAD_CONCAT, SCORE_NONE, SCORE_MAX, SCORE_TOPK, FLAG_STREAM_RELEASE, FLAG_DOUBLE_RING, OPS_PARTIAL,
     RECORD_DTYPE, PAIR_DTYPE, Aggregator, Drain, alto_agg_config, alto_allocator, alto_batch,
     alto_drain, alto_agg_create, alto_agg_push_batch, alto_agg_drain, alto_agg_stats,
     alto_agg_destroy, alto_agg_profile, alto_agg_profile_read, alto_agg_oneshot_noalloc,

@@ -2555,6 +2555,12 @@ struct alto_agg {
   u64 launched;  // batches that launched work (the device's batch epochs)
   u64 drain_first;
   int latched;
+  // output rings: [1] is allocated only with ALTO_FLAG_DOUBLE_RING; pushes
+  // write ring [ring_cur], and a drain hands it out and moves to the other
+  alto_record* ring_rec[2];
+  int32_t* ring_pay[2];
+  alto_topk_pair* ring_topk[2];
+  int ring_cur;
   // measurement hooks
   bool profiling;
   int profile_mode;  // ALTO_PROFILE_STAGES or ALTO_PROFILE_HOT
@@ -2905,7 +2911,7 @@ alto_status validate(const alto_agg_config* c) {
       return ALTO_EINVAL;
   }
   if (nconcat > 1) return ALTO_EINVAL;
-  if (c->flags & ~(int64_t)ALTO_FLAG_STREAM_RELEASE) return ALTO_EINVAL;
+  if (c->flags & ~(int64_t)(ALTO_FLAG_STREAM_RELEASE | ALTO_FLAG_DOUBLE_RING)) return ALTO_EINVAL;
   // streaming release needs the CONCAT level at the leaf parent
   if ((c->flags & ALTO_FLAG_STREAM_RELEASE) && c->payload_op[c->depth - 1] != ALTO_PAYLOAD_CONCAT)
     return ALTO_EINVAL;
@@ -3113,9 +3119,21 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   const u64 scan_tiles = std::max<u64>(std::max<u64>(dense_cap, done_cap), nmax) / kScanTile + 2;
   ALLOC(h->lbs.desc, ulonglong2, 3 * scan_tiles);
   h->lbs.tiles = scan_tiles;
-  ALLOC(d.out_rec, alto_record, std::max<int64_t>(cfg.out_records, 1));
-  ALLOC(d.out_pay, int32_t, std::max<int64_t>(cfg.out_payload_elems, 1));
-  ALLOC(d.out_topk, alto_topk_pair, std::max<int64_t>(cfg.out_topk, 1));
+  const int rings = (cfg.flags & ALTO_FLAG_DOUBLE_RING) ? 2 : 1;
+  for (int r = 0; r < 2; ++r) {
+    h->ring_rec[r] = nullptr;
+    h->ring_pay[r] = nullptr;
+    h->ring_topk[r] = nullptr;
+  }
+  for (int r = 0; r < rings; ++r) {
+    ALLOC(h->ring_rec[r], alto_record, std::max<int64_t>(cfg.out_records, 1));
+    ALLOC(h->ring_pay[r], int32_t, std::max<int64_t>(cfg.out_payload_elems, 1));
+    ALLOC(h->ring_topk[r], alto_topk_pair, std::max<int64_t>(cfg.out_topk, 1));
+  }
+  h->ring_cur = 0;
+  d.out_rec = h->ring_rec[0];
+  d.out_pay = h->ring_pay[0];
+  d.out_topk = h->ring_topk[0];
 #undef ALLOC
   if (ok && cudaMallocHost((void**)&h->h_ctl, sizeof(Ctl)) != cudaSuccess) {
     h->h_ctl = nullptr;
@@ -3241,6 +3259,13 @@ alto_status alto_agg_drain(alto_agg_t* h, void* stream, alto_drain* out) {
   out->payload = h->d.out_pay;
   out->n_topk = (int64_t)c.topk_count;
   out->topk = h->d.out_topk;
+  if (h->ring_rec[1] != nullptr) {
+    // later pushes fill the other ring while the caller reads this one
+    h->ring_cur ^= 1;
+    h->d.out_rec = h->ring_rec[h->ring_cur];
+    h->d.out_pay = h->ring_pay[h->ring_cur];
+    h->d.out_topk = h->ring_topk[h->ring_cur];
+  }
   launch_pdl(k_drain_reset, 1, 1, 0, s, h->d.ctl);
   if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
   return ALTO_OK;

@@ -60,7 +60,7 @@ def _cfg(**kw):
     dict(arena_elems=1 << 32),
     dict(payload_op=[1, 0], stream_release=True),    # streaming release above the leaf parent
     dict(payload_op=[0, 0], stream_release=True),    # streaming release without CONCAT
-    dict(flags=2),                                   # unknown flag
+    dict(flags=4),                                   # unknown flag
 ])
 def test_create_rejects_bad_configs_on_host(bad):
     lib = alto.load_library()
@@ -75,9 +75,11 @@ def test_create_rejects_bad_configs_on_host(bad):
     assert h.value == 12345  # untouched
 
 
-def test_noalloc_refuses_stream_release_on_host():
-    """One batch has nothing to release in a stream: refused before any device work."""
-    cfg = _cfg(stream_release=True)
+@pytest.mark.parametrize("flag", ["stream_release", "double_ring"])
+def test_noalloc_refuses_handle_flags_on_host(flag):
+    """One batch has nothing to release in a stream and writes the caller's
+    buffers, not rings: both flags are refused before any device work."""
+    cfg = _cfg(**{flag: True})
     b = alto.alto_batch()
     b.depth = 2
     counts = (ctypes.c_int64 * 4)()

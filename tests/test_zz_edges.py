@@ -120,3 +120,43 @@ def test_route_small_flow_table_reuses_released_slots():
     slots, routed into four GPU aggregators and released from their records:
     new flows must take the slots of released ones."""
     route_release_and_aggregate(window_stream(20_000, 4, 200, 256, seed=7), max_flows=256)
+
+
+@pytest.mark.parametrize("name,stream_release", [("factcheck", False), ("throughput", True)])
+def test_double_ring_keeps_a_drain_through_the_next(name, stream_release):
+    """With two output rings, what a drain returns stays intact through the
+    next push and drain: each drain's records, payload and top-k pairs, read
+    back only after the following push and drain, equal the oracle's."""
+    import oracle
+    import paper_2403_04311_gb300 as alto
+
+    s = make_stream(name, small=True)
+    caps = stream_caps(s, stream_release=stream_release)
+    caps.update(double_ring=True, stream_release=stream_release)
+    agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, **caps)
+    o = oracle.Oracle.for_stream(s, stream_release=stream_release)
+
+    def check(pending, b):
+        d, od = pending
+        rec, pay, tk = d.host()
+        assert np.array_equal(rec.view(np.uint8), od.records.view(np.uint8)), b
+        assert np.array_equal(pay, od.payload), b
+        assert np.array_equal(tk.view(np.uint8), od.topk.view(np.uint8)), b
+
+    pending, n_rec = None, 0
+    for b in range(s.n_batches):
+        bt = s.batch(b)
+        db = alto.to_device(bt)
+        assert agg.push(db.tags, db.off, db.payload, db.score) == alto.OK
+        d = agg.drain()
+        assert d.status == alto.OK
+        o.push_batch(bt)
+        od = o.drain()
+        n_rec += len(od.records)
+        if pending is not None:
+            check(pending, b - 1)
+        pending = (d, od)
+    check(pending, s.n_batches - 1)
+    agg.close()
+    o.close()
+    assert s.n_batches > 2 and n_rec > 0
