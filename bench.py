@@ -525,6 +525,8 @@ def main():
     ap.add_argument("--latency-batches", type=int, default=16)
     ap.add_argument("--profile-steps", type=int, default=2,
                     help="steps of the separate stage-breakdown pass")
+    ap.add_argument("--double-ring", action="store_true",
+                    help="two output rings: the end-to-end pushes run under the previous read-back")
     ap.add_argument("--max-open-groups", type=int, default=0,
                     help="open-group table capacity (default: every group of the stream)")
     ap.add_argument("--max-batches", type=int, default=0,
@@ -573,6 +575,8 @@ def main():
         caps = stream_caps(s, args.stream_release)
     if args.max_open_groups > 0:
         caps["max_open_groups"] = args.max_open_groups
+    if args.double_ring:
+        caps["double_ring"] = True
     agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, stream=stream, **caps)
     nb = s.n_batches if args.max_batches <= 0 else min(args.max_batches, s.n_batches)
     batches = [alto.to_device(s.batch(b)) for b in range(nb)]
@@ -706,11 +710,13 @@ def main():
     # Copies overlap the pushes as a user of the API would run them: every
     # batch's inputs go up on a copy stream and its push waits for them only;
     # the step's records and payload come back on a second copy stream, while
-    # the next step's inputs go up.  The next step's pushes reuse the output
-    # ring (reset by the drain), so they wait for that read-back.
+    # the next step's inputs go up.  A step's pushes refill the output ring
+    # that an earlier step's read-back copies from, so they wait for it: the
+    # previous step's with one ring, the one before with two.
     cs_in = torch.cuda.Stream()
     cs_out = torch.cuda.Stream()
-    flags = {"out": None}
+    out_events = []
+    ring_lag = 2 if args.double_ring else 1
 
     def e2e_step():
         cs_in.wait_stream(stream)  # the device batch buffers are free once the previous pushes ran
@@ -725,8 +731,8 @@ def main():
                 ev = torch.cuda.Event()
                 ev.record(cs_in)
                 ready.append(ev)
-        if flags["out"] is not None:
-            stream.wait_event(flags["out"])
+        if len(out_events) >= ring_lag:
+            stream.wait_event(out_events[-ring_lag])
         for db, ev in zip(dev, ready):
             stream.wait_event(ev)
             st = agg.push(db.tags, db.off, db.payload, db.score)
@@ -741,12 +747,12 @@ def main():
             pay_host[:npay].copy_(d.payload, non_blocking=True)
             ev = torch.cuda.Event()
             ev.record(cs_out)
-        flags["out"] = ev
+        out_events.append(ev)
         return nr + npay * 4
 
     e2e_step()
     torch.cuda.synchronize()
-    flags["out"] = None
+    out_events.clear()
     barrier(dist)
     torch.cuda.synchronize()
     e_start = torch.cuda.Event(enable_timing=True)
@@ -792,7 +798,8 @@ def main():
                    "span_fraction": s.meta.get("span_fraction"),
                    "l2": "inputs larger than L2 (no flush)", "parallelism": f"replicas x{world}",
                    "stream_release": bool(args.stream_release),
-                   "max_open_groups": int(caps["max_open_groups"])},
+                   "max_open_groups": int(caps["max_open_groups"]),
+                   "double_ring": bool(args.double_ring)},
         "payload_gbps": payload_bytes * world * args.steps / (ms / 1e3) / 1e9,
         "algorithmic_gbps": alg_bytes * world * args.steps / (ms / 1e3) / 1e9,
         "hbm_frac_path": alg_bytes * args.steps / (ms / 1e3) / 1e9 / hbm_gbs,
