@@ -144,3 +144,34 @@ def route_release_and_aggregate(s, L=1, R=4, max_flows=0):
         a.close()
     rt.close()
     assert got == want
+
+
+def route_stream_vs_oracle(s, level, R, policy, batches=None, max_flows=0):
+    """Route the batches of stream s and compare, batch by batch, each
+    fragment's replica, the stable partition, the replica offsets and every
+    replica's sub-batch with the routing oracle's."""
+    bsz = int(max(s.batch_sizes))
+    pay = max(int(s.off[st1] - s.off[st0]) for st0, st1 in zip(s.batch_starts()[:-1], s.batch_starts()[1:]))
+    rt = alto.Router(s.depth, level, R, policy, max_batch_fragments=bsz, max_batch_payload=max(pay, 1),
+                     max_flows=max_flows, with_score=s.score is not None)
+    ro = oracle.RouterOracle(s.depth, level, R, policy)
+    for b in (range(s.n_batches) if batches is None else batches):
+        bt = s.batch(b)
+        db = alto.to_device(bt)
+        assert rt.route(db.tags, db.off, db.payload, db.score) == alto.OK
+        st, fo, po = rt.counts()
+        assert st == alto.OK
+        replica, perm, counts, parts = ro.route(bt)
+        assert np.array_equal(fo, counts)
+        rep_d, perm_d, parts_d = rt.outputs(fo, po)
+        assert np.array_equal(rep_d.cpu().numpy(), replica)
+        assert np.array_equal(perm_d.cpu().numpy(), perm)
+        for r in range(R):
+            t, o, p, sc = parts_d[r]
+            want = parts[r]
+            assert np.array_equal(t.cpu().numpy().view(np.uint64), want["tags"]), (b, r)
+            assert np.array_equal(o.cpu().numpy().astype(np.int64), want["off"]), (b, r)
+            assert np.array_equal(p.cpu().numpy(), want["payload"]), (b, r)
+            if want["score"] is not None:
+                assert np.array_equal(sc.cpu().numpy().view(np.uint32), want["score"].view(np.uint32))
+    rt.close()

@@ -15,49 +15,21 @@ torch = pytest.importorskip("torch")
 import oracle
 import paper_2403_04311_gb300 as alto
 from gen import make_stream
-from gpu_harness import route_release_and_aggregate
+from gpu_harness import route_release_and_aggregate, route_stream_vs_oracle
 
 pytestmark = pytest.mark.gpu
-
-
-def _route_stream(s, level, R, policy, batches=None, max_flows=0):
-    bsz = int(max(s.batch_sizes))
-    pay = max(int(s.off[st1] - s.off[st0]) for st0, st1 in zip(s.batch_starts()[:-1], s.batch_starts()[1:]))
-    rt = alto.Router(s.depth, level, R, policy, max_batch_fragments=bsz, max_batch_payload=max(pay, 1),
-                     max_flows=max_flows, with_score=s.score is not None)
-    ro = oracle.RouterOracle(s.depth, level, R, policy)
-    for b in (range(s.n_batches) if batches is None else batches):
-        bt = s.batch(b)
-        db = alto.to_device(bt)
-        assert rt.route(db.tags, db.off, db.payload, db.score) == alto.OK
-        st, fo, po = rt.counts()
-        assert st == alto.OK
-        replica, perm, counts, parts = ro.route(bt)
-        assert np.array_equal(fo, counts)
-        rep_d, perm_d, parts_d = rt.outputs(fo, po)
-        assert np.array_equal(rep_d.cpu().numpy(), replica)
-        assert np.array_equal(perm_d.cpu().numpy(), perm)
-        for r in range(R):
-            t, o, p, sc = parts_d[r]
-            want = parts[r]
-            assert np.array_equal(t.cpu().numpy().view(np.uint64), want["tags"]), (b, r)
-            assert np.array_equal(o.cpu().numpy().astype(np.int64), want["off"]), (b, r)
-            assert np.array_equal(p.cpu().numpy(), want["payload"]), (b, r)
-            if want["score"] is not None:
-                assert np.array_equal(sc.cpu().numpy().view(np.uint32), want["score"].view(np.uint32))
-    rt.close()
 
 
 @pytest.mark.parametrize("name,level", [("factcheck", 1), ("throughput", 1), ("tot", 0), ("adversarial", 2)])
 @pytest.mark.parametrize("R", [1, 3, 8])
 @pytest.mark.parametrize("policy", [alto.ROUTE_HASH, alto.ROUTE_LEAST_LOADED])
 def test_route_matches_oracle(name, level, R, policy):
-    _route_stream(make_stream(name, small=True), level, R, policy)
+    route_stream_vs_oracle(make_stream(name, small=True), level, R, policy)
 
 
 def test_route_many_replicas():
-    _route_stream(make_stream("throughput", small=True), 2, 1000, alto.ROUTE_LEAST_LOADED)
-    _route_stream(make_stream("throughput", small=True), 2, 1000, alto.ROUTE_HASH)
+    route_stream_vs_oracle(make_stream("throughput", small=True), 2, 1000, alto.ROUTE_LEAST_LOADED)
+    route_stream_vs_oracle(make_stream("throughput", small=True), 2, 1000, alto.ROUTE_HASH)
 
 
 def test_route_errors():
@@ -96,4 +68,4 @@ def test_route_release_and_aggregate():
 @pytest.mark.slow
 def test_route_fullsize_throughput():
     """The 16M-fragment throughput stream, 1M batches, eight replicas placed by load."""
-    _route_stream(make_stream("throughput"), 1, 8, alto.ROUTE_LEAST_LOADED, batches=range(4))
+    route_stream_vs_oracle(make_stream("throughput"), 1, 8, alto.ROUTE_LEAST_LOADED, batches=range(4))

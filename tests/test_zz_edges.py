@@ -1,7 +1,8 @@
 """Edge cases of the CUDA path against the oracle, bit for bit, through the C
 ABI: a small open-group table and a small flow table whose deleted slots
-must be taken again, empty batches, and the largest depth, parent ids and k.
-(This file runs after the main parity files.)"""
+must be taken again, empty batches, the largest depth, parent ids and k, two
+output rings, and batches around a warp and a sort/scan tile.  (This file
+runs after the main parity files.)"""
 import numpy as np
 import pytest
 
@@ -9,8 +10,8 @@ torch = pytest.importorskip("torch")
 
 from fragments import split, to_batch, tree_fragments, window_stream
 from gen import make_stream
-from gpu_harness import (assert_same, route_release_and_aggregate, run_both_stream, run_gpu_batches,
-                         run_oracle_batches, small_caps, stream_caps)
+from gpu_harness import (assert_same, route_release_and_aggregate, route_stream_vs_oracle, run_both_stream,
+                         run_gpu_batches, run_oracle_batches, small_caps, stream_caps)
 
 pytestmark = pytest.mark.gpu
 
@@ -160,3 +161,39 @@ def test_double_ring_keeps_a_drain_through_the_next(name, stream_release):
     agg.close()
     o.close()
     assert s.n_batches > 2 and n_rec > 0
+
+
+_BOUNDARY_SIZES = [1, 31, 32, 33, 4095, 4096, 4097]
+
+
+def _boundary_batches(s):
+    """The stream cut into batches of 1, 31, 32, 33, 4,095, 4,096 and 4,097
+    fragments and the rest: around a warp (32) and around the tile of the
+    radix sort and the scans (4,096 elements)."""
+    import dataclasses
+
+    sizes = _BOUNDARY_SIZES + [s.n - sum(_BOUNDARY_SIZES)]
+    assert sizes[-1] > 0
+    return dataclasses.replace(s, batch_sizes=np.asarray(sizes))
+
+
+@pytest.mark.parametrize("leaf", ["accumulate", "topk", "stream_release"])
+def test_batches_at_warp_and_tile_boundaries(leaf):
+    """Every leaf form on batches around a warp and a sort/scan tile, bit for
+    bit against the oracle."""
+    s = _boundary_batches(window_stream(5_000, 4, 200, 256, seed=11, topk=(leaf == "topk")))
+    o, g = run_both_stream(s, drain_every=1, stream_release=(leaf == "stream_release"))
+    assert all(d.status == 0 for d in o)
+    assert_same(o, g, f"boundary batches/{leaf}")
+
+
+@pytest.mark.parametrize("policy", ["hash", "least_loaded"])
+@pytest.mark.parametrize("R", [8, 1000])
+def test_route_batches_at_warp_and_tile_boundaries(policy, R):
+    """Routing on batches around a warp and a sort/scan tile: each batch's
+    replicas, stable partition (one radix pass for 8 replicas, two for 1,000)
+    and sub-batches equal the routing oracle's."""
+    import paper_2403_04311_gb300 as alto
+
+    s = _boundary_batches(window_stream(5_000, 4, 200, 256, seed=11))
+    route_stream_vs_oracle(s, 1, R, alto.ROUTE_HASH if policy == "hash" else alto.ROUTE_LEAST_LOADED)
