@@ -2635,7 +2635,7 @@ LookbackState lb_region(const LookbackState& lb, int k) {
 }
 
 template <class F>
-void launch_scan3(const LookbackState& lb, int num_sms, Ctl* ctl, const F& f0, const F& f1,
+void launch_scan3(const LookbackState& lb, Ctl* ctl, const F& f0, const F& f1,
                   const F& f2, u64 cap, int site, u64 spin, cudaStream_t s) {
   u64 tiles = (cap + kScanTile - 1) / kScanTile;
   if (tiles == 0) tiles = 1;
@@ -2792,7 +2792,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
                  (M == D - 1) ? d.tab.bstate : nullptr, d.ctl};
     CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
     CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
-    launch_scan3(p.lbs, p.num_sms, d.ctl, f0, f1, f2, dcap, site, spin, s);
+    launch_scan3(p.lbs, d.ctl, f0, f1, f2, dcap, site, spin, s);
     p.launches += 1;
     site += 3;
   }
@@ -2812,7 +2812,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
       c[k].M = M;
       c[k].L = D - 1;
     }
-    launch_scan3(p.lbs, p.num_sms, d.ctl, c[0], c[1], c[2], dcap, site, spin, s);
+    launch_scan3(p.lbs, d.ctl, c[0], c[1], c[2], dcap, site, spin, s);
     p.launches += 1;
     site += 3;
   }
