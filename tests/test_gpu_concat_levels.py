@@ -13,7 +13,6 @@ import json
 import os
 import random
 
-import numpy as np
 import pytest
 
 torch = pytest.importorskip("torch")

@@ -8,7 +8,6 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
-import oracle
 import paper_2403_04311_gb300 as alto
 from fragments import split, to_batch, tree_fragments
 from gen import make_stream

@@ -9,7 +9,6 @@ index), where only the status has to agree."""
 import itertools
 import random
 
-import numpy as np
 import pytest
 
 import oracle

@@ -8,7 +8,6 @@ and writes into buffers the caller owns.  Here two calls in a row, on two
 different batches, must give exactly the records, payload and top-k pairs of
 create + push_batch + drain on a fresh handle (exact equality: the results
 are integers and copied floats).  This file is collected last on purpose."""
-import ctypes
 import dataclasses
 
 import numpy as np
