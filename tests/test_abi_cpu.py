@@ -108,3 +108,44 @@ def test_status_codes_match_oracle_and_header():
     for name in ["EINVAL", "ENOMEM", "ENOSPC", "EDUP", "ELAST", "EINCONSIST", "ECLOSED"]:
         assert int(vals[name]) == getattr(alto, name) == getattr(oracle, name)
     assert alto.RECORD_DTYPE == oracle.RECORD_DTYPE
+
+
+def test_struct_layouts_match_the_header(tmp_path):
+    """Every ctypes structure of the binding, and the record and pair dtypes,
+    have the size and field offsets that a C compiler gives the header's
+    structs (so the binding cannot drift from include/alto_agg.h)."""
+    import shutil
+    import subprocess
+
+    import numpy as np
+
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    structs = [alto.alto_agg_config, alto.alto_allocator, alto.alto_batch, alto.alto_drain,
+               alto._binding.alto_profile, alto.alto_split_args, alto._binding.alto_router_config,
+               alto._binding.alto_routed]
+    lines = ['#include <stddef.h>', '#include <stdio.h>', '#include "alto_agg.h"', 'int main(void) {']
+    want = []
+    for st in structs:
+        name = st.__name__
+        lines.append(f'  printf("%zu\\n", sizeof({name}));')
+        want.append(ctypes.sizeof(st))
+        for fname, _ in st._fields_:
+            lines.append(f'  printf("%zu\\n", offsetof({name}, {fname}));')
+            want.append(getattr(st, fname).offset)
+    for dt, name in [(alto.RECORD_DTYPE, "alto_record"), (alto.PAIR_DTYPE, "alto_topk_pair")]:
+        lines.append(f'  printf("%zu\\n", sizeof({name}));')
+        want.append(dt.itemsize)
+        for fname in dt.names:
+            lines.append(f'  printf("%zu\\n", offsetof({name}, {fname}));')
+            want.append(dt.fields[fname][1])
+    lines += ['  return 0;', '}']
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    include = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.run([cc, "-std=c11", "-I", include, str(src), "-o", str(exe)], check=True)
+    got = [int(x) for x in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()]
+    assert got == want
+    assert np.dtype(alto.RECORD_DTYPE).itemsize == 48
