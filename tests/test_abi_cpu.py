@@ -149,3 +149,20 @@ def test_struct_layouts_match_the_header(tmp_path):
     got = [int(x) for x in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()]
     assert got == want
     assert np.dtype(alto.RECORD_DTYPE).itemsize == 48
+
+
+def test_constants_match_the_header():
+    """Every ALTO_* constant the binding mirrors has the header's value."""
+    txt = open(os.path.join(ROOT, "include", "alto_agg.h")).read()
+    vals = {k: int(v, 0) for k, v in re.findall(r"#define ALTO_(\w+)\s+\(?(-?(?:0x[0-9a-fA-F]+|\d+))\)?", txt)}
+    b = alto._binding
+    pairs = {"ETIMEOUT": b.ETIMEOUT, "ECUDA": b.ECUDA, "MAX_DEPTH": b.MAX_DEPTH,
+             "PAYLOAD_NONE": b.PAYLOAD_NONE, "PAYLOAD_CONCAT": b.PAYLOAD_CONCAT,
+             "SCORE_NONE": b.SCORE_NONE, "SCORE_MAX": b.SCORE_MAX, "SCORE_TOPK": b.SCORE_TOPK,
+             "FLAG_STREAM_RELEASE": b.FLAG_STREAM_RELEASE, "FLAG_DOUBLE_RING": b.FLAG_DOUBLE_RING,
+             "OPS_PARTIAL": b.OPS_PARTIAL, "NUM_STAGES": b.NUM_STAGES, "PROFILE_OFF": b.PROFILE_OFF,
+             "PROFILE_STAGES": b.PROFILE_STAGES, "PROFILE_HOT": b.PROFILE_HOT, "MAX_DELIMS": b.MAX_DELIMS,
+             "ROUTE_HASH": b.ROUTE_HASH, "ROUTE_LEAST_LOADED": b.ROUTE_LEAST_LOADED}
+    for name, v in pairs.items():
+        assert vals[name] == v, name
+    assert len(b.STAGE_NAMES) == b.NUM_STAGES
