@@ -94,7 +94,6 @@ struct Scratch {
   u64* c_arena_base;     // [done_cap + 1] by done index: their buffered spans
   uint4* dense;          // [dense_cap] {stamp, len, owner entry or kNone, position}
   u64* dst;              // [dense_cap + 1]
-  u64* lenscan;          // [n_max + 1]
   u64* pairset;          // [ps_mask + 1]
   u64 ps_mask;
   u32 done_cap;
@@ -2850,7 +2849,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     }
     // plain stream order (no programmatic overlap with its neighbours): the
     // gather is the stage the measurement hooks time on their own
-    k_gather<<<grid, kThreads, 0, s>>>(d, bt);
+    k_gather<<<p.num_sms * blocks_per_sm((const void*)k_gather), kThreads, 0, s>>>(d, bt);
     p.launches += 1;
   }
   p.enter(9);
@@ -2911,7 +2910,8 @@ alto_status validate(const alto_agg_config* c) {
       return ALTO_EINVAL;
   }
   if (nconcat > 1) return ALTO_EINVAL;
-  if (c->flags & ~(int64_t)(ALTO_FLAG_STREAM_RELEASE | ALTO_FLAG_DOUBLE_RING)) return ALTO_EINVAL;
+  if (c->flags & ~(int64_t)(ALTO_FLAG_STREAM_RELEASE | ALTO_FLAG_DOUBLE_RING | ALTO_FLAG_TEST_STALL))
+    return ALTO_EINVAL;
   // streaming release needs the CONCAT level at the leaf parent
   if ((c->flags & ALTO_FLAG_STREAM_RELEASE) && c->payload_op[c->depth - 1] != ALTO_PAYLOAD_CONCAT)
     return ALTO_EINVAL;
@@ -3092,7 +3092,6 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   if (concat >= 0) {
     ALLOC(sc.dense, uint4, std::max<u64>(dense_cap, 1));
     ALLOC(sc.dst, u64, dense_cap + 1);
-    ALLOC(sc.lenscan, u64, nmax + 1);
   }
   if (concat >= 0 && concat < D - 1) {
     ALLOC(sc.c_dense_base, u64, done_cap + 1);
@@ -3147,6 +3146,10 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   }
   // initial state
   cudaMemsetAsync(d.ctl, 0, sizeof(Ctl), s);
+  if (cfg.flags & ALTO_FLAG_TEST_STALL) {
+    static const int kOne = 1;
+    cudaMemcpyAsync(&d.ctl->test_stall, &kOne, sizeof(int), cudaMemcpyHostToDevice, s);
+  }
   cudaMemsetAsync(d.tab.key, 0xFF, sizeof(u64) * T, s);
   cudaMemsetAsync(d.tab.hot, 0, sizeof(Hot) * T, s);
   cudaMemsetAsync(d.tab.cur, 0, sizeof(u64) * T, s);
@@ -3366,6 +3369,7 @@ struct NaDevice {
   unsigned char* base;  // device address of g_noalloc_scratch on that device
 };
 NaDevice g_na_dev[64];
+std::mutex g_na_mu;  // first calls from several host threads set up one entry once
 
 struct NaCarver {
   unsigned char* base;
@@ -3518,9 +3522,13 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
 }
 
 // Clear, in one launch, what every call must find empty: the control block
-// (keeping its epoch, so epoch-stamped arrays stay valid), the table keys,
-// the per-batch accumulators, the completion masks, the leaf-slot set, the
-// free-chunk stacks and the sort histogram.
+// (keeping its epoch), the table keys, the per-batch accumulators, the
+// completion masks, the leaf-slot set, the free-chunk stacks and the sort
+// histogram.  The arrays that are read by epoch stamp (the dense child slots
+// and the per-entry placement state) are cleared too: where they sit in the
+// static array depends on the depth, the CONCAT level and k, so after a call
+// with another layout they would hold whatever that call left there, and a
+// leftover token or key equal to the coming epoch would read as a stamp.
 __global__ void k_na_reset(Dev d, u32* hist, u64 T, u64 PS, u32 nmax) {
   pdl_enter();
   const u64 tid = (u64)blockIdx.x * blockDim.x + threadIdx.x;
@@ -3545,6 +3553,9 @@ __global__ void k_na_reset(Dev d, u32* hist, u64 T, u64 PS, u32 nmax) {
   for (u64 i = tid; i < (nmax + 31) / 32 * 32; i += stride) d.sc.mask[i] = 0;
   for (u64 i = tid; i < nmax / 32 + 1; i += stride) d.sc.mblk[i] = 0;
   for (u64 i = tid; i < 4 * 256; i += stride) hist[i] = 0;
+  for (u64 i = tid; i < T; i += stride) d.tab.bstate[i] = make_uint4(0, 0, 0, 0);
+  if (d.sc.dense != nullptr)
+    for (u64 i = tid; i < d.cfg.dense_cap; i += stride) d.sc.dense[i] = make_uint4(0, 0, 0, 0);
 }
 
 // Counts of the call for the caller: {status, records, payload, top-k pairs}.
@@ -3588,13 +3599,18 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
   // once per device, with that device current: the static array's address
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return ALTO_ECUDA;
-  NaDevice& nd = g_na_dev[dev];
-  if (!nd.ready) {
-    void* ptr = nullptr;
-    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || ptr == nullptr)
-      return ALTO_ECUDA;
-    nd.base = (unsigned char*)ptr;
-    nd.ready = true;
+  unsigned char* base = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_na_mu);
+    NaDevice& nd = g_na_dev[dev];
+    if (!nd.ready) {
+      void* ptr = nullptr;
+      if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || ptr == nullptr)
+        return ALTO_ECUDA;
+      nd.base = (unsigned char*)ptr;
+      nd.ready = true;
+    }
+    base = nd.base;
   }
   int num_sms = 0;
   if (cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
@@ -3602,7 +3618,7 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
 
   NaState st;
   NaCarver cv;
-  na_layout(cfg, nd.base, st, cv);
+  na_layout(cfg, base, st, cv);
   if (!cv.ok) return ALTO_ENOSPC;
   Dev d = st.d;
   d.out_rec = out_records;

@@ -1,13 +1,17 @@
-"""The allocation-free one-shot entry point against the regular path.
+"""The allocation-free one-shot entry point against the oracle and the regular path.
 
 alto_agg_oneshot_noalloc exists for callers that may not allocate device
 memory (a framework that already reserved the device's free memory for its
 own pool, a real-time path that cannot take cudaMalloc's synchronisation, a
 plug-in loaded without an allocator).  It works out of a static device array
-and writes into buffers the caller owns.  Here two calls in a row, on two
-different batches, must give exactly the records, payload and top-k pairs of
-create + push_batch + drain on a fresh handle (exact equality: the results
-are integers and copied floats).  This file is collected last on purpose."""
+and writes into buffers the caller owns.  Each batch goes through it twice in
+a row, and must give exactly the records, payload and top-k pairs of the
+oracle and of create + push_batch + drain on a fresh handle (exact equality:
+the results are integers and copied floats).  The batches follow one another
+with different depths, CONCAT levels and k, so that each call finds the
+static array laid out differently by the call before; one of them carries
+token ids 1..64, values the arrays read by epoch stamp could mistake for a
+stamp if a call did not clear them.  This file is collected last on purpose."""
 import dataclasses
 
 import numpy as np
@@ -15,6 +19,7 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
+import oracle
 import paper_2403_04311_gb300 as alto
 from gen import make_stream
 from gen.streams import make_factcheck
@@ -62,28 +67,50 @@ def _oneshot(s, bt, cap_rec=8192, cap_pay=1 << 18, cap_topk=8192):
             tk[:ntk * 8].cpu().numpy().view(alto.PAIR_DTYPE))
 
 
+def _oracle(s, bt):
+    o = oracle.Oracle.for_stream(s)
+    assert o.push_batch(bt) == oracle.OK
+    d = o.drain()
+    o.close()
+    assert d.status == oracle.OK
+    return d.records, d.payload, d.topk
+
+
 def _cases():
     tiny = make_stream("tiny64")
+    # token ids 1..64: small integers like the epochs the static array's
+    # stamped slots are compared with
+    tiny_small = dict(tiny.batch(0))
+    tiny_small["payload"] = (tiny_small["payload"] % 64 + 1).astype(np.int32)
     # depth 4 with top-k and max levels, whole stream in one batch
     fact = make_factcheck(n_responses=8, batch=4096)
     assert fact.n_batches == 1
     # the same batch with the concatenation two levels above the fragments
     fact_up = dataclasses.replace(fact, payload_op=(0, 1, 0, 0))
-    return [(tiny, tiny.batch(0)), (fact, fact.batch(0)), (fact_up, fact_up.batch(0))]
+    a, b, c = (tiny, tiny_small), (fact, fact.batch(0)), (fact_up, fact_up.batch(0))
+    # every layout after another one, and each again after a change
+    return [a, b, c, a, c, b, a]
 
 
-def test_oneshot_noalloc_matches_regular_path_twice_in_a_row():
+def _same(got, want):
+    assert np.array_equal(got[0].view(np.uint8), want[0].view(np.uint8))
+    assert np.array_equal(got[1], want[1])
+    assert np.array_equal(got[2].view(np.uint8), want[2].view(np.uint8))
+
+
+def test_oneshot_noalloc_matches_oracle_and_regular_path_twice_in_a_row():
     for s, bt in _cases():
         assert bt["n"] <= 4096 and bt["n"] * s.depth <= 16384
         caps = dict(max_batch_fragments=bt["n"], max_batch_payload=int(bt["payload"].size),
                     max_open_groups=1 << 15, arena_elems=1 << 22, out_records=1 << 15,
                     out_payload_elems=1 << 18, out_topk=1 << 15, max_emit_children=1 << 14)
-        want = _regular(s, bt, caps)
-        got = _oneshot(s, bt)
+        want = _oracle(s, bt)
         assert len(want[0]) > 0
-        assert np.array_equal(got[0].view(np.uint8), want[0].view(np.uint8))
-        assert np.array_equal(got[1], want[1])
-        assert np.array_equal(got[2].view(np.uint8), want[2].view(np.uint8))
+        _same(_regular(s, bt, caps), want)
+        first = _oneshot(s, bt)
+        second = _oneshot(s, bt)
+        _same(first, want)
+        _same(second, want)
 
 
 def test_oneshot_noalloc_rejects_oversize_batches():
