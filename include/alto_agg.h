@@ -118,6 +118,16 @@ typedef int alto_status;
  * twice the output capacities' memory.  EINVAL for alto_agg_oneshot_noalloc. */
 #define ALTO_FLAG_DOUBLE_RING 2
 
+/* Failure-path test hook (flags bit 2; the paper has no counterpart): every
+ * look-back wait of a push (the scans' and the radix sort's) waits on a
+ * predecessor's descriptor that nothing publishes, so the first wait of a
+ * scan or sort with more than one tile polls spin_limit times, records
+ * ALTO_ETIMEOUT and stops the batch, as a wait that really ran out does.  The
+ * next drain returns ALTO_ETIMEOUT and the handle stays poisoned; destroy
+ * still succeeds and the CUDA context stays usable.  Only for testing the
+ * timeout path: leave it off.  EINVAL for alto_agg_oneshot_noalloc. */
+#define ALTO_FLAG_TEST_STALL 4
+
 /* Aggregator configuration (Sec. 5: the controller is told which queues are
  * pmap entry/exit points and which data is aggregated; here: the nesting
  * depth and what each level's exit computes).  Zero capacities take the

@@ -38,6 +38,7 @@ struct Ctl {
   int status;              // latched alto_status
   int batch_err;           // priority-encoded error of the current batch
   int abort;               // a device wait gave up: the rest of the batch is skipped
+  int test_stall;          // ALTO_FLAG_TEST_STALL: look-back waits never see a predecessor
   int top[kNumChunks];     // free-chunk stack heights per class
   u32 tile_ctr[kSites];    // dynamic tile counters per launch site
   u32 exit_ctr[kSites];    // CTAs finished per launch site (resets tile_ctr)

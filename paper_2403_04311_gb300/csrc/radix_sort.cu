@@ -156,11 +156,12 @@ __global__ void __launch_bounds__(kSortThreads) k_onesweep(const u32* n_dev, u32
       *slot = ((u64)es << 34) | (1ull << 32) | cnt;
       long long pred = (long long)tile - 1;
       u64 spins = 0;
+      const bool stall = ctl->test_stall != 0;  // test hook: nothing is ever published
       while (pred >= 0) {
         volatile u64* ps = lb + (u64)pred * kRadix + t;
         u64 v = *ps;
         u32 kind = (u32)(v >> 32) & 3u;
-        if ((u32)(v >> 34) != es || kind == 0) {
+        if ((u32)(v >> 34) != es || kind == 0 || stall) {
           if (++spins > spin_limit || *(volatile int*)&ctl->abort) {
             raise_timeout(ctl);
             break;

@@ -77,6 +77,7 @@ __device__ __forceinline__ u64 lb_walk_warp(LookbackState st, u32 tile, u32 es, 
   u64 excl = 0;
   long long top = (long long)tile - 1;
   u64 spins = 0;
+  const bool stall = ctl->test_stall != 0;  // test hook: nothing is ever published
   while (top >= 0) {
     ulonglong2 dsc[4];
     int stop = 128, wait = 128;  // nearest inclusive, nearest unpublished
@@ -88,7 +89,7 @@ __device__ __forceinline__ u64 lb_walk_warp(LookbackState st, u32 tile, u32 es, 
       if (p >= 0) {
         dsc[r] = lb_read(st, p);
         const u32 f = (u32)dsc[r].y;
-        kind = ((f >> 2) == es) ? (f & 3u) : 0u;
+        kind = ((f >> 2) == es && !stall) ? (f & 3u) : 0u;
       }
       const u32 inc = __ballot_sync(0xFFFFFFFFu, kind == 2u);
       const u32 unp = __ballot_sync(0xFFFFFFFFu, kind == 0u);

@@ -60,7 +60,7 @@ def _cfg(**kw):
     dict(arena_elems=1 << 32),
     dict(payload_op=[1, 0], stream_release=True),    # streaming release above the leaf parent
     dict(payload_op=[0, 0], stream_release=True),    # streaming release without CONCAT
-    dict(flags=4),                                   # unknown flag
+    dict(flags=8),                                   # unknown flag
 ])
 def test_create_rejects_bad_configs_on_host(bad):
     lib = alto.load_library()
@@ -75,10 +75,11 @@ def test_create_rejects_bad_configs_on_host(bad):
     assert h.value == 12345  # untouched
 
 
-@pytest.mark.parametrize("flag", ["stream_release", "double_ring"])
+@pytest.mark.parametrize("flag", ["stream_release", "double_ring", "test_stall"])
 def test_noalloc_refuses_handle_flags_on_host(flag):
     """One batch has nothing to release in a stream and writes the caller's
-    buffers, not rings: both flags are refused before any device work."""
+    buffers, not rings, and the wait-stall test hook is for handles only:
+    every flag is refused before any device work."""
     cfg = _cfg(**{flag: True})
     b = alto.alto_batch()
     b.depth = 2
@@ -160,6 +161,7 @@ def test_constants_match_the_header():
              "PAYLOAD_NONE": b.PAYLOAD_NONE, "PAYLOAD_CONCAT": b.PAYLOAD_CONCAT,
              "SCORE_NONE": b.SCORE_NONE, "SCORE_MAX": b.SCORE_MAX, "SCORE_TOPK": b.SCORE_TOPK,
              "FLAG_STREAM_RELEASE": b.FLAG_STREAM_RELEASE, "FLAG_DOUBLE_RING": b.FLAG_DOUBLE_RING,
+             "FLAG_TEST_STALL": b.FLAG_TEST_STALL,
              "OPS_PARTIAL": b.OPS_PARTIAL, "NUM_STAGES": b.NUM_STAGES, "PROFILE_OFF": b.PROFILE_OFF,
              "PROFILE_STAGES": b.PROFILE_STAGES, "PROFILE_HOT": b.PROFILE_HOT, "MAX_DELIMS": b.MAX_DELIMS,
              "ROUTE_HASH": b.ROUTE_HASH, "ROUTE_LEAST_LOADED": b.ROUTE_LEAST_LOADED}
