@@ -140,15 +140,12 @@ def test_bruteforce_stream_release(depth):
 
 
 def test_bruteforce_forest():
-    """Two independent sources interleaved."""
+    """Two independent sources interleaved, at depths 2 and 3."""
     rng = random.Random(7)
-    for shape_a, shape_b in [([2, 1], [1]), ([1, [2]], [[1], 2]), ([3], [2, 2])]:
-        if count_leaves(shape_a) and isinstance(shape_a, list) and isinstance(shape_b, list):
-            pass
+    pairs = [([2, 1], [1]), ([[1], [2]], [[2, 1]]), ([3], [2, 2])]
+    for shape_a, shape_b in pairs:
         da = depth_of(shape_a)
-        db = depth_of(shape_b)
-        if da != db:
-            continue
+        assert da == depth_of(shape_b)
         fa = tree_fragments(shape_a, id_base=100, score_fn=lambda k: SCORES[k % 7])
         fb = tree_fragments(shape_b, id_base=500, score_fn=lambda k: SCORES[(k + 3) % 7])
         frags = fa + fb
