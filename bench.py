@@ -152,6 +152,52 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def host_info():
+    """The host CPU the oracle baselines run on: model name and logical cores."""
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                             text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.strip().lower().startswith("model name:"):
+                model = ln.split(":", 1)[1].strip()
+                break
+    except Exception:
+        pass
+    if model is None:
+        try:
+            with open("/proc/cpuinfo") as f:
+                for ln in f:
+                    if ln.lower().startswith(("model name", "cpu part")):
+                        model = ln.split(":", 1)[1].strip()
+                        break
+        except Exception:
+            pass
+    import platform
+    return {"cpu_model": model or platform.processor() or platform.machine(),
+            "nproc": os.cpu_count(), "arch": platform.machine()}
+
+
+def batch_latency(agg, batches, warm=10, min_samples=64):
+    """Host time of push + drain per batch (the drain synchronises): the first
+    `warm` batches are warm-up, then every batch of the stream at least once
+    (at least `min_samples` batches, passes of the stream in order).  The
+    handle must be at a stream boundary on entry; a pass that the loop leaves
+    unfinished is discarded with the handle."""
+    nb = len(batches)
+    total = warm + max(nb, min_samples)
+    lat = []
+    for i in range(total):
+        db = batches[i % nb]
+        t0 = time.perf_counter()
+        agg.push(db.tags, db.off, db.payload, db.score)
+        agg.drain()
+        if i >= warm:
+            lat.append((time.perf_counter() - t0) * 1e6)
+    lat.sort()
+    return (lat[len(lat) // 2], lat[min(len(lat) - 1, int(0.99 * len(lat)))], len(lat))
+
+
 def algorithmic_bytes(s):
     """Bytes the method itself must move for the stream: tags 8D, offsets 4
     and score 4 per fragment, payload read + write, 48 B per record and 8 B
@@ -201,7 +247,7 @@ def run_reference(args, s, rank, world):
         "data": "synthetic", "config": {"workload": s.name, "fragments": s.n, "depth": s.depth,
                                         "batch": int(s.batch_sizes[0]),
                                         "stream_release": bool(args.stream_release)},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "host": host_info(), "kind": "oracle",
                          "sample": f"first {n} fragments of batch 0 of the {s.name} stream, "
                                    f"one batch per step, single thread"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -234,7 +280,7 @@ def run_split(args, rank, world):
                 "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "int32", "data": "synthetic",
                 "config": {"workload": "split", "streams": n_src, "tokens": n_tok},
-                "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "host": host_info(), "kind": "oracle",
                                  "sample": f"first {k} streams per step, single thread"},
                 "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     import torch
@@ -315,7 +361,7 @@ def run_split(args, rank, world):
         oracle.split_text(si.src_tags[:, :k], si.src_id[:k], si.tok_off[:k + 1],
                           si.tokens[:int(si.tok_off[k])], si.delims)
         dt = time.perf_counter() - t0
-        cpu = {"value": int(si.tok_off[k]) / dt, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+        cpu = {"value": int(si.tok_off[k]) / dt, "unit": "tokens/s", "cores": 1, "host": host_info(), "kind": "oracle",
                "sample": f"first {k} of {n_src} streams ({int(si.tok_off[k])} tokens), single thread"}
     return {"metric": "split_text tokens/s", "value": n_tok * world / (ms / 1e3), "unit": "tokens/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
@@ -359,7 +405,7 @@ def run_route(args, rank, world, R=8):
                 "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
                 "data": "synthetic", "config": {"workload": "route", "replicas": R, "level": L},
-                "cpu_baseline": {"value": value, "unit": "fragments/s", "cores": 1, "kind": "oracle",
+                "cpu_baseline": {"value": value, "unit": "fragments/s", "cores": 1, "host": host_info(), "kind": "oracle",
                                  "sample": f"first {n} fragments of batch 0 per step, single thread"},
                 "e2e": {"value": value, "unit": "fragments/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     import torch
@@ -467,7 +513,7 @@ def run_route(args, rank, world, R=8):
         t0 = time.perf_counter()
         oracle.RouterOracle(s.depth, L, R, oracle.LEAST_LOADED).route(sample)
         dt = time.perf_counter() - t0
-        cpu = {"value": n / dt, "unit": "fragments/s", "cores": 1, "kind": "oracle",
+        cpu = {"value": n / dt, "unit": "fragments/s", "cores": 1, "host": host_info(), "kind": "oracle",
                "sample": f"first {n} fragments of batch 0, single thread"}
     hbm_gbs, peak_kind = peaks()
     # algorithmic bytes of a pass: every fragment's tags and offset read and
@@ -505,7 +551,7 @@ def cpu_baseline(s, budget_s=20.0, stream_release=False):
             break
     dt = time.perf_counter() - t0
     o.close()
-    return {"value": done / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+    return {"value": done / dt, "unit": UNIT, "cores": 1, "host": host_info(), "kind": "oracle",
             "sample": f"first {nb} batch(es) ({done} fragments) of the {s.name} stream in "
                       f"arrival order, single thread, {dt:.1f} s"}
 
@@ -522,7 +568,8 @@ def main():
                     help="streaming release of open CONCAT groups after every push")
     ap.add_argument("--ref-sample", type=float, default=250_000)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--latency-batches", type=int, default=16)
+    ap.add_argument("--latency-batches", type=int, default=64,
+                    help="at least this many timed batches (after 10 warm-up ones) for p50/p99")
     ap.add_argument("--profile-steps", type=int, default=2,
                     help="steps of the separate stage-breakdown pass")
     ap.add_argument("--double-ring", action="store_true",
@@ -770,16 +817,8 @@ def main():
     e2e_value = frags_per_step * world * e_steps / (e_ms / 1e3)
 
     # ---- per-batch latency: push + drain, host clock -------------------------
-    lat = []
-    for hb_i in range(min(args.latency_batches, 2 * s.n_batches)):
-        db = dev[hb_i % len(dev)]
-        t0 = time.perf_counter()
-        agg.push(db.tags, db.off, db.payload, db.score)
-        agg.drain()
-        lat.append((time.perf_counter() - t0) * 1e6)
-    lat_s = sorted(lat)
-    p50 = lat_s[len(lat_s) // 2]
-    p99 = lat_s[min(len(lat_s) - 1, int(0.99 * len(lat_s)))]
+    # (the e2e loop leaves the handle at a stream boundary: every group done)
+    p50, p99, n_lat = batch_latency(agg, dev, warm=10, min_samples=args.latency_batches)
     agg.close()
 
     if rank != 0:
@@ -804,6 +843,7 @@ def main():
         "algorithmic_gbps": alg_bytes * world * args.steps / (ms / 1e3) / 1e9,
         "hbm_frac_path": alg_bytes * args.steps / (ms / 1e3) / 1e9 / hbm_gbs,
         "p50_batch_latency_us": p50, "p99_batch_latency_us": p99,
+        "latency_note": f"push + drain per batch, host clock; {n_lat} batches after 10 warm-up batches",
         "records_per_step": n_records_step, "partial_records_per_step": n_partial_step,
         "roofline": rooflines[dominant],
         "rooflines": rooflines,
