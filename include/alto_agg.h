@@ -128,6 +128,14 @@ typedef int alto_status;
  * timeout path: leave it off.  EINVAL for alto_agg_oneshot_noalloc. */
 #define ALTO_FLAG_TEST_STALL 4
 
+/* Launch every kernel of a push one by one (flags bit 3).  By default a push
+ * of at most 131,072 fragments replays a CUDA graph of its launch sequence,
+ * captured on the handle's first such push (per output ring and profiling
+ * mode): one host launch per push instead of about twenty.  Larger pushes
+ * always launch directly.  Results are the same either way.  EINVAL for
+ * alto_agg_oneshot_noalloc, which always launches directly. */
+#define ALTO_FLAG_DIRECT_LAUNCH 8
+
 /* Aggregator configuration (Sec. 5: the controller is told which queues are
  * pmap entry/exit points and which data is aggregated; here: the nesting
  * depth and what each level's exit computes).  Zero capacities take the

@@ -27,6 +27,7 @@ SCORE_NONE, SCORE_MAX, SCORE_TOPK = 0, 1, 2
 FLAG_STREAM_RELEASE = 1
 FLAG_DOUBLE_RING = 2
 FLAG_TEST_STALL = 4
+FLAG_DIRECT_LAUNCH = 8
 OPS_PARTIAL = 0x80
 
 RECORD_DTYPE = np.dtype([
@@ -182,7 +183,7 @@ def load_library(build: bool = True):
 def make_config(depth, payload_op, score_op, topk_k=None, *, max_batch_fragments,
                 max_batch_payload, max_open_groups=0, arena_elems=0, out_records=0,
                 out_payload_elems=0, out_topk=0, max_emit_children=0, spin_limit=0,
-                stream_release=False, double_ring=False, test_stall=False):
+                stream_release=False, double_ring=False, test_stall=False, direct_launch=False):
     c = alto_agg_config()
     c.depth = depth
     topk_k = topk_k or [0] * depth
@@ -200,7 +201,7 @@ def make_config(depth, payload_op, score_op, topk_k=None, *, max_batch_fragments
     c.max_emit_children = int(max_emit_children)
     c.spin_limit = int(spin_limit)
     c.flags = ((FLAG_STREAM_RELEASE if stream_release else 0) | (FLAG_DOUBLE_RING if double_ring else 0) |
-               (FLAG_TEST_STALL if test_stall else 0))
+               (FLAG_TEST_STALL if test_stall else 0) | (FLAG_DIRECT_LAUNCH if direct_launch else 0))
     return c
 
 

@@ -67,7 +67,8 @@ struct Scratch {
   u32* leaf_seg_of;      // [n_max]
   u32* up_keys;
   u32* up_perm;
-  u32* up_seg_start;     // [n_max + 1]
+  u32* up_seg_start;     // [n_max + 1] sorted levels: segment starts; atomic levels: touched entries
+  u32* up_list2;         // [n_max] atomic levels: touched entries (alternating with up_seg_start)
   u32* it_rep[2];        // items: representative fragment
   u32* it_cseq[2];       // items: done << 31 | completion seq (batch-local)
   u32* it_skey[2];       // items: largest score key of the child
@@ -105,6 +106,7 @@ struct Scratch {
   u32* big_seg;          // [depth][big_cap] segments longer than kBigSeg, per level
   u32 big_cap;
   u32* rel_seg;          // [n_max] streaming: small leaf segments whose groups release a run
+  Batch* batch;          // [1] the push's batch, stored by k_begin (read by graph replays)
 };
 
 struct Dev {
@@ -117,6 +119,18 @@ struct Dev {
   int32_t* out_pay;
   alto_topk_pair* out_topk;
 };
+
+// The batch of the push.  Kernels launched one by one get it by value; in a
+// replay of a push's captured CUDA graph (G) their parameters are those of
+// the capture, and the batch is the copy the graph's first kernel stored.
+template <bool G>
+__device__ __forceinline__ Batch batch_of(const Batch& bv, const Dev& d) {
+  if constexpr (G) {
+    return *d.sc.batch;
+  } else {
+    return bv;
+  }
+}
 
 __device__ __forceinline__ bool poisoned(const Ctl* c) { return halted(c); }
 // Payload-moving kernels also stand down once the batch has any error: its
@@ -159,8 +173,17 @@ __device__ __forceinline__ u32 warp_take(bool want, u32* counter) {
 // No key is ever placed twice, and a walk only grows while other threads take
 // free slots, so it ends.  A key lies within max_probe slots of home; a walk
 // that reaches that distance with no free slot met finds the table full.
+//
+// `publish`: other threads of this launch may add to the new entry's batch
+// accumulators and compare with its chain row as soon as the key is in
+// place (the level kernels that add their items to the parent level).  The
+// insert then leaves the accumulators and `touch` alone (they are clear in a
+// free slot) and, once the chain row is written, sets the entry's ready flag
+// with release order.  Without it (no adder in the launch) the whole record
+// is written, which also brings its line into L2 for the next kernel.
 __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, int* inserted,
-                                  const u64* tags = nullptr, u64 n = 0, u32 rep = 0, int l = 0) {
+                                  const u64* tags = nullptr, u64 n = 0, u32 rep = 0, int l = 0,
+                                  bool publish = false) {
   const u32 home = (u32)mix64(key) & tab.mask;
   const u32 reach = (u32)tab.max_probe;  // at most the table size
   u32 h = home, dist = 0;
@@ -184,12 +207,18 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
     const u64 prev = atomicCAS((unsigned long long*)&tab.key[t], (unsigned long long)want,
                                (unsigned long long)key);
     if (prev == want) {
-      // the whole record: up, last = none, nothing completed, accumulators zero
+      // up, last = none, nothing completed, accumulators clear
       uint4* hw = reinterpret_cast<uint4*>(tab.hot + t);
       hw[0] = make_uint4((u32)up, (u32)(up >> 32), kNone, 0);
-      hw[1] = make_uint4(0, 0, 0, 0);
-      hw[2] = make_uint4(kNone, 0, 0, 0);
-      hw[3] = make_uint4(0, 0, 0, 0);
+      if (publish) {
+        tab.hot[t].maxc1 = 0;
+        tab.hot[t].smax = 0;
+        tab.hot[t].done_epoch = 0;
+      } else {
+        hw[1] = make_uint4(0, 0, 0, 0);
+        hw[2] = make_uint4(kNone, 0, 0, 0);
+        hw[3] = make_uint4(0, 0, 0, 0);
+      }
       if (tab.rel) tab.rel[t] = 0;
       if (tab.vec_n) {
         tab.vec_n[2 * (u64)t] = 0;
@@ -203,6 +232,8 @@ __device__ u32 ht_find_or_insert(const Table& tab, u64 key, u64 up, Ctl* ctl, in
         cb[0] = make_ulonglong2(0, 0);
         cb[1] = make_ulonglong2(0, 0);
       }
+      // the chain row is written: finders of this launch may compare with it
+      if (publish) asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(tab.ready + t), "r"(1u) : "memory");
       *inserted = 1;
       return t;
     }
@@ -445,8 +476,30 @@ __device__ __forceinline__ void chain_reserve(const Table& tab, u32 e, u32 P, u3
 // ---------------------------------------------------------------------------
 // kernels
 // ---------------------------------------------------------------------------
-__global__ void k_begin(Ctl* ctl, u32 n) {
+// Every table record as a free slot has it: no last child, nothing
+// completed, accumulators clear (acc_fmin = none).
+__global__ void k_init_hot(Hot* hot, u64 T) {
   pdl_enter();
+  for (u64 i = (u64)blockIdx.x * blockDim.x + threadIdx.x; i < T; i += (u64)gridDim.x * blockDim.x) {
+    uint4* hw = reinterpret_cast<uint4*>(hot + i);
+    hw[0] = make_uint4(0, 0, kNone, 0);
+    hw[1] = make_uint4(0, 0, 0, 0);
+    hw[2] = make_uint4(kNone, 0, 0, 0);
+    hw[3] = make_uint4(0, 0, 0, 0);
+  }
+}
+
+// Start of a push: store the batch for kernels that read it from device
+// memory (graph replays), reset the output counters a drain handed out
+// (`reset`), and clear the per-batch fields.
+__global__ void k_begin(Ctl* ctl, Batch b, Batch* store, int reset) {
+  pdl_enter();
+  if (store) *store = b;
+  if (reset) {
+    ctl->rec_count = 0;
+    ctl->pay_count = 0;
+    ctl->topk_count = 0;
+  }
   ctl->epoch += 1;
   ctl->batch_err = 0;
   ctl->n_done = 0;
@@ -456,11 +509,13 @@ __global__ void k_begin(Ctl* ctl, u32 n) {
   ctl->n_rel = 0;
   for (int l = 0; l < kMaxDepth; ++l) ctl->n_big[l] = 0;
   for (int l = 0; l < kMaxDepth; ++l) ctl->n_segs[l] = 0;
-  ctl->n = (ctl->status == ALTO_OK) ? n : 0u;
+  ctl->n = (ctl->status == ALTO_OK) ? b.n : 0u;
 }
 
-__global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
+template <bool G>
+__global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch bv) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   __shared__ u32 s_ins;
@@ -491,8 +546,10 @@ __global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch b) {
 }
 
 // Items of level l are the level-(l+1) groups present in the batch.
-__global__ void __launch_bounds__(kThreads) k_items_lookup(Dev d, Batch b, int l, int in_set) {
+template <bool G>
+__global__ void __launch_bounds__(kThreads) k_items_lookup(Dev d, Batch bv, int l, int in_set) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   __shared__ u32 s_ins;
@@ -1070,11 +1127,12 @@ __device__ __forceinline__ void reduce_warp(const Dev& d, const Batch& b, Ctl* c
 // the others one after another by the whole warp; segments longer than
 // kBigSeg are listed for k_reduce_big.  (A small segment whose group makes a
 // streaming release is listed for k_reduce_rel: the release needs a warp.)
-template <bool LEAF>
-__global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, const u32* skeys,
+template <bool LEAF, bool G>
+__global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch bv, int l, const u32* skeys,
                                                      const u32* sperm, const u32* seg_start,
                                                      int in_set) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const u32 nseg = min(ctl->n_segs[l], d.cfg.n_max);
@@ -1114,9 +1172,11 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch b, int l, cons
 }
 
 // Streaming release: the small segments whose groups release a run, a warp each.
-__global__ void __launch_bounds__(kThreads) k_reduce_rel(Dev d, Batch b, const u32* skeys, const u32* sperm,
+template <bool G>
+__global__ void __launch_bounds__(kThreads) k_reduce_rel(Dev d, Batch bv, const u32* skeys, const u32* sperm,
                                                          const u32* seg_start, int in_set) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const int l = d.cfg.depth - 1;
@@ -1137,11 +1197,12 @@ __global__ void __launch_bounds__(kThreads) k_reduce_rel(Dev d, Batch b, const u
 // reductions with the block's warps over strided items, combined in shared
 // memory; each warp keeps a top-k of its items and warp 0 merges them with
 // the entry's list; a streaming release runs on warp 0.
-template <bool LEAF>
-__global__ void __launch_bounds__(kBigThreads) k_reduce_big(Dev d, Batch b, int l, const u32* skeys,
+template <bool LEAF, bool G>
+__global__ void __launch_bounds__(kBigThreads) k_reduce_big(Dev d, Batch bv, int l, const u32* skeys,
                                                             const u32* sperm, const u32* seg_start,
                                                             int in_set) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   constexpr int kW = kBigThreads / 32;
@@ -1230,9 +1291,91 @@ __global__ void __launch_bounds__(kBigThreads) k_reduce_big(Dev d, Batch b, int 
 // upper levels without TOPK: hash-table entries accumulate the batch's items
 // with warp-aggregated atomics; the touched entries are then finalised.
 // ---------------------------------------------------------------------------
-// Items of level l: check ancestry against the entry and accumulate.
-__global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int l, int in_set) {
+// One item of level l per lane (all 32 lanes together; `valid` marks the
+// real ones): the batch's first item of an entry puts the entry on the
+// level's touched list, and every item adds itself to the entry's batch
+// accumulators, warp-aggregated over lanes with the same entry.
+__device__ __forceinline__ void add_items(const Dev& d, Ctl* ctl, bool valid, u32 e, u32 rep, u32 c, u32 f,
+                                          u32 done, u32 cs, u32 sk, u32 ep, u32* list, u32* list_n) {
+  bool first = false;
+  if (valid) first = atomicExch(&d.tab.hot[e].touch, ep) != ep;
+  {
+    const u32 pos = warp_take(first, list_n);
+    if (first) {
+      if (pos < d.cfg.n_max) list[pos] = e;
+      d.tab.hot[e].acc_rep = rep;
+    }
+  }
+  // lanes without an item form their own group; the whole warp takes part
+  const u32 key = valid ? e : kNone;
+  const u32 peers = __match_any_sync(0xFFFFFFFFu, key);
+  if (__all_sync(0xFFFFFFFFu, peers == (1u << (threadIdx.x & 31)))) {
+    if (valid) {
+      if (done) {
+        atomicAdd((unsigned long long*)&d.tab.hot[e].acc_cl, 1ull << 40);
+        atomicMax(&d.tab.hot[e].acc_cs1, cs + 1);
+        if (sk) atomicMax(&d.tab.hot[e].acc_smx, sk);
+      }
+      atomicMax(&d.tab.hot[e].acc_m1, c + 1);
+      if (f) {
+        atomicMin(&d.tab.hot[e].acc_fmin, c);
+        atomicMax(&d.tab.hot[e].acc_fmax1, c + 1);
+      }
+    }
+    return;
+  }
+  const int leader = __ffs(peers) - 1;
+  const u32 cnt = __reduce_add_sync(peers, done);
+  const u32 m1 = __reduce_max_sync(peers, valid ? c + 1 : 0u);
+  const u32 fmin = __reduce_min_sync(peers, (valid && f) ? c : kNone);
+  const u32 fmax1 = __reduce_max_sync(peers, (valid && f) ? c + 1 : 0u);
+  const u32 cs1 = __reduce_max_sync(peers, (valid && done) ? cs + 1 : 0u);
+  const u32 smx = __reduce_max_sync(peers, (valid && done) ? sk : 0u);
+  if (valid && (int)(threadIdx.x & 31) == leader) {
+    if (cnt) atomicAdd((unsigned long long*)&d.tab.hot[e].acc_cl, (unsigned long long)cnt << 40);
+    if (m1) atomicMax(&d.tab.hot[e].acc_m1, m1);
+    if (fmin != kNone) atomicMin(&d.tab.hot[e].acc_fmin, fmin);
+    if (fmax1) atomicMax(&d.tab.hot[e].acc_fmax1, fmax1);
+    if (cs1) atomicMax(&d.tab.hot[e].acc_cs1, cs1);
+    if (smx) atomicMax(&d.tab.hot[e].acc_smx, smx);
+  }
+}
+
+// Ancestry of item `rep` (tags 0..l-1) against entry e's chain row, which the
+// entry's inserter may be writing in this same launch: wait (bounded) until
+// it says the row is written, then read the row from L2 (an L1 line of this
+// SM may predate the write).
+__device__ bool chain_differs_ready(const Dev& d, Ctl* ctl, u32 e, const Batch& b, u32 rep, int l) {
+  if (l == 0) return false;  // a top-level group has no ancestry to compare
+  u64 spins = 0;
+  for (;;) {
+    u32 r;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(r) : "l"(d.tab.ready + e) : "memory");
+    if (r) break;
+    if (*(volatile int*)&ctl->abort) return false;
+    if (++spins > d.cfg.spin_limit) {
+      raise_timeout(ctl);
+      return false;
+    }
+    __nanosleep(32);
+  }
+  const ulonglong2* row = reinterpret_cast<const ulonglong2*>(d.tab.chain + (u64)e * d.tab.chain_len);
+  bool bad = false;
+  for (int q = 0; q < l; q += 2) {
+    const ulonglong2 v = __ldcg(row + (q >> 1));
+    if (b.tags[(u64)q * b.n + rep] != v.x) bad = true;
+    if (q + 1 < l && b.tags[(u64)(q + 1) * b.n + rep] != v.y) bad = true;
+  }
+  return bad;
+}
+
+// Items of level l (after a TOPK level or the sorted leaf level, whose
+// reduce does not look up parents): check ancestry against the entry and
+// accumulate; the touched entries go to `list`.
+template <bool G>
+__global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch bv, int l, int in_set, u32* list) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const u32 ni = min(ctl->n_segs[l + 1], d.cfg.n_max);
@@ -1240,13 +1383,11 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
   const u32* it_rep = d.sc.it_rep[in_set];
   const u32* it_cseq = d.sc.it_cseq[in_set];
   const u32* it_skey = d.sc.it_skey[in_set];
-  u32* list = d.sc.up_seg_start;  // touched entries of this level
   const u64 n = b.n;
   const u32 end = (ni + 31) & ~31u;
   for (u32 x = gtid(); x < end; x += gstride()) {
     const bool valid = x < ni;
     u32 e = 0, rep = 0, c = 0, f = 0, done = 0, cs = 0, sk = 0;
-    bool first = false;
     if (valid) {
       e = d.sc.up_sort_keys0[x] & d.tab.mask;
       rep = it_rep[x];
@@ -1258,51 +1399,8 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
       cs = cf & 0x7FFFFFFFu;
       sk = it_skey[x];
       if (chain_differs(d.tab, e, b.tags, n, rep, l)) raise_err(ctl, ALTO_EINCONSIST);
-      first = atomicExch(&d.tab.hot[e].touch, ep) != ep;
     }
-    {
-      const u32 pos = warp_take(first, &ctl->n_segs[l]);
-      if (first) {
-        if (pos < d.cfg.n_max) list[pos] = e;
-        d.tab.hot[e].acc_rep = rep;
-      }
-    }
-    // lanes past the end form their own group; the whole warp takes part
-    const u32 key = valid ? e : kNone;
-    const u32 peers0 = __match_any_sync(0xFFFFFFFFu, key);
-    if (__all_sync(0xFFFFFFFFu, peers0 == (1u << (threadIdx.x & 31)))) {
-      if (valid) {
-        if (done) {
-          atomicAdd((unsigned long long*)&d.tab.hot[e].acc_cl, 1ull << 40);
-          atomicMax(&d.tab.hot[e].acc_cs1, cs + 1);
-          if (sk) atomicMax(&d.tab.hot[e].acc_smx, sk);
-        }
-        atomicMax(&d.tab.hot[e].acc_m1, c + 1);
-        if (f) {
-          atomicMin(&d.tab.hot[e].acc_fmin, c);
-          atomicMax(&d.tab.hot[e].acc_fmax1, c + 1);
-        }
-      }
-      continue;
-    }
-    {
-      const u32 peers = peers0;
-      const int leader = __ffs(peers) - 1;
-      const u32 cnt = __reduce_add_sync(peers, done);
-      const u32 m1 = __reduce_max_sync(peers, valid ? c + 1 : 0u);
-      const u32 fmin = __reduce_min_sync(peers, (valid && f) ? c : kNone);
-      const u32 fmax1 = __reduce_max_sync(peers, (valid && f) ? c + 1 : 0u);
-      const u32 cs1 = __reduce_max_sync(peers, (valid && done) ? cs + 1 : 0u);
-      const u32 smx = __reduce_max_sync(peers, (valid && done) ? sk : 0u);
-      if (valid && (int)(threadIdx.x & 31) == leader) {
-        if (cnt) atomicAdd((unsigned long long*)&d.tab.hot[e].acc_cl, (unsigned long long)cnt << 40);
-        if (m1) atomicMax(&d.tab.hot[e].acc_m1, m1);
-        if (fmin != kNone) atomicMin(&d.tab.hot[e].acc_fmin, fmin);
-        if (fmax1) atomicMax(&d.tab.hot[e].acc_fmax1, fmax1);
-        if (cs1) atomicMax(&d.tab.hot[e].acc_cs1, cs1);
-        if (smx) atomicMax(&d.tab.hot[e].acc_smx, smx);
-      }
-    }
+    add_items(d, ctl, valid, e, rep, c, f, done, cs, sk, ep, list, &ctl->n_segs[l]);
   }
 }
 
@@ -1310,8 +1408,10 @@ __global__ void __launch_bounds__(kThreads) k_up_accumulate(Dev d, Batch b, int 
 // checks its ancestry against its group's entry and adds itself to the
 // entry's batch accumulators (warp-aggregated over lanes of the same group).
 // 32 registers: eight blocks per SM, so the grid is one wave
-__global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch b) {
+template <bool G>
+__global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch bv) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const int D = d.cfg.depth;
@@ -1393,22 +1493,26 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch b)
 }
 
 // One thread per touched entry: merge, test completion, emit the next items.
-template <bool LEAF>
-__global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l, int in_set) {
+template <bool LEAF, bool G>
+__global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch bv, int l, int in_set,
+                                                          const u32* list, u32* list_next) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
   const int D = d.cfg.depth;
   const bool carry = LEAF && d.cfg.concat_level >= 0;
   const bool receives = !LEAF && chain_parent(d.cfg, l);
   const bool hands_up = chain_level(d.cfg, l);
+  // the level above takes its items right here (no separate accumulate
+  // launch) unless it is a TOPK level, whose items are sorted instead
+  const bool merge = l > 0 && d.cfg.score_op[l - 1] != ALTO_SCORE_TOPK;
   const u32 nt = min(ctl->n_segs[l], d.cfg.n_max);
   const u32 ep = ctl->epoch;
   const u32 ep7 = epoch7(ctl);
   __shared__ u32 s_ins;
   if (threadIdx.x == 0) s_ins = 0;
   __syncthreads();
-  const u32* list = LEAF ? d.sc.leaf_seg_start : d.sc.up_seg_start;
   u32* nx_rep = d.sc.it_rep[in_set ^ 1];
   u32* nx_cseq = d.sc.it_cseq[in_set ^ 1];
   u32* nx_skey = d.sc.it_skey[in_set ^ 1];
@@ -1469,8 +1573,7 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
     // the leaf level allocates the chunks of the reserved growth right here
     if (LEAF && carry) warp_grow(d.tab, d.ar, ctl, grows, e, gv[0], gv[1], gv[2], gv[3]);
     const u32 di = warp_take(complete, &ctl->n_done);
-    if (!valid) continue;
-    if (complete) {
+    if (valid && complete) {
       if (di < d.sc.done_cap) {
         d.sc.done_e[di] = e;
         d.sc.done_lvl[di] = (u32)l;
@@ -1486,21 +1589,33 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch b, int l,
       }
     }
     if (l > 0) {
-      nx_rep[s] = rep;
-      nx_cseq[s] = (complete ? 0x80000000u : 0u) | cmax;
-      nx_skey[s] = smn;
-      // the next level's item is known now: find or insert its parent group
-      const u64 tp = b.tags[(u64)(l - 1) * n + rep];
-      const u64 upp = (l > 1) ? b.tags[(u64)(l - 2) * n + rep] : 0ull;
-      int ins = 0;
-      const u32 e2 = ht_find_or_insert(d.tab, ((u64)(l - 1) << 32) | tag_pid(tp), upp, ctl, &ins,
-                                       b.tags, n, rep, l - 1);
-      if (ins) atomicAdd(&s_ins, 1u);
-      d.sc.up_sort_keys0[s] = (e2 == kNone) ? 0u : e2;
-      if (e2 == kNone) continue;
-      if (ps_insert(d.sc, e2, tag_child(tp), ep7, ctl)) raise_err(ctl, ALTO_EINCONSIST);
-      if (hands_up && complete)
-        chain_reserve(d.tab, e, e2, tag_child(tp), (u64)d.tab.vec_n[2 * (u64)e + 1] + blen);
+      u32 e2 = kNone, c2 = 0, f2 = 0;
+      if (valid) {
+        if (!merge) {
+          nx_rep[s] = rep;
+          nx_cseq[s] = (complete ? 0x80000000u : 0u) | cmax;
+          nx_skey[s] = smn;
+        }
+        // the next level's item is known now: find or insert its parent group
+        const u64 tp = b.tags[(u64)(l - 1) * n + rep];
+        const u64 upp = (l > 1) ? b.tags[(u64)(l - 2) * n + rep] : 0ull;
+        int ins = 0;
+        e2 = ht_find_or_insert(d.tab, ((u64)(l - 1) << 32) | tag_pid(tp), upp, ctl, &ins, b.tags, n, rep,
+                               l - 1, merge);
+        if (ins) atomicAdd(&s_ins, 1u);
+        if (!merge) d.sc.up_sort_keys0[s] = (e2 == kNone) ? 0u : e2;
+        if (e2 != kNone) {
+          c2 = tag_child(tp);
+          f2 = tag_last(tp);
+          if (ps_insert(d.sc, e2, c2, ep7, ctl)) raise_err(ctl, ALTO_EINCONSIST);
+          if (hands_up && complete) chain_reserve(d.tab, e, e2, c2, (u64)d.tab.vec_n[2 * (u64)e + 1] + blen);
+          // an inserter wrote the row from this very fragment's tags
+          if (merge && !ins && chain_differs_ready(d, ctl, e2, b, rep, l - 1)) raise_err(ctl, ALTO_EINCONSIST);
+        }
+      }
+      if (merge)
+        add_items(d, ctl, e2 != kNone, e2, rep, c2, f2, complete ? 1u : 0u, cmax, smn, ep, list_next,
+                  &ctl->n_segs[l - 1]);
     }
   }
   __syncthreads();
@@ -1659,23 +1774,29 @@ struct ChainScan {
   }
 };
 
-__global__ void k_check(Dev d) {
-  pdl_enter();
-  Ctl* ctl = d.ctl;
-  if (poisoned(ctl)) return;
-  bool bad = false;
-  if (ctl->rec_count + ctl->n_done > d.cfg.out_records) bad = true;
-  if (ctl->dense_total + ctl->chain_total > d.cfg.dense_cap) bad = true;
-  if (ctl->topk_count + ctl->topk_total > d.cfg.out_topk) bad = true;
-  if (ctl->n_done > d.sc.done_cap) bad = true;
-  if (bad) {
-    raise_err(ctl, ALTO_ENOSPC);
-    ctl->skip_dense = 1;
+// The batch's output sizes against the capacities, once the record scans
+// have their totals; run by the last CTA of the record-offset scans (volatile
+// reads: other CTAs wrote the totals).
+struct CapCheck {
+  static constexpr bool kActive = true;
+  u64 out_records, dense_cap, out_topk, done_cap;
+  __device__ void operator()(Ctl* ctl) const {
+    volatile Ctl* v = ctl;
+    if (v->status != ALTO_OK || v->abort) return;
+    bool bad = false;
+    if (v->rec_count + v->n_done > out_records) bad = true;
+    if (v->dense_total + v->chain_total > dense_cap) bad = true;
+    if (v->topk_count + v->topk_total > out_topk) bad = true;
+    if (v->n_done > done_cap) bad = true;
+    if (bad) {
+      raise_err(ctl, ALTO_ENOSPC);
+      v->skip_dense = 1;
+    }
+    // allocations of the level kernels may have taken a free stack below zero
+    for (int j = 0; j < kNumChunks; ++j)
+      if (v->top[j] < 0) v->top[j] = 0;
   }
-  // allocations of the level kernels may have taken a free stack below zero
-  for (int j = 0; j < kNumChunks; ++j)
-    if (ctl->top[j] < 0) ctl->top[j] = 0;
-}
+};
 
 // Payload lengths of the leaves in sorted order, scanned: a leaf's position
 // inside its group's new arena data.
@@ -1801,8 +1922,10 @@ __global__ void k_fix_tops(Ctl* ctl) {
 // the spans then copied four at a time, as in the gather, measured slower;
 // so did a warp per carried segment, which leaves a hot group's tens of
 // thousands of leaves to one warp.)
-__global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch b) {
+template <bool G>
+__global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch bv) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (no_copy(ctl)) return;
   const int D = d.cfg.depth;
@@ -1847,8 +1970,10 @@ __global__ void __launch_bounds__(kThreads) k_carry_copy(Dev d, Batch b) {
 
 // Dense child slots of completing CONCAT groups, from this batch's leaves
 // (and, streaming, of the leaves a partial release takes from the batch).
-__global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
+template <bool G>
+__global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch bv) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
   const int D = d.cfg.depth;
@@ -1887,8 +2012,10 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch b) {
 // cursor (one 64-bit atomic: leaf index and payload offset together) and is
 // copied there; a fragment of a group completed by this batch is placed at
 // its dense child slot.
-__global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch b) {
+template <bool G>
+__global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch bv) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (no_copy(ctl)) return;
   const int D = d.cfg.depth;
@@ -2046,6 +2173,10 @@ struct DenseScan {
   const uint4* dense;
   u64* dst;
   Ctl* ctlp;
+  // without levels below M handing spans up, the total is the batch's
+  // payload, checked here against the ring (else k_check2 does it)
+  bool check_payload;
+  u64 out_payload;
   __device__ u64 size(const Ctl* ctl) const {
     return (ctl->skip_dense || ctl->batch_err) ? 0 : ctl->dense_total + ctl->chain_total;
   }
@@ -2061,9 +2192,15 @@ struct DenseScan {
   __device__ void total(Ctl* ctl, u64 t) const {
     dst[size(ctl)] = t;
     ctl->pay_total = t;
+    if (check_payload && !halted(ctl) && !ctl->skip_dense && ctl->pay_count + t > out_payload) {
+      raise_err(ctl, ALTO_ENOSPC);
+      ctl->skip_dense = 1;
+    }
   }
 };
 
+// The payload against the ring when levels below M hand spans up: level M's
+// spans come first, the slots after them are not emitted.
 __global__ void k_check2(Dev d) {
   pdl_enter();
   Ctl* ctl = d.ctl;
@@ -2102,8 +2239,10 @@ constexpr int kSpanLanes = 8;
 constexpr int kSpanFirst = 8;  // elements per lane in the first pass
 
 // 32 registers: eight blocks per SM, the grid is one wave
-__global__ void __launch_bounds__(kThreads, 8) k_gather(Dev d, Batch b) {
+template <bool G>
+__global__ void __launch_bounds__(kThreads, 8) k_gather(Dev d, Batch bv) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
   const int lane = threadIdx.x & 31, sub = lane % kSpanLanes, grp = lane / kSpanLanes;
@@ -2166,8 +2305,10 @@ __global__ void __launch_bounds__(kThreads, 8) k_gather(Dev d, Batch b) {
 // so the level's groups, and their dense slots, form one range.  A warp takes
 // 32 consecutive slots; each lane finds its slot's group by binary search,
 // then the warp copies the spans one after another.
-__global__ void __launch_bounds__(kThreads) k_chain_gather(Dev d, Batch b, int l) {
+template <bool G>
+__global__ void __launch_bounds__(kThreads) k_chain_gather(Dev d, Batch bv, int l) {
   pdl_enter();
+  const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
   const u32 ep = ctl->epoch;
@@ -2449,6 +2590,7 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
         }
       }
       if (!part) {
+        d.tab.ready[e] = 0;
         d.tab.key[e] = kTomb;
         d.tab.cur[e] = 0;  // a slot taken later may receive spans in the launch that inserts it
         atomicAdd(&s_del, 1u);
@@ -2481,11 +2623,27 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
   }
 }
 
+// End of a batch: latch its error, or count its output into the ring.
+__device__ void end_batch(Ctl* ctl) {
+  if (ctl->status != ALTO_OK) return;
+  if (ctl->batch_err) {
+    ctl->status = -(ctl->batch_err & 0xFF);
+    return;
+  }
+  ctl->rec_count += ctl->n_done;
+  ctl->pay_count += ctl->pay_total;
+  ctl->topk_count += ctl->topk_total;
+  ctl->seq_base += ctl->n;
+}
+
 // Turn deleted slots back into free ones where no probe chain runs through
-// them: a tombstone followed (after more tombstones) by a free slot.
+// them: a tombstone followed (after more tombstones) by a free slot.  The
+// batch's records are written by now, so thread 0 also ends the batch (the
+// kernel is the last of a push).
 __global__ void __launch_bounds__(kThreads) k_sweep(Dev d) {
   pdl_enter();
   Ctl* ctl = d.ctl;
+  if (blockIdx.x == 0 && threadIdx.x == 0) end_batch(ctl);
   if (poisoned(ctl)) return;
   const u32 nd = min(ctl->n_done, d.sc.done_cap);
   const u32 mask = d.tab.mask;
@@ -2511,24 +2669,9 @@ __global__ void __launch_bounds__(kThreads) k_sweep(Dev d) {
   }
 }
 
-__global__ void k_end(Ctl* ctl, u32 n) {
+__global__ void k_end(Ctl* ctl) {
   pdl_enter();
-  if (ctl->status != ALTO_OK) return;
-  if (ctl->batch_err) {
-    ctl->status = -(ctl->batch_err & 0xFF);
-    return;
-  }
-  ctl->rec_count += ctl->n_done;
-  ctl->pay_count += ctl->pay_total;
-  ctl->topk_count += ctl->topk_total;
-  ctl->seq_base += n;
-}
-
-__global__ void k_drain_reset(Ctl* ctl) {
-  pdl_enter();
-  ctl->rec_count = 0;
-  ctl->pay_count = 0;
-  ctl->topk_count = 0;
+  end_batch(ctl);
 }
 
 }  // namespace alto
@@ -2570,6 +2713,25 @@ struct alto_agg {
   int64_t stage_launches[ALTO_NUM_STAGES];
   std::vector<cudaEvent_t> ev_free;                   // reusable events
   std::vector<std::vector<cudaEvent_t>> ev_pending;  // per push: stage boundaries
+  // Pushes of up to kGraphMaxBatch fragments replay a CUDA graph of the
+  // push's launch sequence, captured once per (output ring, profiling mode):
+  // one launch from the host instead of twenty-odd.  Only the first node's
+  // parameters (the batch) and, when profiling, the events of the
+  // event-record nodes change from push to push.
+  struct PushGraph {
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    cudaGraphNode_t begin = nullptr;                 // k_begin
+    std::vector<cudaGraphNode_t> ev_node;            // per stage boundary (null: none)
+    int64_t launches = 0;                            // kernels of one replay
+    int64_t stage_launches[ALTO_NUM_STAGES] = {};
+    bool failed = false;                             // capture failed: launch directly
+  };
+  PushGraph graphs[2][3];  // [ring][profiling: off, stages, hot]
+  cudaStream_t cap_stream = nullptr;
+  std::vector<cudaEvent_t> cap_events;  // recorded at capture only (the graphs' templates hold them)
+  bool direct_only = false;   // ALTO_FLAG_DIRECT_LAUNCH
+  bool reset_pending = false; // a drain handed out the ring: the next push resets its counters
 };
 
 namespace {
@@ -2581,6 +2743,7 @@ struct StageClock {
   std::vector<cudaEvent_t> ev;
   int stage = 0;
   int launches_at_start = 0;
+  bool capturing = false;
   StageClock(alto_agg* h_, cudaStream_t s_) : h(h_), s(s_) {}
   cudaEvent_t take() {
     cudaEvent_t e;
@@ -2602,15 +2765,15 @@ struct StageClock {
       cudaEvent_t e = nullptr;
       if (h->profile_mode == ALTO_PROFILE_STAGES || bnd == 2 || bnd == 3 || bnd == 8 || bnd == 9) {
         e = take();
-        if (e) cudaEventRecord(e, s);
+        // inside a stream capture only an external record becomes an
+        // event-record node (a plain one just orders captured streams)
+        if (e) {
+          if (capturing) cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
+          else cudaEventRecord(e, s);
+        }
       }
       ev.push_back(e);
     }
-  }
-  void finish() {
-    if (!h->profiling) return;
-    enter(ALTO_NUM_STAGES);
-    h->ev_pending.push_back(ev);
   }
 };
 
@@ -2633,17 +2796,17 @@ LookbackState lb_region(const LookbackState& lb, int k) {
   return r;
 }
 
-template <class F>
+template <class F, class L>
 void launch_scan3(const LookbackState& lb, Ctl* ctl, const F& f0, const F& f1,
-                  const F& f2, u64 cap, int site, u64 spin, cudaStream_t s) {
+                  const F& f2, u64 cap, int site, u64 spin, cudaStream_t s, const L& last) {
   u64 tiles = (cap + kScanTile - 1) / kScanTile;
   if (tiles == 0) tiles = 1;
   // the record scans run over completed groups (far fewer than fragments):
   // a small persistent grid, so that hundreds of idle CTAs do not contend on
   // the tile and exit counters
   dim3 grid((unsigned)std::min<u64>(tiles, 32), 3);
-  launch_pdl(k_scan3<F>, grid, kScanThreads, 0, s, f0, f1, f2, lb_region(lb, 0), lb_region(lb, 1),
-                                           lb_region(lb, 2), ctl, site, spin);
+  launch_pdl(k_scan3<F, L>, grid, kScanThreads, 0, s, f0, f1, f2, lb_region(lb, 0), lb_region(lb, 1),
+             lb_region(lb, 2), ctl, site, spin, last);
 }
 
 template <class F>
@@ -2658,8 +2821,8 @@ void launch_scan(const LookbackState& lb, int num_sms, Ctl* ctl, const F& f, u64
   launch_pdl(k_scan<F>, grid, kScanThreads, 0, s, f, lb, ctl, site, &ctl->exit_ctr[site], spin);
 }
 
-// What one batch enqueues between k_begin and k_end, for the handle's push
-// and for the one-shot entry point alike.  `stage` (may be null) marks the
+// What one batch enqueues after k_begin, for the handle's push and for the
+// one-shot entry point alike (its last kernel, k_sweep, also ends the batch).  `stage` (may be null) marks the
 // start of each profiling stage; `launches` counts the kernels.
 struct Pipeline {
   Dev d;
@@ -2693,6 +2856,7 @@ int blocks_per_sm(const void* kernel) {
   return nb;
 }
 
+template <bool G>
 void enqueue_batch(Pipeline& p, const Batch& bt) {
   Dev d = p.d;
   cudaStream_t s = p.s;
@@ -2704,11 +2868,14 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   const u64 spin = d.cfg.spin_limit;
   int sl = 0;  // launches inside sort_pairs
   int site = 0;
-  launch_pdl(k_ingest, grid, kThreads, 0, s, d, bt);
+  launch_pdl(k_ingest<G>, grid, kThreads, 0, s, d, bt);
   p.launches += 1;
   // streaming release needs each leaf parent's leaves together: the sorted path
   const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK || d.cfg.stream;
   int set = 0;
+  // touched entries of consecutive levels, alternately
+  u32* lists[2] = {d.sc.up_seg_start, d.sc.up_list2};
+  int li = 0;
   if (leaf_sorted) {
     // leaf level with TOPK: sort fragments by their leaf-parent group so that
     // each group's candidates are contiguous for the segmented top-k
@@ -2723,13 +2890,13 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     SegFind f{d.sc.leaf_keys, d.sc.leaf_seg_start, d.sc.leaf_seg_of, &d.ctl->n, nmax,
               &d.ctl->n_segs[D - 1]};
     launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site + 4, spin, s);
-    launch_pdl(k_reduce<true>, p.num_sms * blocks_per_sm((const void*)k_reduce<true>), kThreads, 0, s, d, bt,
+    launch_pdl(k_reduce<true, G>, p.num_sms * blocks_per_sm((const void*)k_reduce<true, G>), kThreads, 0, s, d, bt,
                D - 1, d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
-    launch_pdl(k_reduce_big<true>, p.num_sms, kBigThreads, 0, s, d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
+    launch_pdl(k_reduce_big<true, G>, p.num_sms, kBigThreads, 0, s, d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
                d.sc.leaf_seg_start, set);
     p.launches += 3;
     if (d.cfg.stream) {
-      launch_pdl(k_reduce_rel, p.num_sms * blocks_per_sm((const void*)k_reduce_rel), kThreads, 0, s, d, bt,
+      launch_pdl(k_reduce_rel<G>, p.num_sms * blocks_per_sm((const void*)k_reduce_rel<G>), kThreads, 0, s, d, bt,
                  d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
       p.launches += 1;
     }
@@ -2737,29 +2904,39 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     // leaf level without TOPK: accumulate into the table in arrival order
     // (plain stream order: the measurement hooks time this kernel on its own)
     p.enter(2);
-    k_leaf_accumulate<<<grid, kThreads, 0, s>>>(d, bt);
+    k_leaf_accumulate<G><<<grid, kThreads, 0, s>>>(d, bt);
     p.enter(3);
-    launch_pdl(k_up_finalize<true>, sgrid, kThreads, 0, s, d, bt, D - 1, set);
+    launch_pdl(k_up_finalize<true, G>, sgrid, kThreads, 0, s, d, bt, D - 1, set,
+               (const u32*)d.sc.leaf_seg_start, lists[li]);
     p.launches += 2;
   }
   site += 5;
   p.enter(4);
-  // an atomic finalize also looks up the parent groups of the items it emits
+  // an atomic finalize looks up the parent groups of the items it emits and,
+  // unless the level above is TOPK, adds the items to them as well
   bool looked_up = !leaf_sorted;
+  bool added = !leaf_sorted && D >= 2 && d.cfg.score_op[D - 2] != ALTO_SCORE_TOPK;
   for (int l = D - 2; l >= 0; --l) {
     set ^= 1;  // items written by the level below
     if (!looked_up) {
-      launch_pdl(k_items_lookup, sgrid, kThreads, 0, s, d, bt, l, set);
+      launch_pdl(k_items_lookup<G>, sgrid, kThreads, 0, s, d, bt, l, set);
       p.launches += 1;
     }
     if (d.cfg.score_op[l] != ALTO_SCORE_TOPK) {
-      launch_pdl(k_up_accumulate, sgrid, kThreads, 0, s, d, bt, l, set);
-      launch_pdl(k_up_finalize<false>, sgrid, kThreads, 0, s, d, bt, l, set);
-      p.launches += 2;
+      if (!added) {
+        launch_pdl(k_up_accumulate<G>, sgrid, kThreads, 0, s, d, bt, l, set, lists[li]);
+        p.launches += 1;
+      }
+      launch_pdl(k_up_finalize<false, G>, sgrid, kThreads, 0, s, d, bt, l, set, (const u32*)lists[li],
+                 lists[li ^ 1]);
+      p.launches += 1;
+      li ^= 1;
       looked_up = true;
+      added = l > 0 && d.cfg.score_op[l - 1] != ALTO_SCORE_TOPK;
       continue;
     }
     looked_up = false;
+    added = false;
     int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nmax, p.tbits, true, *p.up_sort, d.ctl, site, spin,
                         p.num_sms, s, &sl);
     p.launches += sl;
@@ -2770,9 +2947,9 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     SegFind f{d.sc.up_keys, d.sc.up_seg_start, nullptr, &d.ctl->n_segs[l + 1], nmax,
               &d.ctl->n_segs[l]};
     launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site++, spin, s);
-    launch_pdl(k_reduce<false>, p.num_sms * blocks_per_sm((const void*)k_reduce<false>), kThreads, 0, s, d,
+    launch_pdl(k_reduce<false, G>, p.num_sms * blocks_per_sm((const void*)k_reduce<false, G>), kThreads, 0, s, d,
                bt, l, d.sc.up_keys, d.sc.up_perm, d.sc.up_seg_start, set);
-    launch_pdl(k_reduce_big<false>, p.num_sms, kBigThreads, 0, s, d, bt, l, d.sc.up_keys, d.sc.up_perm,
+    launch_pdl(k_reduce_big<false, G>, p.num_sms, kBigThreads, 0, s, d, bt, l, d.sc.up_keys, d.sc.up_perm,
                d.sc.up_seg_start, set);
     p.launches += 3;
   }
@@ -2785,17 +2962,19 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   launch_pdl(k_done_rank, sgrid, kThreads, 0, s, d);
   p.launches += 2;
   const u32 dcap = d.sc.done_cap;
+  const bool chain = M >= 0 && M < D - 1;  // levels below M hand spans up
   {
     CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0,
                  d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask,
                  (M == D - 1) ? d.tab.bstate : nullptr, d.ctl};
     CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
     CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
-    launch_scan3(p.lbs, d.ctl, f0, f1, f2, dcap, site, spin, s);
+    const CapCheck cc{d.cfg.out_records, d.cfg.dense_cap, d.cfg.out_topk, d.sc.done_cap};
+    if (chain) launch_scan3(p.lbs, d.ctl, f0, f1, f2, dcap, site, spin, s, NoLast());
+    else launch_scan3(p.lbs, d.ctl, f0, f1, f2, dcap, site, spin, s, cc);
     p.launches += 1;
     site += 3;
   }
-  const bool chain = M >= 0 && M < D - 1;
   if (chain) {
     ChainScan c[3];
     for (int k = 0; k < 3; ++k) {
@@ -2811,24 +2990,23 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
       c[k].M = M;
       c[k].L = D - 1;
     }
-    launch_scan3(p.lbs, d.ctl, c[0], c[1], c[2], dcap, site, spin, s);
+    launch_scan3(p.lbs, d.ctl, c[0], c[1], c[2], dcap, site, spin, s,
+                 CapCheck{d.cfg.out_records, d.cfg.dense_cap, d.cfg.out_topk, d.sc.done_cap});
     p.launches += 1;
     site += 3;
   }
-  launch_pdl(k_check, 1, 1, 0, s, d);
-  p.launches += 1;
   if (M >= 0) {
     p.enter(6);
     if (leaf_sorted) {
       launch_pdl(k_carry_alloc, sgrid, kThreads, 0, s, d);
       launch_pdl(k_fix_tops, 1, 32, 0, s, d.ctl);
-      launch_pdl(k_carry_copy, grid, kThreads, 0, s, d, bt);
+      launch_pdl(k_carry_copy<G>, grid, kThreads, 0, s, d, bt);
       p.enter(7);
-      launch_pdl(k_dense_batch, grid, kThreads, 0, s, d, bt);
+      launch_pdl(k_dense_batch<G>, grid, kThreads, 0, s, d, bt);
     } else {
       // the leaf finalize already allocated the carried leaves' chunks
       p.enter(7);
-      launch_pdl(k_leaf_place, grid, kThreads, 0, s, d, bt);
+      launch_pdl(k_leaf_place<G>, grid, kThreads, 0, s, d, bt);
     }
     launch_pdl(k_dense_arena<true>, sgrid, kThreads, 0, s, d);
     p.launches += leaf_sorted ? 5 : 2;
@@ -2836,20 +3014,23 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
       launch_pdl(k_dense_arena<false>, sgrid, kThreads, 0, s, d);
       p.launches += 1;
     }
-    DenseScan fd{d.sc.dense, d.sc.dst, d.ctl};
+    DenseScan fd{d.sc.dense, d.sc.dst, d.ctl, !chain, d.cfg.out_payload};
     launch_scan(p.lbs, p.num_sms, d.ctl, fd, d.cfg.dense_cap, site++, spin, s);
-    launch_pdl(k_check2, 1, 1, 0, s, d);
-    p.launches += 2;
+    p.launches += 1;
+    if (chain) {
+      launch_pdl(k_check2, 1, 1, 0, s, d);
+      p.launches += 1;
+    }
     p.enter(8);
     // levels below M hand their concatenations up, deepest first
     for (int l = D - 1; chain && l > M; --l) {
-      launch_pdl(k_chain_gather, p.num_sms * blocks_per_sm((const void*)k_chain_gather), kThreads, 0, s, d,
+      launch_pdl(k_chain_gather<G>, p.num_sms * blocks_per_sm((const void*)k_chain_gather<G>), kThreads, 0, s, d,
                  bt, l);
       p.launches += 1;
     }
     // plain stream order (no programmatic overlap with its neighbours): the
     // gather is the stage the measurement hooks time on their own
-    k_gather<<<p.num_sms * blocks_per_sm((const void*)k_gather), kThreads, 0, s>>>(d, bt);
+    k_gather<G><<<p.num_sms * blocks_per_sm((const void*)k_gather<G>), kThreads, 0, s>>>(d, bt);
     p.launches += 1;
   }
   p.enter(9);
@@ -2874,6 +3055,141 @@ void* dev_alloc(alto_agg* h, size_t bytes, cudaStream_t s) {
   }
   if (p) h->blocks.push_back(p);
   return p;
+}
+
+// Pushes of at most this many fragments replay the captured graph (host
+// launch cost matters there); larger ones launch kernel by kernel, whose
+// kernels read the batch from their parameters rather than device memory.
+constexpr u32 kGraphMaxBatch = 1u << 17;
+
+// Stage bookkeeping of one push's launch sequence: kernels per stage, and the
+// stage-boundary events when profiling.
+struct PushRec {
+  alto_agg* h;
+  StageClock clk;
+  int stage = 0;
+  int64_t l0 = 0;
+  int64_t stage_l[ALTO_NUM_STAGES] = {};
+  PushRec(alto_agg* h_, cudaStream_t s) : h(h_), clk(h_, s) {}
+};
+
+// The whole launch sequence of one push on stream s: k_begin and the
+// pipeline.  G: the kernels read the batch that k_begin stores (graph capture).
+// Returns the number of kernels.
+template <bool G>
+int64_t launch_push(alto_agg* h, cudaStream_t s, const Batch& bt, int reset, PushRec* rec) {
+  Dev d = h->d;
+  Pipeline p;
+  p.d = d;
+  p.leaf_sort = &h->leaf_sort;
+  p.up_sort = &h->up_sort;
+  p.lbs = h->lbs;
+  p.num_sms = h->num_sms;
+  p.tbits = h->tbits;
+  p.nmax = (u32)h->cfg.max_batch_fragments;
+  p.s = s;
+  p.stage = [](void* ctx, int st, int64_t launches) {
+    PushRec* r = (PushRec*)ctx;
+    r->stage_l[r->stage] += launches - r->l0;
+    r->l0 = launches;
+    r->stage = st;
+    r->clk.enter(st);
+  };
+  p.stage_ctx = rec;
+  rec->clk.enter(0);
+  launch_pdl(k_begin, 1, 1, 0, s, d.ctl, bt, d.sc.batch, reset);
+  p.launches += 1;
+  enqueue_batch<G>(p, bt);  // its last kernel also ends the batch
+  p.enter(ALTO_NUM_STAGES);
+  rec->clk.enter(ALTO_NUM_STAGES);
+  return p.launches;
+}
+
+// Capture the launch sequence of a push for the handle's current output ring
+// and profiling mode, on the handle's own stream (nothing runs), and
+// instantiate it.  Every replay sets the parameters of the k_begin node; a
+// profiling capture also holds one event-record node per timed stage
+// boundary, whose event every replay replaces.  On any failure the graph is marked failed and pushes of that
+// kind launch directly.
+bool capture_push(alto_agg* h, alto_agg::PushGraph& g) {
+  g.failed = true;
+  if (!h->cap_stream && cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess) {
+    h->cap_stream = nullptr;
+    cudaGetLastError();
+    return false;
+  }
+  Batch ph;  // k_begin's parameters of the capture; every replay sets its own
+  ph.tags = nullptr;
+  ph.off = nullptr;
+  ph.pay = nullptr;
+  ph.score = nullptr;
+  ph.n = 0;
+  ph.n_payload = 0;
+  if (cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeRelaxed) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  PushRec rec(h, h->cap_stream);
+  rec.clk.capturing = true;
+  const int64_t launches = launch_push<true>(h, h->cap_stream, ph, 0, &rec);
+  for (cudaEvent_t e : rec.clk.ev)
+    if (e) h->cap_events.push_back(e);
+  cudaGraph_t graph = nullptr;
+  if (cudaStreamEndCapture(h->cap_stream, &graph) != cudaSuccess || graph == nullptr) {
+    cudaGetLastError();
+    if (graph) cudaGraphDestroy(graph);
+    return false;
+  }
+  size_t nn = 0;
+  cudaGraphGetNodes(graph, nullptr, &nn);
+  std::vector<cudaGraphNode_t> nodes(nn);
+  if (nn) cudaGraphGetNodes(graph, nodes.data(), &nn);
+  cudaGraphNode_t begin = nullptr;
+  g.ev_node.assign(rec.clk.ev.size(), nullptr);
+  for (cudaGraphNode_t nd : nodes) {
+    cudaGraphNodeType ty;
+    if (cudaGraphNodeGetType(nd, &ty) != cudaSuccess) continue;
+    if (ty == cudaGraphNodeTypeKernel) {
+      cudaKernelNodeParams kp;
+      if (cudaGraphKernelNodeGetParams(nd, &kp) == cudaSuccess && kp.func == (void*)k_begin) begin = nd;
+    } else if (ty == cudaGraphNodeTypeEventRecord) {
+      cudaEvent_t e = nullptr;
+      if (cudaGraphEventRecordNodeGetEvent(nd, &e) != cudaSuccess) continue;
+      for (size_t b = 0; b < rec.clk.ev.size(); ++b)
+        if (rec.clk.ev[b] == e) g.ev_node[b] = nd;
+    }
+  }
+  cudaGetLastError();
+  if (begin == nullptr) {
+    cudaGraphDestroy(graph);
+    return false;
+  }
+  cudaGraphExec_t exec = nullptr;
+  if (cudaGraphInstantiate(&exec, graph, 0) != cudaSuccess || exec == nullptr) {
+    cudaGetLastError();
+    cudaGraphDestroy(graph);
+    return false;
+  }
+  g.graph = graph;
+  g.exec = exec;
+  g.begin = begin;
+  g.launches = launches;
+  for (int i = 0; i < ALTO_NUM_STAGES; ++i) g.stage_launches[i] = rec.stage_l[i];
+  g.failed = false;
+  return true;
+}
+
+void free_graphs(alto_agg* h) {
+  for (auto& row : h->graphs)
+    for (auto& g : row) {
+      if (g.exec) cudaGraphExecDestroy(g.exec);
+      if (g.graph) cudaGraphDestroy(g.graph);
+      g = alto_agg::PushGraph();
+    }
+  for (cudaEvent_t e : h->cap_events) cudaEventDestroy(e);
+  h->cap_events.clear();
+  if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
+  h->cap_stream = nullptr;
 }
 
 void free_all(alto_agg* h, cudaStream_t s) {
@@ -2910,7 +3226,8 @@ alto_status validate(const alto_agg_config* c) {
       return ALTO_EINVAL;
   }
   if (nconcat > 1) return ALTO_EINVAL;
-  if (c->flags & ~(int64_t)(ALTO_FLAG_STREAM_RELEASE | ALTO_FLAG_DOUBLE_RING | ALTO_FLAG_TEST_STALL))
+  if (c->flags & ~(int64_t)(ALTO_FLAG_STREAM_RELEASE | ALTO_FLAG_DOUBLE_RING | ALTO_FLAG_TEST_STALL |
+                            ALTO_FLAG_DIRECT_LAUNCH))
     return ALTO_EINVAL;
   // streaming release needs the CONCAT level at the leaf parent
   if ((c->flags & ALTO_FLAG_STREAM_RELEASE) && c->payload_op[c->depth - 1] != ALTO_PAYLOAD_CONCAT)
@@ -2957,6 +3274,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   h->latched = ALTO_OK;
   h->profiling = false;
   h->profile_mode = ALTO_PROFILE_STAGES;
+  h->direct_only = (cfg.flags & ALTO_FLAG_DIRECT_LAUNCH) != 0;
   h->last_stream = s;
   h->prof_pushes = 0;
   h->launches = 0;
@@ -3008,6 +3326,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(d.tab.cur, u64, T);
   ALLOC(d.tab.dbase, u64, T);
   ALLOC(d.tab.bstate, uint4, T);
+  ALLOC(d.tab.ready, u32, T);
   const bool strm = (cfg.flags & ALTO_FLAG_STREAM_RELEASE) != 0;
   if (strm) {
     ALLOC(d.tab.rel, u32, T);
@@ -3066,6 +3385,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   ALLOC(sc.leaf_seg_start, u32, nmax + 1);
   ALLOC(sc.leaf_seg_of, u32, nmax);
   ALLOC(sc.up_seg_start, u32, nmax + 1);
+  ALLOC(sc.up_list2, u32, nmax);
   for (int b = 0; b < 2; ++b) {
     ALLOC(sc.it_rep[b], u32, nmax);
     ALLOC(sc.it_cseq[b], u32, nmax);
@@ -3101,6 +3421,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     ALLOC(d.tab.app, u64, T);
   }
   ALLOC(sc.pairset, u64, PS);
+  ALLOC(sc.batch, Batch, 1);
   sc.big_cap = (u32)(nmax / kBigSeg + 1);
   ALLOC(sc.big_seg, u32, (u64)D * sc.big_cap);
   sc.ps_mask = PS - 1;
@@ -3151,7 +3472,9 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     cudaMemcpyAsync(&d.ctl->test_stall, &kOne, sizeof(int), cudaMemcpyHostToDevice, s);
   }
   cudaMemsetAsync(d.tab.key, 0xFF, sizeof(u64) * T, s);
-  cudaMemsetAsync(d.tab.hot, 0, sizeof(Hot) * T, s);
+  cudaMemsetAsync(d.tab.ready, 0, sizeof(u32) * T, s);
+  launch_pdl(k_init_hot, (int)std::min<u64>((T + kThreads - 1) / kThreads, (u64)h->num_sms * 8), kThreads, 0, s,
+             d.tab.hot, T);
   cudaMemsetAsync(d.tab.cur, 0, sizeof(u64) * T, s);
   cudaMemsetAsync(sc.mask, 0, sizeof(u32) * ((nmax + 31) / 32 * 32), s);
   cudaMemsetAsync(sc.mblk, 0, sizeof(u32) * (nmax / 32 + 1), s);
@@ -3203,40 +3526,50 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
   h->pushed += 1;
   h->last_stream = s;
   if (h->profiling) h->prof_pushes += 1;
-  struct Clock {
-    alto_agg* h;
-    StageClock clk;
-    int stage;
-    int64_t l0;
-  } ck{h, StageClock(h, s), 0, 0};
-  auto on_stage = [](void* ctx, int st, int64_t launches) {
-    Clock* c = (Clock*)ctx;
-    if (c->h->profiling) c->h->stage_launches[c->stage] += launches - c->l0;
-    c->l0 = launches;
-    c->stage = st;
-    c->clk.enter(st);
-  };
-  Pipeline p;
-  p.d = d;
-  p.leaf_sort = &h->leaf_sort;
-  p.up_sort = &h->up_sort;
-  p.lbs = h->lbs;
-  p.num_sms = h->num_sms;
-  p.tbits = h->tbits;
-  p.nmax = (u32)cfg.max_batch_fragments;
-  p.s = s;
-  p.stage = on_stage;
-  p.stage_ctx = &ck;
-  ck.clk.enter(0);
-  launch_pdl(k_begin, 1, 1, 0, s, d.ctl, n);
-  p.launches += 1;
-  if (n > 0) enqueue_batch(p, bt);
-  else p.enter(9);
-  launch_pdl(k_end, 1, 1, 0, s, d.ctl, n);
-  p.launches += 1;
-  p.enter(ALTO_NUM_STAGES);
-  ck.clk.finish();
-  h->launches += p.launches;
+  const int reset = h->reset_pending ? 1 : 0;
+  h->reset_pending = false;
+  if (!h->direct_only && n <= kGraphMaxBatch) {
+    const int pm = !h->profiling ? 0 : (h->profile_mode == ALTO_PROFILE_HOT ? 2 : 1);
+    alto_agg::PushGraph& g = h->graphs[h->ring_cur][pm];
+    if (g.exec == nullptr && !g.failed) capture_push(h, g);
+    if (g.exec != nullptr) {
+      // this push's batch (and counter reset) as k_begin's parameters
+      Ctl* ctl = d.ctl;
+      Batch* store = d.sc.batch;
+      int rst = reset;
+      void* args[] = {&ctl, &bt, &store, &rst};
+      cudaKernelNodeParams kp;
+      memset(&kp, 0, sizeof(kp));
+      kp.func = (void*)k_begin;
+      kp.gridDim = dim3(1);
+      kp.blockDim = dim3(1);
+      kp.kernelParams = args;
+      if (cudaGraphExecKernelNodeSetParams(g.exec, g.begin, &kp) != cudaSuccess) return ALTO_ECUDA;
+      if (pm) {
+        // fresh events at the timed stage boundaries
+        StageClock clk(h, s);
+        std::vector<cudaEvent_t> ev(g.ev_node.size(), nullptr);
+        for (size_t k = 0; k < ev.size(); ++k) {
+          if (!g.ev_node[k]) continue;
+          ev[k] = clk.take();
+          if (ev[k] && cudaGraphExecEventRecordNodeSetEvent(g.exec, g.ev_node[k], ev[k]) != cudaSuccess)
+            return ALTO_ECUDA;
+        }
+        h->ev_pending.push_back(ev);
+        for (int i = 0; i < ALTO_NUM_STAGES; ++i) h->stage_launches[i] += g.stage_launches[i];
+      }
+      if (cudaGraphLaunch(g.exec, s) != cudaSuccess) return ALTO_ECUDA;
+      h->launches += g.launches;
+      return ALTO_OK;
+    }
+  }
+  PushRec rec(h, s);
+  const int64_t launches = launch_push<false>(h, s, bt, reset, &rec);
+  if (h->profiling) {
+    h->ev_pending.push_back(rec.clk.ev);
+    for (int i = 0; i < ALTO_NUM_STAGES; ++i) h->stage_launches[i] += rec.stage_l[i];
+  }
+  h->launches += launches;
   if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
   return ALTO_OK;
 }
@@ -3256,11 +3589,14 @@ alto_status alto_agg_drain(alto_agg_t* h, void* stream, alto_drain* out) {
     h->latched = c.status;
     return c.status;
   }
-  out->n_records = (int64_t)c.rec_count;
+  // the output counters are reset by the next push that launches work (its
+  // first kernel); until then nothing new has been completed
+  const bool fresh = !h->reset_pending;
+  out->n_records = fresh ? (int64_t)c.rec_count : 0;
   out->records = h->d.out_rec;
-  out->n_payload = (int64_t)c.pay_count;
+  out->n_payload = fresh ? (int64_t)c.pay_count : 0;
   out->payload = h->d.out_pay;
-  out->n_topk = (int64_t)c.topk_count;
+  out->n_topk = fresh ? (int64_t)c.topk_count : 0;
   out->topk = h->d.out_topk;
   if (h->ring_rec[1] != nullptr) {
     // later pushes fill the other ring while the caller reads this one
@@ -3269,8 +3605,7 @@ alto_status alto_agg_drain(alto_agg_t* h, void* stream, alto_drain* out) {
     h->d.out_pay = h->ring_pay[h->ring_cur];
     h->d.out_topk = h->ring_topk[h->ring_cur];
   }
-  launch_pdl(k_drain_reset, 1, 1, 0, s, h->d.ctl);
-  if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
+  h->reset_pending = true;
   return ALTO_OK;
 }
 
@@ -3324,6 +3659,7 @@ alto_status alto_agg_destroy(alto_agg_t* h) {
     for (cudaEvent_t e : ev)
       if (e) cudaEventDestroy(e);
   for (cudaEvent_t e : h->ev_free) cudaEventDestroy(e);
+  free_graphs(h);
   free_all(h, nullptr);
   cudaDeviceSynchronize();
   delete h;
@@ -3431,6 +3767,7 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   d.tab.cur = cv.take<u64>(T);
   d.tab.dbase = cv.take<u64>(T);
   d.tab.bstate = cv.take<uint4>(T);
+  d.tab.ready = cv.take<u32>(T);
   d.tab.leaf_level = D - 1;
   d.tab.mask = (u32)(T - 1);
   d.tab.kk = kk;
@@ -3476,6 +3813,7 @@ void na_layout(const alto_agg_config& cfg, unsigned char* base, NaState& st, NaC
   sc.leaf_seg_start = cv.take<u32>(nmax + 1);
   sc.leaf_seg_of = cv.take<u32>(nmax);
   sc.up_seg_start = cv.take<u32>(nmax + 1);
+  sc.up_list2 = cv.take<u32>(nmax);
   for (int b = 0; b < 2; ++b) {
     sc.it_rep[b] = cv.take<u32>(nmax);
     sc.it_cseq[b] = cv.take<u32>(nmax);
@@ -3548,6 +3886,7 @@ __global__ void k_na_reset(Dev d, u32* hist, u64 T, u64 PS, u32 nmax) {
     hw[2] = make_uint4(kNone, 0, 0, 0);
     hw[3] = make_uint4(0, 0, 0, 0);
     d.tab.cur[i] = 0;
+    d.tab.ready[i] = 0;
   }
   for (u64 i = tid; i < PS; i += stride) d.sc.pairset[i] = 0;
   for (u64 i = tid; i < (nmax + 31) / 32 * 32; i += stride) d.sc.mask[i] = 0;
@@ -3640,7 +3979,7 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
   bt.n_payload = (u64)b->n_payload;
 
   launch_pdl(k_na_reset, num_sms * 2, kThreads, 0, s, d, st.leaf_sort.hist, st.T, st.PS, nmax);
-  launch_pdl(k_begin, 1, 1, 0, s, d.ctl, n);
+  launch_pdl(k_begin, 1, 1, 0, s, d.ctl, bt, (Batch*)nullptr, 0);
   if (n > 0) {
     Pipeline p;
     p.d = d;
@@ -3651,9 +3990,10 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
     p.tbits = st.tbits;
     p.nmax = nmax;
     p.s = s;
-    enqueue_batch(p, bt);
+    enqueue_batch<false>(p, bt);  // its last kernel also ends the batch
+  } else {
+    launch_pdl(k_end, 1, 1, 0, s, d.ctl);
   }
-  launch_pdl(k_end, 1, 1, 0, s, d.ctl, n);
   launch_pdl(k_na_finish, 1, 1, 0, s, d.ctl, out_counts);
   if (cudaGetLastError() != cudaSuccess) return ALTO_ECUDA;
   return ALTO_OK;

@@ -42,6 +42,7 @@ struct Ctl {
   int top[kNumChunks];     // free-chunk stack heights per class
   u32 tile_ctr[kSites];    // dynamic tile counters per launch site
   u32 exit_ctr[kSites];    // CTAs finished per launch site (resets tile_ctr)
+  u32 last_ctr;            // CTAs finished in a multi-scan launch with a last-CTA step
   // per batch (device-computed sizes that later kernels read)
   u32 n;                   // fragments in the batch
   u32 n_items[kMaxDepth];  // items entering level l
@@ -147,7 +148,9 @@ __device__ __forceinline__ u64 chunk_size(int j) { return 1ull << (kChunk0Log + 
 // The fields of an open-group entry that the level kernels read and write
 // together, in one 64-byte record (one access brings them all; a
 // structure-of-arrays table spread them over a dozen cache lines).  The
-// batch accumulators are zero between batches (acc_fmin: kNone).
+// batch accumulators are zero between batches (acc_fmin: kNone), also in
+// free slots, so an insert made while other threads may already add to the
+// new entry (a publishing insert) leaves them, and `touch`, alone.
 struct __align__(64) Hot {
   u64 up;          // tag one level up
   u32 last;        // last child index or kNone
@@ -193,6 +196,10 @@ struct Table {
   // the release of the current batch ends (a partial or the final record)
   u32* rel;        // [T]
   u32* rnew;       // [T]
+  // [T] 1 once a publishing insert has written the entry's chain row (0
+  // while the slot is free): a finder in the launch that inserts the entry
+  // compares ancestry only after that
+  u32* ready;
   int leaf_level;  // D - 1
   int chain_len;   // D - 1, rounded up to even
   u32 mask;        // T - 1

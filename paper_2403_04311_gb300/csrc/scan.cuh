@@ -254,17 +254,35 @@ __global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ct
   scan_body(f, st, ctl, site, exit_ctr, spin_limit);
 }
 
+// No work after the last CTA of a multi-scan launch.
+struct NoLast {
+  static constexpr bool kActive = false;
+  __device__ void operator()(Ctl*) const {}
+};
+
 // Three independent scans in one launch: blockIdx.y selects the scan, each
 // with its own launch site (tile and exit counters) and look-back arrays.
-template <class F>
+// When L is active, the launch's last CTA to finish runs `last` once every
+// scan's total is written (so a check of the totals needs no launch of its
+// own); it must read what other CTAs wrote with volatile loads.
+template <class F, class L>
 __global__ void __launch_bounds__(kScanThreads) k_scan3(F f0, F f1, F f2, LookbackState st0,
                                                         LookbackState st1, LookbackState st2,
-                                                        Ctl* ctl, int site, u64 spin_limit) {
+                                                        Ctl* ctl, int site, u64 spin_limit, L last) {
   pdl_enter();
   const int y = blockIdx.y;
   const F& f = (y == 0) ? f0 : (y == 1) ? f1 : f2;
   const LookbackState st = (y == 0) ? st0 : (y == 1) ? st1 : st2;
   scan_body(f, st, ctl, site + y, &ctl->exit_ctr[site + y], spin_limit);
+  if (L::kActive && threadIdx.x == 0) {
+    __threadfence();
+    const u32 k = atomicAdd(&ctl->last_ctr, 1u);
+    if (k == gridDim.x * gridDim.y - 1) {
+      ctl->last_ctr = 0;
+      __threadfence();
+      last(ctl);
+    }
+  }
 }
 
 }  // namespace alto

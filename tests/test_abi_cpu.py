@@ -60,7 +60,7 @@ def _cfg(**kw):
     dict(arena_elems=1 << 32),
     dict(payload_op=[1, 0], stream_release=True),    # streaming release above the leaf parent
     dict(payload_op=[0, 0], stream_release=True),    # streaming release without CONCAT
-    dict(flags=8),                                   # unknown flag
+    dict(flags=16),                                  # unknown flag
 ])
 def test_create_rejects_bad_configs_on_host(bad):
     lib = alto.load_library()
@@ -75,7 +75,7 @@ def test_create_rejects_bad_configs_on_host(bad):
     assert h.value == 12345  # untouched
 
 
-@pytest.mark.parametrize("flag", ["stream_release", "double_ring", "test_stall"])
+@pytest.mark.parametrize("flag", ["stream_release", "double_ring", "test_stall", "direct_launch"])
 def test_noalloc_refuses_handle_flags_on_host(flag):
     """One batch has nothing to release in a stream and writes the caller's
     buffers, not rings, and the wait-stall test hook is for handles only:
@@ -161,7 +161,7 @@ def test_constants_match_the_header():
              "PAYLOAD_NONE": b.PAYLOAD_NONE, "PAYLOAD_CONCAT": b.PAYLOAD_CONCAT,
              "SCORE_NONE": b.SCORE_NONE, "SCORE_MAX": b.SCORE_MAX, "SCORE_TOPK": b.SCORE_TOPK,
              "FLAG_STREAM_RELEASE": b.FLAG_STREAM_RELEASE, "FLAG_DOUBLE_RING": b.FLAG_DOUBLE_RING,
-             "FLAG_TEST_STALL": b.FLAG_TEST_STALL,
+             "FLAG_TEST_STALL": b.FLAG_TEST_STALL, "FLAG_DIRECT_LAUNCH": b.FLAG_DIRECT_LAUNCH,
              "OPS_PARTIAL": b.OPS_PARTIAL, "NUM_STAGES": b.NUM_STAGES, "PROFILE_OFF": b.PROFILE_OFF,
              "PROFILE_STAGES": b.PROFILE_STAGES, "PROFILE_HOT": b.PROFILE_HOT, "MAX_DELIMS": b.MAX_DELIMS,
              "ROUTE_HASH": b.ROUTE_HASH, "ROUTE_LEAST_LOADED": b.ROUTE_LEAST_LOADED}

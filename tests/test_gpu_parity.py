@@ -11,8 +11,8 @@ torch = pytest.importorskip("torch")
 import paper_2403_04311_gb300 as alto
 from fragments import split, to_batch, tree_fragments
 from gen import make_stream
-from gpu_harness import (assert_same, run_both_stream, run_gpu_batches, run_oracle_batches, small_caps,
-                         stream_caps)
+from gpu_harness import (assert_same, gpu_drain_host, run_both_stream, run_gpu_batches, run_oracle_batches,
+                         small_caps, stream_caps)
 
 pytestmark = pytest.mark.gpu
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
@@ -20,11 +20,41 @@ GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
 
 @pytest.mark.parametrize("name", ["tiny", "tiny64", "factcheck", "throughput", "tokens", "adversarial", "tot"])
 @pytest.mark.parametrize("drain_every", [1, 3])
-def test_workloads_small(name, drain_every):
+@pytest.mark.parametrize("launch", ["graph", "direct"])
+def test_workloads_small(name, drain_every, launch):
+    """Pushes of these small streams replay the captured push graph by
+    default; with ALTO_FLAG_DIRECT_LAUNCH every kernel is launched by itself."""
     s = make_stream(name, small=True)
-    o, g = run_both_stream(s, drain_every=drain_every)
+    caps = dict(stream_caps(s), direct_launch=(launch == "direct"))
+    o, g = run_both_stream(s, drain_every=drain_every, caps=caps)
     assert all(d.status == 0 for d in o)
-    assert_same(o, g, f"{name}/{drain_every}")
+    assert_same(o, g, f"{name}/{drain_every}/{launch}")
+
+
+@pytest.mark.parametrize("mode", ["stages", "hot"])
+def test_graph_replays_while_profiling(mode):
+    """With profiling on, a replayed push records its stage-boundary events
+    through the graph's event-record nodes (fresh events every push): the
+    records still match the oracle and the timed stages have device time."""
+    s = make_stream("factcheck", small=True)
+    agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, **stream_caps(s))
+    agg.profile(alto.PROFILE_STAGES if mode == "stages" else alto.PROFILE_HOT)
+    import oracle
+    o = oracle.Oracle.for_stream(s)
+    for b in range(s.n_batches):
+        bt = s.batch(b)
+        db = alto.to_device(bt)
+        assert agg.push(db.tags, db.off, db.payload, db.score) == alto.OK
+        o.push_batch(bt)
+        assert_same([o.drain()], [gpu_drain_host(agg.drain())], f"{mode} batch {b}")
+    st, prof = agg.profile_read()
+    agg.profile(False)
+    agg.close()
+    o.close()
+    assert st == alto.OK and prof["pushes"] == s.n_batches
+    assert prof["stage_ms"]["gather"] > 0.0
+    if mode == "stages":
+        assert prof["stage_ms"]["ingest"] > 0.0 and prof["stage_ms"]["records"] > 0.0
 
 
 def test_golden_factool_claims():
@@ -93,6 +123,17 @@ def test_bruteforce_streams_on_device():
         _, g = run_gpu_batches(depth, po, so, kk, batches, small_caps(len(frags), 64, depth))
         o = run_oracle_batches(depth, po, so, kk, batches)
         assert_same(o, g, f"{depth} {po} {so} {kk} {cuts}")
+
+
+def test_bruteforce_streams_on_device_direct_launch():
+    """A share of the brute-force streams with every kernel launched by itself."""
+    for depth, po, so, kk, frags, cuts in _brute_cases()[::3]:
+        ws = any(x != 0 for x in so)
+        batches = [to_batch(p, depth, ws) for p in split(frags, cuts)]
+        caps = dict(small_caps(len(frags), 64, depth), direct_launch=True)
+        _, g = run_gpu_batches(depth, po, so, kk, batches, caps)
+        o = run_oracle_batches(depth, po, so, kk, batches)
+        assert_same(o, g, f"direct {depth} {po} {so} {kk} {cuts}")
 
 
 def test_leaf_slot_repeated_in_a_later_batch():
