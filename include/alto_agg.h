@@ -308,7 +308,9 @@ alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg, const alto_batc
                                      alto_topk_pair* out_topk, int64_t cap_topk,
                                      int64_t* out_counts, void* stream);
 
-/* Free everything the handle owns; open groups are discarded.  NULL is OK.
+/* Sec. 3.1: a stream is complete only once its end-of-output delimiter has
+ * arrived, so a group whose last child never came cannot be emitted.  Free
+ * everything the handle owns; such open groups are discarded.  NULL is OK.
  * Always succeeds on a valid or poisoned handle. */
 alto_status alto_agg_destroy(alto_agg_t* h);
 

@@ -500,6 +500,7 @@ __global__ void k_begin(Ctl* ctl, Batch b, Batch* store, int reset) {
     ctl->pay_count = 0;
     ctl->topk_count = 0;
   }
+  ctl->pay_base = ctl->pay_count;
   ctl->epoch += 1;
   ctl->batch_err = 0;
   ctl->n_done = 0;
@@ -1414,13 +1415,18 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch bv
   const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (poisoned(ctl)) return;
+  __shared__ u32 s_cnt, s_base;
+  if (threadIdx.x == 0) s_cnt = 0;
+  __syncthreads();
   const int D = d.cfg.depth;
   const int L = D - 1;
   const u64 n = b.n;
   const bool scores = d.cfg.has_score;
   const u32 ep7 = epoch7(ctl);
   u32* list = d.sc.leaf_seg_start;  // touched leaf-parent entries
-  const u32 end = (b.n + 31) & ~31u;
+  // whole blocks iterate together: the touched entries are appended to the
+  // list with one atomic per block and round
+  const u32 end = (b.n + kThreads - 1) / kThreads * kThreads;
   const int lane = threadIdx.x & 31;
   for (u32 i = gtid(); i < end; i += gstride()) {
     const bool valid = i < b.n;
@@ -1432,29 +1438,28 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch bv
       f = tag_last(t);
       len = b.off[i + 1] - b.off[i];
       if (scores) sk = score_key(b.score[i]);
-      // the chain row and the leaf-slot probe are independent loads: issue both
-      // before acting on either
-      const bool bad = chain_differs(d.tab, e, b.tags, n, i, L);
-      const bool dup = leaf_dup(d.tab, d.sc, e, c, ep7, ctl);
-      if (bad) raise_err(ctl, ALTO_EINCONSIST);
-      if (dup) raise_err(ctl, ALTO_EDUP);
     }
     const u32 key = valid ? e : kNone;
     const u32 peers = __match_any_sync(0xFFFFFFFFu, key);
+    // The accumulator atomics, the chain row loads and the leaf-slot probe
+    // depend on the entry only: all of them go out before any result is used.
     bool first = false;  // this lane made the entry's first contribution of the batch
+    bool bad = false, dup = false;
     if (__all_sync(0xFFFFFFFFu, peers == (1u << lane))) {
       // every lane its own group (the common case): plain atomics, no reductions
       if (valid) {
         Hot* rec = d.tab.hot + e;
         const u64 old = atomicAdd((unsigned long long*)&rec->acc_cl, (1ull << 40) | len);
-        first = old == 0;
         atomicMax(&rec->acc_m1, c + 1);
         atomicMax(&rec->acc_cs1, i + 1);
         if (f) {
-          atomicMin(&d.tab.hot[e].acc_fmin, c);
-          atomicMax(&d.tab.hot[e].acc_fmax1, c + 1);
+          atomicMin(&rec->acc_fmin, c);
+          atomicMax(&rec->acc_fmax1, c + 1);
         }
-        if (scores) atomicMax(&d.tab.hot[e].acc_smx, sk);
+        if (scores) atomicMax(&rec->acc_smx, sk);
+        bad = chain_differs(d.tab, e, b.tags, n, i, L);
+        dup = leaf_dup(d.tab, d.sc, e, c, ep7, ctl);
+        first = old == 0;
       }
     } else {
       const int leader = __ffs(peers) - 1;
@@ -1463,29 +1468,43 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_accumulate(Dev d, Batch bv
       const u32 cs1 = __reduce_max_sync(peers, valid ? i + 1 : 0u);
       const u32 lsum = __reduce_add_sync(peers, len);
       const u32 anyf = __reduce_or_sync(peers, f);
+      const u32 fmin = anyf ? __reduce_min_sync(peers, (valid && f) ? c : kNone) : kNone;
+      const u32 fmax1 = anyf ? __reduce_max_sync(peers, (valid && f) ? c + 1 : 0u) : 0u;
+      const u32 smx = scores ? __reduce_max_sync(peers, valid ? sk : 0u) : 0u;
+      u64 old = 1;
       if (valid && lane == leader) {
         // one returning atomic per group and warp: leaves and payload together
         Hot* rec = d.tab.hot + e;
-        const u64 old = atomicAdd((unsigned long long*)&rec->acc_cl, ((unsigned long long)cnt << 40) | lsum);
-        first = old == 0;
+        old = atomicAdd((unsigned long long*)&rec->acc_cl, ((unsigned long long)cnt << 40) | lsum);
         atomicMax(&rec->acc_m1, m1);
         atomicMax(&rec->acc_cs1, cs1);
-      }
-      if (anyf) {
-        const u32 fmin = __reduce_min_sync(peers, (valid && f) ? c : kNone);
-        const u32 fmax1 = __reduce_max_sync(peers, (valid && f) ? c + 1 : 0u);
-        if (valid && lane == leader && fmax1) {
-          atomicMin(&d.tab.hot[e].acc_fmin, fmin);
-          atomicMax(&d.tab.hot[e].acc_fmax1, fmax1);
+        if (fmax1) {
+          atomicMin(&rec->acc_fmin, fmin);
+          atomicMax(&rec->acc_fmax1, fmax1);
         }
+        if (smx) atomicMax(&rec->acc_smx, smx);
       }
-      if (scores) {
-        const u32 smx = __reduce_max_sync(peers, valid ? sk : 0u);
-        if (valid && lane == leader && smx) atomicMax(&d.tab.hot[e].acc_smx, smx);
+      if (valid) {
+        bad = chain_differs(d.tab, e, b.tags, n, i, L);
+        dup = leaf_dup(d.tab, d.sc, e, c, ep7, ctl);
       }
+      first = old == 0;
     }
-    const u32 pos = warp_take(first, &ctl->n_segs[L]);
+    if (bad) raise_err(ctl, ALTO_EINCONSIST);
+    if (dup) raise_err(ctl, ALTO_EDUP);
+    const u32 m = __ballot_sync(0xFFFFFFFFu, first);
+    const int wl = __ffs(m) - 1;
+    u32 wbase = 0;
+    if (m != 0 && lane == wl) wbase = atomicAdd(&s_cnt, (u32)__popc(m));
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      s_base = s_cnt ? atomicAdd(&ctl->n_segs[L], s_cnt) : 0u;
+      s_cnt = 0;
+    }
+    __syncthreads();
+    if (m != 0) wbase = __shfl_sync(0xFFFFFFFFu, wbase, wl);
     if (first) {
+      const u32 pos = s_base + wbase + __popc(m & lanemask_lt());
       if (pos < d.cfg.n_max) list[pos] = e;
       d.tab.hot[e].acc_rep = i;
     }
@@ -2007,6 +2026,62 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch bv) {
   }
 }
 
+// Dense child slots from the arena: spans buffered by earlier batches (and,
+// above the leaf parent, handed up earlier in this batch).  LEVEL_M: the
+// groups of level M, by emission rank; otherwise the groups of levels M < l,
+// by done index.  (A warp per group with buffered spans, in place of the
+// binary search, measured slower: a few groups hold most of the spans.)
+template <bool LEVEL_M>
+__device__ __forceinline__ void dense_arena_body(const Dev& d, Ctl* ctl, u64 first, u64 stride) {
+  const u32 ep = ctl->epoch;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  const u64 na = LEVEL_M ? ctl->arena_total : ctl->chain_arena;
+  const u64* abase = LEVEL_M ? d.sc.r_arena_base : d.sc.c_arena_base;
+  for (u64 a = first; a < na; a += stride) {
+    // last index x with abase[x] <= a: the one whose spans contain a
+    u32 lo = 0, hi = nd;
+    while (hi - lo > 1) {
+      u32 mid = (lo + hi) >> 1;
+      if (abase[mid] <= a) lo = mid;
+      else hi = mid;
+    }
+    const u32 di = LEVEL_M ? d.sc.r_done[lo] : lo;
+    if (di >= nd) continue;
+    if (!LEVEL_M && (int)d.sc.done_lvl[di] <= d.cfg.concat_level) continue;
+    const u32 e = d.sc.done_e[di] & d.tab.mask;
+    const u64 k = a - abase[lo];
+    const u32 mn = LEVEL_M ? d.sc.r_meta_n[lo] : d.tab.vec_n[2 * (u64)e];
+    if (k >= mn) continue;
+    bool ok1, ok2 = true;
+    u64 ma = vec_addr(d.tab, e, 0, 2 * k, &ok1);
+    if (!ok1) continue;
+    const u32 c = (u32)d.ar.pool[ma];
+    const u32 pos = (u32)d.ar.pool[ma + 1];
+    u32 end;
+    if (k + 1 < mn) {
+      u64 na2 = vec_addr(d.tab, e, 0, 2 * (k + 1) + 1, &ok2);
+      end = ok2 ? (u32)d.ar.pool[na2] : pos;
+    } else {
+      end = d.tab.vec_n[2 * (u64)e + 1];
+    }
+    // streaming: the buffer holds children rel.. only; a partial release
+    // places those below rnew and keeps the rest
+    const u32 rel = (LEVEL_M && d.cfg.stream) ? d.tab.rel[e] : 0u;
+    if (c > d.tab.hot[e].last || end < pos || c < rel) {
+      raise_err(ctl, ALTO_EDUP);
+      continue;
+    }
+    if (LEVEL_M && d.cfg.stream && d.sc.done_part[di] && c >= d.tab.rnew[e]) continue;
+    const u64 slot = d.tab.dbase[e] + (c - rel);
+    if (slot >= d.cfg.dense_cap) continue;
+    u32 old = atomicExch(&d.sc.dense[slot].x, ep);
+    if (old == ep) raise_err(ctl, ALTO_EDUP);
+    d.sc.dense[slot].y = end - pos;
+    d.sc.dense[slot].z = e;
+    d.sc.dense[slot].w = pos;
+  }
+}
+
 // Leaf level without TOPK, per fragment in arrival order, eight lanes each:
 // a fragment of a group left open takes its arena position from the group's
 // cursor (one 64-bit atomic: leaf index and payload offset together) and is
@@ -2106,65 +2181,20 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch bv) {
       }
     }
   }
+  // the completing groups' children buffered by earlier batches take their
+  // dense slots in the same launch: other slots than the fragments' above,
+  // and their latency overlaps that of the fragments
+  if (!ctl->skip_dense) dense_arena_body<true>(d, ctl, gtid(), gstride());
 }
 
-// Dense child slots from the arena: spans buffered by earlier batches (and,
-// above the leaf parent, handed up earlier in this batch).  LEVEL_M: the
-// groups of level M, by emission rank; otherwise the groups of levels M < l,
-// by done index.  (A warp per group with buffered spans, in place of the
-// binary search, measured slower: a few groups hold most of the spans.)
+// The buffered children's dense slots in a launch of their own (the TOPK
+// leaf path, and the levels below M).
 template <bool LEVEL_M>
 __global__ void __launch_bounds__(kThreads) k_dense_arena(Dev d) {
   pdl_enter();
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
-  const u32 ep = ctl->epoch;
-  const u32 nd = min(ctl->n_done, d.sc.done_cap);
-  const u64 na = LEVEL_M ? ctl->arena_total : ctl->chain_arena;
-  const u64* abase = LEVEL_M ? d.sc.r_arena_base : d.sc.c_arena_base;
-  for (u64 a = gtid(); a < na; a += gstride()) {
-    // last index x with abase[x] <= a: the one whose spans contain a
-    u32 lo = 0, hi = nd;
-    while (hi - lo > 1) {
-      u32 mid = (lo + hi) >> 1;
-      if (abase[mid] <= a) lo = mid;
-      else hi = mid;
-    }
-    const u32 di = LEVEL_M ? d.sc.r_done[lo] : lo;
-    if (di >= nd) continue;
-    if (!LEVEL_M && (int)d.sc.done_lvl[di] <= d.cfg.concat_level) continue;
-    const u32 e = d.sc.done_e[di] & d.tab.mask;
-    const u64 k = a - abase[lo];
-    const u32 mn = LEVEL_M ? d.sc.r_meta_n[lo] : d.tab.vec_n[2 * (u64)e];
-    if (k >= mn) continue;
-    bool ok1, ok2 = true;
-    u64 ma = vec_addr(d.tab, e, 0, 2 * k, &ok1);
-    if (!ok1) continue;
-    const u32 c = (u32)d.ar.pool[ma];
-    const u32 pos = (u32)d.ar.pool[ma + 1];
-    u32 end;
-    if (k + 1 < mn) {
-      u64 na2 = vec_addr(d.tab, e, 0, 2 * (k + 1) + 1, &ok2);
-      end = ok2 ? (u32)d.ar.pool[na2] : pos;
-    } else {
-      end = d.tab.vec_n[2 * (u64)e + 1];
-    }
-    // streaming: the buffer holds children rel.. only; a partial release
-    // places those below rnew and keeps the rest
-    const u32 rel = (LEVEL_M && d.cfg.stream) ? d.tab.rel[e] : 0u;
-    if (c > d.tab.hot[e].last || end < pos || c < rel) {
-      raise_err(ctl, ALTO_EDUP);
-      continue;
-    }
-    if (LEVEL_M && d.cfg.stream && d.sc.done_part[di] && c >= d.tab.rnew[e]) continue;
-    const u64 slot = d.tab.dbase[e] + (c - rel);
-    if (slot >= d.cfg.dense_cap) continue;
-    u32 old = atomicExch(&d.sc.dense[slot].x, ep);
-    if (old == ep) raise_err(ctl, ALTO_EDUP);
-    d.sc.dense[slot].y = end - pos;
-    d.sc.dense[slot].z = e;
-    d.sc.dense[slot].w = pos;
-  }
+  dense_arena_body<LEVEL_M>(d, ctl, gtid(), gstride());
 }
 
 // Output offsets of every child span; a slot no child filled means a child
@@ -2249,7 +2279,7 @@ __global__ void __launch_bounds__(kThreads, 8) k_gather(Dev d, Batch bv) {
   constexpr int kGroups = 32 / kSpanLanes;
   const u32 ep = ctl->epoch;
   const u64 total = ctl->dense_total;
-  const u64 base = ctl->pay_count;
+  const u64 base = ctl->pay_base;
   const u64 cap = d.cfg.out_payload;
   int32_t* __restrict__ out = d.out_pay;
   const u64 gw = gtid() >> 5, nw = gstride() >> 5;
@@ -2727,8 +2757,10 @@ struct alto_agg {
     int64_t stage_launches[ALTO_NUM_STAGES] = {};
     bool failed = false;                             // capture failed: launch directly
   };
-  PushGraph graphs[2][3];  // [ring][profiling: off, stages, hot]
+  PushGraph graphs[2][3][4];  // [ring][profiling: off, stages, hot][batch size class]
   cudaStream_t cap_stream = nullptr;
+  cudaStream_t side = nullptr;          // direct launches: records and sweep beside the gather
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   std::vector<cudaEvent_t> cap_events;  // recorded at capture only (the graphs' templates hold them)
   bool direct_only = false;   // ALTO_FLAG_DIRECT_LAUNCH
   bool reset_pending = false; // a drain handed out the ring: the next push resets its counters
@@ -2811,13 +2843,14 @@ void launch_scan3(const LookbackState& lb, Ctl* ctl, const F& f0, const F& f1,
 
 template <class F>
 void launch_scan(const LookbackState& lb, int num_sms, Ctl* ctl, const F& f, u64 cap, int site,
-                 u64 spin, cudaStream_t s) {
+                 u64 spin, cudaStream_t s, int max_grid = 0) {
   u64 tiles = (cap + kScanTile - 1) / kScanTile;
   if (tiles == 0) tiles = 1;
   // up to four CTAs per SM: with a functor that loads and stores per element
   // the extra CTAs hide its latency (one per SM was faster only for a bare
   // sum in isolation)
   int grid = (int)std::min<u64>(tiles, (u64)num_sms * 4);
+  if (max_grid > 0) grid = std::min(grid, max_grid);
   launch_pdl(k_scan<F>, grid, kScanThreads, 0, s, f, lb, ctl, site, &ctl->exit_ctr[site], spin);
 }
 
@@ -2832,9 +2865,17 @@ struct Pipeline {
   int num_sms;
   int tbits;
   u32 nmax;
+  // fragments of the largest batch these launches serve (nmax for a direct
+  // launch, the size class of a captured graph): grids of kernels whose work
+  // the batch size bounds are sized for it
+  u32 nb;
   cudaStream_t s;
   void (*stage)(void* ctx, int st, int64_t launches) = nullptr;
   void* stage_ctx = nullptr;
+  // a second stream (with its fork and join events) on which the records and
+  // the table sweep run beside the payload gather; null: one stream
+  cudaStream_t s2 = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   int64_t launches = 0;
   void enter(int st) {
     if (stage) stage(stage_ctx, st, launches);
@@ -2863,8 +2904,22 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   const int D = d.cfg.depth;
   const int M = d.cfg.concat_level;
   const u32 nmax = p.nmax;
-  const int grid = p.num_sms * 8;   // kernels over fragments or leaves
-  const int sgrid = p.num_sms * 2;  // kernels over groups (fewer items)
+  const u32 nb = std::min(p.nb, nmax);
+  // a grid of at most `full` blocks, no more than `items` of `per` each need
+  // (small batches launch small grids: idle blocks still cost their launch)
+  auto fit = [](int full, u64 items, u64 per) {
+    const u64 need = std::max<u64>(1, (items + per - 1) / per);
+    return (int)std::min<u64>((u64)full, need);
+  };
+  const bool small = nb < nmax;
+  const int grid = fit(p.num_sms * 8, nb, kThreads);    // kernels over fragments or leaves
+  const int sgrid = fit(p.num_sms * 2, nb, kThreads);   // kernels over groups (fewer items)
+  // kernels over completed groups: a fragment completes at most one a level
+  const int dgrid = fit(p.num_sms * 2, (u64)nb * D, kThreads);
+  // kernels whose work the batch does not bound (buffered children of the
+  // groups it completes, payload): one block an SM for a small batch
+  const int ugrid = small ? p.num_sms : p.num_sms * 2;
+  bool forked = false;  // records and sweep on the second stream, beside the gather
   const u64 spin = d.cfg.spin_limit;
   int sl = 0;  // launches inside sort_pairs
   int site = 0;
@@ -2880,7 +2935,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     // leaf level with TOPK: sort fragments by their leaf-parent group so that
     // each group's candidates are contiguous for the segmented top-k
     p.enter(1);
-    int cur = sort_pairs(&d.ctl->n, nmax, p.tbits, true, *p.leaf_sort, d.ctl, site, spin, p.num_sms,
+    int cur = sort_pairs(&d.ctl->n, nb, p.tbits, true, *p.leaf_sort, d.ctl, site, spin, p.num_sms,
                          s, &sl);
     p.launches += sl;
     sl = 0;
@@ -2889,15 +2944,15 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     p.enter(2);
     SegFind f{d.sc.leaf_keys, d.sc.leaf_seg_start, d.sc.leaf_seg_of, &d.ctl->n, nmax,
               &d.ctl->n_segs[D - 1]};
-    launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site + 4, spin, s);
-    launch_pdl(k_reduce<true, G>, p.num_sms * blocks_per_sm((const void*)k_reduce<true, G>), kThreads, 0, s, d, bt,
-               D - 1, d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
-    launch_pdl(k_reduce_big<true, G>, p.num_sms, kBigThreads, 0, s, d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm,
-               d.sc.leaf_seg_start, set);
+    launch_scan(p.lbs, p.num_sms, d.ctl, f, nb, site + 4, spin, s);
+    launch_pdl(k_reduce<true, G>, fit(p.num_sms * blocks_per_sm((const void*)k_reduce<true, G>), nb, kThreads),
+               kThreads, 0, s, d, bt, D - 1, d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
+    launch_pdl(k_reduce_big<true, G>, fit(p.num_sms, nb, kBigSeg), kBigThreads, 0, s, d, bt, D - 1,
+               d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
     p.launches += 3;
     if (d.cfg.stream) {
-      launch_pdl(k_reduce_rel<G>, p.num_sms * blocks_per_sm((const void*)k_reduce_rel<G>), kThreads, 0, s, d, bt,
-                 d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
+      launch_pdl(k_reduce_rel<G>, fit(p.num_sms * blocks_per_sm((const void*)k_reduce_rel<G>), nb, 8), kThreads,
+                 0, s, d, bt, d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
       p.launches += 1;
     }
   } else {
@@ -2937,7 +2992,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     }
     looked_up = false;
     added = false;
-    int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nmax, p.tbits, true, *p.up_sort, d.ctl, site, spin,
+    int c2 = sort_pairs(&d.ctl->n_segs[l + 1], nb, p.tbits, true, *p.up_sort, d.ctl, site, spin,
                         p.num_sms, s, &sl);
     p.launches += sl;
     sl = 0;
@@ -2946,20 +3001,20 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     d.sc.up_perm = p.up_sort->vals[c2];
     SegFind f{d.sc.up_keys, d.sc.up_seg_start, nullptr, &d.ctl->n_segs[l + 1], nmax,
               &d.ctl->n_segs[l]};
-    launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax, site++, spin, s);
-    launch_pdl(k_reduce<false, G>, p.num_sms * blocks_per_sm((const void*)k_reduce<false, G>), kThreads, 0, s, d,
-               bt, l, d.sc.up_keys, d.sc.up_perm, d.sc.up_seg_start, set);
-    launch_pdl(k_reduce_big<false, G>, p.num_sms, kBigThreads, 0, s, d, bt, l, d.sc.up_keys, d.sc.up_perm,
-               d.sc.up_seg_start, set);
+    launch_scan(p.lbs, p.num_sms, d.ctl, f, nb, site++, spin, s);
+    launch_pdl(k_reduce<false, G>, fit(p.num_sms * blocks_per_sm((const void*)k_reduce<false, G>), nb, kThreads),
+               kThreads, 0, s, d, bt, l, d.sc.up_keys, d.sc.up_perm, d.sc.up_seg_start, set);
+    launch_pdl(k_reduce_big<false, G>, fit(p.num_sms, nb, kBigSeg), kBigThreads, 0, s, d, bt, l, d.sc.up_keys,
+               d.sc.up_perm, d.sc.up_seg_start, set);
     p.launches += 3;
   }
   // emission order
   p.enter(5);
   {
     RankScan f{d.sc.mblk, d.sc.prefix, &d.ctl->n};
-    launch_scan(p.lbs, p.num_sms, d.ctl, f, nmax / 32 + 1, site++, spin, s);
+    launch_scan(p.lbs, p.num_sms, d.ctl, f, nb / 32 + 1, site++, spin, s);
   }
-  launch_pdl(k_done_rank, sgrid, kThreads, 0, s, d);
+  launch_pdl(k_done_rank, dgrid, kThreads, 0, s, d);
   p.launches += 2;
   const u32 dcap = d.sc.done_cap;
   const bool chain = M >= 0 && M < D - 1;  // levels below M hand spans up
@@ -2970,8 +3025,9 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
     CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
     const CapCheck cc{d.cfg.out_records, d.cfg.dense_cap, d.cfg.out_topk, d.sc.done_cap};
-    if (chain) launch_scan3(p.lbs, d.ctl, f0, f1, f2, dcap, site, spin, s, NoLast());
-    else launch_scan3(p.lbs, d.ctl, f0, f1, f2, dcap, site, spin, s, cc);
+    const u64 dbound = std::min<u64>(dcap, (u64)nb * D);
+    if (chain) launch_scan3(p.lbs, d.ctl, f0, f1, f2, dbound, site, spin, s, NoLast());
+    else launch_scan3(p.lbs, d.ctl, f0, f1, f2, dbound, site, spin, s, cc);
     p.launches += 1;
     site += 3;
   }
@@ -2990,7 +3046,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
       c[k].M = M;
       c[k].L = D - 1;
     }
-    launch_scan3(p.lbs, d.ctl, c[0], c[1], c[2], dcap, site, spin, s,
+    launch_scan3(p.lbs, d.ctl, c[0], c[1], c[2], std::min<u64>(dcap, (u64)nb * D), site, spin, s,
                  CapCheck{d.cfg.out_records, d.cfg.dense_cap, d.cfg.out_topk, d.sc.done_cap});
     p.launches += 1;
     site += 3;
@@ -3004,18 +3060,19 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
       p.enter(7);
       launch_pdl(k_dense_batch<G>, grid, kThreads, 0, s, d, bt);
     } else {
-      // the leaf finalize already allocated the carried leaves' chunks
+      // the leaf finalize already allocated the carried leaves' chunks; the
+      // placement also places the children buffered by earlier batches
       p.enter(7);
       launch_pdl(k_leaf_place<G>, grid, kThreads, 0, s, d, bt);
     }
-    launch_pdl(k_dense_arena<true>, sgrid, kThreads, 0, s, d);
-    p.launches += leaf_sorted ? 5 : 2;
+    if (leaf_sorted) launch_pdl(k_dense_arena<true>, ugrid, kThreads, 0, s, d);
+    p.launches += leaf_sorted ? 5 : 1;
     if (chain) {
-      launch_pdl(k_dense_arena<false>, sgrid, kThreads, 0, s, d);
+      launch_pdl(k_dense_arena<false>, ugrid, kThreads, 0, s, d);
       p.launches += 1;
     }
     DenseScan fd{d.sc.dense, d.sc.dst, d.ctl, !chain, d.cfg.out_payload};
-    launch_scan(p.lbs, p.num_sms, d.ctl, fd, d.cfg.dense_cap, site++, spin, s);
+    launch_scan(p.lbs, p.num_sms, d.ctl, fd, d.cfg.dense_cap, site++, spin, s, small ? 32 : 0);
     p.launches += 1;
     if (chain) {
       launch_pdl(k_check2, 1, 1, 0, s, d);
@@ -3024,23 +3081,44 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     p.enter(8);
     // levels below M hand their concatenations up, deepest first
     for (int l = D - 1; chain && l > M; --l) {
-      launch_pdl(k_chain_gather<G>, p.num_sms * blocks_per_sm((const void*)k_chain_gather<G>), kThreads, 0, s, d,
-                 bt, l);
+      launch_pdl(k_chain_gather<G>, small ? p.num_sms : p.num_sms * blocks_per_sm((const void*)k_chain_gather<G>),
+                 kThreads, 0, s, d, bt, l);
       p.launches += 1;
+    }
+    // The records and the table sweep touch nothing the gather reads (the
+    // gather takes its ring base from pay_base, not from the counters the
+    // batch's end moves): with a second stream they run beside it, on one
+    // block slot per SM that the gather leaves free.  Not with streaming
+    // release (the buffer compaction after the gather reads the partial
+    // flags the records clear) or CONCAT above the leaf parent.
+    forked = p.s2 != nullptr && !d.cfg.stream && M == D - 1;
+    int gather_grid = small ? p.num_sms : p.num_sms * blocks_per_sm((const void*)k_gather<G>);
+    if (forked) {
+      cudaEventRecord(p.ev_fork, s);
+      cudaStreamWaitEvent(p.s2, p.ev_fork, 0);
+      launch_pdl(k_records, dgrid, kThreads, 0, p.s2, d);
+      launch_pdl(k_sweep, dgrid, kThreads, 0, p.s2, d);
+      cudaEventRecord(p.ev_join, p.s2);
+      p.launches += 2;
+      if (!small) gather_grid -= p.num_sms;
     }
     // plain stream order (no programmatic overlap with its neighbours): the
     // gather is the stage the measurement hooks time on their own
-    k_gather<G><<<p.num_sms * blocks_per_sm((const void*)k_gather<G>), kThreads, 0, s>>>(d, bt);
+    k_gather<G><<<gather_grid, kThreads, 0, s>>>(d, bt);
     p.launches += 1;
   }
   p.enter(9);
+  if (forked) {
+    cudaStreamWaitEvent(s, p.ev_join, 0);
+    return;
+  }
   if (d.cfg.stream) {
     // the released spans are out: drop them from the buffers they came from
-    launch_pdl(k_stream_compact, sgrid, kThreads, 0, s, d);
+    launch_pdl(k_stream_compact, ugrid, kThreads, 0, s, d);
     p.launches += 1;
   }
-  launch_pdl(k_records, sgrid, kThreads, 0, s, d);
-  launch_pdl(k_sweep, sgrid, kThreads, 0, s, d);
+  launch_pdl(k_records, dgrid, kThreads, 0, s, d);
+  launch_pdl(k_sweep, dgrid, kThreads, 0, s, d);
   p.launches += 2;
 }
 
@@ -3057,10 +3135,16 @@ void* dev_alloc(alto_agg* h, size_t bytes, cudaStream_t s) {
   return p;
 }
 
-// Pushes of at most this many fragments replay the captured graph (host
+// Pushes of at most this many fragments replay a captured graph (host
 // launch cost matters there); larger ones launch kernel by kernel, whose
 // kernels read the batch from their parameters rather than device memory.
+// A push replays the graph of the smallest size class that holds it, whose
+// grids are sized for that many fragments.
 constexpr u32 kGraphMaxBatch = 1u << 17;
+constexpr int kGraphClasses = 4;
+__host__ __forceinline__ u32 graph_class_bound(int c) { return 1u << (11 + 2 * c); }  // 2K, 8K, 32K, 128K
+static_assert(sizeof(alto_agg::graphs[0][0]) / sizeof(alto_agg::PushGraph) == kGraphClasses,
+              "one graph per size class");
 
 // Stage bookkeeping of one push's launch sequence: kernels per stage, and the
 // stage-boundary events when profiling.
@@ -3077,7 +3161,7 @@ struct PushRec {
 // pipeline.  G: the kernels read the batch that k_begin stores (graph capture).
 // Returns the number of kernels.
 template <bool G>
-int64_t launch_push(alto_agg* h, cudaStream_t s, const Batch& bt, int reset, PushRec* rec) {
+int64_t launch_push(alto_agg* h, cudaStream_t s, const Batch& bt, int reset, PushRec* rec, u32 nb) {
   Dev d = h->d;
   Pipeline p;
   p.d = d;
@@ -3087,7 +3171,27 @@ int64_t launch_push(alto_agg* h, cudaStream_t s, const Batch& bt, int reset, Pus
   p.num_sms = h->num_sms;
   p.tbits = h->tbits;
   p.nmax = (u32)h->cfg.max_batch_fragments;
+  p.nb = nb;
   p.s = s;
+  // kernel-by-kernel launches run the records beside the gather on the
+  // handle's side stream (not with an event at every stage boundary)
+  if (!G && !(h->profiling && h->profile_mode == ALTO_PROFILE_STAGES)) {
+    if (!h->side && cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) == cudaSuccess) {
+      if (cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+          cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess) {
+        if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+        cudaStreamDestroy(h->side);
+        h->side = nullptr;
+        h->ev_fork = h->ev_join = nullptr;
+      }
+    }
+    cudaGetLastError();
+    if (h->side) {
+      p.s2 = h->side;
+      p.ev_fork = h->ev_fork;
+      p.ev_join = h->ev_join;
+    }
+  }
   p.stage = [](void* ctx, int st, int64_t launches) {
     PushRec* r = (PushRec*)ctx;
     r->stage_l[r->stage] += launches - r->l0;
@@ -3111,13 +3215,14 @@ int64_t launch_push(alto_agg* h, cudaStream_t s, const Batch& bt, int reset, Pus
 // profiling capture also holds one event-record node per timed stage
 // boundary, whose event every replay replaces.  On any failure the graph is marked failed and pushes of that
 // kind launch directly.
-bool capture_push(alto_agg* h, alto_agg::PushGraph& g) {
+bool capture_push(alto_agg* h, alto_agg::PushGraph& g, u32 nb) {
   g.failed = true;
   if (!h->cap_stream && cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess) {
     h->cap_stream = nullptr;
     cudaGetLastError();
     return false;
   }
+
   Batch ph;  // k_begin's parameters of the capture; every replay sets its own
   ph.tags = nullptr;
   ph.off = nullptr;
@@ -3131,7 +3236,7 @@ bool capture_push(alto_agg* h, alto_agg::PushGraph& g) {
   }
   PushRec rec(h, h->cap_stream);
   rec.clk.capturing = true;
-  const int64_t launches = launch_push<true>(h, h->cap_stream, ph, 0, &rec);
+  const int64_t launches = launch_push<true>(h, h->cap_stream, ph, 0, &rec, nb);
   for (cudaEvent_t e : rec.clk.ev)
     if (e) h->cap_events.push_back(e);
   cudaGraph_t graph = nullptr;
@@ -3180,16 +3285,22 @@ bool capture_push(alto_agg* h, alto_agg::PushGraph& g) {
 }
 
 void free_graphs(alto_agg* h) {
-  for (auto& row : h->graphs)
-    for (auto& g : row) {
-      if (g.exec) cudaGraphExecDestroy(g.exec);
-      if (g.graph) cudaGraphDestroy(g.graph);
-      g = alto_agg::PushGraph();
-    }
+  for (auto& ring : h->graphs)
+    for (auto& row : ring)
+      for (auto& g : row) {
+        if (g.exec) cudaGraphExecDestroy(g.exec);
+        if (g.graph) cudaGraphDestroy(g.graph);
+        g = alto_agg::PushGraph();
+      }
   for (cudaEvent_t e : h->cap_events) cudaEventDestroy(e);
   h->cap_events.clear();
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
   h->cap_stream = nullptr;
+  if (h->side) cudaStreamDestroy(h->side);
+  if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+  if (h->ev_join) cudaEventDestroy(h->ev_join);
+  h->side = nullptr;
+  h->ev_fork = h->ev_join = nullptr;
 }
 
 void free_all(alto_agg* h, cudaStream_t s) {
@@ -3530,8 +3641,10 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
   h->reset_pending = false;
   if (!h->direct_only && n <= kGraphMaxBatch) {
     const int pm = !h->profiling ? 0 : (h->profile_mode == ALTO_PROFILE_HOT ? 2 : 1);
-    alto_agg::PushGraph& g = h->graphs[h->ring_cur][pm];
-    if (g.exec == nullptr && !g.failed) capture_push(h, g);
+    int gc = 0;
+    while (gc + 1 < kGraphClasses && n > graph_class_bound(gc)) ++gc;
+    alto_agg::PushGraph& g = h->graphs[h->ring_cur][pm][gc];
+    if (g.exec == nullptr && !g.failed) capture_push(h, g, graph_class_bound(gc));
     if (g.exec != nullptr) {
       // this push's batch (and counter reset) as k_begin's parameters
       Ctl* ctl = d.ctl;
@@ -3564,7 +3677,7 @@ alto_status alto_agg_push_batch(alto_agg_t* h, const alto_batch* b, void* stream
     }
   }
   PushRec rec(h, s);
-  const int64_t launches = launch_push<false>(h, s, bt, reset, &rec);
+  const int64_t launches = launch_push<false>(h, s, bt, reset, &rec, (u32)h->cfg.max_batch_fragments);
   if (h->profiling) {
     h->ev_pending.push_back(rec.clk.ev);
     for (int i = 0; i < ALTO_NUM_STAGES; ++i) h->stage_launches[i] += rec.stage_l[i];
@@ -3987,6 +4100,7 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
     p.up_sort = &st.up_sort;
     p.lbs = st.lbs;
     p.num_sms = num_sms;
+    p.nb = nmax;
     p.tbits = st.tbits;
     p.nmax = nmax;
     p.s = s;

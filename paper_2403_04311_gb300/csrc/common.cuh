@@ -60,6 +60,8 @@ struct Ctl {
   u32 n_big[kMaxDepth];    // segments of level l longer than a warp's share, for the block reduce
   u32 n_rel;               // streaming: small leaf segments left to the warp reduce
   u64 scan_total[kSites];  // totals written by scans
+  u64 pay_base;            // pay_count when the batch started (the gather's base: the
+                           // batch's end may move pay_count while the gather still runs)
 };
 
 // Programmatic dependent launch.  Every kernel of the library is launched

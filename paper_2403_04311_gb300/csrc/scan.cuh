@@ -21,6 +21,12 @@ constexpr int kScanThreads = 512;
 constexpr int kScanItems = 8;
 constexpr int kScanWarps = kScanThreads / 32;
 constexpr int kScanTile = kScanThreads * kScanItems;
+// Scans of at most this many tiles run in the launch's first CTA alone, tile
+// after tile with a running carry: no look-back, no tile or exit counters
+// (the other CTAs return at once).  Small batches' scans are a tile or two,
+// and there the counters and descriptors of a look-back cost more than the
+// scan itself.
+constexpr u32 kScanSmallTiles = 2;
 
 // One 16-byte descriptor per tile, {value, epoch_site << 2 | kind} with kind
 // 1 = the tile's own sum, 2 = the sum of tiles 0..t.  It is written and read
@@ -163,14 +169,21 @@ __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl
   if (ntiles64 > st.tiles) ntiles64 = st.tiles;
   const u32 ntiles = (u32)ntiles64;
   const u32 es = epoch_site(ctl, site);
-  if (t == 0) s_next = take_tile(ctl, site);
+  // every CTA reads the same n, so all take the same path
+  const bool small = ntiles <= kScanSmallTiles;
+  if (small && blockIdx.x != 0) return;
+  __shared__ u64 s_carry;  // small path: sum of the tiles before this one
+  if (t == 0) {
+    s_next = small ? 0u : take_tile(ctl, site);
+    s_carry = 0;
+  }
   __syncthreads();
   u32 tile = s_next;
   __syncthreads();
   u32 r[kScanItems];
   scan_load(f, n, tile, ntiles, r);
   while (tile < ntiles) {
-    if (t == 0) s_next = take_tile(ctl, site);  // read after the barriers below
+    if (t == 0) s_next = small ? tile + 1 : take_tile(ctl, site);  // read after the barriers below
 #pragma unroll
     for (int k = 0; k < kScanItems; ++k) s_v[scan_pad((u32)(k * kScanThreads + t))] = r[k];
     __syncthreads();
@@ -207,17 +220,20 @@ __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl
         rel += w[k];
       }
     }
-    if (warp == 0 && lane == 0) lb_publish(st, tile, es, tile == 0 ? 2u : 1u, agg);
+    if (!small && warp == 0 && lane == 0) lb_publish(st, tile, es, tile == 0 ? 2u : 1u, agg);
     // the next tile's loads go out while warp 0 walks back
     scan_load(f, n, next, ntiles, r);
     if (warp == 0) {
       u64 excl = 0;
-      if (tile != 0) {
+      if (small) {
+        excl = s_carry;
+      } else if (tile != 0) {
         excl = lb_walk_warp(st, tile, es, ctl, spin_limit);
         if (lane == 0) lb_publish(st, tile, es, 2u, excl + agg);
       }
       if (lane == 0) {
         s_excl = excl;
+        if (small) s_carry = excl + agg;
         if (tile == ntiles - 1) f.total(ctl, excl + agg);
       }
     }
@@ -244,7 +260,7 @@ __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl
     __syncthreads();
     tile = next;
   }
-  if (t == 0) finish_ctas(ctl, site, exit_ctr);
+  if (!small && t == 0) finish_ctas(ctl, site, exit_ctr);
 }
 
 template <class F>
