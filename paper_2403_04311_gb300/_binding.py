@@ -10,7 +10,6 @@ from __future__ import annotations
 
 import ctypes
 import os
-from dataclasses import dataclass
 
 import numpy as np
 
@@ -341,14 +340,53 @@ class _DevView:
         }
 
 
-@dataclass
 class Drain:
-    status: int
-    records: object   # torch uint8 tensor (device) of n_records * 48 bytes
-    payload: object   # torch int32 tensor (device)
-    topk: object      # torch uint8 tensor (device) of n_topk * 8 bytes
-    first_batch: int
-    n_batches: int
+    """What one drain returned: status, the batch range, and device views of
+    the records (uint8, 48 bytes each), payload (int32) and top-k pairs (uint8,
+    8 bytes each).  The views are made on first access (they are only valid
+    until the next push, drain or destroy, like the pointers behind them)."""
+
+    __slots__ = ("status", "first_batch", "n_batches", "n_records", "n_payload", "n_topk", "_ptrs", "_views")
+
+    def __init__(self, status, raw=None):
+        self.status = int(status)
+        self.first_batch = int(raw.first_batch) if raw is not None else 0
+        self.n_batches = int(raw.n_batches) if raw is not None else 0
+        ok = raw is not None and self.status == OK
+        self.n_records = int(raw.n_records) if ok else 0
+        self.n_payload = int(raw.n_payload) if ok else 0
+        self.n_topk = int(raw.n_topk) if ok else 0
+        self._ptrs = (raw.records, raw.payload, raw.topk) if ok else None
+        self._views = {}
+
+    def _view(self, k):
+        if self._ptrs is None:
+            return None
+        v = self._views.get(k)
+        if v is None:
+            import torch
+            ptr = self._ptrs[k]
+            nbytes = (self.n_records * 48, self.n_payload * 4, self.n_topk * 8)[k]
+            if not ptr or nbytes == 0:
+                v = torch.zeros(0, dtype=torch.uint8, device="cuda")
+            else:
+                v = torch.as_tensor(_DevView(ptr, nbytes), device="cuda")
+            if k == 1:
+                v = v.view(torch.int32)
+            self._views[k] = v
+        return v
+
+    @property
+    def records(self):
+        return self._view(0)
+
+    @property
+    def payload(self):
+        return self._view(1)
+
+    @property
+    def topk(self):
+        return self._view(2)
 
     def host(self):
         """(records as RECORD_DTYPE, payload int32, topk as PAIR_DTYPE) numpy copies."""
@@ -393,20 +431,7 @@ class Aggregator:
 
     def drain(self) -> Drain:
         st, d = alto_agg_drain(self._h, self.stream.cuda_stream)
-        torch = self._torch
-
-        def view(ptr, nbytes, dtype):
-            if not ptr or nbytes == 0:
-                return torch.zeros(0, dtype=dtype, device="cuda")
-            t = torch.as_tensor(_DevView(ptr, nbytes), device="cuda")
-            return t.view(dtype) if dtype != torch.uint8 else t
-
-        if st != OK:
-            return Drain(st, None, None, None, int(d.first_batch), int(d.n_batches))
-        return Drain(st, view(d.records, d.n_records * 48, torch.uint8),
-                     view(d.payload, d.n_payload * 4, torch.int32),
-                     view(d.topk, d.n_topk * 8, torch.uint8), int(d.first_batch),
-                     int(d.n_batches))
+        return Drain(st, d)
 
     def stats(self):
         return alto_agg_stats(self._h, self.stream.cuda_stream)

@@ -156,6 +156,30 @@ __device__ __forceinline__ u32 warp_take(bool want, u32* counter) {
   return want ? base + __popc(m & lanemask_lt()) : kNone;
 }
 
+// The same with one atomic on `counter` per block (a few thousand warps each
+// appending to one address serialise on it: about 0.65 ns an atomic on the
+// GB300).  All threads of the block call it together; sh.cnt is zero on entry
+// and on return.
+struct BlockTake {
+  u32 cnt;
+  u32 base;
+};
+__device__ __forceinline__ u32 block_take(bool want, u32* counter, BlockTake& sh) {
+  const int lane = threadIdx.x & 31;
+  const u32 m = __ballot_sync(0xFFFFFFFFu, want);
+  const int wl = __ffs(m) - 1;
+  u32 wbase = 0;
+  if (m != 0 && lane == wl) wbase = atomicAdd(&sh.cnt, (u32)__popc(m));
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    sh.base = sh.cnt ? atomicAdd(counter, sh.cnt) : 0u;
+    sh.cnt = 0;
+  }
+  __syncthreads();
+  if (m != 0) wbase = __shfl_sync(0xFFFFFFFFu, wbase, wl);
+  return want ? sh.base + wbase + __popc(m & lanemask_lt()) : kNone;
+}
+
 // ---------------------------------------------------------------------------
 // open-group hash table (linear probing; a slot index is the entry id)
 // ---------------------------------------------------------------------------
@@ -339,14 +363,23 @@ __device__ void free_chunk(const Arena& ar, Ctl* ctl, int j, u32 chunk) {
   if ((u64)pos < ar.stack_cap[j]) ar.stack[ar.stack_off[j] + (u64)pos] = chunk;
 }
 
-// Chunks for the growth of each requesting lane's two vectors of entry e:
+// Chunks for the growth of each requesting thread's two vectors of entry e:
 // every class that starts in [old, new) of a vector (vector 0 holds two int32
-// per leaf).  One free-stack atomic per chunk class and warp; a stack may go
-// negative, and k_check clears that before anything is freed.  All 32 lanes
-// call it together.
-__device__ void warp_grow(const Table& tab, const Arena& ar, Ctl* ctl, bool want, u32 e, u64 old0,
-                          u64 new0, u64 old1, u64 new1) {
-  const int lane = threadIdx.x & 31;
+// per leaf), with one free-stack atomic (and at most one bump atomic) per
+// chunk class and block.  A stack may go negative; the record scans' last
+// CTA (CapCheck) clears that before anything is freed.  All threads of the
+// block call it together; the counters in `sh` are zero on entry and on
+// return.
+struct GrowShared {
+  u32 cnt[kNumChunks];
+  u32 rank[kNumChunks];
+  int old[kNumChunks];
+  u32 avail[kNumChunks];
+  unsigned long long bump[kNumChunks];
+  unsigned long long got;
+};
+__device__ void block_grow(const Table& tab, const Arena& ar, Ctl* ctl, bool want, u32 e, u64 old0,
+                           u64 new0, u64 old1, u64 new1, GrowShared& sh) {
   int jf[kVecs], jl[kVecs];
   const u64 olds[kVecs] = {old0, old1}, news[kVecs] = {new0, new1};
 #pragma unroll
@@ -362,38 +395,37 @@ __device__ void warp_grow(const Table& tab, const Arena& ar, Ctl* ctl, bool want
       }
     }
   }
-  const int lo = __reduce_min_sync(0xFFFFFFFFu, min(jf[0], jf[1]));
-  const int hi = __reduce_max_sync(0xFFFFFFFFu, max(jl[0], jl[1]));
-  u64 got = 0;
-  for (int j = lo; j <= hi; ++j) {
-    const bool w0 = j >= jf[0] && j <= jl[0];
-    const bool w1 = j >= jf[1] && j <= jl[1];
-    const u32 m0 = __ballot_sync(0xFFFFFFFFu, w0), m1 = __ballot_sync(0xFFFFFFFFu, w1);
-    const u32 cnt = __popc(m0) + __popc(m1);
-    if (cnt == 0) continue;
-    const int leader = __ffs(m0 | m1) - 1;
+#pragma unroll
+  for (int v = 0; v < kVecs; ++v)
+    for (int j = jf[v]; j <= jl[v]; ++j) atomicAdd(&sh.cnt[j], 1u);
+  __syncthreads();
+  if (threadIdx.x < kNumChunks) {
+    const int j = threadIdx.x;
+    const u32 cnt = sh.cnt[j];
     int old = 0;
     u32 avail = 0;
     unsigned long long bump = 0;
-    if (lane == leader) {
+    if (cnt) {
       old = atomicSub(&ctl->top[j], (int)cnt);
       avail = (old <= 0) ? 0u : min((u32)old, cnt);
       if (cnt > avail)
         bump = atomicAdd((unsigned long long*)&ctl->bump, (unsigned long long)(cnt - avail) * chunk_size(j));
     }
-    old = __shfl_sync(0xFFFFFFFFu, old, leader);
-    avail = __shfl_sync(0xFFFFFFFFu, avail, leader);
-    bump = __shfl_sync(0xFFFFFFFFu, bump, leader);
-    const u32 lt = lanemask_lt();
+    sh.old[j] = old;
+    sh.avail[j] = avail;
+    sh.bump[j] = bump;
+  }
+  __syncthreads();
+  u64 got = 0;
 #pragma unroll
-    for (int v = 0; v < kVecs; ++v) {
-      if (!(v == 0 ? w0 : w1)) continue;
-      const u32 r = (v == 0) ? __popc(m0 & lt) : __popc(m0) + __popc(m1 & lt);
+  for (int v = 0; v < kVecs; ++v) {
+    for (int j = jf[v]; j <= jl[v]; ++j) {
+      const u32 r = atomicAdd(&sh.rank[j], 1u);
       u32 c;
-      if (r < avail) {
-        c = ar.stack[ar.stack_off[j] + (u64)(old - 1 - (int)r)];
+      if (r < sh.avail[j]) {
+        c = ar.stack[ar.stack_off[j] + (u64)(sh.old[j] - 1 - (int)r)];
       } else {
-        const u64 o = bump + (u64)(r - avail) * chunk_size(j);
+        const u64 o = sh.bump[j] + (u64)(r - sh.avail[j]) * chunk_size(j);
         if (o + chunk_size(j) > ar.elems) {
           raise_err(ctl, ALTO_ENOSPC);
           c = kNone;
@@ -407,7 +439,17 @@ __device__ void warp_grow(const Table& tab, const Arena& ar, Ctl* ctl, bool want
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) got += __shfl_xor_sync(0xFFFFFFFFu, got, o);
-  if (lane == 0 && got) atomicAdd((unsigned long long*)&ctl->arena_used, (unsigned long long)got);
+  if ((threadIdx.x & 31) == 0 && got) atomicAdd(&sh.got, (unsigned long long)got);
+  __syncthreads();
+  if (threadIdx.x < kNumChunks) {
+    sh.cnt[threadIdx.x] = 0;
+    sh.rank[threadIdx.x] = 0;
+  }
+  if (threadIdx.x == 0 && sh.got) {
+    atomicAdd((unsigned long long*)&ctl->arena_used, sh.got);
+    sh.got = 0;
+  }
+  __syncthreads();
 }
 
 // ---------------------------------------------------------------------------
@@ -1297,11 +1339,13 @@ __global__ void __launch_bounds__(kBigThreads) k_reduce_big(Dev d, Batch bv, int
 // level's touched list, and every item adds itself to the entry's batch
 // accumulators, warp-aggregated over lanes with the same entry.
 __device__ __forceinline__ void add_items(const Dev& d, Ctl* ctl, bool valid, u32 e, u32 rep, u32 c, u32 f,
-                                          u32 done, u32 cs, u32 sk, u32 ep, u32* list, u32* list_n) {
+                                          u32 done, u32 cs, u32 sk, u32 ep, u32* list, u32* list_n,
+                                          BlockTake* bsh = nullptr) {
   bool first = false;
   if (valid) first = atomicExch(&d.tab.hot[e].touch, ep) != ep;
   {
-    const u32 pos = warp_take(first, list_n);
+    // (with `bsh`, all threads of the block call this together)
+    const u32 pos = bsh ? block_take(first, list_n, *bsh) : warp_take(first, list_n);
     if (first) {
       if (pos < d.cfg.n_max) list[pos] = e;
       d.tab.hot[e].acc_rep = rep;
@@ -1529,14 +1573,27 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch bv, int l
   const u32 nt = min(ctl->n_segs[l], d.cfg.n_max);
   const u32 ep = ctl->epoch;
   const u32 ep7 = epoch7(ctl);
+  // appends to the done and touched lists and the chunk allocation take one
+  // atomic per block on their shared counters
   __shared__ u32 s_ins;
-  if (threadIdx.x == 0) s_ins = 0;
+  __shared__ BlockTake s_done, s_list;
+  __shared__ GrowShared s_grow;
+  if (threadIdx.x == 0) {
+    s_ins = 0;
+    s_done.cnt = 0;
+    s_list.cnt = 0;
+    s_grow.got = 0;
+  }
+  if (threadIdx.x < kNumChunks) {
+    s_grow.cnt[threadIdx.x] = 0;
+    s_grow.rank[threadIdx.x] = 0;
+  }
   __syncthreads();
   u32* nx_rep = d.sc.it_rep[in_set ^ 1];
   u32* nx_cseq = d.sc.it_cseq[in_set ^ 1];
   u32* nx_skey = d.sc.it_skey[in_set ^ 1];
   const u64 n = b.n;
-  const u32 end = (nt + 31) & ~31u;  // whole warps iterate together
+  const u32 end = (nt + kThreads - 1) / kThreads * kThreads;  // whole blocks iterate together
   for (u32 s = gtid(); s < end; s += gstride()) {
     const bool valid = s < nt;
     u32 e = 0, rep = 0, cmax = 0, smn = 0, blen = 0;
@@ -1590,8 +1647,8 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch bv, int l
       }
     }
     // the leaf level allocates the chunks of the reserved growth right here
-    if (LEAF && carry) warp_grow(d.tab, d.ar, ctl, grows, e, gv[0], gv[1], gv[2], gv[3]);
-    const u32 di = warp_take(complete, &ctl->n_done);
+    if (LEAF && carry) block_grow(d.tab, d.ar, ctl, grows, e, gv[0], gv[1], gv[2], gv[3], s_grow);
+    const u32 di = block_take(complete, &ctl->n_done, s_done);
     if (valid && complete) {
       if (di < d.sc.done_cap) {
         d.sc.done_e[di] = e;
@@ -1634,7 +1691,7 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch bv, int l
       }
       if (merge)
         add_items(d, ctl, e2 != kNone, e2, rep, c2, f2, complete ? 1u : 0u, cmax, smn, ep, list_next,
-                  &ctl->n_segs[l - 1]);
+                  &ctl->n_segs[l - 1], &s_list);
     }
   }
   __syncthreads();
