@@ -97,16 +97,16 @@ typedef int alto_status;
 #define ALTO_SCORE_TOPK 2
 
 /* Streaming release (flags bit 0; Sec. 3.2: the outputs of a pmap are put
- * back in order and passed on as a stream).  With the CONCAT level at the
- * leaf parent (D-1), every push also emits, for each still-open CONCAT group
- * whose run of present children 0..r-1 grew past the r it released before,
- * a partial record: ops = CONCAT | ALTO_OPS_PARTIAL, n_children = r, payload
- * = the newly released children's tokens in child order, score 0, no top-k,
- * completion_seq = the latest arrival among those children.  The group's
- * final record then carries only the children not released before (its other
- * fields are unchanged).  Records stay in (completion_seq, deeper first)
- * order.  EINVAL with no CONCAT level, with CONCAT above the leaf parent, and
- * for alto_agg_oneshot_noalloc. */
+ * back in order and passed on as a stream).  Every push also emits, for each
+ * still-open group of the CONCAT level whose run of complete children
+ * 0..r-1 grew past the r it released before, a partial record: ops = CONCAT
+ * | ALTO_OPS_PARTIAL, n_children = r, payload = the newly released children's
+ * concatenations in child order, score 0, no top-k, completion_seq = the
+ * latest completion seq among those children (at the leaf parent, the latest
+ * arrival).  The group's final record then carries only the children not
+ * released before (its other fields are unchanged).  Records stay in
+ * (completion_seq, deeper first) order.  EINVAL with no CONCAT level and for
+ * alto_agg_oneshot_noalloc. */
 #define ALTO_FLAG_STREAM_RELEASE 1
 #define ALTO_OPS_PARTIAL 0x80
 

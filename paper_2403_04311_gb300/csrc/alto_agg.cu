@@ -566,7 +566,7 @@ __global__ void __launch_bounds__(kThreads) k_ingest(Dev d, Batch bv) {
   __syncthreads();
   const int D = d.cfg.depth;
   const u32 ep7 = epoch7(ctl);
-  const bool sorted_leaf = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK || d.cfg.stream;
+  const bool sorted_leaf = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK || d.cfg.stream_leaf;
   for (u32 i = gtid(); i < b.n; i += gstride()) {
     u32 o0 = b.off[i], o1 = b.off[i + 1];
     if (o1 < o0 || (u64)o1 > b.n_payload) raise_err(ctl, ALTO_EINVAL);
@@ -926,7 +926,7 @@ __device__ void finalize_segment(const Dev& d, const Batch& b, Ctl* ctl, const R
   const int D = d.cfg.depth;
   const u64 n = b.n;
   const bool carry = LEAF && d.cfg.concat_level >= 0;
-  const bool strm = LEAF && d.cfg.stream;
+  const bool strm = LEAF && d.cfg.stream_leaf;
   if (!LEAF && chain_parent(d.cfg, l)) chain_sync(d.tab, d.ar, ctl, e);
   if (red.bad) raise_err(ctl, ALTO_EINCONSIST);
   if (l > 0 && d.tab.hot[e].up != b.tags[(u64)(l - 1) * n + rep0]) raise_err(ctl, ALTO_EINCONSIST);
@@ -1010,7 +1010,7 @@ __device__ __forceinline__ void reduce_small(const Dev& d, const Batch& b, Ctl* 
                                              u32 s, u32 j0, u32 j1, u32 gmask, int sub, bool topk, int K) {
   const u32 e = r.skeys[j0] & d.tab.mask;
   const u32 rep0 = LEAF ? min(r.sperm[j0], r.n_items - 1) : r.it_rep[min(r.sperm[j0], r.n_items - 1)];
-  const bool strm = LEAF && d.cfg.stream;
+  const bool strm = LEAF && d.cfg.stream_leaf;
   const u32 rel = strm ? d.tab.rel[e] : 0u;
   const Chain htag = load_chain(b, r.l, rep0);
   SegRed red;
@@ -1184,7 +1184,7 @@ __global__ void __launch_bounds__(kThreads) k_reduce(Dev d, Batch bv, int l, con
   const u32 gw = gtid() >> 5, nw = gstride() >> 5;
   const bool topk = d.cfg.score_op[l] == ALTO_SCORE_TOPK;
   const int K = d.cfg.topk_k[l];
-  const bool strm = LEAF && d.cfg.stream;
+  const bool strm = LEAF && d.cfg.stream_leaf;
   const ReduceArgs<LEAF> r = reduce_args<LEAF>(d, b, l, skeys, sperm, seg_start, in_set);
   for (u32 sb = gw * 4; sb < nseg; sb += nw * 4) {
     const u32 s = sb + grp;
@@ -1256,7 +1256,7 @@ __global__ void __launch_bounds__(kBigThreads) k_reduce_big(Dev d, Batch bv, int
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const bool topk = d.cfg.score_op[l] == ALTO_SCORE_TOPK;
   const int K = d.cfg.topk_k[l];
-  const bool strm = LEAF && d.cfg.stream;
+  const bool strm = LEAF && d.cfg.stream_leaf;
   const ReduceArgs<LEAF> r = reduce_args<LEAF>(d, b, l, skeys, sperm, seg_start, in_set);
   for (u32 q = blockIdx.x; q < nbig; q += gridDim.x) {
     const u32 s = d.sc.big_seg[(u64)l * d.sc.big_cap + q];
@@ -1698,6 +1698,153 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch bv, int l
   if (threadIdx.x == 0 && s_ins) atomicAdd((unsigned long long*)&ctl->live_groups, (u64)s_ins);
 }
 
+// ---------------------------------------------------------------------------
+// Streaming release with the CONCAT level M above the leaf parent (Sec. 3.2).
+// A group of level M receives its children as spans: a level-(M+1) group
+// that completes appends its concatenation to its parent's buffer.  Right
+// after level M has run, so that its touched list is still there:
+//   k_up_meta      the spans handed up in this batch get their meta entry
+//                  {child index, payload position} in the parent's buffer,
+//                  whose room the parent's finalize allocated;
+//   k_up_release   a warp per touched group of level M left open marks its
+//                  buffered children from `rel` on and finds the first one
+//                  missing: a run that grew is a partial release (a done
+//                  entry of its own, buffered children released);
+//   k_up_rel_seq   a release's completion seq is the latest among its
+//                  children completed in this batch (the one at `rel` is
+//                  one of them, or the run could not have grown);
+//   k_up_rel_mask  the releases take their places in the emission order.
+// The records scan, placement, gather, records and buffer compaction then
+// treat a release as at the leaf parent.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_up_meta(Dev d) {
+  pdl_enter();
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  if (*(const volatile int*)&ctl->batch_err) return;  // a parent entry may be unusable
+  const int M = d.cfg.concat_level;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  for (u32 di = gtid(); di < nd; di += gstride()) {
+    if ((int)d.sc.done_lvl[di] != M + 1) continue;
+    const u32 e = d.sc.done_e[di] & d.tab.mask;
+    const u32 P = d.tab.par[e] & d.tab.mask;
+    const u64 ap = d.tab.app[e];
+    const u64 m = ap >> 40;
+    if (m >= d.tab.vec_n[2 * (u64)P]) continue;
+    bool ok;
+    const u64 a = vec_addr(d.tab, P, 0, 2 * m, &ok);
+    if (!ok) continue;
+    d.ar.pool[a] = (int32_t)d.tab.cidx[e];
+    d.ar.pool[a + 1] = (int32_t)(u32)(ap & kPos40);
+  }
+}
+
+// `list`: level M's touched entries; with `seg_start`, the entries are the
+// sorted keys at the segment starts instead (a TOPK level M).
+__global__ void __launch_bounds__(kThreads) k_up_release(Dev d, const u32* list, const u32* seg_start) {
+  pdl_enter();
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl)) return;
+  if (*(const volatile int*)&ctl->batch_err) return;
+  const int M = d.cfg.concat_level;
+  const u32 nt = min(ctl->n_segs[M], d.cfg.n_max);
+  const u32 ep = ctl->epoch;
+  const int lane = threadIdx.x & 31;
+  const u32 gw = gtid() >> 5, nw = gstride() >> 5;
+  for (u32 w = gw; w < nt; w += nw) {
+    const u32 e = (seg_start ? list[seg_start[w]] : list[w]) & d.tab.mask;
+    if (d.tab.hot[e].done_epoch == ep) continue;  // completed by this batch: its final record
+    const u32 rel = d.tab.rel[e];
+    const u32 B = d.tab.vec_n[2 * (u64)e];
+    if (B == 0) continue;
+    // B buffered children cannot fill B + 1 bits: the run ends inside the map
+    const u64 words = (u64)B / 32 + 1;
+    unsigned long long base = 0;
+    if (lane == 0) base = atomicAdd((unsigned long long*)&ctl->bm_used, (unsigned long long)words);
+    base = __shfl_sync(0xFFFFFFFFu, base, 0);
+    if (base + words > d.sc.bm_cap) {
+      if (lane == 0) raise_err(ctl, ALTO_ENOSPC);
+      continue;
+    }
+    u32* bm = d.sc.bm + base;
+    for (u64 x = lane; x < words; x += 32) bm[x] = 0;
+    __syncwarp();
+    const u64 span = words * 32;
+    for (u32 k = lane; k < B; k += 32) {
+      bool ok;
+      const u64 a = vec_addr(d.tab, e, 0, 2 * (u64)k, &ok);
+      if (!ok) continue;
+      const u32 c = (u32)d.ar.pool[a];
+      if (c >= rel && (u64)(c - rel) < span) atomicOr(&bm[(c - rel) >> 5], 1u << ((c - rel) & 31));
+    }
+    __syncwarp();
+    u32 z = kNone;
+    for (u64 wb = 0; wb < words && z == kNone; wb += 32) {
+      const u64 x = wb + lane;
+      u32 cand = kNone;
+      if (x < words) {
+        const u32 free_bits = ~__ldcg(&bm[x]);
+        if (free_bits) cand = (u32)(x * 32) + (u32)(__ffs(free_bits) - 1);
+      }
+      z = __reduce_min_sync(0xFFFFFFFFu, cand);
+    }
+    if (z == kNone || z == 0) continue;  // child `rel` is still missing (or no room)
+    if (lane == 0) {
+      const u32 di = atomicAdd(&ctl->n_done, 1u);
+      const u32 q = atomicAdd(&ctl->n_rel, 1u);
+      if (di < d.sc.done_cap && q < d.cfg.n_max) {
+        d.sc.done_e[di] = e;
+        d.sc.done_lvl[di] = (u32)M;
+        d.sc.done_cseq[di] = 0;
+        d.sc.done_part[di] = 2u;  // every released child was buffered: the buffer is compacted
+        d.tab.rnew[e] = rel + z;
+        d.tab.hot[e].done_epoch = ep;
+        d.tab.done_idx[e] = di;
+        d.sc.rel_seg[q] = di;
+      } else {
+        raise_err(ctl, ALTO_ENOSPC);
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) k_up_rel_seq(Dev d) {
+  pdl_enter();
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl) || *(const volatile int*)&ctl->batch_err) return;
+  const int M = d.cfg.concat_level;
+  const u32 ep = ctl->epoch;
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  for (u32 di = gtid(); di < nd; di += gstride()) {
+    if ((int)d.sc.done_lvl[di] != M + 1) continue;
+    const u32 e = d.sc.done_e[di] & d.tab.mask;
+    const u32 P = d.tab.par[e] & d.tab.mask;
+    if (d.tab.hot[P].done_epoch != ep) continue;
+    const u32 dp = d.tab.done_idx[P];
+    if (dp >= nd || d.sc.done_part[dp] != 2u) continue;
+    const u32 c = d.tab.cidx[e];
+    if (c >= d.tab.rel[P] && c < d.tab.rnew[P]) atomicMax(&d.sc.done_cseq[dp], d.sc.done_cseq[di]);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) k_up_rel_mask(Dev d) {
+  pdl_enter();
+  Ctl* ctl = d.ctl;
+  if (poisoned(ctl) || *(const volatile int*)&ctl->batch_err) return;
+  const int D = d.cfg.depth, M = d.cfg.concat_level;
+  const u32 nr = min(ctl->n_rel, d.cfg.n_max);
+  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  for (u32 q = gtid(); q < nr; q += gstride()) {
+    const u32 di = d.sc.rel_seg[q];
+    if (di >= nd) continue;
+    const u32 cs = d.sc.done_cseq[di];
+    if (cs < ctl->n) {
+      atomicOr(&d.sc.mask[cs], 1u << (D - 1 - M));
+      atomicAdd(&d.sc.mblk[cs >> 5], 1u);
+    }
+  }
+}
+
 // Emission rank of each completed group: records completed at earlier
 // arrival indices, plus the deeper groups completed at the same index.  The
 // scan runs over runs of 32 seqs (their completion counts); a group adds the
@@ -2069,7 +2216,7 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch bv) {
     if (di >= nd) continue;
     const u32 c = tag_child(b.tags[(u64)(D - 1) * n + i]);
     if (c > d.tab.hot[e].last) continue;
-    const u32 rel = d.cfg.stream ? d.tab.rel[e] : 0u;  // children below were released earlier
+    const u32 rel = d.cfg.stream_leaf ? d.tab.rel[e] : 0u;  // children below were released earlier
     if (c < rel) continue;
     if (sc_mode == 3u && c >= d.tab.rnew[e]) continue;   // kept in the buffer
     const u64 slot = d.tab.dbase[e] + (c - rel);  // the group's first slot, from the count scan
@@ -2570,6 +2717,8 @@ __device__ u64 compact_buffer(const Dev& d, Ctl* ctl, u32 e) {
   if (lane == 0) {
     d.tab.vec_n[2 * (u64)e] = km;
     d.tab.vec_n[2 * (u64)e + 1] = kp;
+    // a group above the leaf parent takes its children's spans at its cursor
+    if (d.cfg.concat_level < d.cfg.depth - 1) d.tab.cur[e] = ((u64)km << 40) | kp;
   }
   return freed;
 }
@@ -2977,13 +3126,23 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   // groups it completes, payload): one block an SM for a small batch
   const int ugrid = small ? p.num_sms : p.num_sms * 2;
   bool forked = false;  // records and sweep on the second stream, beside the gather
+  // streaming release with the CONCAT level above the leaf parent: right
+  // after level M, the releases of its groups left open (see k_up_meta)
+  const bool stream_up = d.cfg.stream && !d.cfg.stream_leaf;
+  auto up_release = [&](const u32* list, const u32* seg_start) {
+    launch_pdl(k_up_meta, dgrid, kThreads, 0, s, d);
+    launch_pdl(k_up_release, ugrid, kThreads, 0, s, d, list, seg_start);
+    launch_pdl(k_up_rel_seq, dgrid, kThreads, 0, s, d);
+    launch_pdl(k_up_rel_mask, dgrid, kThreads, 0, s, d);
+    p.launches += 4;
+  };
   const u64 spin = d.cfg.spin_limit;
   int sl = 0;  // launches inside sort_pairs
   int site = 0;
   launch_pdl(k_ingest<G>, grid, kThreads, 0, s, d, bt);
   p.launches += 1;
   // streaming release needs each leaf parent's leaves together: the sorted path
-  const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK || d.cfg.stream;
+  const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK || d.cfg.stream_leaf;
   int set = 0;
   // touched entries of consecutive levels, alternately
   u32* lists[2] = {d.sc.up_seg_start, d.sc.up_list2};
@@ -3007,7 +3166,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     launch_pdl(k_reduce_big<true, G>, fit(p.num_sms, nb, kBigSeg), kBigThreads, 0, s, d, bt, D - 1,
                d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
     p.launches += 3;
-    if (d.cfg.stream) {
+    if (d.cfg.stream_leaf) {
       launch_pdl(k_reduce_rel<G>, fit(p.num_sms * blocks_per_sm((const void*)k_reduce_rel<G>), nb, 8), kThreads,
                  0, s, d, bt, d.sc.leaf_keys, d.sc.leaf_perm, d.sc.leaf_seg_start, set);
       p.launches += 1;
@@ -3042,6 +3201,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
       launch_pdl(k_up_finalize<false, G>, sgrid, kThreads, 0, s, d, bt, l, set, (const u32*)lists[li],
                  lists[li ^ 1]);
       p.launches += 1;
+      if (stream_up && l == M) up_release(lists[li], nullptr);
       li ^= 1;
       looked_up = true;
       added = l > 0 && d.cfg.score_op[l - 1] != ALTO_SCORE_TOPK;
@@ -3064,6 +3224,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     launch_pdl(k_reduce_big<false, G>, fit(p.num_sms, nb, kBigSeg), kBigThreads, 0, s, d, bt, l, d.sc.up_keys,
                d.sc.up_perm, d.sc.up_seg_start, set);
     p.launches += 3;
+    if (stream_up && l == M) up_release(d.sc.up_keys, d.sc.up_seg_start);
   }
   // emission order
   p.enter(5);
@@ -3397,9 +3558,8 @@ alto_status validate(const alto_agg_config* c) {
   if (c->flags & ~(int64_t)(ALTO_FLAG_STREAM_RELEASE | ALTO_FLAG_DOUBLE_RING | ALTO_FLAG_TEST_STALL |
                             ALTO_FLAG_DIRECT_LAUNCH))
     return ALTO_EINVAL;
-  // streaming release needs the CONCAT level at the leaf parent
-  if ((c->flags & ALTO_FLAG_STREAM_RELEASE) && c->payload_op[c->depth - 1] != ALTO_PAYLOAD_CONCAT)
-    return ALTO_EINVAL;
+  // streaming release needs a CONCAT level
+  if ((c->flags & ALTO_FLAG_STREAM_RELEASE) && nconcat == 0) return ALTO_EINVAL;
   if (c->max_batch_fragments < 1 || c->max_batch_fragments >= (1ll << 30)) return ALTO_EINVAL;
   if (c->max_batch_payload < 0 || c->max_batch_payload >= (1ll << 32)) return ALTO_EINVAL;
   if (c->max_open_groups < 0 || c->max_open_groups > (1ll << 25)) return ALTO_EINVAL;
@@ -3525,6 +3685,7 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   }
   d.cfg.has_score = has_score;
   d.cfg.stream = strm;
+  d.cfg.stream_leaf = strm && d.cfg.concat_level == D - 1;
   d.cfg.n_max = (u32)nmax;
   d.cfg.out_records = (u64)cfg.out_records;
   d.cfg.out_payload = (u64)cfg.out_payload_elems;

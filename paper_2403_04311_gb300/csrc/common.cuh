@@ -223,7 +223,8 @@ struct Cfg {
   int score_op[kMaxDepth];
   int topk_k[kMaxDepth];
   bool has_score;
-  bool stream;          // streaming release at the CONCAT (leaf-parent) level
+  bool stream;          // streaming release at the CONCAT level
+  bool stream_leaf;     // ... and that level is the leaf parent (the sorted leaf path releases)
   u32 n_max;
   u64 out_records, out_payload, out_topk, dense_cap;
   u64 spin_limit;
