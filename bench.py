@@ -578,6 +578,9 @@ def main():
                     help="open-group table capacity (default: every group of the stream)")
     ap.add_argument("--max-batches", type=int, default=0,
                     help="profiling only: push just the first B batches per step")
+    ap.add_argument("--profile-push", type=int, default=-1,
+                    help="profiling only: bracket push B of the first step with cudaProfilerStart/Stop "
+                         "(for a profiler started with profiling off)")
     args = ap.parse_args()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -629,14 +632,24 @@ def main():
     batches = [alto.to_device(s.batch(b)) for b in range(nb)]
     torch.cuda.synchronize()
 
+    profile_push = [args.profile_push]
+
     def step():
         nonlocal agg
         if args.max_batches > 0:
             # a truncated stream leaves groups open: start every step afresh
             agg.close()
             agg = alto.Aggregator(s.depth, s.payload_op, s.score_op, s.topk_k, stream=stream, **caps)
-        for db in batches:
+        for b, db in enumerate(batches):
+            mark = b == profile_push[0]
+            if mark:
+                torch.cuda.synchronize()
+                torch.cuda.profiler.start()
             st = agg.push(db.tags, db.off, db.payload, db.score)
+            if mark:
+                torch.cuda.synchronize()
+                torch.cuda.profiler.stop()
+                profile_push[0] = -1  # the first step only
             if st != alto.OK:
                 raise RuntimeError(f"push failed: {alto.STATUS_NAMES.get(st, st)}")
         d = agg.drain()
