@@ -2291,7 +2291,11 @@ __device__ __forceinline__ void dense_arena_body(const Dev& d, Ctl* ctl, u64 fir
 // cursor (one 64-bit atomic: leaf index and payload offset together) and is
 // copied there; a fragment of a group completed by this batch is placed at
 // its dense child slot.
-template <bool G>
+// PART 1: only the fragments of groups left open (their arena copies need
+// nothing after the leaf finalize, so they may run beside the upper levels);
+// PART 2: only the dense slots (this batch's fragments and the buffered
+// children of the completing groups); PART 3: both.
+template <bool G, int PART>
 __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch bv) {
   pdl_enter();
   const Batch b = batch_of<G>(bv, d);
@@ -2317,6 +2321,7 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch bv) {
       bs = d.tab.bstate[e];
       if (bs.x == ep) mode = bs.y;
       if (mode == 2 && !dense_ok) mode = 0;
+      if (!(PART & mode)) mode = 0;  // mode 1 is PART bit 1, mode 2 PART bit 2
     }
     if (mode == 2) {
       // every child index is below n_children (checked at completion); a
@@ -2388,7 +2393,7 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch bv) {
   // the completing groups' children buffered by earlier batches take their
   // dense slots in the same launch: other slots than the fragments' above,
   // and their latency overlaps that of the fragments
-  if (!ctl->skip_dense) dense_arena_body<true>(d, ctl, gtid(), gstride());
+  if ((PART & 2) && !ctl->skip_dense) dense_arena_body<true>(d, ctl, gtid(), gstride());
 }
 
 // The buffered children's dense slots in a launch of their own (the TOPK
@@ -3126,6 +3131,10 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   // groups it completes, payload): one block an SM for a small batch
   const int ugrid = small ? p.num_sms : p.num_sms * 2;
   bool forked = false;  // records and sweep on the second stream, beside the gather
+  // the side stream takes work beside the main one only without streaming
+  // release (whose compaction and partial flags order the tail)
+  const bool side_ok = p.s2 != nullptr && !d.cfg.stream;
+  bool carry_forked = false;  // the open groups' arena copies on the side stream
   // streaming release with the CONCAT level above the leaf parent: right
   // after level M, the releases of its groups left open (see k_up_meta)
   const bool stream_up = d.cfg.stream && !d.cfg.stream_leaf;
@@ -3180,6 +3189,16 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     launch_pdl(k_up_finalize<true, G>, sgrid, kThreads, 0, s, d, bt, D - 1, set,
                (const u32*)d.sc.leaf_seg_start, lists[li]);
     p.launches += 2;
+    if (side_ok && M == D - 1) {
+      // the open groups' leaves go to the arena on the side stream, beside
+      // the upper levels and the emission order (half the block slots, so
+      // that those latency-bound kernels still find room)
+      carry_forked = true;
+      cudaEventRecord(p.ev_fork, s);
+      cudaStreamWaitEvent(p.s2, p.ev_fork, 0);
+      launch_pdl(k_leaf_place<G, 1>, p.num_sms * 4, kThreads, 0, p.s2, d, bt);
+      p.launches += 1;
+    }
   }
   site += 5;
   p.enter(4);
@@ -3281,7 +3300,8 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
       // the leaf finalize already allocated the carried leaves' chunks; the
       // placement also places the children buffered by earlier batches
       p.enter(7);
-      launch_pdl(k_leaf_place<G>, grid, kThreads, 0, s, d, bt);
+      if (carry_forked) launch_pdl(k_leaf_place<G, 2>, grid, kThreads, 0, s, d, bt);
+      else launch_pdl(k_leaf_place<G, 3>, grid, kThreads, 0, s, d, bt);
     }
     if (leaf_sorted) launch_pdl(k_dense_arena<true>, ugrid, kThreads, 0, s, d);
     p.launches += leaf_sorted ? 5 : 1;
@@ -3309,7 +3329,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     // block slot per SM that the gather leaves free.  Not with streaming
     // release (the buffer compaction after the gather reads the partial
     // flags the records clear) or CONCAT above the leaf parent.
-    forked = p.s2 != nullptr && !d.cfg.stream && M == D - 1;
+    forked = side_ok && M == D - 1;
     int gather_grid = small ? p.num_sms : p.num_sms * blocks_per_sm((const void*)k_gather<G>);
     if (forked) {
       cudaEventRecord(p.ev_fork, s);
@@ -3329,6 +3349,10 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   if (forked) {
     cudaStreamWaitEvent(s, p.ev_join, 0);
     return;
+  }
+  if (carry_forked) {
+    cudaEventRecord(p.ev_join, p.s2);
+    cudaStreamWaitEvent(s, p.ev_join, 0);
   }
   if (d.cfg.stream) {
     // the released spans are out: drop them from the buffers they came from
@@ -3611,7 +3635,8 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     h->stage_launches[i] = 0;
   }
   if (cudaGetDevice(&h->device) != cudaSuccess ||
-      cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device) != cudaSuccess) {
+      cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device) != cudaSuccess ||
+      sort_prepare() != cudaSuccess) {
     delete h;
     return ALTO_ECUDA;
   }
@@ -4277,6 +4302,7 @@ extern "C" alto_status alto_agg_oneshot_noalloc(const alto_agg_config* cfg_in, c
       void* ptr = nullptr;
       if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || ptr == nullptr)
         return ALTO_ECUDA;
+      if (sort_prepare() != cudaSuccess) return ALTO_ECUDA;
       nd.base = (unsigned char*)ptr;
       nd.ready = true;
     }

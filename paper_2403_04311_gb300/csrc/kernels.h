@@ -38,8 +38,13 @@ struct SortBuffers {
 // by the low `bits` bits; the element count is read from n_dev on the device
 // and clamped to n_cap.  Returns the index (0/1) of the buffers holding the
 // result.  Uses launch sites site_base .. site_base + passes - 1.
+// A capacity of at most 8,192 pairs is sorted by one CTA in shared memory
+// (sort_prepare must have run on the device), a larger one by onesweep passes.
 int sort_pairs(const u32* n_dev, u32 n_cap, int bits, bool vals_identity, SortBuffers& b,
                Ctl* ctl, int site_base, u64 spin_limit, int num_sms, cudaStream_t s,
                int* launches);
+
+// Once per device before the first sort: the one-CTA sort's shared memory.
+cudaError_t sort_prepare();
 
 }  // namespace alto

@@ -457,7 +457,8 @@ extern "C" alto_status alto_router_create(const alto_router_config* cfg_in, cons
   h->h_ctl = nullptr;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+      cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      sort_prepare() != cudaSuccess) {
     delete h;
     return ALTO_ECUDA;
   }

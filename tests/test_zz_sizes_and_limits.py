@@ -163,13 +163,15 @@ def test_double_ring_keeps_a_drain_through_the_next(name, stream_release):
     assert s.n_batches > 2 and n_rec > 0
 
 
-_BOUNDARY_SIZES = [1, 31, 32, 33, 4095, 4096, 4097]
+_BOUNDARY_SIZES = [1, 31, 32, 33, 4095, 4096, 4097, 8191, 8192, 8193]
 
 
 def _boundary_batches(s):
-    """The stream cut into batches of 1, 31, 32, 33, 4,095, 4,096 and 4,097
-    fragments and the rest: around a warp (32) and around the tile of the
-    radix sort and the scans (4,096 elements)."""
+    """The stream cut into batches of 1, 31, 32, 33, 4,095, 4,096, 4,097,
+    8,191, 8,192 and 8,193 fragments and the rest: around a warp (32), the
+    tile of the radix sort and the scans (4,096 elements), and the largest
+    sort one CTA takes in shared memory (8,192 pairs; graph replays of pushes
+    up to 8K fragments launch only that form, larger ones both)."""
     import dataclasses
 
     sizes = _BOUNDARY_SIZES + [s.n - sum(_BOUNDARY_SIZES)]
@@ -181,7 +183,7 @@ def _boundary_batches(s):
 def test_batches_at_warp_and_tile_boundaries(leaf):
     """Every leaf form on batches around a warp and a sort/scan tile, bit for
     bit against the oracle."""
-    s = _boundary_batches(window_stream(5_000, 4, 200, 256, seed=11, topk=(leaf == "topk")))
+    s = _boundary_batches(window_stream(40_000, 4, 200, 256, seed=11, topk=(leaf == "topk")))
     o, g = run_both_stream(s, drain_every=1, stream_release=(leaf == "stream_release"))
     assert all(d.status == 0 for d in o)
     assert_same(o, g, f"boundary batches/{leaf}")
@@ -195,5 +197,5 @@ def test_route_batches_at_warp_and_tile_boundaries(policy, R):
     and sub-batches equal the routing oracle's."""
     import paper_2403_04311_gb300 as alto
 
-    s = _boundary_batches(window_stream(5_000, 4, 200, 256, seed=11))
+    s = _boundary_batches(window_stream(40_000, 4, 200, 256, seed=11))
     route_stream_vs_oracle(s, 1, R, alto.ROUTE_HASH if policy == "hash" else alto.ROUTE_LEAST_LOADED)
