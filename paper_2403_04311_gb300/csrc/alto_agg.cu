@@ -1904,6 +1904,10 @@ __global__ void __launch_bounds__(kThreads) k_done_rank(Dev d) {
     d.sc.r_dense_n[r] = (l == M) ? rend - rel : 0u;
     d.sc.r_topk_n[r] = (!part && d.cfg.score_op[l] == ALTO_SCORE_TOPK) ? min(nch, (u32)d.cfg.topk_k[l]) : 0u;
     d.sc.r_meta_n[r] = (l == M) ? d.tab.vec_n[2 * (u64)e] : 0u;
+    // a leaf parent of the CONCAT level: where this batch's leaves go is its
+    // dense base, r_dense_base[r] once the record scans ran (mode 4: by rank;
+    // the scans then write no per-entry state)
+    if (l == M && M == D - 1) d.tab.bstate[e] = make_uint4(ctl->epoch, 4u, r, 0u);
   }
 }
 
@@ -2199,7 +2203,7 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch bv) {
   const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
   if (no_copy(ctl) || ctl->skip_dense) return;
-  const int D = d.cfg.depth;
+  const int D = d.cfg.depth, M = d.cfg.concat_level;
   const u32 ep = ctl->epoch;
   const u64 n = b.n;
   const u32 nd = min(ctl->n_done, d.sc.done_cap);
@@ -2219,7 +2223,11 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch bv) {
     const u32 rel = d.cfg.stream_leaf ? d.tab.rel[e] : 0u;  // children below were released earlier
     if (c < rel) continue;
     if (sc_mode == 3u && c >= d.tab.rnew[e]) continue;   // kept in the buffer
-    const u64 slot = d.tab.dbase[e] + (c - rel);  // the group's first slot, from the count scan
+    // the group's first slot: by rank at the CONCAT level, from the chain
+    // scan below it
+    const u32 rk = d.sc.done_rank[di];
+    if (M == D - 1 && rk >= nd) continue;
+    const u64 slot = ((M == D - 1) ? d.sc.r_dense_base[rk] : d.tab.dbase[e]) + (c - rel);
     if (slot >= d.cfg.dense_cap) continue;
     const u32 old = atomicExch(&d.sc.dense[slot].x, ep);
     if (old == ep) raise_err(ctl, ALTO_EDUP);
@@ -2276,7 +2284,8 @@ __device__ __forceinline__ void dense_arena_body(const Dev& d, Ctl* ctl, u64 fir
       continue;
     }
     if (LEVEL_M && d.cfg.stream && d.sc.done_part[di] && c >= d.tab.rnew[e]) continue;
-    const u64 slot = d.tab.dbase[e] + (c - rel);
+    // level M: its first dense slot by rank; the levels below: by done index
+    const u64 slot = (LEVEL_M ? d.sc.r_dense_base[lo] : d.tab.dbase[e]) + (c - rel);
     if (slot >= d.cfg.dense_cap) continue;
     u32 old = atomicExch(&d.sc.dense[slot].x, ep);
     if (old == ep) raise_err(ctl, ALTO_EDUP);
@@ -2320,6 +2329,16 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch bv) {
       c = tag_child(b.tags[(u64)(D - 1) * n + i]);
       bs = d.tab.bstate[e];
       if (bs.x == ep) mode = bs.y;
+      u64 base = ((u64)bs.w << 32) | bs.z;
+      if (mode == 4) {
+        // a CONCAT-level leaf parent stamped with its rank: its dense base
+        // (the carried-leaves-only launch may run before the record scans,
+        // and does not need it)
+        mode = 2;
+        if (PART & 2) base = (bs.z < d.sc.done_cap) ? d.sc.r_dense_base[bs.z] : dcap;
+      }
+      bs.z = (u32)base;
+      bs.w = (u32)(base >> 32);
       if (mode == 2 && !dense_ok) mode = 0;
       if (!(PART & mode)) mode = 0;  // mode 1 is PART bit 1, mode 2 PART bit 2
     }
@@ -3257,8 +3276,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   const bool chain = M >= 0 && M < D - 1;  // levels below M hand spans up
   {
     CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0,
-                 d.sc.r_done, d.sc.done_e, d.tab.dbase, d.tab.mask,
-                 (M == D - 1) ? d.tab.bstate : nullptr, d.ctl};
+                 nullptr, nullptr, nullptr, d.tab.mask, nullptr, d.ctl};
     CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
     CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
     const CapCheck cc{d.cfg.out_records, d.cfg.dense_cap, d.cfg.out_topk, d.sc.done_cap};
