@@ -43,6 +43,7 @@
 #include "alto_agg.h"
 #include "common.cuh"
 #include "kernels.h"
+
 #include "scan.cuh"
 
 namespace alto {
@@ -107,6 +108,15 @@ struct Scratch {
   u32 big_cap;
   u32* rel_seg;          // [n_max] streaming: small leaf segments whose groups release a run
   Batch* batch;          // [1] the push's batch, stored by k_begin (read by graph replays)
+  // split placement (CONCAT at the leaf parent): the leaf parents ranked
+  // among themselves
+  u32* lblk;             // [n_max/32 + 1] leaf parents completing at the seqs of each run of 32
+  u32* lprefix;          // [n_max/32 + 1] leaf parents completing before each run
+  u32* l_done;           // [done_cap] by leaf rank: done index
+  u32* l_dense_n;        // [done_cap] by leaf rank: children
+  u32* l_meta_n;         // [done_cap] by leaf rank: buffered spans
+  u64* l_dense_base;     // [done_cap + 1] by leaf rank: first dense slot
+  u64* l_arena_base;     // [done_cap + 1] by leaf rank: first buffered span
 };
 
 struct Dev {
@@ -118,6 +128,14 @@ struct Dev {
   alto_record* out_rec;
   int32_t* out_pay;
   alto_topk_pair* out_topk;
+  // Split placement (set per batch by the host): with CONCAT at the leaf
+  // parent, the payload path of the leaf parents that complete (their ranks
+  // among themselves, dense slots, placement, length scan, gather) runs on a
+  // second stream beside the upper levels and the record scans.  Only leaf
+  // parents carry payload, and their order among themselves is their
+  // completion order, so the payload offsets need nothing from the levels
+  // above.
+  int split;
 };
 
 // The batch of the push.  Kernels launched one by one get it by value; in a
@@ -137,6 +155,12 @@ __device__ __forceinline__ bool poisoned(const Ctl* c) { return halted(c); }
 // outputs are undefined and its offsets may not be trustworthy.
 __device__ __forceinline__ bool no_copy(const Ctl* c) {
   return halted(c) || *(const volatile int*)&c->batch_err != 0;
+}
+// A split placement's kernels stand down on the errors raised before the
+// fork (the leaf finalize's snapshot), not on those the upper levels raise
+// beside them: what they find then does not depend on timing.
+__device__ __forceinline__ bool stand_down(const Dev& d, const Ctl* c) {
+  return d.split ? (halted(c) || *(const volatile int*)&c->pre_err != 0) : no_copy(c);
 }
 
 __device__ __forceinline__ u32 gtid() { return blockIdx.x * blockDim.x + threadIdx.x; }
@@ -547,6 +571,8 @@ __global__ void k_begin(Ctl* ctl, Batch b, Batch* store, int reset) {
   ctl->batch_err = 0;
   ctl->n_done = 0;
   ctl->skip_dense = 0;
+  ctl->skip_rec = 0;
+  ctl->pre_err = 0;
   ctl->dense_total = ctl->arena_total = ctl->pay_total = ctl->topk_total = ctl->n_emit = 0;
   ctl->bm_used = 0;
   ctl->n_rel = 0;
@@ -1659,6 +1685,8 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch bv, int l
         if (cmax < n) {
           atomicOr(&d.sc.mask[cmax], 1u << (D - 1 - l));
           atomicAdd(&d.sc.mblk[cmax >> 5], 1u);
+          // split placement: leaf parents are ranked among themselves
+          if (LEAF && d.split) atomicAdd(&d.sc.lblk[cmax >> 5], 1u);
         }
       } else {
         raise_err(ctl, ALTO_ENOSPC);
@@ -1696,6 +1724,18 @@ __global__ void __launch_bounds__(kThreads) k_up_finalize(Dev d, Batch bv, int l
   }
   __syncthreads();
   if (threadIdx.x == 0 && s_ins) atomicAdd((unsigned long long*)&ctl->live_groups, (u64)s_ins);
+  if (LEAF && d.split && threadIdx.x == 0) {
+    // the last CTA to finish leaves the batch's errors so far for the split
+    // placement (the block barrier above orders this CTA's raises before the
+    // fence; the other CTAs fenced theirs before counting)
+    __threadfence();
+    if (atomicAdd(&ctl->fin_ctr, 1u) == gridDim.x - 1) {
+      __threadfence();
+      ctl->fin_ctr = 0;
+      ctl->pre_err = *(volatile int*)&ctl->batch_err;
+      ctl->n_done_leaf = *(volatile u32*)&ctl->n_done;  // the upper levels append after these
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -1907,7 +1947,7 @@ __global__ void __launch_bounds__(kThreads) k_done_rank(Dev d) {
     // a leaf parent of the CONCAT level: where this batch's leaves go is its
     // dense base, r_dense_base[r] once the record scans ran (mode 4: by rank;
     // the scans then write no per-entry state)
-    if (l == M && M == D - 1) d.tab.bstate[e] = make_uint4(ctl->epoch, 4u, r, 0u);
+    if (l == M && M == D - 1 && !d.split) d.tab.bstate[e] = make_uint4(ctl->epoch, 4u, r, 0u);
   }
 }
 
@@ -1940,6 +1980,7 @@ struct CountScan {
     }
   }
   __device__ void total(Ctl* ctl, u64 t) const {
+    if (which == 3) return;  // an unused scan of a three-scan launch
     out_off[size(nullptr)] = t;
     if (which == 0) ctl->dense_total = t;
     else if (which == 1) ctl->topk_total = t;
@@ -2006,7 +2047,11 @@ struct ChainScan {
 // reads: other CTAs wrote the totals).
 struct CapCheck {
   static constexpr bool kActive = true;
+  static constexpr bool kSide = false;
   u64 out_records, dense_cap, out_topk, done_cap;
+  // split placement: the placement beside these scans checks the dense slots
+  // and the payload itself, and only the records stand down here
+  bool split = false;
   __device__ void operator()(Ctl* ctl) const {
     volatile Ctl* v = ctl;
     if (v->status != ALTO_OK || v->abort) return;
@@ -2017,11 +2062,79 @@ struct CapCheck {
     if (v->n_done > done_cap) bad = true;
     if (bad) {
       raise_err(ctl, ALTO_ENOSPC);
-      v->skip_dense = 1;
+      v->skip_rec = 1;
+      if (!split) v->skip_dense = 1;
     }
     // allocations of the level kernels may have taken a free stack below zero
     for (int j = 0; j < kNumChunks; ++j)
       if (v->top[j] < 0) v->top[j] = 0;
+  }
+};
+
+// Split placement, first step: the leaf parents completing before each run
+// of 32 arrival indices (the leaf finalize counted them per run).
+struct LeafRunScan {
+  const u32* lblk;
+  u32* lprefix;
+  __device__ u64 size(const Ctl* ctl) const { return (ctl->n + 31) >> 5; }
+  __device__ u64 value(u64 i) const { return lblk[i]; }
+  // only runs that completed a leaf parent are ever looked up
+  __device__ void out(u64 i, u64 excl, u64 v) const {
+    if (v) lprefix[i] = (u32)excl;
+  }
+  __device__ void total(Ctl*, u64) const {}
+};
+
+// Split placement: each leaf parent's rank among the leaf parents completing
+// in the batch (their emission order restricted to the leaf level: by
+// completion seq, at most one a seq), its children and buffered spans by
+// that rank, and its placement state (mode 4: its dense base by rank).  The
+// leaf parents are the done list's first n_done_leaf entries; the upper
+// levels append theirs, and set other bits of the masks, beside this kernel.
+__global__ void __launch_bounds__(kThreads) k_leaf_rank(Dev d) {
+  pdl_enter();
+  Ctl* ctl = d.ctl;
+  if (halted(ctl)) return;
+  const u32 nl = min(ctl->n_done_leaf, d.sc.done_cap);
+  for (u32 di = gtid(); di < nl; di += gstride()) {
+    const u32 e = d.sc.done_e[di] & d.tab.mask;
+    const u32 cs = d.sc.done_cseq[di];
+    if (cs >= ctl->n) continue;
+    const u32 b0 = cs & ~31u;
+    const uint4* m4 = reinterpret_cast<const uint4*>(d.sc.mask + b0);
+    u32 before = 0;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const uint4 v = m4[q];
+      const u32 s0 = b0 + 4 * q;
+      before += (s0 < cs ? (v.x & 1u) : 0) + (s0 + 1 < cs ? (v.y & 1u) : 0) + (s0 + 2 < cs ? (v.z & 1u) : 0) +
+                (s0 + 3 < cs ? (v.w & 1u) : 0);
+    }
+    const u32 r = d.sc.lprefix[cs >> 5] + before;
+    // the run's count is consumed (the next batch starts from zero)
+    d.sc.lblk[cs >> 5] = 0;
+    if (r >= nl) continue;
+    d.sc.l_done[r] = di;
+    d.sc.l_dense_n[r] = d.tab.hot[e].last + 1;
+    d.sc.l_meta_n[r] = d.tab.vec_n[2 * (u64)e];
+    d.tab.bstate[e] = make_uint4(ctl->epoch, 4u, r, 0u);
+  }
+}
+
+// The split placement's dense slots against their capacity, once its scans
+// have their totals (the placement, the length scan and the gather then
+// stand down).
+struct LeafCheck {
+  static constexpr bool kActive = true;
+  static constexpr bool kSide = true;
+  u64 dense_cap;
+  __device__ void operator()(Ctl* ctl) const {
+    volatile Ctl* v = ctl;
+    if (v->status != ALTO_OK || v->abort) return;
+    if (v->dense_total > dense_cap) {
+      raise_err(ctl, ALTO_ENOSPC);
+      v->skip_dense = 1;
+    }
   }
 };
 
@@ -2243,12 +2356,17 @@ __global__ void __launch_bounds__(kThreads) k_dense_batch(Dev d, Batch bv) {
 // groups of level M, by emission rank; otherwise the groups of levels M < l,
 // by done index.  (A warp per group with buffered spans, in place of the
 // binary search, measured slower: a few groups hold most of the spans.)
-template <bool LEVEL_M>
+template <bool LEVEL_M, bool SPLIT = false>
 __device__ __forceinline__ void dense_arena_body(const Dev& d, Ctl* ctl, u64 first, u64 stride) {
   const u32 ep = ctl->epoch;
-  const u32 nd = min(ctl->n_done, d.sc.done_cap);
+  // split placement: the leaf parents by their rank among themselves (the
+  // done list grows beside it)
+  const u32 nd = min(SPLIT ? ctl->n_done_leaf : ctl->n_done, d.sc.done_cap);
   const u64 na = LEVEL_M ? ctl->arena_total : ctl->chain_arena;
-  const u64* abase = LEVEL_M ? d.sc.r_arena_base : d.sc.c_arena_base;
+  const u64* abase = SPLIT ? d.sc.l_arena_base : LEVEL_M ? d.sc.r_arena_base : d.sc.c_arena_base;
+  const u32* by_rank = SPLIT ? d.sc.l_done : d.sc.r_done;
+  const u32* meta_n = SPLIT ? d.sc.l_meta_n : d.sc.r_meta_n;
+  const u64* dense_base = SPLIT ? d.sc.l_dense_base : d.sc.r_dense_base;
   for (u64 a = first; a < na; a += stride) {
     // last index x with abase[x] <= a: the one whose spans contain a
     u32 lo = 0, hi = nd;
@@ -2257,12 +2375,13 @@ __device__ __forceinline__ void dense_arena_body(const Dev& d, Ctl* ctl, u64 fir
       if (abase[mid] <= a) lo = mid;
       else hi = mid;
     }
-    const u32 di = LEVEL_M ? d.sc.r_done[lo] : lo;
+    const u32 di = LEVEL_M ? by_rank[lo] : lo;
     if (di >= nd) continue;
     if (!LEVEL_M && (int)d.sc.done_lvl[di] <= d.cfg.concat_level) continue;
     const u32 e = d.sc.done_e[di] & d.tab.mask;
     const u64 k = a - abase[lo];
-    const u32 mn = LEVEL_M ? d.sc.r_meta_n[lo] : d.tab.vec_n[2 * (u64)e];
+    const u32 mn = LEVEL_M ? meta_n[lo] : d.tab.vec_n[2 * (u64)e];
+    const u64 dbase = LEVEL_M ? dense_base[lo] : d.tab.dbase[e];
     if (k >= mn) continue;
     bool ok1, ok2 = true;
     u64 ma = vec_addr(d.tab, e, 0, 2 * k, &ok1);
@@ -2284,8 +2403,9 @@ __device__ __forceinline__ void dense_arena_body(const Dev& d, Ctl* ctl, u64 fir
       continue;
     }
     if (LEVEL_M && d.cfg.stream && d.sc.done_part[di] && c >= d.tab.rnew[e]) continue;
-    // level M: its first dense slot by rank; the levels below: by done index
-    const u64 slot = (LEVEL_M ? d.sc.r_dense_base[lo] : d.tab.dbase[e]) + (c - rel);
+    // level M: its first dense slot by rank (split: by its rank among the
+    // leaf parents); the levels below: by done index
+    const u64 slot = dbase + (c - rel);
     if (slot >= d.cfg.dense_cap) continue;
     u32 old = atomicExch(&d.sc.dense[slot].x, ep);
     if (old == ep) raise_err(ctl, ALTO_EDUP);
@@ -2309,7 +2429,7 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch bv) {
   pdl_enter();
   const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
-  if (no_copy(ctl)) return;
+  if (stand_down(d, ctl)) return;
   const int D = d.cfg.depth;
   const u32 ep = ctl->epoch;
   const u64 n = b.n;
@@ -2335,7 +2455,7 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch bv) {
         // (the carried-leaves-only launch may run before the record scans,
         // and does not need it)
         mode = 2;
-        if (PART & 2) base = (bs.z < d.sc.done_cap) ? d.sc.r_dense_base[bs.z] : dcap;
+        if (PART & 2) base = (bs.z < d.sc.done_cap) ? (d.split ? d.sc.l_dense_base : d.sc.r_dense_base)[bs.z] : dcap;
       }
       bs.z = (u32)base;
       bs.w = (u32)(base >> 32);
@@ -2412,7 +2532,10 @@ __global__ void __launch_bounds__(kThreads, 8) k_leaf_place(Dev d, Batch bv) {
   // the completing groups' children buffered by earlier batches take their
   // dense slots in the same launch: other slots than the fragments' above,
   // and their latency overlaps that of the fragments
-  if ((PART & 2) && !ctl->skip_dense) dense_arena_body<true>(d, ctl, gtid(), gstride());
+  if ((PART & 2) && !ctl->skip_dense) {
+    if (d.split) dense_arena_body<true, true>(d, ctl, gtid(), gstride());
+    else dense_arena_body<true>(d, ctl, gtid(), gstride());
+  }
 }
 
 // The buffered children's dense slots in a launch of their own (the TOPK
@@ -2435,8 +2558,10 @@ struct DenseScan {
   // payload, checked here against the ring (else k_check2 does it)
   bool check_payload;
   u64 out_payload;
+  bool split = false;  // split placement: stands down on the errors raised before the fork
   __device__ u64 size(const Ctl* ctl) const {
-    return (ctl->skip_dense || ctl->batch_err) ? 0 : ctl->dense_total + ctl->chain_total;
+    return (ctl->skip_dense || (split ? ctl->pre_err : ctl->batch_err)) ? 0
+                                                                         : ctl->dense_total + ctl->chain_total;
   }
   __device__ u64 value(u64 j) const {
     uint4 v = dense[j];
@@ -2502,7 +2627,7 @@ __global__ void __launch_bounds__(kThreads, 8) k_gather(Dev d, Batch bv) {
   pdl_enter();
   const Batch b = batch_of<G>(bv, d);
   Ctl* ctl = d.ctl;
-  if (no_copy(ctl) || ctl->skip_dense) return;
+  if (stand_down(d, ctl) || ctl->skip_dense) return;
   const int lane = threadIdx.x & 31, sub = lane % kSpanLanes, grp = lane / kSpanLanes;
   constexpr int kGroups = 32 / kSpanLanes;
   const u32 ep = ctl->epoch;
@@ -2782,7 +2907,7 @@ __global__ void __launch_bounds__(kThreads) k_records(Dev d) {
   }
   const int M = d.cfg.concat_level;
   const u32 nd = min(ctl->n_done, d.sc.done_cap);
-  const bool skip = ctl->skip_dense;
+  const bool skip = ctl->skip_dense || ctl->skip_rec;
   for (u32 base = blockIdx.x * blockDim.x; base < nd; base += gridDim.x * blockDim.x) {
     if (threadIdx.x < kNumChunks) {
       s_cnt[threadIdx.x] = 0;
@@ -2989,8 +3114,12 @@ struct alto_agg {
   };
   PushGraph graphs[2][3][4];  // [ring][profiling: off, stages, hot][batch size class]
   cudaStream_t cap_stream = nullptr;
-  cudaStream_t side = nullptr;          // direct launches: records and sweep beside the gather
-  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  // direct launches: the side streams (records and sweep beside the gather;
+  // with a split placement the leaf parents' payload path and the arena
+  // copies) and their events
+  cudaStream_t side = nullptr, side3 = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr, ev_dense = nullptr, ev_join3 = nullptr;
+  LookbackState lbs2{};                 // the split placement's look-back state
   std::vector<cudaEvent_t> cap_events;  // recorded at capture only (the graphs' templates hold them)
   bool direct_only = false;   // ALTO_FLAG_DIRECT_LAUNCH
   bool reset_pending = false; // a drain handed out the ring: the next push resets its counters
@@ -3020,8 +3149,9 @@ struct StageClock {
   // mark the start of stage `st` (stages must be entered in order); in the hot
   // mode only the boundaries around the leaf accumulate and the gather get an
   // event
-  void enter(int st) {
+  void enter(int st, cudaStream_t on = nullptr) {
     if (!h->profiling) return;
+    if (!on) on = s;
     while ((int)ev.size() <= st) {
       const int bnd = (int)ev.size();
       cudaEvent_t e = nullptr;
@@ -3030,8 +3160,8 @@ struct StageClock {
         // inside a stream capture only an external record becomes an
         // event-record node (a plain one just orders captured streams)
         if (e) {
-          if (capturing) cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
-          else cudaEventRecord(e, s);
+          if (capturing) cudaEventRecordWithFlags(e, on, cudaEventRecordExternal);
+          else cudaEventRecord(e, on);
         }
       }
       ev.push_back(e);
@@ -3103,14 +3233,33 @@ struct Pipeline {
   void (*stage)(void* ctx, int st, int64_t launches) = nullptr;
   void* stage_ctx = nullptr;
   // a second stream (with its fork and join events) on which the records and
-  // the table sweep run beside the payload gather; null: one stream
+  // the table sweep run beside the payload gather, or, with a split
+  // placement, the completing leaf parents' payload path; null: one stream
   cudaStream_t s2 = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  // split placement: a third stream for the open groups' arena copies, the
+  // second stream's look-back state, and the events after its length scan
+  // and at the end of the third stream
+  cudaStream_t s3 = nullptr;
+  cudaEvent_t ev_dense = nullptr, ev_join3 = nullptr;
+  LookbackState lbs2{};
   int64_t launches = 0;
+  void (*stage_on)(void* ctx, int st, int64_t launches, cudaStream_t on) = nullptr;
   void enter(int st) {
     if (stage) stage(stage_ctx, st, launches);
   }
+  // a stage boundary recorded on another stream (split placement: the gather)
+  void enter_on(int st, cudaStream_t on) {
+    if (stage_on) stage_on(stage_ctx, st, launches, on);
+    else enter(st);
+  }
 };
+
+// Launch sites of the split placement's scans (its rank scan, three
+// record-style scans and its length scan): above every site the main
+// stream's scans take (at most 5 + 5 (kMaxDepth - 1) + 4).
+constexpr int kSplitSite = kSites - 5;
+static_assert(5 + 5 * (kMaxDepth - 1) + 4 <= kSplitSite, "scan launch sites overlap");
 
 // Blocks of 256 threads of `kernel` resident per SM (cached per kernel): a
 // grid-stride kernel whose grid is exactly one wave has no ragged tail.
@@ -3153,7 +3302,15 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   // the side stream takes work beside the main one only without streaming
   // release (whose compaction and partial flags order the tail)
   const bool side_ok = p.s2 != nullptr && !d.cfg.stream;
-  bool carry_forked = false;  // the open groups' arena copies on the side stream
+  // streaming release needs each leaf parent's leaves together: the sorted path
+  const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK || d.cfg.stream_leaf;
+  // Split placement (CONCAT at the leaf parent, atomic leaf level): right
+  // after the leaf finalize, the open groups' arena copies go to the third
+  // stream and the completing leaf parents' payload path (their offsets by
+  // arrival index, the placement, the length scan, the gather) to the second,
+  // beside the upper levels and the record scans on this one.
+  const bool split = side_ok && p.s3 != nullptr && M == D - 1 && !leaf_sorted;
+  d.split = split ? 1 : 0;
   // streaming release with the CONCAT level above the leaf parent: right
   // after level M, the releases of its groups left open (see k_up_meta)
   const bool stream_up = d.cfg.stream && !d.cfg.stream_leaf;
@@ -3165,12 +3322,11 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     p.launches += 4;
   };
   const u64 spin = d.cfg.spin_limit;
+  const u32 dcap = d.sc.done_cap;
   int sl = 0;  // launches inside sort_pairs
   int site = 0;
   launch_pdl(k_ingest<G>, grid, kThreads, 0, s, d, bt);
   p.launches += 1;
-  // streaming release needs each leaf parent's leaves together: the sorted path
-  const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK || d.cfg.stream_leaf;
   int set = 0;
   // touched entries of consecutive levels, alternately
   u32* lists[2] = {d.sc.up_seg_start, d.sc.up_list2};
@@ -3208,15 +3364,42 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     launch_pdl(k_up_finalize<true, G>, sgrid, kThreads, 0, s, d, bt, D - 1, set,
                (const u32*)d.sc.leaf_seg_start, lists[li]);
     p.launches += 2;
-    if (side_ok && M == D - 1) {
-      // the open groups' leaves go to the arena on the side stream, beside
-      // the upper levels and the emission order (half the block slots, so
-      // that those latency-bound kernels still find room)
-      carry_forked = true;
+    if (split) {
       cudaEventRecord(p.ev_fork, s);
+      // the open groups' leaves to the arena (half the block slots, so that
+      // the latency-bound kernels beside them still find room)
+      cudaStreamWaitEvent(p.s3, p.ev_fork, 0);
+      launch_pdl(k_leaf_place<G, 1>, p.num_sms * 4, kThreads, 0, p.s3, d, bt);
+      cudaEventRecord(p.ev_join3, p.s3);
+      // the completing leaf parents ranked among themselves, their dense
+      // slots and buffered spans by that rank, their placement and the
+      // length scan; the records on this stream wait for those
       cudaStreamWaitEvent(p.s2, p.ev_fork, 0);
-      launch_pdl(k_leaf_place<G, 1>, p.num_sms * 4, kThreads, 0, p.s2, d, bt);
-      p.launches += 1;
+      LeafRunScan fr{d.sc.lblk, d.sc.lprefix};
+      launch_scan(p.lbs2, p.num_sms, d.ctl, fr, nb / 32 + 1, kSplitSite, spin, p.s2);
+      launch_pdl(k_leaf_rank, dgrid, kThreads, 0, p.s2, d);
+      {
+        const u32* nl = &d.ctl->n_done_leaf;
+        CountScan l0{d.sc.l_dense_n, d.sc.l_dense_base, nl, dcap, 0};
+        CountScan l1{d.sc.l_meta_n, d.sc.l_arena_base, nl, dcap, 2};
+        CountScan l2{nullptr, nullptr, nl, 0, 3};
+        launch_scan3(p.lbs2, d.ctl, l0, l1, l2, std::min<u64>(dcap, nb), kSplitSite + 1, spin, p.s2,
+                     LeafCheck{d.cfg.dense_cap});
+      }
+      // three quarters of the block slots: the upper levels and the record
+      // scans run beside it
+      launch_pdl(k_leaf_place<G, 2>, std::min(grid, p.num_sms * 6), kThreads, 0, p.s2, d, bt);
+      DenseScan fd{d.sc.dense, d.sc.dst, d.ctl, true, d.cfg.out_payload, true};
+      launch_scan(p.lbs2, p.num_sms, d.ctl, fd, d.cfg.dense_cap, kSplitSite + 4, spin, p.s2, small ? 32 : 0);
+      cudaEventRecord(p.ev_dense, p.s2);
+      // the gather leaves one block slot per SM to the records and the sweep
+      int gather_grid = small ? p.num_sms : p.num_sms * blocks_per_sm((const void*)k_gather<G>);
+      if (!small) gather_grid -= p.num_sms;
+      p.enter_on(8, p.s2);
+      k_gather<G><<<gather_grid, kThreads, 0, p.s2>>>(d, bt);
+      p.enter_on(9, p.s2);
+      cudaEventRecord(p.ev_join, p.s2);
+      p.launches += 7;
     }
   }
   site += 5;
@@ -3272,14 +3455,13 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   }
   launch_pdl(k_done_rank, dgrid, kThreads, 0, s, d);
   p.launches += 2;
-  const u32 dcap = d.sc.done_cap;
   const bool chain = M >= 0 && M < D - 1;  // levels below M hand spans up
   {
     CountScan f0{d.sc.r_dense_n, d.sc.r_dense_base, &d.ctl->n_done, dcap, 0,
                  nullptr, nullptr, nullptr, d.tab.mask, nullptr, d.ctl};
     CountScan f1{d.sc.r_topk_n, d.sc.r_topk_off, &d.ctl->n_done, dcap, 1};
     CountScan f2{d.sc.r_meta_n, d.sc.r_arena_base, &d.ctl->n_done, dcap, 2};
-    const CapCheck cc{d.cfg.out_records, d.cfg.dense_cap, d.cfg.out_topk, d.sc.done_cap};
+    const CapCheck cc{d.cfg.out_records, d.cfg.dense_cap, d.cfg.out_topk, d.sc.done_cap, split};
     const u64 dbound = std::min<u64>(dcap, (u64)nb * D);
     if (chain) launch_scan3(p.lbs, d.ctl, f0, f1, f2, dbound, site, spin, s, NoLast());
     else launch_scan3(p.lbs, d.ctl, f0, f1, f2, dbound, site, spin, s, cc);
@@ -3306,6 +3488,18 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     p.launches += 1;
     site += 3;
   }
+  if (split) {
+    // the records take their payload offsets from the length scan; the
+    // sweep ends the batch, so it also waits for the arena copies
+    cudaStreamWaitEvent(s, p.ev_dense, 0);
+    launch_pdl(k_records, dgrid, kThreads, 0, s, d);
+    cudaStreamWaitEvent(s, p.ev_join3, 0);
+    launch_pdl(k_sweep, dgrid, kThreads, 0, s, d);
+    cudaStreamWaitEvent(s, p.ev_join, 0);
+    p.launches += 2;
+    p.enter(9);
+    return;
+  }
   if (M >= 0) {
     p.enter(6);
     if (leaf_sorted) {
@@ -3318,8 +3512,7 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
       // the leaf finalize already allocated the carried leaves' chunks; the
       // placement also places the children buffered by earlier batches
       p.enter(7);
-      if (carry_forked) launch_pdl(k_leaf_place<G, 2>, grid, kThreads, 0, s, d, bt);
-      else launch_pdl(k_leaf_place<G, 3>, grid, kThreads, 0, s, d, bt);
+      launch_pdl(k_leaf_place<G, 3>, grid, kThreads, 0, s, d, bt);
     }
     if (leaf_sorted) launch_pdl(k_dense_arena<true>, ugrid, kThreads, 0, s, d);
     p.launches += leaf_sorted ? 5 : 1;
@@ -3368,10 +3561,6 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     cudaStreamWaitEvent(s, p.ev_join, 0);
     return;
   }
-  if (carry_forked) {
-    cudaEventRecord(p.ev_join, p.s2);
-    cudaStreamWaitEvent(s, p.ev_join, 0);
-  }
   if (d.cfg.stream) {
     // the released spans are out: drop them from the buffers they came from
     launch_pdl(k_stream_compact, ugrid, kThreads, 0, s, d);
@@ -3417,6 +3606,28 @@ struct PushRec {
   PushRec(alto_agg* h_, cudaStream_t s) : h(h_), clk(h_, s) {}
 };
 
+void free_side_streams(alto_agg* h) {
+  for (cudaStream_t* x : {&h->side, &h->side3})
+    if (*x) cudaStreamDestroy(*x);
+  for (cudaEvent_t* x : {&h->ev_fork, &h->ev_join, &h->ev_dense, &h->ev_join3})
+    if (*x) cudaEventDestroy(*x);
+  h->side = h->side3 = nullptr;
+  h->ev_fork = h->ev_join = h->ev_dense = h->ev_join3 = nullptr;
+}
+
+// The side streams and their events, made once; false (and none kept) if
+// any could not be made: the push then runs on its own stream alone.
+bool make_side_streams(alto_agg* h) {
+  if (h->side) return true;
+  bool ok = cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) == cudaSuccess &&
+            cudaStreamCreateWithFlags(&h->side3, cudaStreamNonBlocking) == cudaSuccess;
+  for (cudaEvent_t* x : {&h->ev_fork, &h->ev_join, &h->ev_dense, &h->ev_join3})
+    ok = ok && cudaEventCreateWithFlags(x, cudaEventDisableTiming) == cudaSuccess;
+  if (!ok) free_side_streams(h);
+  cudaGetLastError();
+  return ok;
+}
+
 // The whole launch sequence of one push on stream s: k_begin and the
 // pipeline.  G: the kernels read the batch that k_begin stores (graph capture).
 // Returns the number of kernels.
@@ -3433,24 +3644,16 @@ int64_t launch_push(alto_agg* h, cudaStream_t s, const Batch& bt, int reset, Pus
   p.nmax = (u32)h->cfg.max_batch_fragments;
   p.nb = nb;
   p.s = s;
-  // kernel-by-kernel launches run the records beside the gather on the
-  // handle's side stream (not with an event at every stage boundary)
-  if (!G && !(h->profiling && h->profile_mode == ALTO_PROFILE_STAGES)) {
-    if (!h->side && cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) == cudaSuccess) {
-      if (cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
-          cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess) {
-        if (h->ev_fork) cudaEventDestroy(h->ev_fork);
-        cudaStreamDestroy(h->side);
-        h->side = nullptr;
-        h->ev_fork = h->ev_join = nullptr;
-      }
-    }
-    cudaGetLastError();
-    if (h->side) {
-      p.s2 = h->side;
-      p.ev_fork = h->ev_fork;
-      p.ev_join = h->ev_join;
-    }
+  // kernel-by-kernel launches put work beside the main stream on the
+  // handle's side streams (not with an event at every stage boundary)
+  if (!G && !(h->profiling && h->profile_mode == ALTO_PROFILE_STAGES) && make_side_streams(h)) {
+    p.s2 = h->side;
+    p.s3 = h->side3;
+    p.ev_fork = h->ev_fork;
+    p.ev_join = h->ev_join;
+    p.ev_dense = h->ev_dense;
+    p.ev_join3 = h->ev_join3;
+    p.lbs2 = h->lbs2;
   }
   p.stage = [](void* ctx, int st, int64_t launches) {
     PushRec* r = (PushRec*)ctx;
@@ -3458,6 +3661,13 @@ int64_t launch_push(alto_agg* h, cudaStream_t s, const Batch& bt, int reset, Pus
     r->l0 = launches;
     r->stage = st;
     r->clk.enter(st);
+  };
+  p.stage_on = [](void* ctx, int st, int64_t launches, cudaStream_t on) {
+    PushRec* r = (PushRec*)ctx;
+    r->stage_l[r->stage] += launches - r->l0;
+    r->l0 = launches;
+    r->stage = st;
+    r->clk.enter(st, on);
   };
   p.stage_ctx = rec;
   rec->clk.enter(0);
@@ -3556,11 +3766,7 @@ void free_graphs(alto_agg* h) {
   h->cap_events.clear();
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
   h->cap_stream = nullptr;
-  if (h->side) cudaStreamDestroy(h->side);
-  if (h->ev_fork) cudaEventDestroy(h->ev_fork);
-  if (h->ev_join) cudaEventDestroy(h->ev_join);
-  h->side = nullptr;
-  h->ev_fork = h->ev_join = nullptr;
+  free_side_streams(h);
 }
 
 void free_all(alto_agg* h, cudaStream_t s) {
@@ -3792,6 +3998,15 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     ALLOC(d.tab.cidx, u32, T);
     ALLOC(d.tab.app, u64, T);
   }
+  if (concat == D - 1) {
+    ALLOC(sc.lblk, u32, nmax / 32 + 1);
+    ALLOC(sc.lprefix, u32, nmax / 32 + 1);
+    ALLOC(sc.l_done, u32, done_cap);
+    ALLOC(sc.l_dense_n, u32, done_cap);
+    ALLOC(sc.l_meta_n, u32, done_cap);
+    ALLOC(sc.l_dense_base, u64, done_cap + 1);
+    ALLOC(sc.l_arena_base, u64, done_cap + 1);
+  }
   ALLOC(sc.pairset, u64, PS);
   ALLOC(sc.batch, Batch, 1);
   sc.big_cap = (u32)(nmax / kBigSeg + 1);
@@ -3809,8 +4024,12 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
     ALLOC(sc.rel_seg, u32, nmax);
   }
   const u64 scan_tiles = std::max<u64>(std::max<u64>(dense_cap, done_cap), nmax) / kScanTile + 2;
-  ALLOC(h->lbs.desc, ulonglong2, 3 * scan_tiles);
+  // three look-back regions for the main stream's scans, three for the
+  // split placement's
+  ALLOC(h->lbs.desc, ulonglong2, 6 * scan_tiles);
   h->lbs.tiles = scan_tiles;
+  h->lbs2.desc = h->lbs.desc ? h->lbs.desc + 3 * scan_tiles : nullptr;
+  h->lbs2.tiles = scan_tiles;
   const int rings = (cfg.flags & ALTO_FLAG_DOUBLE_RING) ? 2 : 1;
   for (int r = 0; r < 2; ++r) {
     h->ring_rec[r] = nullptr;
@@ -3853,7 +4072,8 @@ alto_status alto_agg_create(const alto_agg_config* cfg_in, const alto_allocator*
   cudaMemsetAsync(sc.pairset, 0, sizeof(u64) * PS, s);
   cudaMemsetAsync(h->leaf_sort.hist, 0, sizeof(u32) * 4 * 256, s);
   cudaMemsetAsync(h->leaf_sort.lookback, 0, sizeof(u64) * sort_tiles * 256, s);
-  cudaMemsetAsync(h->lbs.desc, 0, sizeof(ulonglong2) * 3 * scan_tiles, s);
+  cudaMemsetAsync(h->lbs.desc, 0, sizeof(ulonglong2) * 6 * scan_tiles, s);
+  if (concat == D - 1) cudaMemsetAsync(sc.lblk, 0, sizeof(u32) * (nmax / 32 + 1), s);
   if (concat >= 0) cudaMemsetAsync(sc.dense, 0, sizeof(uint4) * std::max<u64>(dense_cap, 1), s);
   if (strm) cudaMemsetAsync(sc.done_part, 0, sizeof(u32) * done_cap, s);
   if (cudaGetLastError() != cudaSuccess) {

@@ -49,6 +49,12 @@ struct Ctl {
   u32 n_segs[kMaxDepth];   // distinct level-l groups in the batch
   u32 n_done;              // groups completed by the batch
   u32 skip_dense;          // set when a capacity check failed for this batch
+  u32 skip_rec;            // the record scans' capacity check failed: no records (with a
+                           // split placement that check leaves skip_dense to the placement's own)
+  int pre_err;             // split placement: batch_err as the leaf finalize left it
+  u32 n_done_leaf;         // split placement: leaf parents completed (done list 0..n-1)
+  u32 fin_ctr;             // split placement: leaf finalize CTAs finished
+  u32 last_ctr2;           // as last_ctr, for the split placement's scans
   u64 dense_total;         // children of CONCAT groups completing in this batch
   u64 arena_total;         // buffered leaves of those groups
   u64 pay_total;           // payload elements emitted by this batch

@@ -264,7 +264,7 @@ __device__ __forceinline__ void scan_body(const F& f, LookbackState st, Ctl* ctl
 }
 
 template <class F>
-__global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ctl* ctl, int site,
+__global__ void __launch_bounds__(kScanThreads, 2) k_scan(F f, LookbackState st, Ctl* ctl, int site,
                                                        u32* exit_ctr, u64 spin_limit) {
   pdl_enter();
   scan_body(f, st, ctl, site, exit_ctr, spin_limit);
@@ -273,6 +273,7 @@ __global__ void __launch_bounds__(kScanThreads) k_scan(F f, LookbackState st, Ct
 // No work after the last CTA of a multi-scan launch.
 struct NoLast {
   static constexpr bool kActive = false;
+  static constexpr bool kSide = false;
   __device__ void operator()(Ctl*) const {}
 };
 
@@ -280,21 +281,25 @@ struct NoLast {
 // with its own launch site (tile and exit counters) and look-back arrays.
 // When L is active, the launch's last CTA to finish runs `last` once every
 // scan's total is written (so a check of the totals needs no launch of its
-// own); it must read what other CTAs wrote with volatile loads.
+// own); it must read what other CTAs wrote with volatile loads.  L::kSide
+// selects the CTA counter of a launch that may run beside another one.
 template <class F, class L>
-__global__ void __launch_bounds__(kScanThreads) k_scan3(F f0, F f1, F f2, LookbackState st0,
+__global__ void __launch_bounds__(kScanThreads, 2) k_scan3(F f0, F f1, F f2, LookbackState st0,
                                                         LookbackState st1, LookbackState st2,
                                                         Ctl* ctl, int site, u64 spin_limit, L last) {
   pdl_enter();
   const int y = blockIdx.y;
-  const F& f = (y == 0) ? f0 : (y == 1) ? f1 : f2;
-  const LookbackState st = (y == 0) ? st0 : (y == 1) ? st1 : st2;
-  scan_body(f, st, ctl, site + y, &ctl->exit_ctr[site + y], spin_limit);
+  // one inlined body per scan: selecting a functor at run time would copy it
+  // to local memory
+  if (y == 0) scan_body(f0, st0, ctl, site, &ctl->exit_ctr[site], spin_limit);
+  else if (y == 1) scan_body(f1, st1, ctl, site + 1, &ctl->exit_ctr[site + 1], spin_limit);
+  else scan_body(f2, st2, ctl, site + 2, &ctl->exit_ctr[site + 2], spin_limit);
   if (L::kActive && threadIdx.x == 0) {
     __threadfence();
-    const u32 k = atomicAdd(&ctl->last_ctr, 1u);
+    u32* ctr = L::kSide ? &ctl->last_ctr2 : &ctl->last_ctr;
+    const u32 k = atomicAdd(ctr, 1u);
     if (k == gridDim.x * gridDim.y - 1) {
-      ctl->last_ctr = 0;
+      *ctr = 0;
       __threadfence();
       last(ctl);
     }
