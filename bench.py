@@ -665,17 +665,15 @@ def main():
     n_partial_step = int(((d.records.view(-1, 48)[:, 41] & 0x80) != 0).sum().item()) if n_records_step else 0
 
     # ---- timed region: device-resident inputs -------------------------------
-    # CUDA events on the push stream around the two heaviest kernels only (the
-    # leaf accumulate and the gather, four events a push), so that every other
-    # kernel boundary runs as it does without measurement.  Pushes of at most
-    # 128K fragments replay a captured graph, where four event nodes add about
-    # 25 us to an 8K-fragment push: those workloads time the two kernels in a
-    # separate pass right after the timed region instead.
-    hot_in_timed = int(max(s.batch_sizes)) > (1 << 17)
+    # No events inside the pushes: four event records a push around the two
+    # heaviest kernels (the leaf accumulate and the gather) cost 3.5% of the
+    # 16M-fragment pass (each one ends a programmatic overlap of neighbouring
+    # kernels) and, as event nodes of a replayed graph, about 25 us of an
+    # 8K-fragment push.  The two kernels are timed with those events in a
+    # separate pass of the same pushes right after the timed region.
     sampler = ClockSampler(local_rank)
     agg.profile(alto.PROFILE_HOT)
-    if not hot_in_timed:
-        agg.profile(False)  # the launch count restarts; no events
+    agg.profile(False)  # the launch count restarts; no events
     barrier(dist)
     torch.cuda.synchronize()
     sampler.start()
@@ -690,19 +688,17 @@ def main():
     clocks = sampler.stop()
     _st, prof = agg.profile_read()
     agg.profile(False)
-    kernel_timing = "CUDA events around the two kernels inside the timed region"
-    if not hot_in_timed:
-        launches_timed = prof["launches"]
-        k_steps = max(1, min(args.steps, 3))
-        agg.profile(alto.PROFILE_HOT)
-        for _ in range(k_steps):
-            step()
-        torch.cuda.synchronize()
-        _st, prof = agg.profile_read()
-        agg.profile(False)
-        prof["launches"] = launches_timed
-        kernel_timing = (f"CUDA events around the two kernels in a separate pass of {k_steps} step(s) "
-                         "after the timed region (the pushes replay a captured graph)")
+    launches_timed = prof["launches"]
+    k_steps = max(1, min(args.steps, 3))
+    agg.profile(alto.PROFILE_HOT)
+    for _ in range(k_steps):
+        step()
+    torch.cuda.synchronize()
+    _st, prof = agg.profile_read()
+    agg.profile(False)
+    prof["launches"] = launches_timed
+    kernel_timing = (f"CUDA events around the two kernels in a separate pass of {k_steps} step(s) "
+                     "right after the timed region (events inside the pushes slow the path)")
     ms = max_over_ranks(t_start.elapsed_time(t_end), dist)
     ms_per_step = ms / args.steps
     frags_per_step = s.n

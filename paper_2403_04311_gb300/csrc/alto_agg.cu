@@ -3644,9 +3644,10 @@ int64_t launch_push(alto_agg* h, cudaStream_t s, const Batch& bt, int reset, Pus
   p.nmax = (u32)h->cfg.max_batch_fragments;
   p.nb = nb;
   p.s = s;
-  // kernel-by-kernel launches put work beside the main stream on the
-  // handle's side streams (not with an event at every stage boundary)
-  if (!G && !(h->profiling && h->profile_mode == ALTO_PROFILE_STAGES) && make_side_streams(h)) {
+  // work beside the main stream goes to the handle's side streams (in a
+  // capture they become branches of the graph; not with an event at every
+  // stage boundary)
+  if (!(h->profiling && h->profile_mode == ALTO_PROFILE_STAGES) && make_side_streams(h)) {
     p.s2 = h->side;
     p.s3 = h->side3;
     p.ev_fork = h->ev_fork;
