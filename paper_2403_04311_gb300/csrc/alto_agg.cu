@@ -3366,10 +3366,9 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
     p.launches += 2;
     if (split) {
       cudaEventRecord(p.ev_fork, s);
-      // the open groups' leaves to the arena (half the block slots, so that
-      // the latency-bound kernels beside them still find room)
+      // the open groups' leaves to the arena
       cudaStreamWaitEvent(p.s3, p.ev_fork, 0);
-      launch_pdl(k_leaf_place<G, 1>, p.num_sms * 4, kThreads, 0, p.s3, d, bt);
+      launch_pdl(k_leaf_place<G, 1>, grid, kThreads, 0, p.s3, d, bt);
       cudaEventRecord(p.ev_join3, p.s3);
       // the completing leaf parents ranked among themselves, their dense
       // slots and buffered spans by that rank, their placement and the
@@ -3619,7 +3618,11 @@ void free_side_streams(alto_agg* h) {
 // any could not be made: the push then runs on its own stream alone.
 bool make_side_streams(alto_agg* h) {
   if (h->side) return true;
-  bool ok = cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) == cudaSuccess &&
+  // the second stream carries the split placement's critical path: its
+  // blocks go first when blocks of the other streams retire
+  int lo_pr = 0, hi_pr = 0;
+  if (cudaDeviceGetStreamPriorityRange(&lo_pr, &hi_pr) != cudaSuccess) lo_pr = hi_pr = 0;
+  bool ok = cudaStreamCreateWithPriority(&h->side, cudaStreamNonBlocking, hi_pr) == cudaSuccess &&
             cudaStreamCreateWithFlags(&h->side3, cudaStreamNonBlocking) == cudaSuccess;
   for (cudaEvent_t* x : {&h->ev_fork, &h->ev_join, &h->ev_dense, &h->ev_join3})
     ok = ok && cudaEventCreateWithFlags(x, cudaEventDisableTiming) == cudaSuccess;
