@@ -3306,9 +3306,9 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
   const bool leaf_sorted = d.cfg.score_op[D - 1] == ALTO_SCORE_TOPK || d.cfg.stream_leaf;
   // Split placement (CONCAT at the leaf parent, atomic leaf level): right
   // after the leaf finalize, the open groups' arena copies go to the third
-  // stream and the completing leaf parents' payload path (their offsets by
-  // arrival index, the placement, the length scan, the gather) to the second,
-  // beside the upper levels and the record scans on this one.
+  // stream and the completing leaf parents' payload path (their ranks among
+  // themselves and offsets, the placement, the length scan, the gather) to
+  // the second, beside the upper levels and the record scans on this one.
   const bool split = side_ok && p.s3 != nullptr && M == D - 1 && !leaf_sorted;
   d.split = split ? 1 : 0;
   // streaming release with the CONCAT level above the leaf parent: right
