@@ -574,6 +574,7 @@ __global__ void k_begin(Ctl* ctl, Batch b, Batch* store, int reset) {
   ctl->skip_rec = 0;
   ctl->pre_err = 0;
   ctl->dense_total = ctl->arena_total = ctl->pay_total = ctl->topk_total = ctl->n_emit = 0;
+  ctl->leaf_dense_total = ctl->leaf_arena_total = 0;
   ctl->bm_used = 0;
   ctl->n_rel = 0;
   for (int l = 0; l < kMaxDepth; ++l) ctl->n_big[l] = 0;
@@ -1957,7 +1958,7 @@ struct CountScan {
   u64* out_off;
   const u32* n_dev;
   u32 cap;
-  int which;  // 0 dense, 1 topk, 2 arena
+  int which;  // 0 dense, 1 topk, 2 arena; split placement: 3 unused, 4 dense, 5 arena
   // dense only: also leave each completing group's first slot in its entry
   const u32* r_done = nullptr;
   const u32* done_e = nullptr;
@@ -1984,7 +1985,9 @@ struct CountScan {
     out_off[size(nullptr)] = t;
     if (which == 0) ctl->dense_total = t;
     else if (which == 1) ctl->topk_total = t;
-    else ctl->arena_total = t;
+    else if (which == 2) ctl->arena_total = t;
+    else if (which == 4) ctl->leaf_dense_total = t;
+    else ctl->leaf_arena_total = t;
   }
 };
 
@@ -2131,7 +2134,7 @@ struct LeafCheck {
   __device__ void operator()(Ctl* ctl) const {
     volatile Ctl* v = ctl;
     if (v->status != ALTO_OK || v->abort) return;
-    if (v->dense_total > dense_cap) {
+    if (v->leaf_dense_total > dense_cap) {
       raise_err(ctl, ALTO_ENOSPC);
       v->skip_dense = 1;
     }
@@ -2362,7 +2365,7 @@ __device__ __forceinline__ void dense_arena_body(const Dev& d, Ctl* ctl, u64 fir
   // split placement: the leaf parents by their rank among themselves (the
   // done list grows beside it)
   const u32 nd = min(SPLIT ? ctl->n_done_leaf : ctl->n_done, d.sc.done_cap);
-  const u64 na = LEVEL_M ? ctl->arena_total : ctl->chain_arena;
+  const u64 na = SPLIT ? ctl->leaf_arena_total : LEVEL_M ? ctl->arena_total : ctl->chain_arena;
   const u64* abase = SPLIT ? d.sc.l_arena_base : LEVEL_M ? d.sc.r_arena_base : d.sc.c_arena_base;
   const u32* by_rank = SPLIT ? d.sc.l_done : d.sc.r_done;
   const u32* meta_n = SPLIT ? d.sc.l_meta_n : d.sc.r_meta_n;
@@ -2560,8 +2563,8 @@ struct DenseScan {
   u64 out_payload;
   bool split = false;  // split placement: stands down on the errors raised before the fork
   __device__ u64 size(const Ctl* ctl) const {
-    return (ctl->skip_dense || (split ? ctl->pre_err : ctl->batch_err)) ? 0
-                                                                         : ctl->dense_total + ctl->chain_total;
+    if (split) return (ctl->skip_dense || ctl->pre_err) ? 0 : ctl->leaf_dense_total;
+    return (ctl->skip_dense || ctl->batch_err) ? 0 : ctl->dense_total + ctl->chain_total;
   }
   __device__ u64 value(u64 j) const {
     uint4 v = dense[j];
@@ -2631,7 +2634,7 @@ __global__ void __launch_bounds__(kThreads, 8) k_gather(Dev d, Batch bv) {
   const int lane = threadIdx.x & 31, sub = lane % kSpanLanes, grp = lane / kSpanLanes;
   constexpr int kGroups = 32 / kSpanLanes;
   const u32 ep = ctl->epoch;
-  const u64 total = ctl->dense_total;
+  const u64 total = d.split ? ctl->leaf_dense_total : ctl->dense_total;
   const u64 base = ctl->pay_base;
   const u64 cap = d.cfg.out_payload;
   int32_t* __restrict__ out = d.out_pay;
@@ -3379,8 +3382,8 @@ void enqueue_batch(Pipeline& p, const Batch& bt) {
       launch_pdl(k_leaf_rank, dgrid, kThreads, 0, p.s2, d);
       {
         const u32* nl = &d.ctl->n_done_leaf;
-        CountScan l0{d.sc.l_dense_n, d.sc.l_dense_base, nl, dcap, 0};
-        CountScan l1{d.sc.l_meta_n, d.sc.l_arena_base, nl, dcap, 2};
+        CountScan l0{d.sc.l_dense_n, d.sc.l_dense_base, nl, dcap, 4};
+        CountScan l1{d.sc.l_meta_n, d.sc.l_arena_base, nl, dcap, 5};
         CountScan l2{nullptr, nullptr, nl, 0, 3};
         launch_scan3(p.lbs2, d.ctl, l0, l1, l2, std::min<u64>(dcap, nb), kSplitSite + 1, spin, p.s2,
                      LeafCheck{d.cfg.dense_cap});

@@ -53,6 +53,8 @@ struct Ctl {
                            // split placement that check leaves skip_dense to the placement's own)
   int pre_err;             // split placement: batch_err as the leaf finalize left it
   u32 n_done_leaf;         // split placement: leaf parents completed (done list 0..n-1)
+  u64 leaf_dense_total;    // split placement: its own totals (the record scans beside it
+  u64 leaf_arena_total;    // write dense_total and arena_total, which it never reads)
   u32 fin_ctr;             // split placement: leaf finalize CTAs finished
   u32 last_ctr2;           // as last_ctr, for the split placement's scans
   u64 dense_total;         // children of CONCAT groups completing in this batch
